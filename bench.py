@@ -1,0 +1,387 @@
+#!/usr/bin/env python
+"""Throughput of the flow-matching denoise of the pi0.5-shaped action expert on GB300.
+
+One step = one jpi_denoise call: a full 10-step Euler denoise of one 50 x 32 action chunk at
+batch 1 over an 816-token prefix KV (18 layers, width 1024, 8 x 256 heads, GeGLU 4096, bf16
+weights). Inputs are seeded synthetic tensors already resident in HBM when the timed region
+starts; every call streams 6.2 GB of weights, far more than the 129 MB L2, so no flush is
+needed between iterations.
+
+Prints one JSON line (rank 0). `--impl reference` times the fp64 CPU oracle instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "action chunks/s (10-step denoise, batch 1, pi0.5-shaped expert)"
+UNIT = "chunks/s"
+WORKLOAD = dict(batch=1, prefix=816, chunk=50, steps=10)
+WORKLOAD_NAME = ("pi0.5-shaped action expert (18 x W1024, 8x256 heads, 1 KV head, GeGLU 4096), "
+                 "batch 1, prefix 816, chunk 50 x 32, 10 Euler steps")
+OP_NAMES = {2: "norm+qkv+rope", 3: "attention", 4: "o_proj+residual", 5: "norm+gate_up+geglu",
+            6: "down_proj+residual"}
+
+# DRAM bytes per launch from an ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
+# valid only while the kernel sources hash to `source_sha256`.
+NCU_TRAFFIC = {}
+
+
+def source_sha() -> str:
+    d = os.path.join(ROOT, "paper_2607_12659_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in sorted(os.listdir(d)):
+        if f.endswith((".cu", ".h")):
+            h.update(open(os.path.join(d, f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def algorithmic_bytes(cfg, B, P, C, N):
+    """Bytes an ideal denoise must move: weights once per step (bf16), the time/modulation
+    weights once per call, the prefix KV once, inputs and outputs."""
+    W, H, D, F, L, A = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim, cfg.n_layers, cfg.action_dim
+    per_step = (L * (H * D * W * 2 + 2 * D * W + 3 * F * W) + (cfg.state_dim + 2 * A) * W) * 2
+    time_w = (W * cfg.time_dim + W * W + (6 * L + 2) * W * W) * 2
+    kv = B * L * P * D * 2 * 2
+    io = B * (cfg.state_dim + 2 * C * A) * 4
+    return N * per_step + time_w + kv + io
+
+
+def op_bytes(cfg, op, B, P, C):
+    """Algorithmic bytes of one launch of a layer op (weights + activation reads/writes)."""
+    W, H, D, F = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim
+    Mt = B * (C + 1)
+    if op == 2:
+        return (H + 2) * D * W * 2 + Mt * W * 4 + Mt * (H + 2) * D * 2
+    if op == 3:
+        return B * (P + C + 1) * D * 2 * 2 + Mt * H * D * 2 * 2
+    if op == 4:
+        return W * H * D * 2 + Mt * H * D * 2 + Mt * W * 4 * 2
+    if op == 5:
+        return 2 * F * W * 2 + Mt * W * 4 + Mt * F * 2
+    if op == 6:
+        return F * W * 2 + Mt * F * 2 + Mt * W * 4 * 2
+    raise ValueError(op)
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["hbm_gbs"], d.get("bf16_tflops"), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in getattr(self, "lines", []):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_baseline_child():
+    """Times the fp64 oracle on one full request of the workload (runs in a subprocess whose
+    BLAS thread count is fixed by the parent)."""
+    import numpy as np
+    import oracle
+    from synth import PI05, make_requests, make_weights
+    B, P, C, N = (WORKLOAD[k] for k in ("batch", "prefix", "chunk", "steps"))
+    w = oracle.to_f64(make_weights(PI05, 2000))
+    r = make_requests(PI05, 2001, 1, P, C)
+    args = (r["prefix_k"][:, 0].astype(np.float64), r["prefix_v"][:, 0].astype(np.float64), w, PI05)
+    oracle.expert_forward(r["noise"][0].astype(np.float64), r["state"][0].astype(np.float64), 0.0, *args)
+    t0 = time.perf_counter()
+    oracle.denoise(r["noise"][0], r["state"][0].astype(np.float64), N, *args)
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt}))
+
+
+def run_cpu_baseline(cores: int) -> dict:
+    env = dict(os.environ, OPENBLAS_NUM_THREADS=str(cores), OMP_NUM_THREADS=str(cores),
+               MKL_NUM_THREADS=str(cores))
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-baseline-child"],
+                       capture_output=True, text=True, env=env, timeout=900)
+    if r.returncode != 0:
+        return {"value": None, "unit": UNIT, "cores": cores, "kind": "oracle",
+                "sample": "failed: " + r.stderr.strip().splitlines()[-1][:200] if r.stderr else "failed"}
+    sec = json.loads(r.stdout.strip().splitlines()[-1])["seconds"]
+    return {"value": 1.0 / sec, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"one full request: 10-step denoise at batch 1 (P 816, C 50), fp64 numpy "
+                      f"oracle, {sec:.2f} s"}
+
+
+def reference_arm(args):
+    """The fp64 CPU oracle on this host's cores; a step is one Euler step (one expert pass)
+    of the batch-1 workload, and chunks/s = 1 / (10 x mean step time)."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import numpy as np
+    import oracle
+    from synth import PI05, make_requests, make_weights
+    cores = os.cpu_count() or 1
+    B, P, C, N = (WORKLOAD[k] for k in ("batch", "prefix", "chunk", "steps"))
+    w = oracle.to_f64(make_weights(PI05, 2000))
+    r = make_requests(PI05, 2001, 1, P, C)
+    a = (r["prefix_k"][:, 0].astype(np.float64), r["prefix_v"][:, 0].astype(np.float64), w, PI05)
+    x, s = r["noise"][0].astype(np.float64), r["state"][0].astype(np.float64)
+    times = []
+    for i in range(args.warmup + args.steps):
+        t = (i % N) / N
+        t0 = time.perf_counter()
+        x = x + (1.0 / N) * oracle.expert_forward(x, s, t, *a)
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    step = statistics.mean(times)
+    value = 1.0 / (N * step)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD_NAME, **WORKLOAD,
+                   "reference_step": "one Euler step (one expert pass) of the workload"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"{args.steps} Euler steps of one batch-1 request, fp64 numpy oracle"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def our_arm(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_12659_gb300 import build, jpi
+    from synth import PI05, make_requests, make_weights
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if rank == 0:
+        build.build()
+    if world > 1:
+        dist.barrier()
+    jpi.load()
+
+    B, P, C, N = (WORKLOAD[k] for k in ("batch", "prefix", "chunk", "steps"))
+    cfg = PI05
+    w = make_weights(cfg, 2000)
+    ex = jpi.Expert(cfg, w, max_batch=B, max_prefix=P, max_chunk=C, max_steps=N)
+    del w
+    r = make_requests(cfg, 2001 + rank, B, P, C)
+    ex.set_prefix_kv(torch.from_numpy(r["prefix_k"]).cuda().to(torch.bfloat16),
+                     torch.from_numpy(r["prefix_v"]).cuda().to(torch.bfloat16))
+    state = torch.from_numpy(r["state"]).cuda()
+    noise = torch.from_numpy(r["noise"]).cuda()
+    out = torch.empty_like(noise)
+    stream = torch.cuda.current_stream()
+
+    t0 = time.perf_counter()
+    ex.denoise(state, noise, N, out)              # first call captures the graph
+    torch.cuda.synchronize()
+    capture_s = time.perf_counter() - t0
+    for _ in range(max(args.warmup - 1, 0)):
+        ex.denoise(state, noise, N, out)
+    torch.cuda.synchronize()
+    ex.device_status()
+
+    # ---- timed region: K denoise calls, device events on the launching stream ----
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        evs[0].record(stream)
+        for i in range(args.steps):
+            ex.denoise(state, noise, N, out)
+            evs[i + 1].record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
+    total_ms = evs[0].elapsed_time(evs[-1])
+    ex.device_status()
+    t_max = total_ms
+    if world > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        t_max = float(t.item())
+    ms_per_step = t_max / args.steps
+    value = world * B * args.steps / (t_max / 1e3)
+
+    # ---- end to end through the host-buffer entry point (pinned host memory) ----
+    hs = torch.from_numpy(r["state"]).pin_memory()
+    hn = torch.from_numpy(r["noise"]).pin_memory()
+    ho = torch.empty_like(hn).pin_memory()
+    hs_np, hn_np, ho_np = hs.numpy(), hn.numpy(), ho.numpy()
+    for _ in range(2):
+        ex.denoise_host(hs_np, hn_np, N, ho_np)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        ex.denoise_host(hs_np, hn_np, N, ho_np)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([e2e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = world * B * args.steps / (e2e_ms / 1e3)
+    same = bool(np.array_equal(ho_np, out.cpu().numpy()))
+
+    # ---- per-op durations (each op alone, back to back, events on the launching stream) ----
+    reps = 20
+    op_ms = {}
+    for op in OP_NAMES:
+        jpi.jpi_profile_op(ex.handle, op, 0, B, C, N, 3, stream)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        jpi.jpi_profile_op(ex.handle, op, 0, B, C, N, reps, stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        op_ms[op] = a.elapsed_time(b) / reps
+    dom = max(op_ms, key=op_ms.get)
+    hbm_peak, tc_peak, peak_src = measured_peaks()
+    dom_bytes = op_bytes(cfg, dom, B, P, C)
+    achieved = dom_bytes / (op_ms[dom] * 1e-3) / 1e9
+    sha = source_sha()
+    tr = NCU_TRAFFIC.get(OP_NAMES[dom])
+    traffic = tr["bytes"] if tr and tr.get("source_sha256") == sha else None
+
+    n_kernels = ctypes_count(jpi, ex, B, C, N)
+    alg = algorithmic_bytes(cfg, B, P, C, N)
+    path_bw = alg / (ms_per_step * 1e-3) / 1e9
+
+    if rank == 0:
+        cpu = run_cpu_baseline(os.cpu_count() or 1) if world == 1 and not args.no_cpu_baseline else None
+        clocks = clk.summary()
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD_NAME, **WORKLOAD,
+                       "l2": "no flush: each call streams 6.2 GB of weights (> 129 MB L2)",
+                       "parallelism": f"replicas x{world}"},
+            "us_per_denoise": {"median": statistics.median(per) * 1e3,
+                               "p10": sorted(per)[max(0, int(0.1 * len(per)) - 0)] * 1e3,
+                               "p90": sorted(per)[min(len(per) - 1, int(0.9 * len(per)))] * 1e3},
+            "path_roofline": {"bound": "hbm", "algorithmic_bytes": alg, "achieved_gbs": path_bw,
+                              "peak_gbs": hbm_peak, "frac": path_bw / hbm_peak,
+                              "roofline_us": alg / hbm_peak / 1e3},
+            "roofline": {"bound": "hbm", "kernel": OP_NAMES[dom], "achieved": achieved,
+                         "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+                         "traffic": traffic, "peak_source": peak_src,
+                         "bytes_per_launch": dom_bytes, "us_per_launch": op_ms[dom] * 1e3},
+            "op_us": {OP_NAMES[k]: v * 1e3 for k, v in op_ms.items()},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": UNIT,
+                    "h2d_bytes_per_step": int(hs.numel() * 4 + hn.numel() * 4),
+                    "d2h_bytes_per_step": int(ho.numel() * 4), "matches_device_path": same},
+            "gpu_launches": n_kernels * args.steps,
+            "kernels_per_denoise": n_kernels,
+            "graph_capture_s": capture_s,
+            "clocks": clocks,
+            "source_sha256": sha,
+        }
+        print(json.dumps(line), flush=True)
+    ex.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def ctypes_count(jpi, ex, B, C, N) -> int:
+    import ctypes
+    cnt = ctypes.c_int()
+    jpi._check(jpi.load().jpi_graph_kernel_count(ex.handle, B, C, N, ctypes.byref(cnt)),
+               "jpi_graph_kernel_count")
+    return cnt.value
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-baseline-child", action="store_true", help=argparse.SUPPRESS)
+    args = ap.parse_args()
+    if args.cpu_baseline_child:
+        cpu_baseline_child()
+        return
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        our_arm(args)
+
+
+if __name__ == "__main__":
+    main()

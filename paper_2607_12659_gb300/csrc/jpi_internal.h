@@ -1,0 +1,156 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+#include <cstddef>
+#include <map>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "../../include/jpi.h"
+
+namespace jpi {
+
+// Last-error message of the calling host thread.
+void set_error(const char* fmt, ...);
+void clear_error();
+
+#define JPI_CUDA_TRY(expr)                                                        \
+    do {                                                                          \
+        cudaError_t e_ = (expr);                                                  \
+        if (e_ != cudaSuccess) {                                                  \
+            ::jpi::set_error("%s failed: %s (%s:%d)", #expr, cudaGetErrorString(e_), \
+                             __FILE__, __LINE__);                                 \
+            return JPI_ERR_CUDA;                                                  \
+        }                                                                         \
+    } while (0)
+
+#define JPI_TRY(expr)                        \
+    do {                                     \
+        jpi_status s_ = (expr);              \
+        if (s_ != JPI_OK) return s_;         \
+    } while (0)
+
+// Device error codes written by bounded waits inside kernels (first writer wins).
+enum DeviceError : int {
+    DEV_OK = 0,
+    DEV_TIMEOUT_WEIGHTS = 1,   // weight tile TMA never completed
+    DEV_TIMEOUT_MMA = 2,       // tensor-core commit never arrived
+    DEV_BAD_SHAPE = 3,         // a kernel saw a shape it cannot tile
+};
+
+// Offsets (in rows of W) of the modulation vectors inside one step's modulation row block.
+// Layer l: attention (sigma, beta, gamma) at 6 l + {0,1,2}, MLP at 6 l + {3,4,5};
+// the final norm's (sigma, beta) at 6 L + {0, 1}.
+inline int mod_rows(int L) { return 6 * L + 2; }
+
+// Plain (un-tiled) layer weights used by the CUDA-core kernels.
+struct LayerPlain {
+    void* wqkv;   // [(H+2) D][W]: rows of wq, then wk, then wv
+    void* wo;     // [W][H D]
+    void* wg;     // [F][W]
+    void* wu;     // [F][W]
+    void* wd;     // [W][F]
+};
+
+// Tensor-core (tcgen05) layer weights: tiles of 128 rows x 64 K-elements (16 KiB of bf16),
+// stored tile-contiguously in [row tile][k block] order so that one bulk tensor copy moves one
+// contiguous tile. Row order inside the QKV and gate/up matrices is permuted so that the rows
+// an epilogue pairs (the two halves of a rotary pair, or a gate row and its up row) sit in
+// rows r and r + 64 of the same tile.
+struct LayerTiled {
+    __nv_bfloat16* qkv;    // [(H+2) D / 128 tiles][W / 64][128][64]
+    __nv_bfloat16* o;      // [W / 128][H D / 64][128][64]
+    __nv_bfloat16* gu;     // [2 F / 128][W / 64][128][64]
+    __nv_bfloat16* down;   // [W / 128][F / 64][128][64]
+};
+
+struct GraphKey {
+    int batch, chunk, steps, prefix;
+    bool operator<(const GraphKey& o) const {
+        return std::tie(batch, chunk, steps, prefix) < std::tie(o.batch, o.chunk, o.steps, o.prefix);
+    }
+};
+
+}  // namespace jpi
+
+struct jpi_handle {
+    jpi_config cfg;
+    int device = 0;
+    bool bf16 = true;
+    bool tc = false;          // tensor-core kernels in use (bf16 mode with supported dims)
+
+    // Dimensions.
+    int L, W, H, D, F, A, Sd, dt, HD, QKV;   // QKV = (H + 2) D
+    int maxB, maxP, maxC, maxS, maxN, maxMt, kv_rows;
+
+    // ---- Device memory (all allocated in create) ----
+    std::vector<void*> allocations;
+    size_t device_bytes = 0;
+
+    // Weights. Element type is bf16 in JPI_BF16 mode, fp32 in JPI_FP32 mode ("TW").
+    std::vector<jpi::LayerPlain> plain;
+    std::vector<jpi::LayerTiled> tiled;
+    void* mod_w = nullptr;       // [(6L+2) W][W] TW, all modulation matrices stacked
+    float* mod_b = nullptr;      // [(6L+2) W]
+    void* time_in_w = nullptr;   // [W][d_t] TW
+    float* time_in_b = nullptr;  // [W]
+    void* time_out_w = nullptr;  // [W][W] TW
+    float* time_out_b = nullptr; // [W]
+    float* state_in_w = nullptr; // [W][S_d] fp32
+    float* state_in_b = nullptr;
+    float* action_in_w = nullptr;   // [W][A] fp32
+    float* action_in_b = nullptr;
+    float* action_out_w = nullptr;  // [A][W] fp32
+    float* action_out_b = nullptr;
+    float2* rope_tab = nullptr;     // [maxP + maxS][D/2] (cos, sin); null when rope_base == 0
+
+    // KV store: [L][maxB][kv_rows][D], element type TW; rows 0..P-1 prefix, P..P+S-1 suffix.
+    void* kv_k = nullptr;
+    void* kv_v = nullptr;
+
+    // Activations.
+    float* h = nullptr;         // [maxMt][W] residual stream
+    float* x = nullptr;         // [maxB][maxC][A] current actions
+    float* state = nullptr;     // [maxB][S_d] staged state
+    float* out = nullptr;       // [maxB][maxC][A] staged output
+    float* temb = nullptr;      // [maxN][d_t] time embeddings
+    float* c1 = nullptr;        // [maxN][W]
+    float* cond = nullptr;      // [maxN][W]
+    float* mods = nullptr;      // [maxN][(6L+2) W]
+    void* act = nullptr;        // [maxMt][max(W, F)] GEMM input (TW type)
+    float* qkv = nullptr;       // [maxMt][QKV] raw projections (CUDA-core path)
+    void* q = nullptr;          // [maxMt][H][D] rotated queries (TW type)
+    void* o = nullptr;          // [maxMt][H D] attention output (TW type)
+    void* z = nullptr;          // [maxMt][F] GeGLU output (TW type)
+    int* dev_err = nullptr;     // device error word
+
+    // State.
+    int cur_batch = 0, cur_prefix = 0;
+    bool prefix_ready = false;
+    cudaStream_t cap_stream = nullptr;
+    std::map<jpi::GraphKey, cudaGraphExec_t> graphs;
+    std::map<jpi::GraphKey, int> graph_kernels;
+};
+
+namespace jpi {
+
+// Kernel launchers (kernels_simt.cu). All enqueue on `st` and return JPI_OK or JPI_ERR_CUDA.
+jpi_status configure_simt_kernels(jpi_handle* h);
+jpi_status launch_time_embed(jpi_handle* h, int nsteps, double t_override, cudaStream_t st);
+jpi_status launch_time_conditioning(jpi_handle* h, int nsteps, cudaStream_t st);
+jpi_status launch_embed(jpi_handle* h, int batch, int chunk, const float* x, cudaStream_t st);
+jpi_status launch_layer_simt(jpi_handle* h, int layer, int step, int batch, int chunk,
+                             cudaStream_t st);
+// One sub-step of a layer (ops 2..6 of jpi_profile_op).
+jpi_status launch_op_simt(jpi_handle* h, int op, int layer, int step, int batch, int chunk,
+                          cudaStream_t st);
+jpi_status launch_final(jpi_handle* h, int step, int batch, int chunk, float delta,
+                        float* x_inout, float* v_out, float* out_copy, cudaStream_t st);
+jpi_status launch_convert_kv(jpi_handle* h, const void* src, int src_fp32, void* dst,
+                             int batch, int prefix_len, cudaStream_t st);
+
+}  // namespace jpi

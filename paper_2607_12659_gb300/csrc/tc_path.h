@@ -1,0 +1,22 @@
+// Tensor-core (tcgen05 + TMA) path of the bf16 expert layers.
+#pragma once
+#include "jpi_internal.h"
+
+namespace jpi {
+
+// True when the handle's dimensions are tiled by the tensor-core kernels.
+bool tc_supported(const jpi_handle* h);
+// Packs the per-layer projection/MLP matrices into the tiled bf16 layout (see LayerTiled).
+jpi_status tc_pack_layers(jpi_handle* h, const jpi_weights* w, float* tmp, bool on_device);
+// Builds tensor maps, workspaces and kernel attributes once the buffers exist.
+jpi_status tc_prepare(jpi_handle* h);
+// Enqueues one expert layer (norm + QKV + rotary, attention, O-proj, norm + GeGLU, down).
+jpi_status tc_launch_layer(jpi_handle* h, int layer, int step, int batch, int chunk,
+                           cudaStream_t st);
+// One sub-step of a layer (ops 2..6 of jpi_profile_op).
+jpi_status tc_launch_op(jpi_handle* h, int op, int layer, int step, int batch, int chunk,
+                        cudaStream_t st);
+// Frees what tc_prepare created outside the handle's allocation list.
+void tc_release(jpi_handle* h);
+
+}  // namespace jpi

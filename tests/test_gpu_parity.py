@@ -1,0 +1,170 @@
+"""Parity of the CUDA path (through the C-ABI) with the fp64 CPU oracle on seeded inputs.
+
+Configurations: the tiny fp32 expert; a small bf16 expert spanning several weight tiles with
+ragged token counts; the pi0.5-shaped expert at batch 1 (816-token prefix, 50 x 32 chunk,
+10 steps); its sweep over prefix length, chunk and step count; batches 4/8/16 with
+per-request prefixes; and batch 64 with 2048-token prefixes (sampled requests).
+"""
+
+import numpy as np
+import pytest
+
+import oracle
+from synth import PI05, TINY, make_requests, make_weights
+from tests.gpu_util import (SMALL_BF16, assert_close, errors, gpu_denoise, lib, make_expert,
+                            oracle_denoise, to_dev_kv)
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.fail("the gpu tests need a CUDA device")
+    torch.cuda.set_device(0)
+    lib()
+
+
+# ------------------------------------------------------------------ tiny fp32 (verification mode)
+
+@pytest.fixture(scope="module")
+def tiny():
+    w = make_weights(TINY, 0)
+    ex = make_expert(TINY, w, max_batch=3, max_prefix=64, max_chunk=8, max_steps=4)
+    yield w, ex
+    ex.close()
+
+
+def test_tiny_fp32_denoise(tiny):
+    w, ex = tiny
+    r = make_requests(TINY, 1, 1, 64, 8)
+    got = gpu_denoise(ex, TINY, r, 4)
+    assert_close(got, oracle_denoise(TINY, w, r, 4), TINY, "tiny fp32")
+
+
+@pytest.mark.parametrize("B,P,C,N", [(1, 1, 1, 1), (2, 63, 5, 3), (3, 17, 8, 2)])
+def test_tiny_fp32_ragged_shapes(tiny, B, P, C, N):
+    w, ex = tiny
+    r = make_requests(TINY, 7, B, P, C)
+    got = gpu_denoise(ex, TINY, r, N)
+    assert_close(got, oracle_denoise(TINY, w, r, N), TINY, f"tiny fp32 B{B} P{P} C{C} N{N}")
+
+
+def test_tiny_fp32_forward_velocity_and_hidden(tiny):
+    w, ex = tiny
+    r = make_requests(TINY, 3, 2, 40, 6)
+    k, v = to_dev_kv(r, TINY)
+    ex.set_prefix_kv(k, v)
+    x = torch.from_numpy(r["noise"]).cuda()
+    vel, hres = ex.forward(torch.from_numpy(r["state"]).cuda(), x, 0.37)
+    torch.cuda.synchronize()
+    ref_v, ref_h = oracle.forward_batch(r["noise"], r["state"], 0.37, r["prefix_k"], r["prefix_v"], w, TINY)
+    assert_close(vel.cpu().numpy(), ref_v, TINY, "forward v")
+    scale = np.abs(ref_h).max()
+    assert np.abs(hres.cpu().numpy() - ref_h).max() <= 1e-4 * max(1.0, scale)
+
+
+# ------------------------------------------------------------------ small bf16, several tiles
+
+@pytest.fixture(scope="module")
+def small():
+    w = make_weights(SMALL_BF16, 11, mod_bias_std=0.5)
+    ex = make_expert(SMALL_BF16, w, max_batch=5, max_prefix=300, max_chunk=70, max_steps=6)
+    yield w, ex
+    ex.close()
+
+
+@pytest.mark.parametrize("B,P,C,N", [(1, 100, 13, 3), (2, 257, 50, 2), (5, 64, 70, 1), (3, 1, 1, 4)])
+def test_small_bf16_denoise(small, B, P, C, N):
+    w, ex = small
+    r = make_requests(SMALL_BF16, 12, B, P, C)
+    got = gpu_denoise(ex, SMALL_BF16, r, N)
+    assert_close(got, oracle_denoise(SMALL_BF16, w, r, N), SMALL_BF16, f"small bf16 B{B} P{P} C{C} N{N}")
+
+
+def test_small_bf16_forward_hidden_state(small):
+    w, ex = small
+    r = make_requests(SMALL_BF16, 13, 2, 150, 20)
+    k, v = to_dev_kv(r, SMALL_BF16)
+    ex.set_prefix_kv(k, v)
+    vel, hres = ex.forward(torch.from_numpy(r["state"]).cuda(), torch.from_numpy(r["noise"]).cuda(), 0.55)
+    torch.cuda.synchronize()
+    ref_v, ref_h = oracle.forward_batch(r["noise"], r["state"], 0.55, r["prefix_k"], r["prefix_v"], w, SMALL_BF16)
+    assert_close(vel.cpu().numpy(), ref_v, SMALL_BF16, "small forward v")
+    _, rel = errors(hres.cpu().numpy(), ref_h)
+    assert rel <= 1e-2, f"hidden state rel-L2 {rel:.3g}"
+
+
+# ------------------------------------------------------------------ pi0.5-shaped expert
+
+@pytest.fixture(scope="module")
+def pi05():
+    w = oracle.to_f64(make_weights(PI05, 2000))
+    w32 = {k: v for k, v in w.items() if k != "__f64__"}
+    ex = make_expert(PI05, w32, max_batch=16, max_prefix=1536, max_chunk=50, max_steps=10)
+    yield w, ex
+    ex.close()
+
+
+def test_pi05_batch1_prefix816_chunk50_steps10(pi05):
+    w, ex = pi05
+    r = make_requests(PI05, 2001, 1, 816, 50)
+    got = gpu_denoise(ex, PI05, r, 10)
+    max_abs, rel = assert_close(got, oracle_denoise(PI05, w, r, 10), PI05, "pi0.5 B1 P816 C50 N10")
+    print(f"pi0.5 config: max-abs {max_abs:.3g} rel-L2 {rel:.3g}")
+
+
+@pytest.mark.parametrize("P", [256, 512, 816, 1536])
+@pytest.mark.parametrize("C", [10, 50])
+@pytest.mark.parametrize("N", [1, 5, 10])
+def test_pi05_sweep(pi05, P, C, N):
+    w, ex = pi05
+    r = make_requests(PI05, 3000 + P + C + N, 1, P, C)
+    got = gpu_denoise(ex, PI05, r, N)
+    assert_close(got, oracle_denoise(PI05, w, r, N), PI05, f"sweep P{P} C{C} N{N}")
+
+
+@pytest.mark.parametrize("B", [4, 8, 16])
+def test_pi05_batches_sampled_requests(pi05, B):
+    w, ex = pi05
+    r = make_requests(PI05, 4000 + B, B, 816, 50)
+    got = gpu_denoise(ex, PI05, r, 10)
+    sample = sorted({0, B // 2, B - 1})
+    assert_close(got[sample], oracle_denoise(PI05, w, r, 10, sample), PI05, f"batch {B}")
+    # Batch independence: request b alone gives the same actions as inside the batch.
+    b = B - 1
+    r1 = make_requests(PI05, 4000 + B, 1, 816, 50, first_request=b)
+    one = gpu_denoise(ex, PI05, r1, 10)
+    assert np.abs(one[0] - got[b]).max() <= 1e-5
+
+
+def test_pi05_high_gain_forward():
+    """Gates of O(1) (modulation biases ~N(0,1)) so every sublayer visibly moves the output."""
+    w = make_weights(PI05.with_(n_layers=4), 2100, mod_bias_std=1.0)
+    cfg = PI05.with_(n_layers=4)
+    ex = make_expert(cfg, w, max_batch=2, max_prefix=816, max_chunk=50, max_steps=1)
+    try:
+        r = make_requests(cfg, 2101, 2, 816, 50)
+        k, v = to_dev_kv(r, cfg)
+        ex.set_prefix_kv(k, v)
+        vel, hres = ex.forward(torch.from_numpy(r["state"]).cuda(), torch.from_numpy(r["noise"]).cuda(), 0.3)
+        torch.cuda.synchronize()
+        ref_v, ref_h = oracle.forward_batch(r["noise"], r["state"], 0.3, r["prefix_k"], r["prefix_v"], w, cfg)
+        assert_close(vel.cpu().numpy(), ref_v, cfg, "high-gain forward v")
+        _, rel = errors(hres.cpu().numpy(), ref_h)
+        assert rel <= 1e-2, f"high-gain hidden rel-L2 {rel:.3g}"
+    finally:
+        ex.close()
+
+
+def test_pi05_batch64_prefix2048_sampled():
+    w = make_weights(PI05, 2000)
+    ex = make_expert(PI05, w, max_batch=64, max_prefix=2048, max_chunk=50, max_steps=10)
+    try:
+        r = make_requests(PI05, 5000, 64, 2048, 50)
+        got = gpu_denoise(ex, PI05, r, 10)
+        sample = [0, 21, 42, 63]
+        assert_close(got[sample], oracle_denoise(PI05, w, r, 10, sample), PI05, "batch 64 P2048")
+    finally:
+        ex.close()
