@@ -93,13 +93,13 @@ def attention(q: np.ndarray, K: np.ndarray, V: np.ndarray, visible: np.ndarray) 
     App. A: queries come from the action-noise tokens, keys/values are the LLM layer's KV
     cache concatenated with the suffix tokens' own keys/values.
     """
-    D = q.shape[-1]
-    scores = np.einsum("shd,nd->shn", q, K) / np.sqrt(F64(D))
+    S, H, D = q.shape
+    scores = (q.reshape(S * H, D) @ K.T).reshape(S, H, -1) / np.sqrt(F64(D))
     scores = np.where(visible[:, None, :], scores, -np.inf)
     scores = scores - scores.max(axis=-1, keepdims=True)
     p = np.exp(scores)
     p = p / p.sum(axis=-1, keepdims=True)
-    return np.einsum("shn,nd->shd", p, V)
+    return (p.reshape(S * H, -1) @ V).reshape(S, H, D)
 
 
 def gelu_tanh(y: np.ndarray) -> np.ndarray:
@@ -168,10 +168,14 @@ def denoise(noise: np.ndarray, s: np.ndarray, num_steps: int, prefix_k: np.ndarr
 
 
 def to_f64(w: dict) -> dict:
-    """Weights as fp64 (per-layer lists preserved)."""
-    out = {}
-    for k, v in w.items():
-        out[k] = [np.asarray(a, F64) for a in v] if isinstance(v, list) else np.asarray(v, F64)
+    """Weights as fp64 (per-layer lists preserved); converts tensors on a few threads."""
+    from concurrent.futures import ThreadPoolExecutor
+    if w.get("__f64__"):
+        return w
+    with ThreadPoolExecutor(max_workers=8) as ex:
+        out = {k: (list(ex.map(lambda a: np.asarray(a, F64), v)) if isinstance(v, list)
+                   else np.asarray(v, F64)) for k, v in w.items()}
+    out["__f64__"] = True
     return out
 
 

@@ -6,8 +6,9 @@ models": 18 layers, width 1024, 8 heads x 256) and its LLM prefix (Gemma 2B, 256
 seed fixes every value bit for bit on any machine.
 
 Draw order (fixed, part of the input recipe):
-  weights: Generator(PCG64(seed)); the global tensors in ``GLOBAL_WEIGHTS`` order, then for
-           each layer the tensors in ``LAYER_WEIGHTS`` order.
+  weights: tensor j in the order "global tensors in ``GLOBAL_WEIGHTS`` order, then for each
+           layer the tensors in ``LAYER_WEIGHTS`` order" is drawn from its own
+           Generator(PCG64([seed, j])) (independent streams, so tensors are drawn in parallel).
   request b: Generator(PCG64([seed, b])); prefix K for every layer, prefix V for every layer,
            then the state vector, then the action noise.
 Weight matrices are N(0, std^2); biases N(0, bias_std^2) (the three modulation biases can be
@@ -20,6 +21,8 @@ exact values; biases, state and noise stay fp32.
 from __future__ import annotations
 
 from dataclasses import dataclass, replace
+
+from concurrent.futures import ThreadPoolExecutor
 
 import numpy as np
 
@@ -86,10 +89,11 @@ def weight_shapes(cfg: ExpertConfig) -> dict:
 
 
 def round_to_bf16(a: np.ndarray) -> np.ndarray:
-    """fp32 array whose values are ``a`` rounded to bf16 (nearest, ties to even)."""
-    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
-    return u.astype(np.uint32).view(np.float32)
+    """fp32 array whose values are ``a`` rounded to bf16 (nearest, ties to even); finite input."""
+    u = np.array(a, dtype=np.float32, copy=True).view(np.uint32)
+    u += np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))
+    u &= np.uint32(0xFFFF0000)
+    return u.view(np.float32)
 
 
 def _draw(rng: np.random.Generator, shape, std: float) -> np.ndarray:
@@ -109,21 +113,28 @@ def make_weights(cfg: ExpertConfig, seed: int, std: float = 0.02, bias_std: floa
     if mod_bias_std is None:
         mod_bias_std = bias_std
     shapes = weight_shapes(cfg)
-    rng = np.random.Generator(np.random.PCG64(seed))
     bf16 = cfg.precision == "bf16"
+    order = [(name, None) for name in GLOBAL_WEIGHTS] + [
+        (name, l) for l in range(cfg.n_layers) for name in LAYER_WEIGHTS]
 
-    def one(name):
+    def one(j):
+        name = order[j][0]
+        rng = np.random.Generator(np.random.PCG64([seed, j]))
         shp = shapes[name]
         if len(shp) == 2:
             x = _draw(rng, shp, std)
             return round_to_bf16(x) if bf16 else x
         return _draw(rng, shp, mod_bias_std if name in _MOD_BIASES else bias_std)
 
-    out = {name: one(name) for name in GLOBAL_WEIGHTS}
-    per_layer = {name: [] for name in LAYER_WEIGHTS}
-    for _ in range(cfg.n_layers):
-        for name in LAYER_WEIGHTS:
-            per_layer[name].append(one(name))
+    with ThreadPoolExecutor(max_workers=8) as ex:
+        arrays = list(ex.map(one, range(len(order))))
+    out = {}
+    per_layer = {name: [None] * cfg.n_layers for name in LAYER_WEIGHTS}
+    for (name, l), a in zip(order, arrays):
+        if l is None:
+            out[name] = a
+        else:
+            per_layer[name][l] = a
     out.update(per_layer)
     return out
 
@@ -141,7 +152,7 @@ def make_requests(cfg: ExpertConfig, seed: int, batch: int, prefix_len: int, chu
     V = np.empty((L, batch, prefix_len, D), np.float32)
     state = np.empty((batch, cfg.state_dim), np.float32)
     noise = np.empty((batch, chunk, cfg.action_dim), np.float32)
-    for b in range(batch):
+    def one(b):
         rng = np.random.Generator(np.random.PCG64([seed, first_request + b]))
         for l in range(L):
             K[l, b] = _draw(rng, (prefix_len, D), 1.0)
@@ -149,6 +160,9 @@ def make_requests(cfg: ExpertConfig, seed: int, batch: int, prefix_len: int, chu
             V[l, b] = _draw(rng, (prefix_len, D), 1.0)
         state[b] = _draw(rng, (cfg.state_dim,), 1.0)
         noise[b] = _draw(rng, (chunk, cfg.action_dim), 1.0)
+
+    with ThreadPoolExecutor(max_workers=8) as ex:
+        list(ex.map(one, range(batch)))
     if bf16:
         K = round_to_bf16(K)
         V = round_to_bf16(V)
