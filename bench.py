@@ -314,7 +314,7 @@ def our_arm(args):
     tr = NCU_TRAFFIC.get(OP_NAMES[dom])
     traffic = tr["bytes"] if tr and tr.get("source_sha256") == sha else None
 
-    n_kernels = ctypes_count(jpi, ex, B, C, N)
+    n_kernels = jpi.jpi_graph_kernel_count(ex.handle, B, C, N)
     alg = algorithmic_bytes(cfg, B, P, C, N)
     path_bw = alg / (ms_per_step * 1e-3) / 1e9
 
@@ -353,14 +353,6 @@ def our_arm(args):
     ex.close()
     if world > 1:
         dist.destroy_process_group()
-
-
-def ctypes_count(jpi, ex, B, C, N) -> int:
-    import ctypes
-    cnt = ctypes.c_int()
-    jpi._check(jpi.load().jpi_graph_kernel_count(ex.handle, B, C, N, ctypes.byref(cnt)),
-               "jpi_graph_kernel_count")
-    return cnt.value
 
 
 def main():

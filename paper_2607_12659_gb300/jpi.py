@@ -68,6 +68,8 @@ _SIGS = {
                            c_void_p, c_void_p],
     "jpi_device_status": [c_void_p],
     "jpi_memory_usage": [c_void_p, POINTER(c_longlong)],
+    "jpi_graph_kernel_count": [c_void_p, c_int, c_int, c_int, POINTER(c_int)],
+    "jpi_profile_op": [c_void_p, c_int, c_int, c_int, c_int, c_int, c_int, c_void_p],
 }
 
 _lib = None
@@ -173,6 +175,18 @@ def jpi_memory_usage(h) -> int:
     b = c_longlong()
     _check(load().jpi_memory_usage(h, byref(b)), "jpi_memory_usage")
     return b.value
+
+
+def jpi_graph_kernel_count(h, batch, chunk, num_steps) -> int:
+    n = c_int()
+    _check(load().jpi_graph_kernel_count(h, batch, chunk, num_steps, byref(n)),
+           "jpi_graph_kernel_count")
+    return n.value
+
+
+def jpi_profile_op(h, op, layer, batch, chunk, num_steps, reps, stream=None):
+    _check(load().jpi_profile_op(h, op, layer, batch, chunk, num_steps, reps, _stream(stream)),
+           "jpi_profile_op")
 
 
 def jpi_last_error() -> str:
