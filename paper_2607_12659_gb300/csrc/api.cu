@@ -131,6 +131,7 @@ jpi_status pack_weights(jpi_handle* h, const jpi_weights* w) {
     if ((size_t)F * W > maxe) maxe = (size_t)F * W;
     if ((size_t)HD * W > maxe) maxe = (size_t)HD * W;
     if ((size_t)W * dt > maxe) maxe = (size_t)W * dt;
+    if ((size_t)h->QKV * W > maxe) maxe = (size_t)h->QKV * W;
     if (!up.on_device || b16) JPI_TRY(dev_alloc(h, &up.tmp, maxe));
 
     // Small fp32 tensors.
@@ -222,6 +223,8 @@ jpi_status alloc_buffers(jpi_handle* h) {
     JPI_CUDA_TRY(cudaMemset(h->kv_k, 0, kv * ts));
     JPI_CUDA_TRY(cudaMemset(h->kv_v, 0, kv * ts));
     JPI_CUDA_TRY(cudaMemset(h->h, 0, Mt * W * sizeof(float)));
+    JPI_TRY(dev_alloc(h, &h->ss, (size_t)((W + 127) / 128) * Mt));
+    JPI_CUDA_TRY(cudaMemset(h->ss, 0, (size_t)((W + 127) / 128) * Mt * sizeof(float)));
     JPI_TRY(dev_alloc(h, &h->dev_err, 4));
     JPI_CUDA_TRY(cudaMemset(h->dev_err, 0, 4 * sizeof(int)));
     if (h->cfg.rope_base > 0.f) {

@@ -1,6 +1,7 @@
 // Internal declarations shared by the library's translation units.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <cstdint>
@@ -68,6 +69,13 @@ struct LayerTiled {
     __nv_bfloat16* down;   // [W / 128][F / 64][128][64]
 };
 
+// Work split of one tensor-core projection: `ntiles` 128-row weight tiles, each reduced over
+// K by a cluster of `splits` CTAs that own `kpb` 64-wide K blocks apiece.
+struct GemmPlan {
+    int rows = 0, K = 0, ntiles = 0, nkb = 0, kpb = 0, splits = 0, ctas = 0;
+    size_t smem = 0;
+};
+
 struct GraphKey {
     int batch, chunk, steps, prefix;
     bool operator<(const GraphKey& o) const {
@@ -82,6 +90,7 @@ struct jpi_handle {
     int device = 0;
     bool bf16 = true;
     bool tc = false;          // tensor-core kernels in use (bf16 mode with supported dims)
+    bool pdl = true;          // programmatic dependent launch between tensor-core kernels
 
     // Dimensions.
     int L, W, H, D, F, A, Sd, dt, HD, QKV;   // QKV = (H + 2) D
@@ -126,7 +135,12 @@ struct jpi_handle {
     void* q = nullptr;          // [maxMt][H][D] rotated queries (TW type)
     void* o = nullptr;          // [maxMt][H D] attention output (TW type)
     void* z = nullptr;          // [maxMt][F] GeGLU output (TW type)
+    float* ss = nullptr;        // [W / 128][maxMt] per-token sums of h^2 over 128-feature slices
     int* dev_err = nullptr;     // device error word
+
+    // Tensor-core path: plans and tensor maps (4 per layer: QKV, O, gate/up, down).
+    jpi::GemmPlan plans[4];
+    std::vector<CUtensorMap> tmaps;
 
     // State.
     int cur_batch = 0, cur_prefix = 0;

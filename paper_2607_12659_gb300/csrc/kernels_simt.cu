@@ -110,10 +110,13 @@ __global__ void k_gemv_multi(const TW* __restrict__ Wm, const float* __restrict_
 
 // ---------------------------------------------------------------------------------------------
 // Token embedding: row 0 of each request is the state token, rows 1..C the action tokens.
-__global__ void k_embed(float* __restrict__ hres, const float* __restrict__ state,
-                        const float* __restrict__ x, const float* __restrict__ Ws,
-                        const float* __restrict__ bs, const float* __restrict__ Wa,
-                        const float* __restrict__ ba, int S, int C, int W, int Sd, int A) {
+// Block = 128 features of one token; with `ss` it also writes that slice's sum of squares
+// (ss[slice][m]) for the next RMSNorm of the tensor-core path.
+__global__ void __launch_bounds__(128) k_embed(
+    float* __restrict__ hres, float* __restrict__ ss, int ss_ld, const float* __restrict__ state,
+    const float* __restrict__ x, const float* __restrict__ Ws, const float* __restrict__ bs,
+    const float* __restrict__ Wa, const float* __restrict__ ba, int S, int C, int W, int Sd, int A) {
+    __shared__ float scratch[32];
     const int m = blockIdx.y;
     const int b = m / S, i = m % S;
     const float* in;
@@ -125,10 +128,17 @@ __global__ void k_embed(float* __restrict__ hres, const float* __restrict__ stat
     } else {
         in = x + ((size_t)b * C + (i - 1)) * A; Wm = Wa; bias = ba; K = A;
     }
-    for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < W; n += gridDim.x * blockDim.x) {
+    const int n = blockIdx.x * 128 + threadIdx.x;
+    float v = 0.f;
+    if (n < W) {
         float acc = 0.f;
         for (int k = 0; k < K; ++k) acc = fmaf(Wm[(size_t)n * K + k], in[k], acc);
-        hres[(size_t)m * W + n] = acc + bias[n];
+        v = acc + bias[n];
+        hres[(size_t)m * W + n] = v;
+    }
+    if (ss) {
+        const float t = block_sum(v * v, scratch);
+        if (threadIdx.x == 0) ss[(size_t)blockIdx.x * ss_ld + m] = t;
     }
 }
 
@@ -384,7 +394,7 @@ template <typename T>
 jpi_status op_simt(jpi_handle* h, int op, int l, int step, int B, int C, cudaStream_t st) {
     const int S = C + 1, Mt = B * S, W = h->W, F = h->F, HD = h->HD, D = h->D;
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * W + (size_t)6 * l * W;
-    const LayerPlain& lw = h->plain[l];
+    const LayerPlain* lwp = (size_t)l < h->plain.size() ? &h->plain[l] : nullptr;
     T* act = (T*)h->act;
     const size_t kv_layer = (size_t)l * h->maxB * h->kv_rows * D;
     T* kst = (T*)h->kv_k + kv_layer;
@@ -392,11 +402,15 @@ jpi_status op_simt(jpi_handle* h, int op, int l, int step, int B, int C, cudaStr
     const float eps = h->cfg.rms_eps;
     const dim3 blk(256);
     const int mtiles = (Mt + GB_M - 1) / GB_M;
+    if (op != 3 && !lwp) {
+        set_error("layer %d has no CUDA-core weights", l);
+        return JPI_ERR_INVALID_ARG;
+    }
     switch (op) {
         case 2:
             k_rms_mod<T><<<Mt, blk, 0, st>>>(h->h, ms, ms + W, act, W, W, eps);
             k_gemm_simt<T, T, EPI_STORE><<<dim3((h->QKV + GB_N - 1) / GB_N, mtiles), blk, 0, st>>>(
-                act, W, (const T*)lw.wqkv, nullptr, Mt, h->QKV, W, h->qkv, h->QKV, nullptr, nullptr, 0);
+                act, W, (const T*)lwp->wqkv, nullptr, Mt, h->QKV, W, h->qkv, h->QKV, nullptr, nullptr, 0);
             k_qkv_post<T, T><<<Mt, blk, 0, st>>>(h->qkv, (T*)h->q, kst, vst, h->rope_tab, S, h->H, D,
                                                  h->cur_prefix, h->kv_rows);
             break;
@@ -409,16 +423,16 @@ jpi_status op_simt(jpi_handle* h, int op, int l, int step, int B, int C, cudaStr
         }
         case 4:
             k_gemm_simt<T, T, EPI_RESID><<<dim3((W + GB_N - 1) / GB_N, mtiles), blk, 0, st>>>(
-                (const T*)h->o, HD, (const T*)lw.wo, nullptr, Mt, W, HD, h->h, W, ms + 2 * W, nullptr, 0);
+                (const T*)h->o, HD, (const T*)lwp->wo, nullptr, Mt, W, HD, h->h, W, ms + 2 * W, nullptr, 0);
             break;
         case 5:
             k_rms_mod<T><<<Mt, blk, 0, st>>>(h->h, ms + 3 * W, ms + 4 * W, act, W, W, eps);
             k_gemm_simt<T, T, EPI_GEGLU><<<dim3((F + GB_N - 1) / GB_N, mtiles), blk, 0, st>>>(
-                act, W, (const T*)lw.wg, (const T*)lw.wu, Mt, F, W, nullptr, 0, nullptr, (T*)h->z, F);
+                act, W, (const T*)lwp->wg, (const T*)lwp->wu, Mt, F, W, nullptr, 0, nullptr, (T*)h->z, F);
             break;
         case 6:
             k_gemm_simt<T, T, EPI_RESID><<<dim3((W + GB_N - 1) / GB_N, mtiles), blk, 0, st>>>(
-                (const T*)h->z, F, (const T*)lw.wd, nullptr, Mt, W, F, h->h, W, ms + 5 * W, nullptr, 0);
+                (const T*)h->z, F, (const T*)lwp->wd, nullptr, Mt, W, F, h->h, W, ms + 5 * W, nullptr, 0);
             break;
         default:
             set_error("unknown layer op %d", op);
@@ -480,9 +494,9 @@ jpi_status launch_time_conditioning(jpi_handle* h, int nsteps, cudaStream_t st) 
 
 jpi_status launch_embed(jpi_handle* h, int B, int C, const float* x, cudaStream_t st) {
     const int S = C + 1;
-    k_embed<<<dim3((h->W + 255) / 256, B * S), 256, 0, st>>>(
-        h->h, h->state, x, h->state_in_w, h->state_in_b, h->action_in_w, h->action_in_b, S, C,
-        h->W, h->Sd, h->A);
+    k_embed<<<dim3((h->W + 127) / 128, B * S), 128, 0, st>>>(
+        h->h, h->tc ? h->ss : nullptr, h->maxMt, h->state, x, h->state_in_w, h->state_in_b,
+        h->action_in_w, h->action_in_b, S, C, h->W, h->Sd, h->A);
     return check_launch("embed");
 }
 
