@@ -101,7 +101,7 @@ inline void* tw_offset(const jpi_handle* h, void* base, size_t elems) {
 
 jpi_status check_config(const jpi_config* c) {
     if (!c) return fail(JPI_ERR_INVALID_ARG, "config is NULL");
-    if (c->n_layers < 1 || c->width < 32 || c->n_heads < 1 || c->head_dim < 32 ||
+    if (c->n_layers < 1 || c->width < 32 || c->width % 32 || c->n_heads < 1 || c->head_dim < 32 ||
         c->mlp_dim < 32 || c->action_dim < 1 || c->state_dim < 1 || c->time_dim < 4)
         return fail(JPI_ERR_INVALID_ARG, "config has a dimension below its minimum");
     if (c->n_kv_heads != 1) return fail(JPI_ERR_UNSUPPORTED, "n_kv_heads must be 1");
@@ -223,6 +223,8 @@ jpi_status alloc_buffers(jpi_handle* h) {
     JPI_CUDA_TRY(cudaMemset(h->kv_k, 0, kv * ts));
     JPI_CUDA_TRY(cudaMemset(h->kv_v, 0, kv * ts));
     JPI_CUDA_TRY(cudaMemset(h->h, 0, Mt * W * sizeof(float)));
+    JPI_TRY(dev_alloc(h, (char**)&h->hx, Mt * W * 2));
+    JPI_CUDA_TRY(cudaMemset(h->hx, 0, Mt * W * 2));
     JPI_TRY(dev_alloc(h, &h->ss, (size_t)((W + 127) / 128) * Mt));
     JPI_CUDA_TRY(cudaMemset(h->ss, 0, (size_t)((W + 127) / 128) * Mt * sizeof(float)));
     JPI_TRY(dev_alloc(h, &h->dev_err, 4));

@@ -1,0 +1,423 @@
+// Attention of the suffix queries over [prefix KV ; suffix KV] with one shared KV head, on
+// tensor cores (bf16 operands, fp32 accumulation and softmax).
+//
+// App. A of the paper: at every expert layer the queries come from the action-noise tokens
+// (here the state token and the C action tokens) and the keys/values are the matching LLM
+// layer's KV cache concatenated with the suffix tokens' own keys/values. With a single KV head
+// every query head of every suffix token attends to the same K/V rows, so one request's
+// S x H query rows form one dense [S*H][D] x [D][P+S] problem; rows are ordered token-major
+// (row = i * H + head). The state row (i = 0) sees the prefix and itself only.
+//
+// Grid: (64-row query blocks, key splits, requests). The key splits of one query block form a
+// thread-block cluster: each CTA runs an online softmax over its key range (blocks of 64 keys
+// staged in shared memory with cp.async), then the cluster combines the partial (max, sum,
+// output) triples through distributed shared memory in split order, so the result does not
+// depend on timing.
+
+#include "jpi_internal.h"
+#include "ptx.h"
+
+#include <cooperative_groups.h>
+
+namespace cg = cooperative_groups;
+
+namespace jpi {
+namespace {
+
+constexpr int AT_ROWS = 64;      // query rows per CTA (4 warps x 16)
+constexpr int AT_KEYS = 64;      // keys per shared-memory block
+constexpr int AT_THREADS = 128;
+constexpr int AT_MAX_SPLITS = 16;
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Byte offset of 16-byte chunk `c` of row `r` in a [rows][D] bf16 tile whose chunks are
+// XOR-swizzled by (r mod 8), so 8 rows read at one logical column hit 8 distinct bank groups.
+template <int D>
+__device__ __forceinline__ uint32_t sw_off(int r, int c) {
+    return (uint32_t)(r * (D * 2) + ((c ^ (r & 7)) << 4));
+}
+
+struct AttnArgs {
+    const __nv_bfloat16* q;     // [Mt][H][D]
+    const __nv_bfloat16* kst;   // [maxB][kv_rows][D] (this layer)
+    const __nv_bfloat16* vst;
+    __nv_bfloat16* o;           // [Mt][H * D]
+    int S, H, P, kv_rows, chunk, nsplit;
+    float scale_log2;           // log2(e) / sqrt(D)
+    int* err;
+};
+
+// Shared bytes of q/k/v, or of the 64 partial rows plus the received slices (at most
+// 64 + 15 rows: ceil(64 / splits) rows from each of up to 16 splits), whichever is larger.
+template <int D>
+__host__ __device__ constexpr int attn_region() {
+    return (3 * AT_ROWS * D * 2 > (2 * AT_ROWS + AT_MAX_SPLITS - 1) * (D + 4) * 4)
+               ? 3 * AT_ROWS * D * 2
+               : (2 * AT_ROWS + AT_MAX_SPLITS - 1) * (D + 4) * 4;
+}
+
+template <int D>
+__global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ AttnArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((128u - (ptx::smem_u32(smem_raw) & 127u)) & 127u);
+    uint8_t* qs = smem;                                  // [64][D] bf16
+    uint8_t* ks = qs + AT_ROWS * D * 2;                  // [64][D] bf16
+    uint8_t* vs = ks + AT_KEYS * D * 2;                  // [64][D] bf16
+    // After the key loop: this split's partial rows [64][D + 4] (O unnormalised, then m, l) over
+    // q/k, and the slices other splits send for the rows this CTA owns right after it.
+    float* opart = (float*)smem;
+    float* recv = opart + AT_ROWS * (D + 4);             // [splits][rows_per][D + 4]
+    float* coef = (float*)(smem + attn_region<D>());     // [64][AT_MAX_SPLITS]
+    uint64_t* rbar = (uint64_t*)(coef + AT_ROWS * AT_MAX_SPLITS);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int rb = blockIdx.x, split = blockIdx.y, b = blockIdx.z;
+    const int nrows = a.S * a.H, nk = a.P + a.S;
+    const int row0 = rb * AT_ROWS;
+    const int k_begin = split * a.chunk, k_end = min(nk, k_begin + a.chunk);
+    constexpr int DC = D / 8;                            // 16-byte chunks per row
+    if (tid == 0) {
+        ptx::mbar_init(rbar, 1);
+        ptx::fence_mbar_init();
+    }
+
+    // Prefix keys/values were written before this graph ran: the first block's prefix rows are
+    // fetched before the dependency wait; the suffix rows (written by the QKV kernel) after it.
+    const __nv_bfloat16* kb_ = a.kst + (size_t)b * a.kv_rows * D;
+    const __nv_bfloat16* vb_ = a.vst + (size_t)b * a.kv_rows * D;
+    const uint32_t qs_u = ptx::smem_u32(qs), ks_u = ptx::smem_u32(ks), vs_u = ptx::smem_u32(vs);
+    auto load_kv = [&](int key0, int r_from, int r_to) {
+        for (int idx = tid; idx < AT_KEYS * DC; idx += AT_THREADS) {
+            const int r = idx / DC, c = idx % DC;
+            if (r < r_from || r >= r_to) continue;
+            const bool ok = key0 + r < k_end;
+            const size_t off = (size_t)(ok ? key0 + r : 0) * D + c * 8;
+            cp_async16(ks_u + sw_off<D>(r, c), kb_ + off, ok);
+            cp_async16(vs_u + sw_off<D>(r, c), vb_ + off, ok);
+        }
+    };
+    const int first_suffix_row = min(AT_KEYS, max(0, a.P - k_begin));
+    load_kv(k_begin, 0, first_suffix_row);
+
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
+
+    // Query block (rows beyond this request's S*H rows are zero).
+    const __nv_bfloat16* qb = a.q + (size_t)b * nrows * D;
+    for (int idx = tid; idx < AT_ROWS * DC; idx += AT_THREADS) {
+        const int r = idx / DC, c = idx % DC;
+        const bool ok = row0 + r < nrows;
+        cp_async16(qs_u + sw_off<D>(r, c), qb + (size_t)(ok ? row0 + r : 0) * D + c * 8, ok);
+    }
+    load_kv(k_begin, first_suffix_row, AT_KEYS);
+
+    // Per-thread rows g and g + 8 of this warp's 16; their visible key count.
+    const int g = lane >> 2, cq = lane & 3;
+    int nvis[2];
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+        const int R = row0 + warp * 16 + g + hh * 8;
+        const int i = R / a.H;
+        nvis[hh] = (R < nrows && i == 0) ? a.P + 1 : nk;
+    }
+
+    float oacc[D / 8][4];
+#pragma unroll
+    for (int n = 0; n < D / 8; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.f;
+    float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+
+    for (int key0 = k_begin; key0 < k_end; key0 += AT_KEYS) {
+        __syncthreads();
+        if (key0 != k_begin) load_kv(key0, 0, AT_KEYS);
+        cp_async_wait_all();
+        __syncthreads();
+
+        // S = Q K^T for this warp's 16 rows x 64 keys.
+        float sacc[AT_KEYS / 8][4];
+#pragma unroll
+        for (int n = 0; n < AT_KEYS / 8; ++n) sacc[n][0] = sacc[n][1] = sacc[n][2] = sacc[n][3] = 0.f;
+#pragma unroll
+        for (int kc = 0; kc < D / 16; ++kc) {
+            uint32_t a0, a1, a2, a3;
+            {
+                const int r = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int c = kc * 2 + (lane >> 4);
+                ldsm_x4(qs_u + sw_off<D>(r, c), a0, a1, a2, a3);
+            }
+#pragma unroll
+            for (int nt = 0; nt < AT_KEYS / 8; nt += 2) {
+                uint32_t b0, b1, b2, b3;
+                const int r = (nt + (lane >> 4)) * 8 + (lane & 7);
+                const int c = kc * 2 + ((lane >> 3) & 1);
+                ldsm_x4(ks_u + sw_off<D>(r, c), b0, b1, b2, b3);
+                mma16816(sacc[nt], a0, a1, a2, a3, b0, b1);
+                mma16816(sacc[nt + 1], a0, a1, a2, a3, b2, b3);
+            }
+        }
+        // Scale to log2 units, mask, online softmax.
+        float bmax[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+        for (int nt = 0; nt < AT_KEYS / 8; ++nt)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int key = key0 + nt * 8 + 2 * cq + (e & 1);
+                const int hh = e >> 1;
+                const float s = (key < k_end && key < nvis[hh]) ? sacc[nt][e] * a.scale_log2 : -INFINITY;
+                sacc[nt][e] = s;
+                bmax[hh] = fmaxf(bmax[hh], s);
+            }
+        float alpha[2], mnew[2];
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            bmax[hh] = fmaxf(bmax[hh], __shfl_xor_sync(0xffffffffu, bmax[hh], 1));
+            bmax[hh] = fmaxf(bmax[hh], __shfl_xor_sync(0xffffffffu, bmax[hh], 2));
+            mnew[hh] = fmaxf(m_run[hh], bmax[hh]);
+            alpha[hh] = (mnew[hh] == -INFINITY) ? 1.f : exp2f(m_run[hh] - mnew[hh]);
+        }
+        float psum[2] = {0.f, 0.f};
+#pragma unroll
+        for (int nt = 0; nt < AT_KEYS / 8; ++nt)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int hh = e >> 1;
+                const float p = (sacc[nt][e] == -INFINITY) ? 0.f : exp2f(sacc[nt][e] - mnew[hh]);
+                sacc[nt][e] = p;
+                psum[hh] += p;
+            }
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            psum[hh] += __shfl_xor_sync(0xffffffffu, psum[hh], 1);
+            psum[hh] += __shfl_xor_sync(0xffffffffu, psum[hh], 2);
+            l_run[hh] = l_run[hh] * alpha[hh] + psum[hh];
+            m_run[hh] = mnew[hh];
+        }
+#pragma unroll
+        for (int n = 0; n < D / 8; ++n) {
+            oacc[n][0] *= alpha[0];
+            oacc[n][1] *= alpha[0];
+            oacc[n][2] *= alpha[1];
+            oacc[n][3] *= alpha[1];
+        }
+        // O += P V: the S accumulators of key tiles (2j, 2j+1) are the A operand of k-step j.
+#pragma unroll
+        for (int j = 0; j < AT_KEYS / 16; ++j) {
+            const uint32_t a0 = pack_bf16x2(sacc[2 * j][0], sacc[2 * j][1]);
+            const uint32_t a1 = pack_bf16x2(sacc[2 * j][2], sacc[2 * j][3]);
+            const uint32_t a2 = pack_bf16x2(sacc[2 * j + 1][0], sacc[2 * j + 1][1]);
+            const uint32_t a3 = pack_bf16x2(sacc[2 * j + 1][2], sacc[2 * j + 1][3]);
+#pragma unroll
+            for (int dt = 0; dt < D / 8; dt += 2) {
+                uint32_t b0, b1, b2, b3;
+                const int r = j * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int c = dt + (lane >> 4);
+                ldsm_x4_t(vs_u + sw_off<D>(r, c), b0, b1, b2, b3);
+                mma16816(oacc[dt], a0, a1, a2, a3, b0, b1);
+                mma16816(oacc[dt + 1], a0, a1, a2, a3, b2, b3);
+            }
+        }
+    }
+
+    // Partial rows of this split (O unnormalised, then m and l in the row padding).
+    __syncthreads();
+#pragma unroll
+    for (int n = 0; n < D / 8; ++n) {
+        const int r = warp * 16 + g, col = n * 8 + 2 * cq;
+        *(float2*)(opart + r * (D + 4) + col) = make_float2(oacc[n][0], oacc[n][1]);
+        *(float2*)(opart + (r + 8) * (D + 4) + col) = make_float2(oacc[n][2], oacc[n][3]);
+    }
+    if (cq == 0) {
+        *(float2*)(opart + (warp * 16 + g) * (D + 4) + D) = make_float2(m_run[0], l_run[0]);
+        *(float2*)(opart + (warp * 16 + g + 8) * (D + 4) + D) = make_float2(m_run[1], l_run[1]);
+    }
+    // Rows [s * rows_per, ...) of the 64 belong to split rank s, which combines them.
+    const int ns = a.nsplit;
+    const int rank = (int)ptx::cluster_rank();
+    const int rows_per = (AT_ROWS + ns - 1) / ns;
+    const int r_lo = min(AT_ROWS, rank * rows_per), r_hi = min(AT_ROWS, r_lo + rows_per);
+    const uint32_t row_bytes = (uint32_t)((D + 4) * 4);
+    if (tid == 32) ptx::mbar_expect_tx(rbar, (uint32_t)(ns * (r_hi - r_lo)) * row_bytes);
+    ptx::fence_proxy_async_smem();
+    // Every split is done with q/k/v (the receive buffers overlap them) and every receive
+    // barrier is initialised past this point.
+    ptx::cluster_sync_all();
+    if (tid == 0) {
+        const uint32_t recv_u = ptx::smem_u32(recv + (size_t)rank * rows_per * (D + 4));
+        const uint32_t bar_u = ptx::smem_u32(rbar);
+        for (int s = 0; s < ns; ++s) {
+            const int lo = min(AT_ROWS, s * rows_per), hi = min(AT_ROWS, lo + rows_per);
+            if (hi <= lo) continue;
+            ptx::bulk_copy_to_cluster(ptx::dsmem_map(recv_u, (uint32_t)s), opart + (size_t)lo * (D + 4),
+                                      (uint32_t)(hi - lo) * row_bytes, ptx::dsmem_map(bar_u, (uint32_t)s));
+        }
+    }
+    const bool got = ptx::mbar_wait_bounded(rbar, 0, 200ull * 1000 * 1000);
+
+    // Combine the splits in rank order for the owned rows, from local shared memory.
+    for (int r = r_lo + tid; r < r_hi; r += AT_THREADS) {
+        float mx = -INFINITY;
+        for (int s = 0; s < ns; ++s)
+            mx = fmaxf(mx, recv[((size_t)s * rows_per + (r - r_lo)) * (D + 4) + D]);
+        float L = 0.f;
+        for (int s = 0; s < ns; ++s) {
+            const float* rr = recv + ((size_t)s * rows_per + (r - r_lo)) * (D + 4) + D;
+            const float w = (mx == -INFINITY) ? 0.f : exp2f(rr[0] - mx);
+            coef[r * AT_MAX_SPLITS + s] = w;
+            L += w * rr[1];
+        }
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        for (int s = 0; s < ns; ++s) coef[r * AT_MAX_SPLITS + s] *= inv;
+    }
+    __syncthreads();
+    const int nrow_here = r_hi - r_lo;
+    for (int idx = tid; idx < nrow_here * (D / 4); idx += AT_THREADS) {
+        const int r = r_lo + idx / (D / 4), d = (idx % (D / 4)) * 4;
+        const int R = row0 + r;
+        if (R >= nrows || !got) continue;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int s = 0; s < ns; ++s) {
+            const float c = coef[r * AT_MAX_SPLITS + s];
+            const float4 v = *(const float4*)(recv + ((size_t)s * rows_per + (r - r_lo)) * (D + 4) + d);
+            acc.x = fmaf(c, v.x, acc.x);
+            acc.y = fmaf(c, v.y, acc.y);
+            acc.z = fmaf(c, v.z, acc.z);
+            acc.w = fmaf(c, v.w, acc.w);
+        }
+        const int i = R / a.H, head = R - i * a.H;
+        const size_t tok = (size_t)b * a.S + i;
+        uint2 packed = make_uint2(pack_bf16x2(acc.x, acc.y), pack_bf16x2(acc.z, acc.w));
+        *(uint2*)(a.o + (tok * a.H + head) * D + d) = packed;
+    }
+    if (tid == 0 && !got) atomicCAS(a.err, 0, (int)DEV_TIMEOUT_MMA);
+    // No split exits while a copy out of its shared memory may still be in flight.
+    ptx::cluster_sync_all();
+}
+
+template <int D>
+size_t attn_smem() {
+    return 128 + attn_region<D>() + sizeof(float) * AT_ROWS * AT_MAX_SPLITS + 16;
+}
+
+template <int D>
+jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
+    const int S = C + 1, nrows = S * h->H, nk = h->cur_prefix + S;
+    const int rblocks = (nrows + AT_ROWS - 1) / AT_ROWS;
+    // Enough key splits for one request to put about two CTAs on every SM, at most 16 (one
+    // cluster). The split depends on the request's sizes only, never on the batch, so a request
+    // gives bitwise the same output alone or inside any batch.
+    int want = (2 * h->num_sms + rblocks - 1) / rblocks;
+    want = want < 1 ? 1 : (want > h->attn_max_splits ? h->attn_max_splits : want);
+    int chunk = (nk + want - 1) / want;
+    chunk = (chunk + 15) / 16 * 16;
+    const int ns = (nk + chunk - 1) / chunk;
+    AttnArgs a;
+    const size_t kv_layer = (size_t)l * h->maxB * h->kv_rows * h->D;
+    a.q = (const __nv_bfloat16*)h->q;
+    a.kst = (const __nv_bfloat16*)h->kv_k + kv_layer;
+    a.vst = (const __nv_bfloat16*)h->kv_v + kv_layer;
+    a.o = (__nv_bfloat16*)h->o;
+    a.S = S;
+    a.H = h->H;
+    a.P = h->cur_prefix;
+    a.kv_rows = h->kv_rows;
+    a.chunk = chunk;
+    a.nsplit = ns;
+    a.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
+    a.err = h->dev_err;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(rblocks, ns, B);
+    cfg.blockDim = dim3(AT_THREADS);
+    cfg.dynamicSmemBytes = attn_smem<D>();
+    cfg.stream = st;
+    cudaLaunchAttribute attrs[2];
+    int n = 0;
+    attrs[n].id = cudaLaunchAttributeClusterDimension;
+    attrs[n].val.clusterDim.x = 1;
+    attrs[n].val.clusterDim.y = ns;
+    attrs[n].val.clusterDim.z = 1;
+    ++n;
+    if (h->pdl) {
+        attrs[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attrs[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    cfg.attrs = attrs;
+    cfg.numAttrs = n;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_tc<D>, a);
+    if (e != cudaSuccess) {
+        set_error("attention launch failed: %s", cudaGetErrorString(e));
+        return JPI_ERR_CUDA;
+    }
+    return JPI_OK;
+}
+
+template <int D>
+jpi_status prepare_d(jpi_handle* h) {
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_attn_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)attn_smem<D>()));
+    if (cudaFuncSetAttribute(k_attn_tc<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+        cudaGetLastError();
+        h->attn_max_splits = 8;
+    } else {
+        h->attn_max_splits = AT_MAX_SPLITS;
+    }
+    return JPI_OK;
+}
+
+}  // namespace
+
+bool attn_tc_supported(const jpi_handle* h) {
+    return h->D == 64 || h->D == 128 || h->D == 256;
+}
+
+jpi_status attn_tc_prepare(jpi_handle* h) {
+    switch (h->D) {
+        case 64: return prepare_d<64>(h);
+        case 128: return prepare_d<128>(h);
+        case 256: return prepare_d<256>(h);
+        default:
+            set_error("attention head_dim %d is not tiled", h->D);
+            return JPI_ERR_UNSUPPORTED;
+    }
+}
+
+jpi_status launch_attn_tc(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
+    switch (h->D) {
+        case 64: return launch_attn_d<64>(h, l, B, C, st);
+        case 128: return launch_attn_d<128>(h, l, B, C, st);
+        case 256: return launch_attn_d<256>(h, l, B, C, st);
+        default:
+            set_error("attention head_dim %d is not tiled", h->D);
+            return JPI_ERR_UNSUPPORTED;
+    }
+}
+
+}  // namespace jpi

@@ -1,0 +1,289 @@
+// The tensor-core projection kernel (included by tc_path.cu, inside jpi's anonymous namespace).
+//
+// One CTA = one (128-row weight tile, K range) unit; the CTAs of a cluster share the tile and
+// split its K range. Per 64-token tile:
+//   1. B operand: bulk tensor copies of the bf16/fp16 activation blocks; for the RMSNorm-fed
+//      projections the norm and the time-conditioned scale/shift are applied in place.
+//   2. tcgen05.mma of the weight blocks (loaded before the grid-dependency wait) into TMEM.
+//   3. Split-K reduction: after a cluster barrier (every CTA's MMA is done, so its weight and
+//      operand buffers are free), each CTA pushes the rows owned by every rank of the cluster to
+//      that rank with bulk shared::cluster copies (completion counted on the owner's mbarrier);
+//      the owner sums its received slices in rank order from its own shared memory. With a
+//      single token tile the receive buffer reuses the weight region.
+//   4. Epilogue on the owned rows, then a cluster barrier before buffers are reused.
+
+template <int KIND>
+__global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_constant__ CUtensorMap wmap,
+                                                          const __grid_constant__ CUtensorMap xmap,
+                                                          const __grid_constant__ GemmArgs a) {
+    constexpr bool NORM_IN = (KIND == G_QKV || KIND == G_GU);
+    constexpr bool RESID = (KIND == G_O || KIND == G_DOWN);
+    constexpr uint32_t IDESC = ptx::idesc_bf16_f32(TILE_ROWS, NT);
+
+    extern __shared__ uint8_t smem_raw[];
+    // Offsetting the shared array itself (not a cast through an integer) keeps every access
+    // below in the shared state space.
+    uint8_t* smem = smem_raw + ((1024u - (ptx::smem_u32(smem_raw) & 1023u)) & 1023u);
+    const int xp_bytes = max(a.kpb * XBLK_BYTES, TILE_ROWS * PSTRIDE * 4);
+    uint8_t* wsm = smem;                                   // kpb weight tiles
+    uint8_t* xsm = wsm + a.kpb * TILE_BYTES;               // X blocks, then the outgoing partial
+    float* part = (float*)xsm;                             // [128][PSTRIDE] this CTA's fp32 product
+    // [splits][2 * npairs][PSTRIDE] received slices: in the weight region or after the partial.
+    float* recv = a.recv_alias ? (float*)wsm : (float*)(xsm + xp_bytes);
+    float* slots = (float*)(xsm + xp_bytes + (a.recv_alias ? 0 : RECV_BYTES));   // [MAX_SPLITS][NT]
+    float* rinv = slots + MAX_SPLITS * NT;                 // [NT]
+    float* sspart = rinv + NT;                             // [GEMM_THREADS][4]
+    float* sig = sspart + 4 * GEMM_THREADS;                // [8 * KBLK] this CTA's sigma slice
+    float* bet = sig + 8 * KBLK;                           // [8 * KBLK] this CTA's beta slice
+    uint64_t* bars = (uint64_t*)(bet + 8 * KBLK);          // weights, X, MMA done, received
+    uint32_t* tmem_slot = (uint32_t*)(bars + 4);
+    int* flag = (int*)(tmem_slot + 1);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int rank = (int)ptx::cluster_rank();
+    const int tile = blockIdx.x / a.splits;
+    const int kb0 = rank * a.kpb;
+    const int npairs = 64 / a.splits, p0 = rank * npairs;
+    const int nitems = npairs * QUADS;
+
+    if (warp == 0) {
+        ptx::tmem_alloc(tmem_slot, NT);
+        ptx::tmem_relinquish();
+    }
+    if (tid == 0) {
+        for (int i = 0; i < 4; ++i) ptx::mbar_init(&bars[i], 1);
+        ptx::fence_mbar_init();
+        *flag = 0;
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    // Weight tiles depend on nothing upstream: start streaming them before the dependency wait.
+    if (tid == 0) {
+        const uint64_t pol = ptx::l2_policy_evict_first();
+        ptx::mbar_expect_tx(&bars[0], (uint32_t)(a.kpb * TILE_BYTES));
+        for (int j = 0; j < a.kpb; ++j)
+            ptx::tma_load_2d(wsm + j * TILE_BYTES, &wmap, &bars[0], 0,
+                             (tile * a.nkb + kb0 + j) * TILE_ROWS, pol);
+    }
+    // The modulation vectors come from the time-conditioning kernels, which precede this launch
+    // by at least two kernels; a dependent launch starts only after its predecessor has passed
+    // its own dependency wait, so they are complete here and can be read before ours.
+    if (NORM_IN) {
+        for (int i = tid; i < a.kpb * KBLK; i += GEMM_THREADS) {
+            sig[i] = a.sigma[kb0 * KBLK + i];
+            bet[i] = a.beta[kb0 * KBLK + i];
+        }
+    }
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
+
+    const int ntt = (a.Mt + NT - 1) / NT;
+    for (int tt = 0; tt < ntt; ++tt) {
+        const int tok0 = tt * NT;
+        // ---- 1. B operand ----
+        if (tid == 0) {
+            const uint64_t pol = ptx::l2_policy_evict_first();
+            ptx::mbar_expect_tx(&bars[1], (uint32_t)(a.kpb * XBLK_BYTES));
+            for (int j = 0; j < a.kpb; ++j)
+                ptx::tma_load_2d(xsm + j * XBLK_BYTES, &xmap, &bars[1], (kb0 + j) * KBLK, tok0, pol);
+        }
+        if (tid == 32) ptx::mbar_expect_tx(&bars[3], (uint32_t)(TILE_ROWS * PSTRIDE * 4));
+        if (NORM_IN) {
+            if (tid >= 64 && tid < 64 + NT) {
+                const int tok = tok0 + tid - 64;
+                float r = 0.f;
+                if (tok < a.Mt) {
+                    float s = 0.f;
+                    for (int sl = 0; sl < a.nslot; ++sl) s += a.ss[(size_t)sl * a.ss_ld + tok];
+                    r = rsqrtf(s * a.inv_w + a.eps);
+                }
+                rinv[tid - 64] = r;
+            }
+        }
+        if (!ptx::mbar_wait_bounded(&bars[1], tt & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_WEIGHTS;
+        if (NORM_IN) {
+            __syncthreads();
+            // In place: u = h * rinv * (1 + sigma) + beta on each swizzled 16-byte chunk.
+            for (int idx = tid; idx < a.kpb * NT * 8; idx += GEMM_THREADS) {
+                const int j = idx / (NT * 8), t = (idx >> 3) % NT, q = idx & 7;
+                const int c = q ^ (t & 7);                         // logical chunk of row t
+                const int kl = j * KBLK + c * 8;                   // index into this CTA's slice
+                uint4* p = (uint4*)(xsm + j * XBLK_BYTES + t * 128 + q * 16);
+                const uint4 v = *p;
+                const float r = rinv[t];
+                const float4 s0 = *(const float4*)(sig + kl), s1 = *(const float4*)(sig + kl + 4);
+                const float4 b0 = *(const float4*)(bet + kl), b1 = *(const float4*)(bet + kl + 4);
+                const float2 h0 = unpack_half2(v.x), h1 = unpack_half2(v.y);
+                const float2 h2 = unpack_half2(v.z), h3 = unpack_half2(v.w);
+                uint4 o;
+                o.x = pack_bf16x2(h0.x * r * (1.f + s0.x) + b0.x, h0.y * r * (1.f + s0.y) + b0.y);
+                o.y = pack_bf16x2(h1.x * r * (1.f + s0.z) + b0.z, h1.y * r * (1.f + s0.w) + b0.w);
+                o.z = pack_bf16x2(h2.x * r * (1.f + s1.x) + b1.x, h2.y * r * (1.f + s1.y) + b1.y);
+                o.w = pack_bf16x2(h3.x * r * (1.f + s1.z) + b1.z, h3.y * r * (1.f + s1.w) + b1.w);
+                if (tok0 + t >= a.Mt) o = make_uint4(0u, 0u, 0u, 0u);
+                *p = o;
+            }
+            ptx::fence_proxy_async_smem();
+        }
+        __syncthreads();
+
+        // ---- 2. MMA: D[128 rows][NT tokens] over this CTA's K blocks ----
+        if (tid == 0 && *flag == 0) {
+            if (tt == 0 && !ptx::mbar_wait_bounded(&bars[0], 0, WAIT_LIMIT_NS)) {
+                *flag = DEV_TIMEOUT_WEIGHTS;
+            } else {
+                ptx::tc_fence_after();
+                const uint32_t wbase = ptx::smem_u32(wsm), xbase = ptx::smem_u32(xsm);
+                for (int j = 0; j < a.kpb; ++j)
+#pragma unroll
+                    for (int kk = 0; kk < KBLK / 16; ++kk)
+                        ptx::mma_bf16(tmem, ptx::desc_sw128(wbase + j * TILE_BYTES + kk * 32),
+                                      ptx::desc_sw128(xbase + j * XBLK_BYTES + kk * 32), IDESC,
+                                      (j | kk) != 0);
+                ptx::mma_commit(&bars[2]);
+            }
+        }
+        // Epilogue inputs from global memory that do not depend on the product: issued now so
+        // their latency overlaps the MMA and the exchange (first item of this thread only).
+        float hv1[4] = {0.f, 0.f, 0.f, 0.f}, hv2[4] = {0.f, 0.f, 0.f, 0.f};
+        float2 cs[4] = {make_float2(1.f, 0.f), make_float2(1.f, 0.f), make_float2(1.f, 0.f), make_float2(1.f, 0.f)};
+        auto prefetch = [&](int item) {
+            const int p = p0 + item / QUADS, t0 = (item % QUADS) * 4;
+            const int f1 = tile * TILE_ROWS + p, f2 = f1 + 64;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int tok = tok0 + t0 + e;
+                hv1[e] = hv2[e] = 0.f;
+                cs[e] = make_float2(1.f, 0.f);
+                if (tok < a.Mt) {
+                    if (RESID) {
+                        hv1[e] = a.hres[(size_t)tok * a.W + f1];
+                        hv2[e] = a.hres[(size_t)tok * a.W + f2];
+                    }
+                    if (KIND == G_QKV && a.rope) {
+                        const int hd = a.D >> 1, pair = tile * 64 + p;
+                        const int sec = pair / hd, d = pair - sec * hd;
+                        if (sec <= a.H) cs[e] = __ldg(a.rope + (size_t)(a.P + tok % a.S) * hd + d);
+                    }
+                }
+            }
+        };
+        if (tid < nitems) prefetch(tid);
+        if (*flag == 0 && !ptx::mbar_wait_bounded(&bars[2], tt & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
+        __syncthreads();
+        const bool ok = *flag == 0;
+        ptx::tc_fence_after();
+
+        // ---- 3a. TMEM -> fp32 partial in shared memory (warp w: lanes 32 (w mod 4), half w / 4) ----
+        if (ok) {
+            const int row = (warp & 3) * 32 + lane, cbase = (warp >> 2) * (NT / 2);
+#pragma unroll
+            for (int c0 = 0; c0 < NT / 2; c0 += 16) {
+                uint32_t r[16];
+                ptx::tmem_ld_x16(tmem + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(cbase + c0), r);
+                ptx::tmem_ld_wait();
+                float4* dst = (float4*)(part + row * PSTRIDE + cbase + c0);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4)
+                    dst[q4] = make_float4(__uint_as_float(r[4 * q4]), __uint_as_float(r[4 * q4 + 1]),
+                                          __uint_as_float(r[4 * q4 + 2]), __uint_as_float(r[4 * q4 + 3]));
+            }
+        }
+        ptx::tc_fence_before();
+        ptx::fence_proxy_async_smem();
+        // Every CTA's MMA is complete (its buffers may be overwritten) and every receive
+        // barrier is initialised past this point.
+        ptx::cluster_sync_all();
+
+        // ---- 3b. push each rank's rows (pairs r*npairs.. and +64) to that rank ----
+        if (tid == 0) {
+            const uint32_t chunk = (uint32_t)(npairs * PSTRIDE * 4);
+            const uint32_t recv_u = ptx::smem_u32(recv + (size_t)rank * 2 * npairs * PSTRIDE);
+            const uint32_t bar_u = ptx::smem_u32(&bars[3]);
+            for (int r = 0; r < a.splits; ++r) {
+                const uint32_t dst = ptx::dsmem_map(recv_u, (uint32_t)r);
+                const uint32_t rbar = ptx::dsmem_map(bar_u, (uint32_t)r);
+                ptx::bulk_copy_to_cluster(dst, part + (size_t)r * npairs * PSTRIDE, chunk, rbar);
+                ptx::bulk_copy_to_cluster(dst + chunk, part + (size_t)(r * npairs + 64) * PSTRIDE, chunk, rbar);
+            }
+        }
+        if (!ptx::mbar_wait_bounded(&bars[3], tt & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
+
+        // ---- 4. rank-ordered sum of the received slices + epilogue; item = (pair, 4 tokens) ----
+        float ssq[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int item = tid; item < nitems; item += GEMM_THREADS) {
+            if (item != tid) prefetch(item);
+            const int pi = item / QUADS, t0 = (item % QUADS) * 4, p = p0 + pi;
+            float4 y1 = make_float4(0.f, 0.f, 0.f, 0.f), y2 = y1;
+            for (int r = 0; r < a.splits; ++r) {
+                f4add(y1, *(const float4*)(recv + ((size_t)r * 2 * npairs + pi) * PSTRIDE + t0));
+                f4add(y2, *(const float4*)(recv + ((size_t)r * 2 * npairs + npairs + pi) * PSTRIDE + t0));
+            }
+            if (!ok) continue;
+            const int f1 = tile * TILE_ROWS + p, f2 = f1 + 64;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int tok = tok0 + t0 + e;
+                if (tok >= a.Mt) continue;
+                const float u1 = f4get(y1, e), u2 = f4get(y2, e);
+                if (KIND == G_QKV) {
+                    const int hd = a.D >> 1, pair = tile * 64 + p;
+                    const int sec = pair / hd, d = pair - sec * hd;
+                    const int b = tok / a.S, pos = a.P + (tok - b * a.S);
+                    float r1 = u1, r2 = u2;
+                    if (sec <= a.H) {
+                        r1 = u1 * cs[e].x - u2 * cs[e].y;
+                        r2 = u2 * cs[e].x + u1 * cs[e].y;
+                    }
+                    __nv_bfloat16* dst = (sec < a.H) ? a.q + ((size_t)tok * a.H + sec) * a.D
+                                                     : (sec == a.H ? a.kst : a.vst) + ((size_t)b * a.kv_rows + pos) * a.D;
+                    dst[d] = __float2bfloat16_rn(r1);
+                    dst[d + hd] = __float2bfloat16_rn(r2);
+                } else if (KIND == G_GU) {
+                    a.z[(size_t)tok * a.F + tile * 64 + p] = __float2bfloat16_rn(gelu_tanh(u1) * u2);
+                } else {
+                    const float n1 = hv1[e] + a.gamma[f1] * u1;
+                    const float n2 = hv2[e] + a.gamma[f2] * u2;
+                    a.hres[(size_t)tok * a.W + f1] = n1;
+                    a.hres[(size_t)tok * a.W + f2] = n2;
+                    a.hx[(size_t)tok * a.W + f1] = __float2half_rn(n1);
+                    a.hx[(size_t)tok * a.W + f2] = __float2half_rn(n2);
+                    if (!(fabsf(n1) <= 65504.f && fabsf(n2) <= 65504.f)) set_device_error(a.err, DEV_FP16_RANGE);
+                    ssq[e] = fmaf(n1, n1, fmaf(n2, n2, ssq[e]));
+                }
+            }
+        }
+        if (RESID) {
+            // Per-token sum over this CTA's features (threads with equal tid mod QUADS share a
+            // token quad), pushed to rank 0, which sums the ranks in order after the barrier.
+#pragma unroll
+            for (int e = 0; e < 4; ++e) sspart[tid * 4 + e] = ssq[e];
+            __syncthreads();
+            if (tid < NT) {
+                const int qd = tid >> 2, e = tid & 3;
+                float s = 0.f;
+                for (int m = qd; m < GEMM_THREADS; m += QUADS) s += sspart[m * 4 + e];
+                ptx::dsmem_st_f32(ptx::dsmem_map(ptx::smem_u32(slots + rank * NT + tid), 0u), s);
+            }
+        }
+        // All copies into and out of this CTA's buffers are complete past this barrier.
+        ptx::cluster_sync_all();
+        if (RESID && rank == 0 && tid < NT && ok) {
+            const int tok = tok0 + tid;
+            if (tok < a.Mt) {
+                float s = 0.f;
+                for (int r = 0; r < a.splits; ++r) s += slots[r * NT + tid];
+                a.ss_out[(size_t)tile * a.ss_ld + tok] = s;
+            }
+        }
+    }
+
+    if (tid == 0 && *flag != 0) set_device_error(a.err, *flag);
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    if (warp == 0) ptx::tmem_dealloc(tmem, NT);
+}

@@ -4,6 +4,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cstdint>
 #include <cstddef>
 #include <map>
@@ -11,7 +12,7 @@
 #include <tuple>
 #include <vector>
 
-#include "../../include/jpi.h"
+#include "jpi.h"
 
 namespace jpi {
 
@@ -41,6 +42,7 @@ enum DeviceError : int {
     DEV_TIMEOUT_WEIGHTS = 1,   // weight tile TMA never completed
     DEV_TIMEOUT_MMA = 2,       // tensor-core commit never arrived
     DEV_BAD_SHAPE = 3,         // a kernel saw a shape it cannot tile
+    DEV_FP16_RANGE = 4,        // a residual-stream value exceeded the fp16 range of its copy
 };
 
 // Offsets (in rows of W) of the modulation vectors inside one step's modulation row block.
@@ -73,6 +75,7 @@ struct LayerTiled {
 // K by a cluster of `splits` CTAs that own `kpb` 64-wide K blocks apiece.
 struct GemmPlan {
     int rows = 0, K = 0, ntiles = 0, nkb = 0, kpb = 0, splits = 0, ctas = 0;
+    int recv_alias = 0;   // received split-K slices overwrite the weight tiles
     size_t smem = 0;
 };
 
@@ -91,6 +94,8 @@ struct jpi_handle {
     bool bf16 = true;
     bool tc = false;          // tensor-core kernels in use (bf16 mode with supported dims)
     bool pdl = true;          // programmatic dependent launch between tensor-core kernels
+    int num_sms = 0;
+    int attn_max_splits = 8;  // largest key-split cluster of the attention kernel
 
     // Dimensions.
     int L, W, H, D, F, A, Sd, dt, HD, QKV;   // QKV = (H + 2) D
@@ -136,11 +141,14 @@ struct jpi_handle {
     void* o = nullptr;          // [maxMt][H D] attention output (TW type)
     void* z = nullptr;          // [maxMt][F] GeGLU output (TW type)
     float* ss = nullptr;        // [W / 128][maxMt] per-token sums of h^2 over 128-feature slices
+    void* hx = nullptr;         // [maxMt][W] fp16 copy of h, read by the norm-fed GEMMs
     int* dev_err = nullptr;     // device error word
 
-    // Tensor-core path: plans and tensor maps (4 per layer: QKV, O, gate/up, down).
-    jpi::GemmPlan plans[4];
+    // Tensor-core path: plans ([0] one 64-token tile, [1] several) and tensor maps
+    // (4 per layer: QKV, O, gate/up, down).
+    jpi::GemmPlan plans[2][4];
     std::vector<CUtensorMap> tmaps;
+    CUtensorMap xmaps[3];       // B operands: hx, o, z
 
     // State.
     int cur_batch = 0, cur_prefix = 0;

@@ -108,12 +108,88 @@ __global__ void k_gemv_multi(const TW* __restrict__ Wm, const float* __restrict_
     }
 }
 
+// Y[n][r] = sum_k W[r][k] X[n][k] + b[r] for all n < NG step times at once: the stacked
+// modulation matrix (6 L + 2) W rows is streamed from HBM exactly once per call. Each thread
+// owns MOD_RT consecutive rows; per 16-wide K slab it loads 32 bytes of every row (full
+// sectors) and reads each X value as a shared-memory broadcast, so the inner loop is FMAs.
+constexpr int MOD_RT = 4;
+
+template <typename TW> struct Slab;                 // 16 consecutive weights of one row
+template <> struct Slab<__nv_bfloat16> {
+    uint4 v[2];
+    __device__ __forceinline__ void load(const __nv_bfloat16* p) {
+        v[0] = __ldg((const uint4*)p);
+        v[1] = __ldg((const uint4*)p + 1);
+    }
+    __device__ __forceinline__ float get(int i) const {
+        const uint32_t u = (&v[0].x)[i >> 1];
+        return __uint_as_float((i & 1) ? (u & 0xFFFF0000u) : (u << 16));
+    }
+};
+template <> struct Slab<float> {
+    float4 v[4];
+    __device__ __forceinline__ void load(const float* p) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v[i] = __ldg((const float4*)p + i);
+    }
+    __device__ __forceinline__ float get(int i) const { return (&v[0].x)[i]; }
+};
+
+template <typename TW, int NG>
+__global__ void __launch_bounds__(256) k_mod_gemv(const TW* __restrict__ Wm, const float* __restrict__ bias,
+                                                   const float* __restrict__ X, float* __restrict__ Y,
+                                                   int R, int K) {
+    extern __shared__ float xs[];                     // [NG][K]
+    for (int i = threadIdx.x; i < NG * K; i += blockDim.x) xs[i] = X[i];
+    __syncthreads();
+    const int r0 = (blockIdx.x * blockDim.x + threadIdx.x) * MOD_RT;
+    if (r0 >= R) return;
+    float acc[MOD_RT][NG];
+#pragma unroll
+    for (int rr = 0; rr < MOD_RT; ++rr)
+#pragma unroll
+        for (int n = 0; n < NG; ++n) acc[rr][n] = 0.f;
+    const TW* rowp[MOD_RT];
+#pragma unroll
+    for (int rr = 0; rr < MOD_RT; ++rr) rowp[rr] = Wm + (size_t)min(r0 + rr, R - 1) * K;
+    Slab<TW> cur[MOD_RT], nxt[MOD_RT];
+#pragma unroll
+    for (int rr = 0; rr < MOD_RT; ++rr) cur[rr].load(rowp[rr]);
+    for (int k0 = 0; k0 < K; k0 += 16) {
+        if (k0 + 16 < K) {
+#pragma unroll
+            for (int rr = 0; rr < MOD_RT; ++rr) nxt[rr].load(rowp[rr] + k0 + 16);
+        }
+#pragma unroll
+        for (int kk = 0; kk < 16; ++kk) {
+            float w[MOD_RT];
+#pragma unroll
+            for (int rr = 0; rr < MOD_RT; ++rr) w[rr] = cur[rr].get(kk);
+#pragma unroll
+            for (int n = 0; n < NG; ++n) {
+                const float xv = xs[n * K + k0 + kk];
+#pragma unroll
+                for (int rr = 0; rr < MOD_RT; ++rr) acc[rr][n] = fmaf(w[rr], xv, acc[rr][n]);
+            }
+        }
+#pragma unroll
+        for (int rr = 0; rr < MOD_RT; ++rr) cur[rr] = nxt[rr];
+    }
+#pragma unroll
+    for (int n = 0; n < NG; ++n)
+#pragma unroll
+        for (int rr = 0; rr < MOD_RT; ++rr)
+            if (r0 + rr < R) Y[(size_t)n * R + r0 + rr] = acc[rr][n] + bias[r0 + rr];
+}
+
 // ---------------------------------------------------------------------------------------------
 // Token embedding: row 0 of each request is the state token, rows 1..C the action tokens.
 // Block = 128 features of one token; with `ss` it also writes that slice's sum of squares
 // (ss[slice][m]) for the next RMSNorm of the tensor-core path.
 __global__ void __launch_bounds__(128) k_embed(
-    float* __restrict__ hres, float* __restrict__ ss, int ss_ld, const float* __restrict__ state,
+    float* __restrict__ hres, __half* __restrict__ hx, int* __restrict__ err, float* __restrict__ ss,
+    int ss_ld,
+    const float* __restrict__ state,
     const float* __restrict__ x, const float* __restrict__ Ws, const float* __restrict__ bs,
     const float* __restrict__ Wa, const float* __restrict__ ba, int S, int C, int W, int Sd, int A) {
     __shared__ float scratch[32];
@@ -135,6 +211,10 @@ __global__ void __launch_bounds__(128) k_embed(
         for (int k = 0; k < K; ++k) acc = fmaf(Wm[(size_t)n * K + k], in[k], acc);
         v = acc + bias[n];
         hres[(size_t)m * W + n] = v;
+        if (hx) {
+            hx[(size_t)m * W + n] = __float2half_rn(v);
+            if (!(fabsf(v) <= 65504.f)) atomicCAS(err, 0, (int)DEV_FP16_RANGE);
+        }
     }
     if (ss) {
         const float t = block_sum(v * v, scratch);
@@ -445,6 +525,42 @@ jpi_status op_simt(jpi_handle* h, int op, int l, int step, int B, int C, cudaStr
 // stays at 8 x max(W, d_t) floats whatever the step count.
 constexpr int TC_GROUP = 8;
 
+// Modulation step times per pass of k_mod_gemv (its shared copy of X is MOD_GROUP x W floats).
+constexpr int MOD_GROUP = 16;
+
+template <typename T, int NG>
+void launch_mod_gemv(jpi_handle* h, const float* X, float* Y, int R, cudaStream_t st) {
+    const int W = h->W;
+    int threads = (R / MOD_RT + h->num_sms - 1) / h->num_sms;   // about one CTA per SM
+    threads = (threads + 31) / 32 * 32;
+    threads = threads < 64 ? 64 : (threads > 256 ? 256 : threads);
+    const int grid = (R + threads * MOD_RT - 1) / (threads * MOD_RT);
+    k_mod_gemv<T, NG><<<grid, threads, sizeof(float) * NG * W, st>>>((const T*)h->mod_w, h->mod_b, X, Y, R, W);
+}
+
+template <typename T>
+void mod_gemv(jpi_handle* h, int g, const float* X, float* Y, int R, cudaStream_t st) {
+    switch (g) {
+#define JPI_MOD_CASE(n) case n: launch_mod_gemv<T, n>(h, X, Y, R, st); break;
+        JPI_MOD_CASE(1) JPI_MOD_CASE(2) JPI_MOD_CASE(3) JPI_MOD_CASE(4) JPI_MOD_CASE(5) JPI_MOD_CASE(6)
+        JPI_MOD_CASE(7) JPI_MOD_CASE(8) JPI_MOD_CASE(9) JPI_MOD_CASE(10) JPI_MOD_CASE(11)
+        JPI_MOD_CASE(12) JPI_MOD_CASE(13) JPI_MOD_CASE(14) JPI_MOD_CASE(15) JPI_MOD_CASE(16)
+#undef JPI_MOD_CASE
+        default: break;
+    }
+}
+
+template <typename T>
+jpi_status set_mod_attrs(int smem) {
+#define JPI_MOD_ATTR(n) \
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_mod_gemv<T, n>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    JPI_MOD_ATTR(1) JPI_MOD_ATTR(2) JPI_MOD_ATTR(3) JPI_MOD_ATTR(4) JPI_MOD_ATTR(5) JPI_MOD_ATTR(6)
+    JPI_MOD_ATTR(7) JPI_MOD_ATTR(8) JPI_MOD_ATTR(9) JPI_MOD_ATTR(10) JPI_MOD_ATTR(11) JPI_MOD_ATTR(12)
+    JPI_MOD_ATTR(13) JPI_MOD_ATTR(14) JPI_MOD_ATTR(15) JPI_MOD_ATTR(16)
+#undef JPI_MOD_ATTR
+    return JPI_OK;
+}
+
 template <typename T>
 jpi_status time_cond(jpi_handle* h, int N, cudaStream_t st) {
     const int W = h->W, dt = h->dt;
@@ -456,8 +572,10 @@ jpi_status time_cond(jpi_handle* h, int N, cudaStream_t st) {
             (const T*)h->time_in_w, h->time_in_b, h->temb + (size_t)n0 * dt, h->c1 + (size_t)n0 * W, W, dt, g);
         k_gemv_multi<T, true><<<grid_for((long long)W * 32, 256, 1024), blk, sizeof(float) * g * W, st>>>(
             (const T*)h->time_out_w, h->time_out_b, h->c1 + (size_t)n0 * W, h->cond + (size_t)n0 * W, W, W, g);
-        k_gemv_multi<T, false><<<grid_for((long long)R * 32, 256, 8192), blk, sizeof(float) * g * W, st>>>(
-            (const T*)h->mod_w, h->mod_b, h->cond + (size_t)n0 * W, h->mods + (size_t)n0 * R, R, W, g);
+    }
+    for (int n0 = 0; n0 < N; n0 += MOD_GROUP) {
+        const int g = (N - n0) < MOD_GROUP ? (N - n0) : MOD_GROUP;
+        mod_gemv<T>(h, g, h->cond + (size_t)n0 * W, h->mods + (size_t)n0 * R, R, st);
     }
     return check_launch("time conditioning");
 }
@@ -468,16 +586,22 @@ jpi_status configure_simt_kernels(jpi_handle* h) {
     const int D = h->D, H = h->H;
     const int att_smem = (int)(sizeof(float) * ((size_t)H * D + 32 * (D + 1) + 32 * D));
     const int gemv_smem = (int)(sizeof(float) * (size_t)TC_GROUP * (h->W > h->dt ? h->W : h->dt));
+    const int mod_smem = (int)(sizeof(float) * (size_t)MOD_GROUP * h->W);
+    int dev = 0;
+    JPI_CUDA_TRY(cudaGetDevice(&dev));
+    JPI_CUDA_TRY(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev));
     if (h->bf16) {
         using T = __nv_bfloat16;
         JPI_CUDA_TRY(cudaFuncSetAttribute(k_attn_simt<T, T, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, att_smem));
         JPI_CUDA_TRY(cudaFuncSetAttribute(k_gemv_multi<T, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, gemv_smem));
         JPI_CUDA_TRY(cudaFuncSetAttribute(k_gemv_multi<T, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, gemv_smem));
+        JPI_TRY(set_mod_attrs<T>(mod_smem));
     } else {
         using T = float;
         JPI_CUDA_TRY(cudaFuncSetAttribute(k_attn_simt<T, T, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, att_smem));
         JPI_CUDA_TRY(cudaFuncSetAttribute(k_gemv_multi<T, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, gemv_smem));
         JPI_CUDA_TRY(cudaFuncSetAttribute(k_gemv_multi<T, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, gemv_smem));
+        JPI_TRY(set_mod_attrs<float>(mod_smem));
     }
     return JPI_OK;
 }
@@ -495,7 +619,8 @@ jpi_status launch_time_conditioning(jpi_handle* h, int nsteps, cudaStream_t st) 
 jpi_status launch_embed(jpi_handle* h, int B, int C, const float* x, cudaStream_t st) {
     const int S = C + 1;
     k_embed<<<dim3((h->W + 127) / 128, B * S), 128, 0, st>>>(
-        h->h, h->tc ? h->ss : nullptr, h->maxMt, h->state, x, h->state_in_w, h->state_in_b,
+        h->h, h->tc ? (__half*)h->hx : nullptr, h->dev_err, h->tc ? h->ss : nullptr, h->maxMt, h->state,
+        x, h->state_in_w, h->state_in_b,
         h->action_in_w, h->action_in_b, S, C, h->W, h->Sd, h->A);
     return check_launch("embed");
 }

@@ -16,6 +16,10 @@ jpi_status tc_launch_layer(jpi_handle* h, int layer, int step, int batch, int ch
 // One sub-step of a layer (ops 2..6 of jpi_profile_op).
 jpi_status tc_launch_op(jpi_handle* h, int op, int layer, int step, int batch, int chunk,
                         cudaStream_t st);
+// Tensor-core attention (attn_tc.cu).
+bool attn_tc_supported(const jpi_handle* h);
+jpi_status attn_tc_prepare(jpi_handle* h);
+jpi_status launch_attn_tc(jpi_handle* h, int layer, int batch, int chunk, cudaStream_t st);
 // Frees what tc_prepare created outside the handle's allocation list.
 void tc_release(jpi_handle* h);
 
