@@ -185,6 +185,26 @@ JPI_API jpi_status jpi_expert_forward(jpi_handle* h, const float* state, const f
                                       void* stream);
 
 /*
+ * jpi_expert_forward without allocation of its own, for callers that cannot call cudaMalloc
+ * (code that runs inside a stream capture, or under an allocator that owns all device memory
+ * once start-up is over). Same arguments, results and errors as jpi_expert_forward.
+ * The paper has no counterpart; this is a deployment convenience.
+ *   - It allocates nothing: no cudaMalloc, cudaFree or allocating library routine. The scratch
+ *     of its time-conditioning stage (sinusoidal embedding, time-MLP hidden layer, conditioning
+ *     vector; 96 KiB) is a fixed device array in the library, which every GPU that loads the
+ *     library holds until the process exits. width and time_dim above 8192 return
+ *     JPI_ERR_SHAPE. The rest of the evaluation uses the handle's buffers, as
+ *     jpi_expert_forward does.
+ *   - The first call on a device resolves the array's device address (cudaGetSymbolAddress);
+ *     make that first call before any stream capture on that device.
+ *   - Every call shares the one array and overwrites it in full: calls that overlap on the GPU
+ *     (on different streams, or with different handles) race on it.
+ */
+JPI_API jpi_status jpi_expert_forward_noalloc(jpi_handle* h, const float* state, const float* x_t,
+                                              float t, int batch, int chunk, float* out_v,
+                                              float* out_h, void* stream);
+
+/*
  * Synchronise the handle's device work and report device-side errors: JPI_OK, or
  * JPI_ERR_DEVICE_TIMEOUT if a bounded wait inside a kernel gave up (the kernel then skipped
  * its work and returned; outputs of that call are invalid), or JPI_ERR_CUDA.

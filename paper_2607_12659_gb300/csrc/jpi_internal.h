@@ -164,6 +164,8 @@ namespace jpi {
 jpi_status configure_simt_kernels(jpi_handle* h);
 jpi_status launch_time_embed(jpi_handle* h, int nsteps, double t_override, cudaStream_t st);
 jpi_status launch_time_conditioning(jpi_handle* h, int nsteps, cudaStream_t st);
+jpi_status launch_time_conditioning_into(jpi_handle* h, double t, float* temb, float* c1,
+                                         float* cond, cudaStream_t st);
 jpi_status launch_embed(jpi_handle* h, int batch, int chunk, const float* x, cudaStream_t st);
 jpi_status launch_layer_simt(jpi_handle* h, int layer, int step, int batch, int chunk,
                              cudaStream_t st);

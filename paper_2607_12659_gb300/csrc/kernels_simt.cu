@@ -616,6 +616,33 @@ jpi_status launch_time_conditioning(jpi_handle* h, int nsteps, cudaStream_t st) 
     return h->bf16 ? time_cond<__nv_bfloat16>(h, nsteps, st) : time_cond<float>(h, nsteps, st);
 }
 
+// Time conditioning of one step time with caller-chosen scratch: sinusoid into temb [d_t],
+// time-MLP hidden layer into c1 [W], conditioning vector into cond [W]; the modulation
+// vectors go to the handle's step-0 slot, as with launch_time_conditioning(h, 1, ...).
+jpi_status launch_time_conditioning_into(jpi_handle* h, double t, float* temb, float* c1,
+                                         float* cond, cudaStream_t st) {
+    const int W = h->W, dt = h->dt;
+    const int R = mod_rows(h->L) * W;
+    k_time_embed<<<1, 128, 0, st>>>(temb, 1, dt, h->cfg.t_min_period, h->cfg.t_max_period, t);
+    const dim3 blk(256);
+    if (h->bf16) {
+        using T = __nv_bfloat16;
+        k_gemv_multi<T, true><<<grid_for((long long)W * 32, 256, 1024), blk, sizeof(float) * dt, st>>>(
+            (const T*)h->time_in_w, h->time_in_b, temb, c1, W, dt, 1);
+        k_gemv_multi<T, true><<<grid_for((long long)W * 32, 256, 1024), blk, sizeof(float) * W, st>>>(
+            (const T*)h->time_out_w, h->time_out_b, c1, cond, W, W, 1);
+        mod_gemv<T>(h, 1, cond, h->mods, R, st);
+    } else {
+        using T = float;
+        k_gemv_multi<T, true><<<grid_for((long long)W * 32, 256, 1024), blk, sizeof(float) * dt, st>>>(
+            (const T*)h->time_in_w, h->time_in_b, temb, c1, W, dt, 1);
+        k_gemv_multi<T, true><<<grid_for((long long)W * 32, 256, 1024), blk, sizeof(float) * W, st>>>(
+            (const T*)h->time_out_w, h->time_out_b, c1, cond, W, W, 1);
+        mod_gemv<T>(h, 1, cond, h->mods, R, st);
+    }
+    return check_launch("time conditioning (caller scratch)");
+}
+
 jpi_status launch_embed(jpi_handle* h, int B, int C, const float* x, cudaStream_t st) {
     const int S = C + 1;
     k_embed<<<dim3((h->W + 127) / 128, B * S), 128, 0, st>>>(

@@ -70,6 +70,8 @@ _SIGS = {
     "jpi_memory_usage": [c_void_p, POINTER(c_longlong)],
     "jpi_graph_kernel_count": [c_void_p, c_int, c_int, c_int, POINTER(c_int)],
     "jpi_profile_op": [c_void_p, c_int, c_int, c_int, c_int, c_int, c_int, c_void_p],
+    "jpi_expert_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_float, c_int, c_int, c_void_p,
+                                   c_void_p, c_void_p],
 }
 
 _lib = None
@@ -165,6 +167,13 @@ def jpi_expert_forward(h, state, x_t, t, batch, chunk, out_v, out_h=None, stream
     _check(load().jpi_expert_forward(h, _ptr(state), _ptr(x_t), float(t), batch, chunk,
                                      _ptr(out_v), _ptr(out_h), _stream(stream)),
            "jpi_expert_forward")
+
+
+def jpi_expert_forward_noalloc(h, state, x_t, t, batch, chunk, out_v, out_h=None, stream=None):
+    """jpi_expert_forward with its time-conditioning scratch in the library's fixed array."""
+    _check(load().jpi_expert_forward_noalloc(h, _ptr(state), _ptr(x_t), float(t), batch, chunk,
+                                             _ptr(out_v), _ptr(out_h), _stream(stream)),
+           "jpi_expert_forward_noalloc")
 
 
 def jpi_device_status(h):
