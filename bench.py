@@ -355,8 +355,33 @@ def our_arm(args):
         dist.destroy_process_group()
 
 
+def profile_forward(args):
+    """Small case for kernel captures: the workload's expert, two eager expert passes."""
+    import torch
+    from paper_2607_12659_gb300 import build, jpi
+    from synth import PI05, make_requests, make_weights
+    build.build()
+    jpi.load()
+    torch.cuda.set_device(0)
+    B, P, C = WORKLOAD["batch"], WORKLOAD["prefix"], WORKLOAD["chunk"]
+    ex = jpi.Expert(PI05, make_weights(PI05, 2000), max_batch=B, max_prefix=P, max_chunk=C,
+                    max_steps=WORKLOAD["steps"])
+    r = make_requests(PI05, 2001, B, P, C)
+    ex.set_prefix_kv(torch.from_numpy(r["prefix_k"]).cuda().to(torch.bfloat16),
+                     torch.from_numpy(r["prefix_v"]).cuda().to(torch.bfloat16))
+    s, x = torch.from_numpy(r["state"]).cuda(), torch.from_numpy(r["noise"]).cuda()
+    for _ in range(args.forward_passes):
+        ex.forward(s, x, 0.0)
+    torch.cuda.synchronize()
+    ex.device_status()
+    print(json.dumps({"profile_forward": "ok", "passes": args.forward_passes}))
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--profile-forward", action="store_true",
+                    help="run eager expert passes of the workload (small case for ncu captures)")
+    ap.add_argument("--forward-passes", type=int, default=2)
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
@@ -366,6 +391,9 @@ def main():
     args = ap.parse_args()
     if args.cpu_baseline_child:
         cpu_baseline_child()
+        return
+    if args.profile_forward:
+        profile_forward(args)
         return
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

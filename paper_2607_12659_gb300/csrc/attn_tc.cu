@@ -76,13 +76,18 @@ struct AttnArgs {
     int* err;
 };
 
+// One exchanged partial row: D fp16 values of O, then m and l (fp32), padded to 16 bytes.
+template <int D>
+__host__ __device__ constexpr int attn_row_bytes() {
+    return 2 * D + 16;
+}
 // Shared bytes of q/k/v, or of the 64 partial rows plus the received slices (at most
 // 64 + 15 rows: ceil(64 / splits) rows from each of up to 16 splits), whichever is larger.
 template <int D>
 __host__ __device__ constexpr int attn_region() {
-    return (3 * AT_ROWS * D * 2 > (2 * AT_ROWS + AT_MAX_SPLITS - 1) * (D + 4) * 4)
+    return (3 * AT_ROWS * D * 2 > (2 * AT_ROWS + AT_MAX_SPLITS - 1) * attn_row_bytes<D>())
                ? 3 * AT_ROWS * D * 2
-               : (2 * AT_ROWS + AT_MAX_SPLITS - 1) * (D + 4) * 4;
+               : (2 * AT_ROWS + AT_MAX_SPLITS - 1) * attn_row_bytes<D>();
 }
 
 template <int D>
@@ -92,10 +97,12 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     uint8_t* qs = smem;                                  // [64][D] bf16
     uint8_t* ks = qs + AT_ROWS * D * 2;                  // [64][D] bf16
     uint8_t* vs = ks + AT_KEYS * D * 2;                  // [64][D] bf16
-    // After the key loop: this split's partial rows [64][D + 4] (O unnormalised, then m, l) over
-    // q/k, and the slices other splits send for the rows this CTA owns right after it.
-    float* opart = (float*)smem;
-    float* recv = opart + AT_ROWS * (D + 4);             // [splits][rows_per][D + 4]
+    // After the key loop: this split's partial rows (O unnormalised in fp16, then m and l in
+    // fp32; attn_row_bytes each) over q/k, and right after them the slices other splits send
+    // for the rows this CTA owns ([splits][rows_per] rows).
+    constexpr int ROWB = attn_row_bytes<D>();
+    uint8_t* opart = smem;
+    uint8_t* recv = opart + AT_ROWS * ROWB;
     float* coef = (float*)(smem + attn_region<D>());     // [64][AT_MAX_SPLITS]
     uint64_t* rbar = (uint64_t*)(coef + AT_ROWS * AT_MAX_SPLITS);
 
@@ -246,52 +253,59 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         }
     }
 
-    // Partial rows of this split (O unnormalised, then m and l in the row padding).
+    // Partial rows of this split: O unnormalised in fp16 (a value beyond the fp16 range raises a
+    // device error), then m and l in fp32.
     __syncthreads();
+    bool range_ok = true;
 #pragma unroll
     for (int n = 0; n < D / 8; ++n) {
         const int r = warp * 16 + g, col = n * 8 + 2 * cq;
-        *(float2*)(opart + r * (D + 4) + col) = make_float2(oacc[n][0], oacc[n][1]);
-        *(float2*)(opart + (r + 8) * (D + 4) + col) = make_float2(oacc[n][2], oacc[n][3]);
+        range_ok &= fabsf(oacc[n][0]) <= 65000.f && fabsf(oacc[n][1]) <= 65000.f &&
+                    fabsf(oacc[n][2]) <= 65000.f && fabsf(oacc[n][3]) <= 65000.f;
+        *(__half2*)(opart + r * ROWB + col * 2) = __floats2half2_rn(oacc[n][0], oacc[n][1]);
+        *(__half2*)(opart + (r + 8) * ROWB + col * 2) = __floats2half2_rn(oacc[n][2], oacc[n][3]);
     }
+    if (!range_ok) atomicCAS(a.err, 0, (int)DEV_FP16_RANGE);
     if (cq == 0) {
-        *(float2*)(opart + (warp * 16 + g) * (D + 4) + D) = make_float2(m_run[0], l_run[0]);
-        *(float2*)(opart + (warp * 16 + g + 8) * (D + 4) + D) = make_float2(m_run[1], l_run[1]);
+        *(float2*)(opart + (warp * 16 + g) * ROWB + 2 * D) = make_float2(m_run[0], l_run[0]);
+        *(float2*)(opart + (warp * 16 + g + 8) * ROWB + 2 * D) = make_float2(m_run[1], l_run[1]);
     }
     // Rows [s * rows_per, ...) of the 64 belong to split rank s, which combines them.
     const int ns = a.nsplit;
     const int rank = (int)ptx::cluster_rank();
     const int rows_per = (AT_ROWS + ns - 1) / ns;
     const int r_lo = min(AT_ROWS, rank * rows_per), r_hi = min(AT_ROWS, r_lo + rows_per);
-    const uint32_t row_bytes = (uint32_t)((D + 4) * 4);
-    if (tid == 32) ptx::mbar_expect_tx(rbar, (uint32_t)(ns * (r_hi - r_lo)) * row_bytes);
+    if (tid == 32) ptx::mbar_expect_tx(rbar, (uint32_t)((ns - 1) * (r_hi - r_lo) * ROWB));
     ptx::fence_proxy_async_smem();
     // Every split is done with q/k/v (the receive buffers overlap them) and every receive
     // barrier is initialised past this point.
     ptx::cluster_sync_all();
     if (tid == 0) {
-        const uint32_t recv_u = ptx::smem_u32(recv + (size_t)rank * rows_per * (D + 4));
+        const uint32_t recv_u = ptx::smem_u32(recv + (size_t)rank * rows_per * ROWB);
         const uint32_t bar_u = ptx::smem_u32(rbar);
         for (int s = 0; s < ns; ++s) {
             const int lo = min(AT_ROWS, s * rows_per), hi = min(AT_ROWS, lo + rows_per);
-            if (hi <= lo) continue;
-            ptx::bulk_copy_to_cluster(ptx::dsmem_map(recv_u, (uint32_t)s), opart + (size_t)lo * (D + 4),
-                                      (uint32_t)(hi - lo) * row_bytes, ptx::dsmem_map(bar_u, (uint32_t)s));
+            if (hi <= lo || s == rank) continue;
+            ptx::bulk_copy_to_cluster(ptx::dsmem_map(recv_u, (uint32_t)s), opart + (size_t)lo * ROWB,
+                                      (uint32_t)((hi - lo) * ROWB), ptx::dsmem_map(bar_u, (uint32_t)s));
         }
     }
     const bool got = ptx::mbar_wait_bounded(rbar, 0, 200ull * 1000 * 1000);
+    // Row r of split s: this CTA's own partial, or the slice split s sent.
+    auto srow = [&](int s, int r) -> const uint8_t* {
+        return s == rank ? opart + (size_t)r * ROWB : recv + ((size_t)s * rows_per + (r - r_lo)) * ROWB;
+    };
 
     // Combine the splits in rank order for the owned rows, from local shared memory.
     for (int r = r_lo + tid; r < r_hi; r += AT_THREADS) {
         float mx = -INFINITY;
-        for (int s = 0; s < ns; ++s)
-            mx = fmaxf(mx, recv[((size_t)s * rows_per + (r - r_lo)) * (D + 4) + D]);
+        for (int s = 0; s < ns; ++s) mx = fmaxf(mx, *(const float*)(srow(s, r) + 2 * D));
         float L = 0.f;
         for (int s = 0; s < ns; ++s) {
-            const float* rr = recv + ((size_t)s * rows_per + (r - r_lo)) * (D + 4) + D;
-            const float w = (mx == -INFINITY) ? 0.f : exp2f(rr[0] - mx);
+            const float2 ml = *(const float2*)(srow(s, r) + 2 * D);
+            const float w = (mx == -INFINITY) ? 0.f : exp2f(ml.x - mx);
             coef[r * AT_MAX_SPLITS + s] = w;
-            L += w * rr[1];
+            L += w * ml.y;
         }
         const float inv = L > 0.f ? 1.f / L : 0.f;
         for (int s = 0; s < ns; ++s) coef[r * AT_MAX_SPLITS + s] *= inv;
@@ -305,11 +319,13 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int s = 0; s < ns; ++s) {
             const float c = coef[r * AT_MAX_SPLITS + s];
-            const float4 v = *(const float4*)(recv + ((size_t)s * rows_per + (r - r_lo)) * (D + 4) + d);
-            acc.x = fmaf(c, v.x, acc.x);
-            acc.y = fmaf(c, v.y, acc.y);
-            acc.z = fmaf(c, v.z, acc.z);
-            acc.w = fmaf(c, v.w, acc.w);
+            const uint2 hv = *(const uint2*)(srow(s, r) + 2 * d);
+            const float2 v01 = __half22float2(*reinterpret_cast<const __half2*>(&hv.x));
+            const float2 v23 = __half22float2(*reinterpret_cast<const __half2*>(&hv.y));
+            acc.x = fmaf(c, v01.x, acc.x);
+            acc.y = fmaf(c, v01.y, acc.y);
+            acc.z = fmaf(c, v23.x, acc.z);
+            acc.w = fmaf(c, v23.y, acc.w);
         }
         const int i = R / a.H, head = R - i * a.H;
         const size_t tok = (size_t)b * a.S + i;

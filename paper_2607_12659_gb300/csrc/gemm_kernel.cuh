@@ -24,12 +24,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
     // Offsetting the shared array itself (not a cast through an integer) keeps every access
     // below in the shared state space.
     uint8_t* smem = smem_raw + ((1024u - (ptx::smem_u32(smem_raw) & 1023u)) & 1023u);
-    const int xp_bytes = max(a.kpb * XBLK_BYTES, TILE_ROWS * PSTRIDE * 4);
+    const int xp_bytes = max(a.kpb * XBLK_BYTES, RECV_BYTES);
     uint8_t* wsm = smem;                                   // kpb weight tiles
     uint8_t* xsm = wsm + a.kpb * TILE_BYTES;               // X blocks, then the outgoing partial
-    float* part = (float*)xsm;                             // [128][PSTRIDE] this CTA's fp32 product
+    __half* part = (__half*)xsm;                           // [128][PSTRIDE] this CTA's product
     // [splits][2 * npairs][PSTRIDE] received slices: in the weight region or after the partial.
-    float* recv = a.recv_alias ? (float*)wsm : (float*)(xsm + xp_bytes);
+    __half* recv = a.recv_alias ? (__half*)wsm : (__half*)(xsm + xp_bytes);
     float* slots = (float*)(xsm + xp_bytes + (a.recv_alias ? 0 : RECV_BYTES));   // [MAX_SPLITS][NT]
     float* rinv = slots + MAX_SPLITS * NT;                 // [NT]
     float* sspart = rinv + NT;                             // [GEMM_THREADS][4]
@@ -90,7 +90,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
             for (int j = 0; j < a.kpb; ++j)
                 ptx::tma_load_2d(xsm + j * XBLK_BYTES, &xmap, &bars[1], (kb0 + j) * KBLK, tok0, pol);
         }
-        if (tid == 32) ptx::mbar_expect_tx(&bars[3], (uint32_t)(TILE_ROWS * PSTRIDE * 4));
+        if (tid == 32)
+            ptx::mbar_expect_tx(&bars[3], (uint32_t)((a.splits - 1) * 2 * npairs * PSTRIDE * 2));
         if (NORM_IN) {
             if (tid >= 64 && tid < 64 + NT) {
                 const int tok = tok0 + tid - 64;
@@ -177,20 +178,30 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         const bool ok = *flag == 0;
         ptx::tc_fence_after();
 
-        // ---- 3a. TMEM -> fp32 partial in shared memory (warp w: lanes 32 (w mod 4), half w / 4) ----
+        // ---- 3a. TMEM -> fp16 partial in shared memory (warp w: lanes 32 (w mod 4), half w / 4).
+        // fp16 halves the bytes the cluster exchanges; a partial beyond the fp16 range raises a
+        // device error instead of overflowing silently.
         if (ok) {
             const int row = (warp & 3) * 32 + lane, cbase = (warp >> 2) * (NT / 2);
+            bool range_ok = true;
 #pragma unroll
             for (int c0 = 0; c0 < NT / 2; c0 += 16) {
                 uint32_t r[16];
                 ptx::tmem_ld_x16(tmem + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(cbase + c0), r);
                 ptx::tmem_ld_wait();
-                float4* dst = (float4*)(part + row * PSTRIDE + cbase + c0);
+                uint32_t hp[8];
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4)
-                    dst[q4] = make_float4(__uint_as_float(r[4 * q4]), __uint_as_float(r[4 * q4 + 1]),
-                                          __uint_as_float(r[4 * q4 + 2]), __uint_as_float(r[4 * q4 + 3]));
+                for (int i = 0; i < 8; ++i) {
+                    const float v0 = __uint_as_float(r[2 * i]), v1 = __uint_as_float(r[2 * i + 1]);
+                    range_ok &= fabsf(v0) <= 65000.f && fabsf(v1) <= 65000.f;
+                    __half2 hv = __floats2half2_rn(v0, v1);
+                    hp[i] = *reinterpret_cast<uint32_t*>(&hv);
+                }
+                uint4* dst = (uint4*)(part + row * PSTRIDE + cbase + c0);
+                dst[0] = make_uint4(hp[0], hp[1], hp[2], hp[3]);
+                dst[1] = make_uint4(hp[4], hp[5], hp[6], hp[7]);
             }
+            if (!range_ok) set_device_error(a.err, DEV_FP16_RANGE);
         }
         ptx::tc_fence_before();
         ptx::fence_proxy_async_smem();
@@ -198,12 +209,13 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         // barrier is initialised past this point.
         ptx::cluster_sync_all();
 
-        // ---- 3b. push each rank's rows (pairs r*npairs.. and +64) to that rank ----
+        // ---- 3b. push each other rank's rows (pairs r*npairs.. and +64) to that rank ----
         if (tid == 0) {
-            const uint32_t chunk = (uint32_t)(npairs * PSTRIDE * 4);
+            const uint32_t chunk = (uint32_t)(npairs * PSTRIDE * 2);
             const uint32_t recv_u = ptx::smem_u32(recv + (size_t)rank * 2 * npairs * PSTRIDE);
             const uint32_t bar_u = ptx::smem_u32(&bars[3]);
             for (int r = 0; r < a.splits; ++r) {
+                if (r == rank) continue;
                 const uint32_t dst = ptx::dsmem_map(recv_u, (uint32_t)r);
                 const uint32_t rbar = ptx::dsmem_map(bar_u, (uint32_t)r);
                 ptx::bulk_copy_to_cluster(dst, part + (size_t)r * npairs * PSTRIDE, chunk, rbar);
@@ -212,15 +224,19 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         }
         if (!ptx::mbar_wait_bounded(&bars[3], tt & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
 
-        // ---- 4. rank-ordered sum of the received slices + epilogue; item = (pair, 4 tokens) ----
+        // ---- 4. rank-ordered sum of the slices (own rows read in place) + epilogue ----
         float ssq[4] = {0.f, 0.f, 0.f, 0.f};
         for (int item = tid; item < nitems; item += GEMM_THREADS) {
             if (item != tid) prefetch(item);
             const int pi = item / QUADS, t0 = (item % QUADS) * 4, p = p0 + pi;
             float4 y1 = make_float4(0.f, 0.f, 0.f, 0.f), y2 = y1;
             for (int r = 0; r < a.splits; ++r) {
-                f4add(y1, *(const float4*)(recv + ((size_t)r * 2 * npairs + pi) * PSTRIDE + t0));
-                f4add(y2, *(const float4*)(recv + ((size_t)r * 2 * npairs + npairs + pi) * PSTRIDE + t0));
+                const __half* s1 = (r == rank) ? part + (size_t)p * PSTRIDE + t0
+                                               : recv + ((size_t)r * 2 * npairs + pi) * PSTRIDE + t0;
+                const __half* s2 = (r == rank) ? part + (size_t)(p + 64) * PSTRIDE + t0
+                                               : recv + ((size_t)r * 2 * npairs + npairs + pi) * PSTRIDE + t0;
+                f4add(y1, half4_to_float4(*(const uint2*)s1));
+                f4add(y2, half4_to_float4(*(const uint2*)s2));
             }
             if (!ok) continue;
             const int f1 = tile * TILE_ROWS + p, f2 = f1 + 64;

@@ -33,11 +33,11 @@ constexpr int TILE_ROWS = 128;                 // weight rows per tile (M)
 constexpr int KBLK = 64;                       // K elements per block: one 128-byte swizzle row
 constexpr int TILE_BYTES = TILE_ROWS * KBLK * 2;
 constexpr int XBLK_BYTES = NT * KBLK * 2;
-constexpr int PSTRIDE = NT + 4;                // fp32 partial row stride (floats)
+constexpr int PSTRIDE = NT + 8;                // fp16 partial row stride (halves, 144 bytes)
 constexpr int GEMM_THREADS = 256;
 constexpr int MAX_SPLITS = 16;
 constexpr int QUADS = NT / 4;                  // token quads per tile
-constexpr int RECV_BYTES = TILE_ROWS * PSTRIDE * 4;   // received split-K slices of one tile
+constexpr int RECV_BYTES = TILE_ROWS * PSTRIDE * 2;   // split-K slices of one tile (fp16)
 constexpr uint64_t WAIT_LIMIT_NS = 200ull * 1000 * 1000;   // 0.2 s
 
 enum GemmKind { G_QKV = 0, G_O = 1, G_GU = 2, G_DOWN = 3 };
@@ -88,6 +88,11 @@ __device__ __forceinline__ void set_device_error(int* err, int code) { atomicCAS
 
 __device__ __forceinline__ float f4get(const float4& v, int e) {
     return e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
+}
+__device__ __forceinline__ float4 half4_to_float4(uint2 v) {
+    const float2 lo = __half22float2(*reinterpret_cast<__half2*>(&v.x));
+    const float2 hi = __half22float2(*reinterpret_cast<__half2*>(&v.y));
+    return make_float4(lo.x, lo.y, hi.x, hi.y);
 }
 __device__ __forceinline__ void f4add(float4& a, const float4& b) {
     a.x += b.x;
