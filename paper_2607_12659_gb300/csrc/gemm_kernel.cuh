@@ -107,25 +107,34 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         if (!ptx::mbar_wait_bounded(&bars[1], tt & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_WEIGHTS;
         if (NORM_IN) {
             __syncthreads();
-            // In place: u = h * rinv * (1 + sigma) + beta on each swizzled 16-byte chunk.
-            for (int idx = tid; idx < a.kpb * NT * 8; idx += GEMM_THREADS) {
-                const int j = idx / (NT * 8), t = (idx >> 3) % NT, q = idx & 7;
-                const int c = q ^ (t & 7);                         // logical chunk of row t
-                const int kl = j * KBLK + c * 8;                   // index into this CTA's slice
-                uint4* p = (uint4*)(xsm + j * XBLK_BYTES + t * 128 + q * 16);
-                const uint4 v = *p;
-                const float r = rinv[t];
+            // In place: u = h * rinv * (1 + sigma) + beta on each swizzled 16-byte chunk. Thread
+            // = physical chunk q of rows tr and tr + 32 (GEMM_THREADS / 8 == 32); both rows hold
+            // the same logical chunk c = q ^ (tr mod 8), so sigma/beta are read once per block.
+            static_assert(GEMM_THREADS == 8 * 32, "transform mapping assumes 256 threads");
+            const int q = tid & 7, tr = tid >> 3, c = q ^ (tr & 7);
+            const float r0 = (tok0 + tr < a.Mt) ? rinv[tr] : 0.f;
+            const float r1 = (tok0 + tr + 32 < a.Mt) ? rinv[tr + 32] : 0.f;
+            for (int j = 0; j < a.kpb; ++j) {
+                const int kl = j * KBLK + c * 8;
+                uint4* p0 = (uint4*)(xsm + j * XBLK_BYTES + tr * 128 + q * 16);
+                uint4* p1 = p0 + 32 * 128 / 16;
+                const uint4 v0 = *p0, v1 = *p1;
                 const float4 s0 = *(const float4*)(sig + kl), s1 = *(const float4*)(sig + kl + 4);
                 const float4 b0 = *(const float4*)(bet + kl), b1 = *(const float4*)(bet + kl + 4);
-                const float2 h0 = unpack_half2(v.x), h1 = unpack_half2(v.y);
-                const float2 h2 = unpack_half2(v.z), h3 = unpack_half2(v.w);
-                uint4 o;
-                o.x = pack_bf16x2(h0.x * r * (1.f + s0.x) + b0.x, h0.y * r * (1.f + s0.y) + b0.y);
-                o.y = pack_bf16x2(h1.x * r * (1.f + s0.z) + b0.z, h1.y * r * (1.f + s0.w) + b0.w);
-                o.z = pack_bf16x2(h2.x * r * (1.f + s1.x) + b1.x, h2.y * r * (1.f + s1.y) + b1.y);
-                o.w = pack_bf16x2(h3.x * r * (1.f + s1.z) + b1.z, h3.y * r * (1.f + s1.w) + b1.w);
-                if (tok0 + t >= a.Mt) o = make_uint4(0u, 0u, 0u, 0u);
-                *p = o;
+                const float g[8] = {1.f + s0.x, 1.f + s0.y, 1.f + s0.z, 1.f + s0.w,
+                                    1.f + s1.x, 1.f + s1.y, 1.f + s1.z, 1.f + s1.w};
+                const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+                const uint32_t in0[4] = {v0.x, v0.y, v0.z, v0.w}, in1[4] = {v1.x, v1.y, v1.z, v1.w};
+                uint32_t o0[4], o1[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 h0 = unpack_half2(in0[e]), h1 = unpack_half2(in1[e]);
+                    // Padding tokens (>= Mt) become exactly zero: rinv 0 and no shift.
+                    o0[e] = r0 != 0.f ? pack_bf16x2(h0.x * r0 * g[2 * e] + bb[2 * e], h0.y * r0 * g[2 * e + 1] + bb[2 * e + 1]) : 0u;
+                    o1[e] = r1 != 0.f ? pack_bf16x2(h1.x * r1 * g[2 * e] + bb[2 * e], h1.y * r1 * g[2 * e + 1] + bb[2 * e + 1]) : 0u;
+                }
+                *p0 = make_uint4(o0[0], o0[1], o0[2], o0[3]);
+                *p1 = make_uint4(o1[0], o1[1], o1[2], o1[3]);
             }
             ptx::fence_proxy_async_smem();
         }
