@@ -225,8 +225,9 @@ jpi_status alloc_buffers(jpi_handle* h) {
     JPI_CUDA_TRY(cudaMemset(h->h, 0, Mt * W * sizeof(float)));
     JPI_TRY(dev_alloc(h, (char**)&h->hx, Mt * W * 2));
     JPI_CUDA_TRY(cudaMemset(h->hx, 0, Mt * W * 2));
-    JPI_TRY(dev_alloc(h, &h->ss, (size_t)((W + 127) / 128) * Mt));
-    JPI_CUDA_TRY(cudaMemset(h->ss, 0, (size_t)((W + 127) / 128) * Mt * sizeof(float)));
+    const size_t ss_slots = (size_t)((W + 127) / 128) * MAX_SPLIT_K;
+    JPI_TRY(dev_alloc(h, &h->ss, ss_slots * Mt));
+    JPI_CUDA_TRY(cudaMemset(h->ss, 0, ss_slots * Mt * sizeof(float)));
     JPI_TRY(dev_alloc(h, &h->dev_err, 4));
     JPI_CUDA_TRY(cudaMemset(h->dev_err, 0, 4 * sizeof(int)));
     if (h->cfg.rope_base > 0.f) {

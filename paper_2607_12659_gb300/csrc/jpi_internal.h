@@ -50,6 +50,10 @@ enum DeviceError : int {
 // the final norm's (sigma, beta) at 6 L + {0, 1}.
 inline int mod_rows(int L) { return 6 * L + 2; }
 
+// Largest split of a projection's K range over the CTAs of a cluster. The per-token sums of
+// squares of the residual stream are kept in up to (W / 128) x MAX_SPLIT_K slots.
+constexpr int MAX_SPLIT_K = 16;
+
 // Plain (un-tiled) layer weights used by the CUDA-core kernels.
 struct LayerPlain {
     void* wqkv;   // [(H+2) D][W]: rows of wq, then wk, then wv
@@ -75,7 +79,6 @@ struct LayerTiled {
 // K by a cluster of `splits` CTAs that own `kpb` 64-wide K blocks apiece.
 struct GemmPlan {
     int rows = 0, K = 0, ntiles = 0, nkb = 0, kpb = 0, splits = 0, ctas = 0;
-    int recv_alias = 0;   // received split-K slices overwrite the weight tiles
     size_t smem = 0;
 };
 
@@ -144,9 +147,9 @@ struct jpi_handle {
     void* hx = nullptr;         // [maxMt][W] fp16 copy of h, read by the norm-fed GEMMs
     int* dev_err = nullptr;     // device error word
 
-    // Tensor-core path: plans ([0] one 64-token tile, [1] several) and tensor maps
-    // (4 per layer: QKV, O, gate/up, down).
-    jpi::GemmPlan plans[2][4];
+    // Tensor-core path: one plan per projection (QKV, O, gate/up, down) and tensor maps
+    // (4 per layer, same order).
+    jpi::GemmPlan plans[4];
     std::vector<CUtensorMap> tmaps;
     CUtensorMap xmaps[3];       // B operands: hx, o, z
 

@@ -33,21 +33,18 @@ constexpr int TILE_ROWS = 128;                 // weight rows per tile (M)
 constexpr int KBLK = 64;                       // K elements per block: one 128-byte swizzle row
 constexpr int TILE_BYTES = TILE_ROWS * KBLK * 2;
 constexpr int XBLK_BYTES = NT * KBLK * 2;
-constexpr int PSTRIDE = NT + 8;                // fp16 partial row stride (halves, 144 bytes)
+constexpr int PART_BYTES = TILE_ROWS * NT * 2;  // fp16 partial of one tile (128-byte rows)
 constexpr int GEMM_THREADS = 256;
-constexpr int MAX_SPLITS = 16;
 constexpr int QUADS = NT / 4;                  // token quads per tile
-constexpr int RECV_BYTES = TILE_ROWS * PSTRIDE * 2;   // split-K slices of one tile (fp16)
 constexpr uint64_t WAIT_LIMIT_NS = 200ull * 1000 * 1000;   // 0.2 s
 
 enum GemmKind { G_QKV = 0, G_O = 1, G_GU = 2, G_DOWN = 3 };
 
 struct GemmArgs {
     int Mt, K, nkb, kpb, splits;
-    int recv_alias;          // 1: received slices overwrite the weight tiles (single token tile)
     // RMSNorm-fed projections (QKV, gate/up): u = h * rinv * (1 + sigma) + beta, with rinv from
     // the per-token sums of squares left by the producer of h.
-    const float* ss;         // [nslot][ss_ld]: sum of h^2 over each 128-feature slice
+    const float* ss;         // [nslot][ss_ld]: sums of h^2 over disjoint feature ranges
     int nslot, ss_ld;
     const float* sigma;
     const float* beta;
@@ -56,7 +53,7 @@ struct GemmArgs {
     float* hres;
     __half* hx;              // fp16 copy of the residual stream (B operand of the next norm-fed GEMM)
     const float* gamma;
-    float* ss_out;
+    float* ss_out;           // slot (tile * splits + rank): this CTA's features
     int W;
     // QKV epilogue.
     __nv_bfloat16* q;
@@ -101,24 +98,45 @@ __device__ __forceinline__ void f4add(float4& a, const float4& b) {
     a.w += b.w;
 }
 
+// Shared-memory layout of one GEMM CTA (byte offsets from the 1024-aligned base).
+struct GemmSmem {
+    int x, recv, misc, ssred, bars, total;
+};
+__host__ __device__ __forceinline__ GemmSmem gemm_layout(int kpb, int splits, bool norm_in) {
+    GemmSmem L;
+    const int xbytes = kpb * XBLK_BYTES > PART_BYTES ? kpb * XBLK_BYTES : PART_BYTES;
+    const int ssred_bytes = 2 * NT * (int)sizeof(float);
+    L.x = kpb * TILE_BYTES;
+    L.recv = L.x + xbytes;
+    L.misc = L.recv + (splits - 1) * (TILE_ROWS / splits) * NT * 2;
+    int end = L.misc + (norm_in ? (4 * NT + 2 * kpb * KBLK) * (int)sizeof(float) : 0);
+    if (norm_in) {
+        L.ssred = L.misc;                               // unused by the norm-fed kinds
+    } else if (xbytes >= PART_BYTES + ssred_bytes) {
+        L.ssred = L.x + PART_BYTES;                     // X blocks are dead once the MMA is done
+    } else {
+        L.ssred = end;
+        end += ssred_bytes;
+    }
+    L.bars = (end + 7) & ~7;
+    L.total = L.bars + 64;
+    return L;
+}
+
 #include "gemm_kernel.cuh"
 
 // ---------------------------------------------------------------------------------------------
 // Host side: packing, plans, tensor maps, launches.
 
-bool recv_in_weights(int kpb, bool single_tile) {
-    return single_tile && (size_t)kpb * TILE_BYTES >= (size_t)RECV_BYTES;
+size_t gemm_smem(int kpb, int splits, bool norm_in) {
+    return 1024 + (size_t)gemm_layout(kpb, splits, norm_in).total;
 }
 
-size_t gemm_smem(int kpb, bool single_tile) {
-    const size_t xp = std::max((size_t)kpb * XBLK_BYTES, (size_t)RECV_BYTES);
-    return 1024 + (size_t)kpb * TILE_BYTES + xp + (recv_in_weights(kpb, single_tile) ? 0 : RECV_BYTES) +
-           sizeof(float) * (MAX_SPLITS * NT + NT + 4 * GEMM_THREADS + 16 * KBLK) + 64;
-}
-
-// Chooses the K blocks per CTA: one wave on the device, little weight per SM, and shared
-// memory small enough (<= 113 KB) for the next kernel's CTAs to start prefetching alongside.
-bool make_plan(int rows, int K, int max_cluster, int num_sms, bool single_tile, GemmPlan* out) {
+// Chooses the K blocks per CTA: one wave on the device, then at most 8 CTAs per cluster (each
+// extra rank adds two pushes to every CTA's exchange and a slice to every owner's sum, which
+// measured slower than streaming more weight per CTA), then little weight per SM, then shared
+// memory small enough (<= 113 KB) for two CTAs per SM.
+bool make_plan(int rows, int K, int max_cluster, int num_sms, bool norm_in, GemmPlan* out) {
     if (rows % TILE_ROWS || K % KBLK) return false;
     GemmPlan best;
     long best_score = -1;
@@ -126,20 +144,19 @@ bool make_plan(int rows, int K, int max_cluster, int num_sms, bool single_tile, 
     for (int kpb = 1; kpb <= 8; kpb *= 2) {
         if (nkb % kpb) continue;
         const int splits = nkb / kpb;
-        if (splits > max_cluster || 64 % splits) continue;
-        const size_t smem = gemm_smem(kpb, single_tile);
+        if (splits > std::min(max_cluster, MAX_SPLIT_K) || 64 % splits) continue;
+        const size_t smem = gemm_smem(kpb, splits, norm_in);
         if (smem > 227 * 1024) continue;
         const int res = std::min(2, (int)((228 * 1024) / (smem + 1024)));
         const int ctas = ntiles * splits;
         const long waves = (ctas + (long)num_sms * res - 1) / ((long)num_sms * res);
         const long per_sm = (ctas + num_sms - 1) / num_sms;
-        const long score = waves * 10000 + (smem > 113 * 1024 ? 1000 : 0) + per_sm * kpb * 10 +
-                           (ctas > num_sms ? 1 : 0);
+        const long score = waves * 10000 + std::max(splits - 8, 0) * 100 + per_sm * kpb * 10 +
+                           (smem > 113 * 1024 ? 5 : 0) + (ctas > num_sms ? 1 : 0);
         if (best_score < 0 || score < best_score) {
             best_score = score;
             best.rows = rows; best.K = K; best.ntiles = ntiles; best.nkb = nkb; best.kpb = kpb;
             best.splits = splits; best.ctas = ctas; best.smem = smem;
-            best.recv_alias = recv_in_weights(kpb, single_tile) ? 1 : 0;
         }
     }
     if (best_score < 0) return false;
@@ -267,7 +284,6 @@ GemmArgs base_args(jpi_handle* h, int B, int C, const GemmPlan& pl) {
     a.nkb = pl.nkb;
     a.kpb = pl.kpb;
     a.splits = pl.splits;
-    a.recv_alias = pl.recv_alias;
     a.ss = h->ss;
     a.nslot = h->W / TILE_ROWS;
     a.ss_ld = h->maxMt;
@@ -356,27 +372,17 @@ jpi_status tc_prepare(jpi_handle* h) {
     }
     const int rows[4] = {h->QKV, h->W, 2 * h->F, h->W};
     const int ks[4] = {h->W, h->HD, h->W, h->F};
-    // The K split (and so the summation order) is chosen once per projection and shared by the
-    // one-tile and several-tile variants, which differ only in where the received slices live:
-    // a request's result does not depend on how many other requests share its batch.
+    // The K split (and so the summation order) is chosen once per projection, for every batch
+    // size: a request's result does not depend on how many other requests share its batch.
     for (int g = 0; g < 4; ++g) {
-        if (!make_plan(rows[g], ks[g], max_cluster, sms, true, &h->plans[0][g])) {
+        if (!make_plan(rows[g], ks[g], max_cluster, sms, g == G_QKV || g == G_GU, &h->plans[g])) {
             set_error("no tensor-core tiling for a %d x %d projection", rows[g], ks[g]);
-            return JPI_ERR_UNSUPPORTED;
-        }
-        h->plans[1][g] = h->plans[0][g];
-        h->plans[1][g].recv_alias = 0;
-        h->plans[1][g].smem = gemm_smem(h->plans[0][g].kpb, false);
-        if (h->plans[1][g].smem > 227 * 1024) {
-            set_error("the several-tile variant of a %d x %d projection needs too much shared memory",
-                      rows[g], ks[g]);
             return JPI_ERR_UNSUPPORTED;
         }
     }
     // A cluster of `splits` CTAs must fit on the device at this shared-memory size.
-    for (int vg = 0; vg < 8; ++vg) {
-        const int g = vg % 4;
-        const GemmPlan& pl = h->plans[vg / 4][g];
+    for (int g = 0; g < 4; ++g) {
+        const GemmPlan& pl = h->plans[g];
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(pl.ctas);
         cfg.blockDim = dim3(GEMM_THREADS);
@@ -423,13 +429,16 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
     const int W = h->W;
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * W + (size_t)6 * l * W;
     const size_t kv_layer = (size_t)l * h->maxB * h->kv_rows * h->D;
-    const jpi::GemmPlan* plans = h->plans[B * (C + 1) <= NT ? 0 : 1];
+    const jpi::GemmPlan* plans = h->plans;
     switch (op) {
         case 2: {
             const GemmPlan& pl = plans[G_QKV];
             GemmArgs a = base_args(h, B, C, pl);
             a.sigma = ms;
             a.beta = ms + W;
+            // Sums of squares left by the embedding (one per 128 features) or the previous
+            // layer's down projection (one per CTA).
+            if (l > 0) a.nslot = plans[G_DOWN].ntiles * plans[G_DOWN].splits;
             a.q = (__nv_bfloat16*)h->q;
             a.kst = (__nv_bfloat16*)h->kv_k + kv_layer;
             a.vst = (__nv_bfloat16*)h->kv_v + kv_layer;
@@ -453,6 +462,7 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
             GemmArgs a = base_args(h, B, C, pl);
             a.sigma = ms + 3 * W;
             a.beta = ms + 4 * W;
+            a.nslot = plans[G_O].ntiles * plans[G_O].splits;   // left by the output projection
             a.z = (__nv_bfloat16*)h->z;
             return launch_gemm<G_GU>(h, pl, h->tmaps[4 * l + G_GU], h->xmaps[0], a, st);
         }
