@@ -8,11 +8,15 @@
 // S x H query rows form one dense [S*H][D] x [D][P+S] problem; rows are ordered token-major
 // (row = i * H + head). The state row (i = 0) sees the prefix and itself only.
 //
-// Grid: (64-row query blocks, key splits, requests). The key splits of one query block form a
-// thread-block cluster: each CTA runs an online softmax over its key range (blocks of 64 keys
-// staged in shared memory with cp.async), then the cluster combines the partial (max, sum,
-// output) triples through distributed shared memory in split order, so the result does not
-// depend on timing.
+// Grid: (32-row query blocks, key splits, requests). The key splits of one query block form a
+// thread-block cluster. Inside a CTA, warp w takes query rows 16 (w mod 2) .. + 15 and key half
+// w / 2 of every 64-key block (staged in shared memory with cp.async), with its own online
+// softmax; the two key halves of a row group are merged in shared memory, and the cluster then
+// combines the per-split (max, sum, output) triples through distributed shared memory in split
+// order, so the result does not depend on timing. Each split pushes the rows owned by every other
+// split into that split's dedicated receive buffer as soon as its own rows are final; the only
+// cluster-wide waits are one before the first push (receive barriers initialised) and one before
+// exit (every copy out of this CTA has landed).
 
 #include "jpi_internal.h"
 #include "ptx.h"
@@ -24,10 +28,12 @@ namespace cg = cooperative_groups;
 namespace jpi {
 namespace {
 
-constexpr int AT_ROWS = 64;      // query rows per CTA (4 warps x 16)
-constexpr int AT_KEYS = 64;      // keys per shared-memory block
-constexpr int AT_THREADS = 128;
+constexpr int AT_ROWS = 32;      // query rows per CTA (2 row groups of 16)
+constexpr int AT_KEYS = 64;      // keys per shared-memory block (2 halves of 32)
+constexpr int AT_THREADS = 128;  // 4 warps: (row group, key half)
 constexpr int AT_MAX_SPLITS = 16;
+// Most rows one split receives: (splits - 1) x ceil(32 / splits), largest at 15 splits.
+constexpr int AT_MAX_RECV_ROWS = 42;
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
@@ -81,41 +87,67 @@ template <int D>
 __host__ __device__ constexpr int attn_row_bytes() {
     return 2 * D + 16;
 }
-// Shared bytes of q/k/v, or of the 64 partial rows plus the received slices (at most
-// 64 + 15 rows: ceil(64 / splits) rows from each of up to 16 splits), whichever is larger.
+// Row stride (floats) of the fp32 staging of the second key half: 8 floats of padding put the
+// 4 rows a half-warp writes at one column (8-byte accesses) on disjoint banks.
 template <int D>
-__host__ __device__ constexpr int attn_region() {
-    return (3 * AT_ROWS * D * 2 > (2 * AT_ROWS + AT_MAX_SPLITS - 1) * attn_row_bytes<D>())
-               ? 3 * AT_ROWS * D * 2
-               : (2 * AT_ROWS + AT_MAX_SPLITS - 1) * attn_row_bytes<D>();
+__host__ __device__ constexpr int attn_ofp_stride() {
+    return D + 8;
 }
+// Shared-memory layout (bytes from the 128-aligned base): q/k/v, reused after the key loop for
+// the second key half's fp32 output and (m, l) and then this split's partial rows; the receive
+// buffer; the combine coefficients; the receive barrier.
+template <int D>
+struct AttnSmem {
+    static constexpr int QKV = (AT_ROWS + 2 * AT_KEYS) * D * 2;
+    static constexpr int OFP = AT_ROWS * attn_ofp_stride<D>() * 4;
+    static constexpr int ML1 = OFP;                              // [32] float2 after the fp32 rows
+    static constexpr int OPART = OFP + AT_ROWS * 8;              // [32][row bytes]
+    static constexpr int REGION_USED = OPART + AT_ROWS * attn_row_bytes<D>();
+    static constexpr int REGION = QKV > REGION_USED ? QKV : REGION_USED;
+    static constexpr int RECV = REGION;                          // [AT_MAX_RECV_ROWS][row bytes]
+    static constexpr int COEF = RECV + AT_MAX_RECV_ROWS * attn_row_bytes<D>();   // [32][16] floats
+    static constexpr int BAR = COEF + AT_ROWS * AT_MAX_SPLITS * 4;
+    static constexpr int TOTAL = BAR + 16;
+};
 
 template <int D>
 __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ AttnArgs a) {
+    using L = AttnSmem<D>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((128u - (ptx::smem_u32(smem_raw) & 127u)) & 127u);
-    uint8_t* qs = smem;                                  // [64][D] bf16
+    uint8_t* qs = smem;                                  // [32][D] bf16
     uint8_t* ks = qs + AT_ROWS * D * 2;                  // [64][D] bf16
     uint8_t* vs = ks + AT_KEYS * D * 2;                  // [64][D] bf16
-    // After the key loop: this split's partial rows (O unnormalised in fp16, then m and l in
-    // fp32; attn_row_bytes each) over q/k, and right after them the slices other splits send
-    // for the rows this CTA owns ([splits][rows_per] rows).
     constexpr int ROWB = attn_row_bytes<D>();
-    uint8_t* opart = smem;
-    uint8_t* recv = opart + AT_ROWS * ROWB;
-    float* coef = (float*)(smem + attn_region<D>());     // [64][AT_MAX_SPLITS]
-    uint64_t* rbar = (uint64_t*)(coef + AT_ROWS * AT_MAX_SPLITS);
+    constexpr int OS = attn_ofp_stride<D>();
+    float* ofp = (float*)smem;                           // [32][OS] second key half's O (fp32)
+    float2* ml1 = (float2*)(smem + L::ML1);              // [32] its (m, l)
+    uint8_t* opart = smem + L::OPART;                    // [32][ROWB] this split's partial rows
+    uint8_t* recv = smem + L::RECV;                      // [(splits - 1) x rows_per][ROWB]
+    float* coef = (float*)(smem + L::COEF);              // [32][AT_MAX_SPLITS]
+    uint64_t* rbar = (uint64_t*)(smem + L::BAR);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int rb = blockIdx.x, split = blockIdx.y, b = blockIdx.z;
+    const int rg = warp & 1, kh = warp >> 1;             // row group, key half
+    const int rb = blockIdx.x, b = blockIdx.z;
     const int nrows = a.S * a.H, nk = a.P + a.S;
     const int row0 = rb * AT_ROWS;
-    const int k_begin = split * a.chunk, k_end = min(nk, k_begin + a.chunk);
+    const int ns = a.nsplit;
+    const int rank = (int)ptx::cluster_rank();           // == blockIdx.y (cluster spans the splits)
+    const int k_begin = rank * a.chunk, k_end = min(nk, k_begin + a.chunk);
+    // Rows [s * rows_per, ...) of the 32 belong to split s, which combines them.
+    const int rows_per = (AT_ROWS + ns - 1) / ns;
+    const int r_lo = min(AT_ROWS, rank * rows_per), r_hi = min(AT_ROWS, r_lo + rows_per);
     constexpr int DC = D / 8;                            // 16-byte chunks per row
     if (tid == 0) {
         ptx::mbar_init(rbar, 1);
         ptx::fence_mbar_init();
+        ptx::mbar_expect_tx(rbar, (uint32_t)((ns - 1) * (r_hi - r_lo) * ROWB));
     }
+    __syncthreads();
+    // Receive barriers are initialised cluster-wide before anyone pushes: arrive now, wait
+    // before the first push.
+    ptx::cluster_arrive();
 
     // Prefix keys/values were written before this graph ran: the first block's prefix rows are
     // fetched before the dependency wait; the suffix rows (written by the QKV kernel) after it.
@@ -152,7 +184,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     int nvis[2];
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
-        const int R = row0 + warp * 16 + g + hh * 8;
+        const int R = row0 + rg * 16 + g + hh * 8;
         const int i = R / a.H;
         nvis[hh] = (R < nrows && i == 0) ? a.P + 1 : nk;
     }
@@ -161,6 +193,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
 #pragma unroll
     for (int n = 0; n < D / 8; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.f;
     float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+    constexpr int HK = AT_KEYS / 2;                      // keys per half
 
     for (int key0 = k_begin; key0 < k_end; key0 += AT_KEYS) {
         __syncthreads();
@@ -168,22 +201,22 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         cp_async_wait_all();
         __syncthreads();
 
-        // S = Q K^T for this warp's 16 rows x 64 keys.
-        float sacc[AT_KEYS / 8][4];
+        // S = Q K^T for this warp's 16 rows x 32 keys.
+        float sacc[HK / 8][4];
 #pragma unroll
-        for (int n = 0; n < AT_KEYS / 8; ++n) sacc[n][0] = sacc[n][1] = sacc[n][2] = sacc[n][3] = 0.f;
+        for (int n = 0; n < HK / 8; ++n) sacc[n][0] = sacc[n][1] = sacc[n][2] = sacc[n][3] = 0.f;
 #pragma unroll
         for (int kc = 0; kc < D / 16; ++kc) {
             uint32_t a0, a1, a2, a3;
             {
-                const int r = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int r = rg * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                 const int c = kc * 2 + (lane >> 4);
                 ldsm_x4(qs_u + sw_off<D>(r, c), a0, a1, a2, a3);
             }
 #pragma unroll
-            for (int nt = 0; nt < AT_KEYS / 8; nt += 2) {
+            for (int nt = 0; nt < HK / 8; nt += 2) {
                 uint32_t b0, b1, b2, b3;
-                const int r = (nt + (lane >> 4)) * 8 + (lane & 7);
+                const int r = kh * HK + (nt + (lane >> 4)) * 8 + (lane & 7);
                 const int c = kc * 2 + ((lane >> 3) & 1);
                 ldsm_x4(ks_u + sw_off<D>(r, c), b0, b1, b2, b3);
                 mma16816(sacc[nt], a0, a1, a2, a3, b0, b1);
@@ -193,10 +226,10 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         // Scale to log2 units, mask, online softmax.
         float bmax[2] = {-INFINITY, -INFINITY};
 #pragma unroll
-        for (int nt = 0; nt < AT_KEYS / 8; ++nt)
+        for (int nt = 0; nt < HK / 8; ++nt)
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-                const int key = key0 + nt * 8 + 2 * cq + (e & 1);
+                const int key = key0 + kh * HK + nt * 8 + 2 * cq + (e & 1);
                 const int hh = e >> 1;
                 const float s = (key < k_end && key < nvis[hh]) ? sacc[nt][e] * a.scale_log2 : -INFINITY;
                 sacc[nt][e] = s;
@@ -212,7 +245,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         }
         float psum[2] = {0.f, 0.f};
 #pragma unroll
-        for (int nt = 0; nt < AT_KEYS / 8; ++nt)
+        for (int nt = 0; nt < HK / 8; ++nt)
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int hh = e >> 1;
@@ -236,7 +269,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         }
         // O += P V: the S accumulators of key tiles (2j, 2j+1) are the A operand of k-step j.
 #pragma unroll
-        for (int j = 0; j < AT_KEYS / 16; ++j) {
+        for (int j = 0; j < HK / 16; ++j) {
             const uint32_t a0 = pack_bf16x2(sacc[2 * j][0], sacc[2 * j][1]);
             const uint32_t a1 = pack_bf16x2(sacc[2 * j][2], sacc[2 * j][3]);
             const uint32_t a2 = pack_bf16x2(sacc[2 * j + 1][0], sacc[2 * j + 1][1]);
@@ -244,7 +277,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
 #pragma unroll
             for (int dt = 0; dt < D / 8; dt += 2) {
                 uint32_t b0, b1, b2, b3;
-                const int r = j * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int r = kh * HK + j * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                 const int c = dt + (lane >> 4);
                 ldsm_x4_t(vs_u + sw_off<D>(r, c), b0, b1, b2, b3);
                 mma16816(oacc[dt], a0, a1, a2, a3, b0, b1);
@@ -253,72 +286,104 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         }
     }
 
-    // Partial rows of this split: O unnormalised in fp16 (a value beyond the fp16 range raises a
-    // device error), then m and l in fp32.
+    // ---- merge the two key halves of each row group (q/k/v are dead past this barrier) ----
     __syncthreads();
-    bool range_ok = true;
+    const int ra = rg * 16 + g, rb2 = ra + 8;             // this thread's two rows
+    if (kh == 1) {
 #pragma unroll
-    for (int n = 0; n < D / 8; ++n) {
-        const int r = warp * 16 + g, col = n * 8 + 2 * cq;
-        range_ok &= fabsf(oacc[n][0]) <= 65000.f && fabsf(oacc[n][1]) <= 65000.f &&
-                    fabsf(oacc[n][2]) <= 65000.f && fabsf(oacc[n][3]) <= 65000.f;
-        *(__half2*)(opart + r * ROWB + col * 2) = __floats2half2_rn(oacc[n][0], oacc[n][1]);
-        *(__half2*)(opart + (r + 8) * ROWB + col * 2) = __floats2half2_rn(oacc[n][2], oacc[n][3]);
+        for (int n = 0; n < D / 8; ++n) {
+            const int col = n * 8 + 2 * cq;
+            *(float2*)(ofp + ra * OS + col) = make_float2(oacc[n][0], oacc[n][1]);
+            *(float2*)(ofp + rb2 * OS + col) = make_float2(oacc[n][2], oacc[n][3]);
+        }
+        if (cq == 0) {
+            ml1[ra] = make_float2(m_run[0], l_run[0]);
+            ml1[rb2] = make_float2(m_run[1], l_run[1]);
+        }
     }
-    if (!range_ok) atomicCAS(a.err, 0, (int)DEV_FP16_RANGE);
-    if (cq == 0) {
-        *(float2*)(opart + (warp * 16 + g) * ROWB + 2 * D) = make_float2(m_run[0], l_run[0]);
-        *(float2*)(opart + (warp * 16 + g + 8) * ROWB + 2 * D) = make_float2(m_run[1], l_run[1]);
+    __syncthreads();
+    if (kh == 0) {
+        // Partial rows of this split: O unnormalised in fp16 (a value beyond the fp16 range
+        // raises a device error), then m and l in fp32.
+        float w0[2], w1[2];
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const float2 o1 = ml1[hh ? rb2 : ra];
+            const float m = fmaxf(m_run[hh], o1.x);
+            w0[hh] = (m_run[hh] == -INFINITY) ? 0.f : exp2f(m_run[hh] - m);
+            w1[hh] = (o1.x == -INFINITY) ? 0.f : exp2f(o1.x - m);
+            const float l = l_run[hh] * w0[hh] + o1.y * w1[hh];
+            if (cq == 0) *(float2*)(opart + (hh ? rb2 : ra) * ROWB + 2 * D) = make_float2(m, l);
+        }
+        bool range_ok = true;
+#pragma unroll
+        for (int n = 0; n < D / 8; ++n) {
+            const int col = n * 8 + 2 * cq;
+            const float2 p0 = *(const float2*)(ofp + ra * OS + col);
+            const float2 p1 = *(const float2*)(ofp + rb2 * OS + col);
+            const float v0 = oacc[n][0] * w0[0] + p0.x * w1[0], v1 = oacc[n][1] * w0[0] + p0.y * w1[0];
+            const float v2 = oacc[n][2] * w0[1] + p1.x * w1[1], v3 = oacc[n][3] * w0[1] + p1.y * w1[1];
+            range_ok &= fabsf(v0) <= 65000.f && fabsf(v1) <= 65000.f && fabsf(v2) <= 65000.f &&
+                        fabsf(v3) <= 65000.f;
+            *(__half2*)(opart + ra * ROWB + col * 2) = __floats2half2_rn(v0, v1);
+            *(__half2*)(opart + rb2 * ROWB + col * 2) = __floats2half2_rn(v2, v3);
+        }
+        if (!range_ok) atomicCAS(a.err, 0, (int)DEV_FP16_RANGE);
     }
-    // Rows [s * rows_per, ...) of the 64 belong to split rank s, which combines them.
-    const int ns = a.nsplit;
-    const int rank = (int)ptx::cluster_rank();
-    const int rows_per = (AT_ROWS + ns - 1) / ns;
-    const int r_lo = min(AT_ROWS, rank * rows_per), r_hi = min(AT_ROWS, r_lo + rows_per);
-    if (tid == 32) ptx::mbar_expect_tx(rbar, (uint32_t)((ns - 1) * (r_hi - r_lo) * ROWB));
     ptx::fence_proxy_async_smem();
-    // Every split is done with q/k/v (the receive buffers overlap them) and every receive
-    // barrier is initialised past this point.
-    ptx::cluster_sync_all();
+    __syncthreads();
+
+    // ---- exchange: push every other split's rows into its receive buffer ----
+    ptx::cluster_wait();
     if (tid == 0) {
-        const uint32_t recv_u = ptx::smem_u32(recv + (size_t)rank * rows_per * ROWB);
         const uint32_t bar_u = ptx::smem_u32(rbar);
         for (int s = 0; s < ns; ++s) {
             const int lo = min(AT_ROWS, s * rows_per), hi = min(AT_ROWS, lo + rows_per);
             if (hi <= lo || s == rank) continue;
-            ptx::bulk_copy_to_cluster(ptx::dsmem_map(recv_u, (uint32_t)s), opart + (size_t)lo * ROWB,
+            const int slot = rank < s ? rank : rank - 1;   // split s stores senders != s in order
+            const uint32_t dst = ptx::smem_u32(recv + (size_t)slot * rows_per * ROWB);
+            ptx::bulk_copy_to_cluster(ptx::dsmem_map(dst, (uint32_t)s), opart + (size_t)lo * ROWB,
                                       (uint32_t)((hi - lo) * ROWB), ptx::dsmem_map(bar_u, (uint32_t)s));
         }
     }
     const bool got = ptx::mbar_wait_bounded(rbar, 0, 200ull * 1000 * 1000);
+    // Everything addressed to this split has landed (seen through its own barrier); once all
+    // splits arrive, every copy out of this CTA has landed too.
+    ptx::cluster_arrive_relaxed();
     // Row r of split s: this CTA's own partial, or the slice split s sent.
     auto srow = [&](int s, int r) -> const uint8_t* {
-        return s == rank ? opart + (size_t)r * ROWB : recv + ((size_t)s * rows_per + (r - r_lo)) * ROWB;
+        if (s == rank) return opart + (size_t)r * ROWB;
+        const int slot = s < rank ? s : s - 1;
+        return recv + ((size_t)slot * rows_per + (r - r_lo)) * ROWB;
     };
 
-    // Combine the splits in rank order for the owned rows, from local shared memory.
-    for (int r = r_lo + tid; r < r_hi; r += AT_THREADS) {
-        float mx = -INFINITY;
-        for (int s = 0; s < ns; ++s) mx = fmaxf(mx, *(const float*)(srow(s, r) + 2 * D));
-        float L = 0.f;
-        for (int s = 0; s < ns; ++s) {
-            const float2 ml = *(const float2*)(srow(s, r) + 2 * D);
-            const float w = (mx == -INFINITY) ? 0.f : exp2f(ml.x - mx);
-            coef[r * AT_MAX_SPLITS + s] = w;
-            L += w * ml.y;
-        }
-        const float inv = L > 0.f ? 1.f / L : 0.f;
-        for (int s = 0; s < ns; ++s) coef[r * AT_MAX_SPLITS + s] *= inv;
+    // ---- combine the splits for the owned rows, in split order ----
+    // Coefficients: 16 lanes per row (lane s = split s), max and sum by butterflies.
+    const int nrow_here = r_hi - r_lo;
+    for (int base = 0; base < nrow_here * AT_MAX_SPLITS; base += AT_THREADS) {
+        const int idx = base + tid;
+        const int r = r_lo + idx / AT_MAX_SPLITS, s = idx % AT_MAX_SPLITS;
+        const bool valid = idx < nrow_here * AT_MAX_SPLITS && s < ns;
+        const float2 ml = valid ? *(const float2*)(srow(s, r) + 2 * D) : make_float2(-INFINITY, 0.f);
+        float mx = ml.x;
+#pragma unroll
+        for (int o = 1; o < AT_MAX_SPLITS; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        const float w = (ml.x == -INFINITY) ? 0.f : exp2f(ml.x - mx);
+        float L = w * ml.y;
+#pragma unroll
+        for (int o = 1; o < AT_MAX_SPLITS; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+        if (idx < nrow_here * AT_MAX_SPLITS) coef[(r - r_lo) * AT_MAX_SPLITS + s] = L > 0.f ? w / L : 0.f;
     }
     __syncthreads();
-    const int nrow_here = r_hi - r_lo;
     for (int idx = tid; idx < nrow_here * (D / 4); idx += AT_THREADS) {
         const int r = r_lo + idx / (D / 4), d = (idx % (D / 4)) * 4;
         const int R = row0 + r;
         if (R >= nrows || !got) continue;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int s = 0; s < ns; ++s) {
-            const float c = coef[r * AT_MAX_SPLITS + s];
+#pragma unroll
+        for (int s = 0; s < AT_MAX_SPLITS; ++s) {
+            if (s >= ns) break;
+            const float c = coef[(r - r_lo) * AT_MAX_SPLITS + s];
             const uint2 hv = *(const uint2*)(srow(s, r) + 2 * d);
             const float2 v01 = __half22float2(*reinterpret_cast<const __half2*>(&hv.x));
             const float2 v23 = __half22float2(*reinterpret_cast<const __half2*>(&hv.y));
@@ -334,12 +399,12 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     }
     if (tid == 0 && !got) atomicCAS(a.err, 0, (int)DEV_TIMEOUT_MMA);
     // No split exits while a copy out of its shared memory may still be in flight.
-    ptx::cluster_sync_all();
+    ptx::cluster_wait();
 }
 
 template <int D>
 size_t attn_smem() {
-    return 128 + attn_region<D>() + sizeof(float) * AT_ROWS * AT_MAX_SPLITS + 16;
+    return 128 + (size_t)AttnSmem<D>::TOTAL;
 }
 
 template <int D>
