@@ -223,8 +223,9 @@ jpi_status alloc_buffers(jpi_handle* h) {
     JPI_CUDA_TRY(cudaMemset(h->kv_k, 0, kv * ts));
     JPI_CUDA_TRY(cudaMemset(h->kv_v, 0, kv * ts));
     JPI_CUDA_TRY(cudaMemset(h->h, 0, Mt * W * sizeof(float)));
-    JPI_TRY(dev_alloc(h, (char**)&h->hx, Mt * W * 2));
-    JPI_CUDA_TRY(cudaMemset(h->hx, 0, Mt * W * 2));
+    const size_t xs_rows = (size_t)xs_tiles((int)Mt) * 64;
+    JPI_TRY(dev_alloc(h, (char**)&h->hx, xs_rows * W * 2));
+    JPI_CUDA_TRY(cudaMemset(h->hx, 0, xs_rows * W * 2));
     const size_t ss_slots = (size_t)((W + 127) / 128) * MAX_SPLIT_K;
     JPI_TRY(dev_alloc(h, &h->ss, ss_slots * Mt));
     JPI_CUDA_TRY(cudaMemset(h->ss, 0, ss_slots * Mt * sizeof(float)));
@@ -262,7 +263,7 @@ void free_handle(jpi_handle* h) {
 // One Euler step (or one forward): token embedding, L layers, final norm + projection.
 jpi_status enqueue_step(jpi_handle* h, int step, int B, int C, float delta, float* v_out,
                         cudaStream_t st) {
-    JPI_TRY(launch_embed(h, B, C, h->x, st));
+    JPI_TRY(launch_embed(h, step, B, C, h->x, st));
     for (int l = 0; l < h->L; ++l) {
         if (h->tc)
             JPI_TRY(tc_launch_layer(h, l, step, B, C, st));
@@ -528,7 +529,7 @@ JPI_API jpi_status jpi_profile_op(jpi_handle* h, int op, int layer, int batch, i
                 JPI_TRY(launch_time_embed(h, num_steps, -1.0, st));
                 JPI_TRY(launch_time_conditioning(h, num_steps, st));
                 break;
-            case 1: JPI_TRY(launch_embed(h, batch, chunk, h->x, st)); break;
+            case 1: JPI_TRY(launch_embed(h, 0, batch, chunk, h->x, st)); break;
             case 7:
                 JPI_TRY(launch_final(h, 0, batch, chunk, 0.f, nullptr, h->out, nullptr, st));
                 break;

@@ -54,6 +54,14 @@ inline int mod_rows(int L) { return 6 * L + 2; }
 // squares of the residual stream are kept in up to (W / 128) x MAX_SPLIT_K slots.
 constexpr int MAX_SPLIT_K = 16;
 
+// Operand of the RMSNorm-fed projections on the tensor-core path: xs = bf16((1 + sigma) * h) for
+// the next norm's scale sigma, in tiles of 64 rows: 63 token rows, then one row holding the
+// norm's shift beta. The projection of a tile then carries W * beta in its last column, and the
+// per-token 1 / rms(h) is applied to the product (Sec. 4 norm folded into the matmul).
+constexpr int XS_TOKENS = 63;
+__host__ __device__ inline int xs_row(int t) { return (t / XS_TOKENS) * 64 + t % XS_TOKENS; }
+__host__ __device__ inline int xs_tiles(int Mt) { return (Mt + XS_TOKENS - 1) / XS_TOKENS; }
+
 // Plain (un-tiled) layer weights used by the CUDA-core kernels.
 struct LayerPlain {
     void* wqkv;   // [(H+2) D][W]: rows of wq, then wk, then wv
@@ -144,7 +152,7 @@ struct jpi_handle {
     void* o = nullptr;          // [maxMt][H D] attention output (TW type)
     void* z = nullptr;          // [maxMt][F] GeGLU output (TW type)
     float* ss = nullptr;        // [W / 128][maxMt] per-token sums of h^2 over 128-feature slices
-    void* hx = nullptr;         // [maxMt][W] fp16 copy of h, read by the norm-fed GEMMs
+    void* hx = nullptr;         // [xs_tiles(maxMt) x 64][W] bf16 scaled h (+ beta rows), see xs_row
     int* dev_err = nullptr;     // device error word
 
     // Tensor-core path: one plan per projection (QKV, O, gate/up, down) and tensor maps
@@ -169,7 +177,7 @@ jpi_status launch_time_embed(jpi_handle* h, int nsteps, double t_override, cudaS
 jpi_status launch_time_conditioning(jpi_handle* h, int nsteps, cudaStream_t st);
 jpi_status launch_time_conditioning_into(jpi_handle* h, double t, float* temb, float* c1,
                                          float* cond, cudaStream_t st);
-jpi_status launch_embed(jpi_handle* h, int batch, int chunk, const float* x, cudaStream_t st);
+jpi_status launch_embed(jpi_handle* h, int step, int batch, int chunk, const float* x, cudaStream_t st);
 jpi_status launch_layer_simt(jpi_handle* h, int layer, int step, int batch, int chunk,
                              cudaStream_t st);
 // One sub-step of a layer (ops 2..6 of jpi_profile_op).

@@ -184,11 +184,12 @@ __global__ void __launch_bounds__(256) k_mod_gemv(const TW* __restrict__ Wm, con
 
 // ---------------------------------------------------------------------------------------------
 // Token embedding: row 0 of each request is the state token, rows 1..C the action tokens.
-// Block = 128 features of one token; with `ss` it also writes that slice's sum of squares
-// (ss[slice][m]) for the next RMSNorm of the tensor-core path.
+// Block = 128 features of one token. For the tensor-core path it also writes the operand of
+// the first layer's norm-fed projection (xs = bf16((1 + sigma) * h) at row xs_row(m), and beta in
+// the last row of tile m while m < xs_tiles) and that slice's sum of squares (ss[slice][m]).
 __global__ void __launch_bounds__(128) k_embed(
-    float* __restrict__ hres, __half* __restrict__ hx, int* __restrict__ err, float* __restrict__ ss,
-    int ss_ld,
+    float* __restrict__ hres, __nv_bfloat16* __restrict__ xs, const float* __restrict__ sigma,
+    const float* __restrict__ beta, float* __restrict__ ss, int ss_ld,
     const float* __restrict__ state,
     const float* __restrict__ x, const float* __restrict__ Ws, const float* __restrict__ bs,
     const float* __restrict__ Wa, const float* __restrict__ ba, int S, int C, int W, int Sd, int A) {
@@ -211,9 +212,9 @@ __global__ void __launch_bounds__(128) k_embed(
         for (int k = 0; k < K; ++k) acc = fmaf(Wm[(size_t)n * K + k], in[k], acc);
         v = acc + bias[n];
         hres[(size_t)m * W + n] = v;
-        if (hx) {
-            hx[(size_t)m * W + n] = __float2half_rn(v);
-            if (!(fabsf(v) <= 65504.f)) atomicCAS(err, 0, (int)DEV_FP16_RANGE);
+        if (xs) {
+            xs[(size_t)xs_row(m) * W + n] = __float2bfloat16_rn((1.f + sigma[n]) * v);
+            if (m < xs_tiles(gridDim.y)) xs[((size_t)m * 64 + 63) * W + n] = __float2bfloat16_rn(beta[n]);
         }
     }
     if (ss) {
@@ -643,10 +644,13 @@ jpi_status launch_time_conditioning_into(jpi_handle* h, double t, float* temb, f
     return check_launch("time conditioning (caller scratch)");
 }
 
-jpi_status launch_embed(jpi_handle* h, int B, int C, const float* x, cudaStream_t st) {
+jpi_status launch_embed(jpi_handle* h, int step, int B, int C, const float* x, cudaStream_t st) {
     const int S = C + 1;
+    // Scale and shift of layer 0's attention norm at this step.
+    const float* ms = h->mods + (size_t)step * mod_rows(h->L) * h->W;
     k_embed<<<dim3((h->W + 127) / 128, B * S), 128, 0, st>>>(
-        h->h, h->tc ? (__half*)h->hx : nullptr, h->dev_err, h->tc ? h->ss : nullptr, h->maxMt, h->state,
+        h->h, h->tc ? (__nv_bfloat16*)h->hx : nullptr, ms, ms + h->W, h->tc ? h->ss : nullptr, h->maxMt,
+        h->state,
         x, h->state_in_w, h->state_in_b,
         h->action_in_w, h->action_in_b, S, C, h->W, h->Sd, h->A);
     return check_launch("embed");

@@ -62,7 +62,7 @@ extern "C" JPI_API jpi_status jpi_expert_forward_noalloc(jpi_handle* h, const fl
     JPI_CUDA_TRY(cudaMemcpyAsync(h->x, x_t, (size_t)batch * chunk * h->A * sizeof(float),
                                  cudaMemcpyDeviceToDevice, st));
     JPI_TRY(jpi::launch_time_conditioning_into(h, (double)t, temb, c1, cond, st));
-    JPI_TRY(jpi::launch_embed(h, batch, chunk, h->x, st));
+    JPI_TRY(jpi::launch_embed(h, 0, batch, chunk, h->x, st));
     for (int l = 0; l < h->L; ++l) {
         if (h->tc)
             JPI_TRY(jpi::tc_launch_layer(h, l, 0, batch, chunk, st));

@@ -42,16 +42,17 @@ enum GemmKind { G_QKV = 0, G_O = 1, G_GU = 2, G_DOWN = 3 };
 
 struct GemmArgs {
     int Mt, K, nkb, kpb, splits;
-    // RMSNorm-fed projections (QKV, gate/up): u = h * rinv * (1 + sigma) + beta, with rinv from
-    // the per-token sums of squares left by the producer of h.
+    // RMSNorm-fed projections (QKV, gate/up): W u = rinv * (W xs) + W beta, with xs = (1 + sigma) h
+    // and beta packed as tiles of 63 tokens + 1 beta row by the producer of h, and rinv from the
+    // per-token sums of squares it left.
     const float* ss;         // [nslot][ss_ld]: sums of h^2 over disjoint feature ranges
     int nslot, ss_ld;
-    const float* sigma;
-    const float* beta;
     float eps, inv_w;
     // Gated residual epilogue (O, down).
     float* hres;
-    __half* hx;              // fp16 copy of the residual stream (B operand of the next norm-fed GEMM)
+    __nv_bfloat16* xs;       // operand of the next norm-fed GEMM (null: none follows)
+    const float* sigma_next; // that norm's scale and shift
+    const float* beta_next;
     const float* gamma;
     float* ss_out;           // slot (tile * splits + rank): this CTA's features
     int W;
@@ -109,7 +110,7 @@ __host__ __device__ __forceinline__ GemmSmem gemm_layout(int kpb, int splits, bo
     L.x = kpb * TILE_BYTES;
     L.recv = L.x + xbytes;
     L.misc = L.recv + (splits - 1) * (TILE_ROWS / splits) * NT * 2;
-    int end = L.misc + (norm_in ? (4 * NT + 2 * kpb * KBLK) * (int)sizeof(float) : 0);
+    int end = L.misc + (norm_in ? 4 * NT * (int)sizeof(float) : 0);   // ss partials + rinv
     if (norm_in) {
         L.ssred = L.misc;                               // unused by the norm-fed kinds
     } else if (xbytes >= PART_BYTES + ssred_bytes) {
@@ -119,7 +120,7 @@ __host__ __device__ __forceinline__ GemmSmem gemm_layout(int kpb, int splits, bo
         end += ssred_bytes;
     }
     L.bars = (end + 7) & ~7;
-    L.total = L.bars + 64;
+    L.total = L.bars + 64;   // 4 mbarriers, the TMEM address, the error flag
     return L;
 }
 
@@ -418,8 +419,9 @@ jpi_status tc_prepare(jpi_handle* h) {
         JPI_TRY(make_tmap(t.down, (uint64_t)d_rows / TILE_ROWS * (h->F / KBLK) * TILE_ROWS, KBLK, TILE_ROWS,
                           &h->tmaps[4 * l + G_DOWN]));
     }
-    // B operands: fp16 residual copy, attention output, GeGLU output ([maxMt][K] row-major).
-    JPI_TRY(make_tmap(h->hx, h->maxMt, h->W, NT, &h->xmaps[0], CU_TENSOR_MAP_DATA_TYPE_FLOAT16));
+    // B operands: scaled residual stream in tiles of 63 tokens + beta, attention output and GeGLU
+    // output ([rows][K] row-major).
+    JPI_TRY(make_tmap(h->hx, (uint64_t)xs_tiles(h->maxMt) * 64, h->W, NT, &h->xmaps[0]));
     JPI_TRY(make_tmap(h->o, h->maxMt, h->HD, NT, &h->xmaps[1]));
     JPI_TRY(make_tmap(h->z, h->maxMt, h->F, NT, &h->xmaps[2]));
     return JPI_OK;
@@ -434,8 +436,6 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
         case 2: {
             const GemmPlan& pl = plans[G_QKV];
             GemmArgs a = base_args(h, B, C, pl);
-            a.sigma = ms;
-            a.beta = ms + W;
             // Sums of squares left by the embedding (one per 128 features) or the previous
             // layer's down projection (one per CTA).
             if (l > 0) a.nslot = plans[G_DOWN].ntiles * plans[G_DOWN].splits;
@@ -452,7 +452,9 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
             const GemmPlan& pl = plans[G_O];
             GemmArgs a = base_args(h, B, C, pl);
             a.hres = h->h;
-            a.hx = (__half*)h->hx;
+            a.xs = (__nv_bfloat16*)h->hx;
+            a.sigma_next = ms + 3 * W;   // the MLP norm of this layer
+            a.beta_next = ms + 4 * W;
             a.gamma = ms + 2 * W;
             a.ss_out = h->ss;
             return launch_gemm<G_O>(h, pl, h->tmaps[4 * l + G_O], h->xmaps[1], a, st);
@@ -460,8 +462,6 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
         case 5: {
             const GemmPlan& pl = plans[G_GU];
             GemmArgs a = base_args(h, B, C, pl);
-            a.sigma = ms + 3 * W;
-            a.beta = ms + 4 * W;
             a.nslot = plans[G_O].ntiles * plans[G_O].splits;   // left by the output projection
             a.z = (__nv_bfloat16*)h->z;
             return launch_gemm<G_GU>(h, pl, h->tmaps[4 * l + G_GU], h->xmaps[0], a, st);
@@ -470,7 +470,11 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
             const GemmPlan& pl = plans[G_DOWN];
             GemmArgs a = base_args(h, B, C, pl);
             a.hres = h->h;
-            a.hx = (__half*)h->hx;
+            if (l + 1 < h->L) {           // the attention norm of the next layer
+                a.xs = (__nv_bfloat16*)h->hx;
+                a.sigma_next = ms + 6 * W;
+                a.beta_next = ms + 7 * W;
+            }
             a.gamma = ms + 5 * W;
             a.ss_out = h->ss;
             return launch_gemm<G_DOWN>(h, pl, h->tmaps[4 * l + G_DOWN], h->xmaps[2], a, st);
