@@ -76,6 +76,45 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
             ptx::tma_load_2d(wsm + j * TILE_BYTES, &wmap, &bars[0], 0,
                              (tile * a.nkb + kb0 + j) * TILE_ROWS, pol);
     }
+    // Epilogue inputs from global memory that do not depend on the product (first item of this
+    // thread only). For the first token tile they are read before the dependency wait: the rotary
+    // table is constant, the modulation vectors come from kernels that finished long before, and
+    // the residual stream h was last written two projections back (the previous norm-fed kernel
+    // passed its own dependency wait, so that writer has completed). Later tiles issue them after
+    // the TMEM read-out, which global loads in flight slow down.
+    float hv1[4] = {0.f, 0.f, 0.f, 0.f}, hv2[4] = {0.f, 0.f, 0.f, 0.f}, g1 = 0.f, g2 = 0.f;
+    float sn1 = 0.f, sn2 = 0.f;
+    float2 cs[4] = {make_float2(1.f, 0.f), make_float2(1.f, 0.f), make_float2(1.f, 0.f), make_float2(1.f, 0.f)};
+    auto prefetch = [&](int item, int tok0) {
+        const int p = p0 + item % npairs, t0 = (item / npairs) * 4;
+        const int f1 = tile * TILE_ROWS + p, f2 = f1 + 64;
+        if (RESID) {
+            g1 = a.gamma[f1];
+            g2 = a.gamma[f2];
+            if (a.xs) {
+                sn1 = a.sigma_next[f1];
+                sn2 = a.sigma_next[f2];
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int tok = tok0 + t0 + e;
+            hv1[e] = hv2[e] = 0.f;
+            cs[e] = make_float2(1.f, 0.f);
+            if (t0 + e < TT && tok < a.Mt) {
+                if (RESID) {
+                    hv1[e] = a.hres[(size_t)tok * a.W + f1];
+                    hv2[e] = a.hres[(size_t)tok * a.W + f2];
+                }
+                if (KIND == G_QKV && a.rope) {
+                    const int hd = a.D >> 1, pair = tile * 64 + p;
+                    const int sec = pair / hd, d = pair - sec * hd;
+                    if (sec <= a.H) cs[e] = __ldg(a.rope + (size_t)(a.P + tok % a.S) * hd + d);
+                }
+            }
+        }
+    };
+    if (tid < nitems) prefetch(tid, 0);
     // Every CTA's receive barrier is initialised before any CTA pushes into it: arrive now, wait
     // before the first push (the round trip overlaps the previous kernel and this one's loads).
     ptx::cluster_arrive();
@@ -143,41 +182,6 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
                 rinv_s[c] = r;
             }
         }
-        // Epilogue inputs from global memory that do not depend on the product. They are issued
-        // after the TMEM read-out (global loads in flight slow tcgen05.ld down), so their latency
-        // overlaps the exchange (first item of this thread only).
-        float hv1[4] = {0.f, 0.f, 0.f, 0.f}, hv2[4] = {0.f, 0.f, 0.f, 0.f}, g1 = 0.f, g2 = 0.f;
-        float sn1 = 0.f, sn2 = 0.f;
-        float2 cs[4] = {make_float2(1.f, 0.f), make_float2(1.f, 0.f), make_float2(1.f, 0.f), make_float2(1.f, 0.f)};
-        auto prefetch = [&](int item) {
-            const int p = p0 + item % npairs, t0 = (item / npairs) * 4;
-            const int f1 = tile * TILE_ROWS + p, f2 = f1 + 64;
-            if (RESID) {
-                g1 = a.gamma[f1];
-                g2 = a.gamma[f2];
-                if (a.xs) {
-                    sn1 = a.sigma_next[f1];
-                    sn2 = a.sigma_next[f2];
-                }
-            }
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int tok = tok0 + t0 + e;
-                hv1[e] = hv2[e] = 0.f;
-                cs[e] = make_float2(1.f, 0.f);
-                if (t0 + e < TT && tok < a.Mt) {
-                    if (RESID) {
-                        hv1[e] = a.hres[(size_t)tok * a.W + f1];
-                        hv2[e] = a.hres[(size_t)tok * a.W + f2];
-                    }
-                    if (KIND == G_QKV && a.rope) {
-                        const int hd = a.D >> 1, pair = tile * 64 + p;
-                        const int sec = pair / hd, d = pair - sec * hd;
-                        if (sec <= a.H) cs[e] = __ldg(a.rope + (size_t)(a.P + tok % a.S) * hd + d);
-                    }
-                }
-            }
-        };
         if (!ptx::mbar_wait_bounded(&bars[2], tt & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
         __syncthreads();
         const bool ok = *flag == 0;
@@ -216,7 +220,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         }
         ptx::tc_fence_before();
         ptx::fence_proxy_async_smem();
-        if (tid < nitems) prefetch(tid);
+        if (tt > 0 && tid < nitems) prefetch(tid, tok0);
         __syncthreads();
 
         // ---- 3b. push each other rank's rows (pairs r*npairs.. and +64) to that rank ----
@@ -242,7 +246,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         // ---- 4. rank-ordered sum of the slices (own rows read in place) + epilogue ----
         float ssq[4] = {0.f, 0.f, 0.f, 0.f};
         for (int item = tid; item < nitems; item += GEMM_THREADS) {
-            if (item != tid) prefetch(item);
+            if (item != tid) prefetch(item, tok0);
             const int pi = item % npairs, quad = item / npairs, t0 = quad * 4, p = p0 + pi;
             // Offsets of columns t0..t0+3 and of column 63 inside a swizzled row with key p mod 8
             // (= (p + 64) mod 8).
