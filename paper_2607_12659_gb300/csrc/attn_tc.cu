@@ -168,7 +168,6 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     load_kv(k_begin, 0, first_suffix_row);
 
     ptx::grid_dep_wait();
-    ptx::grid_dep_launch();
 
     // Query block (rows beyond this request's S*H rows are zero).
     const __nv_bfloat16* qb = a.q + (size_t)b * nrows * D;
@@ -350,6 +349,9 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     // Everything addressed to this split has landed (seen through its own barrier); once all
     // splits arrive, every copy out of this CTA has landed too.
     ptx::cluster_arrive_relaxed();
+    // The next kernel may start now (its weight prefetch no longer competes with this one's
+    // loads and exchange).
+    ptx::grid_dep_launch();
     // Row r of split s: this CTA's own partial, or the slice split s sent.
     auto srow = [&](int s, int r) -> const uint8_t* {
         if (s == rank) return opart + (size_t)r * ROWB;

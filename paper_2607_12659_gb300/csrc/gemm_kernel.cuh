@@ -119,7 +119,6 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
     // before the first push (the round trip overlaps the previous kernel and this one's loads).
     ptx::cluster_arrive();
     ptx::grid_dep_wait();
-    ptx::grid_dep_launch();
 
     const int ntt = (a.Mt + TT - 1) / TT;
     for (int tt = 0; tt < ntt; ++tt) {
@@ -242,6 +241,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         // ranks arrive, every copy out of this CTA's partial has completed as well. Nothing else
         // is published through this barrier, so the arrival is relaxed.
         if (last) ptx::cluster_arrive_relaxed();
+        // The next kernel may start now: its weight prefetch would otherwise compete with this
+        // kernel's operand loads, MMAs and exchange for memory and shared-memory bandwidth.
+        if (tt == 0) ptx::grid_dep_launch();
 
         // ---- 4. rank-ordered sum of the slices (own rows read in place) + epilogue ----
         float ssq[4] = {0.f, 0.f, 0.f, 0.f};
