@@ -87,21 +87,22 @@ template <int D>
 __host__ __device__ constexpr int attn_row_bytes() {
     return 2 * D + 16;
 }
-// Row stride (floats) of the fp32 staging of the second key half: 8 floats of padding put the
-// 4 rows a half-warp writes at one column (8-byte accesses) on disjoint banks.
+// Row stride (floats) of the fp32 staging of one key half's output columns that the other key
+// half merges (D / 2 columns): 8 floats of padding put the 4 rows a half-warp writes at one column
+// (8-byte accesses) on disjoint banks.
 template <int D>
 __host__ __device__ constexpr int attn_ofp_stride() {
-    return D + 8;
+    return D / 2 + 8;
 }
 // Shared-memory layout (bytes from the 128-aligned base): q/k/v, reused after the key loop for
-// the second key half's fp32 output and (m, l) and then this split's partial rows; the receive
+// each key half's hand-over columns (fp32) and (m, l), then this split's partial rows; the receive
 // buffer; the combine coefficients; the receive barrier.
 template <int D>
 struct AttnSmem {
     static constexpr int QKV = (AT_ROWS + 2 * AT_KEYS) * D * 2;
-    static constexpr int OFP = AT_ROWS * attn_ofp_stride<D>() * 4;
-    static constexpr int ML1 = OFP;                              // [32] float2 after the fp32 rows
-    static constexpr int OPART = OFP + AT_ROWS * 8;              // [32][row bytes]
+    static constexpr int OFP = 2 * AT_ROWS * attn_ofp_stride<D>() * 4;   // [2 halves][32][OS]
+    static constexpr int ML = OFP;                               // [2 halves][32] float2
+    static constexpr int OPART = ML + 2 * AT_ROWS * 8;           // [32][row bytes]
     static constexpr int REGION_USED = OPART + AT_ROWS * attn_row_bytes<D>();
     static constexpr int REGION = QKV > REGION_USED ? QKV : REGION_USED;
     static constexpr int RECV = REGION;                          // [AT_MAX_RECV_ROWS][row bytes]
@@ -120,8 +121,8 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     uint8_t* vs = ks + AT_KEYS * D * 2;                  // [64][D] bf16
     constexpr int ROWB = attn_row_bytes<D>();
     constexpr int OS = attn_ofp_stride<D>();
-    float* ofp = (float*)smem;                           // [32][OS] second key half's O (fp32)
-    float2* ml1 = (float2*)(smem + L::ML1);              // [32] its (m, l)
+    float* ofp = (float*)smem;                           // [2][32][OS] columns handed over
+    float2* mls = (float2*)(smem + L::ML);               // [2][32] (m, l) of each key half
     uint8_t* opart = smem + L::OPART;                    // [32][ROWB] this split's partial rows
     uint8_t* recv = smem + L::RECV;                      // [(splits - 1) x rows_per][ROWB]
     float* coef = (float*)(smem + L::COEF);              // [32][AT_MAX_SPLITS]
@@ -286,46 +287,76 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     }
 
     // ---- merge the two key halves of each row group (q/k/v are dead past this barrier) ----
+    // Key half kh merges output columns [kh D/2, (kh + 1) D/2): it hands the other half of its
+    // columns over in fp32, then combines its own with the ones handed to it.
     __syncthreads();
     const int ra = rg * 16 + g, rb2 = ra + 8;             // this thread's two rows
-    if (kh == 1) {
+    constexpr int NH = D / 16;                           // n-tiles per column half
+    float* give = ofp + (size_t)kh * AT_ROWS * OS;       // this half's hand-over rows
+    const float* take = ofp + (size_t)(1 - kh) * AT_ROWS * OS;
+    if (kh == 0) {
 #pragma unroll
-        for (int n = 0; n < D / 8; ++n) {
-            const int col = n * 8 + 2 * cq;
-            *(float2*)(ofp + ra * OS + col) = make_float2(oacc[n][0], oacc[n][1]);
-            *(float2*)(ofp + rb2 * OS + col) = make_float2(oacc[n][2], oacc[n][3]);
+        for (int n = NH; n < 2 * NH; ++n) {
+            const int col = (n - NH) * 8 + 2 * cq;
+            *(float2*)(give + ra * OS + col) = make_float2(oacc[n][0], oacc[n][1]);
+            *(float2*)(give + rb2 * OS + col) = make_float2(oacc[n][2], oacc[n][3]);
         }
-        if (cq == 0) {
-            ml1[ra] = make_float2(m_run[0], l_run[0]);
-            ml1[rb2] = make_float2(m_run[1], l_run[1]);
+    } else {
+#pragma unroll
+        for (int n = 0; n < NH; ++n) {
+            const int col = n * 8 + 2 * cq;
+            *(float2*)(give + ra * OS + col) = make_float2(oacc[n][0], oacc[n][1]);
+            *(float2*)(give + rb2 * OS + col) = make_float2(oacc[n][2], oacc[n][3]);
         }
     }
+    if (cq == 0) {
+        mls[kh * AT_ROWS + ra] = make_float2(m_run[0], l_run[0]);
+        mls[kh * AT_ROWS + rb2] = make_float2(m_run[1], l_run[1]);
+    }
     __syncthreads();
-    if (kh == 0) {
+    {
         // Partial rows of this split: O unnormalised in fp16 (a value beyond the fp16 range
-        // raises a device error), then m and l in fp32.
+        // raises a device error), then m and l in fp32. o = o_half0 w0 + o_half1 w1.
         float w0[2], w1[2];
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
-            const float2 o1 = ml1[hh ? rb2 : ra];
-            const float m = fmaxf(m_run[hh], o1.x);
-            w0[hh] = (m_run[hh] == -INFINITY) ? 0.f : exp2f(m_run[hh] - m);
-            w1[hh] = (o1.x == -INFINITY) ? 0.f : exp2f(o1.x - m);
-            const float l = l_run[hh] * w0[hh] + o1.y * w1[hh];
-            if (cq == 0) *(float2*)(opart + (hh ? rb2 : ra) * ROWB + 2 * D) = make_float2(m, l);
+            const int r = hh ? rb2 : ra;
+            const float2 h0 = mls[r], h1 = mls[AT_ROWS + r];
+            const float m = fmaxf(h0.x, h1.x);
+            w0[hh] = (h0.x == -INFINITY) ? 0.f : exp2f(h0.x - m);
+            w1[hh] = (h1.x == -INFINITY) ? 0.f : exp2f(h1.x - m);
+            const float l = __fmaf_rn(h1.y, w1[hh], __fmul_rn(h0.y, w0[hh]));
+            if (kh == 0 && cq == 0) *(float2*)(opart + r * ROWB + 2 * D) = make_float2(m, l);
         }
         bool range_ok = true;
-#pragma unroll
-        for (int n = 0; n < D / 8; ++n) {
+        auto merge = [&](int n, float2 t0, float2 t1, bool own_first) {
+            // own_first: this warp is key half 0 (its values carry w0).
             const int col = n * 8 + 2 * cq;
-            const float2 p0 = *(const float2*)(ofp + ra * OS + col);
-            const float2 p1 = *(const float2*)(ofp + rb2 * OS + col);
-            const float v0 = oacc[n][0] * w0[0] + p0.x * w1[0], v1 = oacc[n][1] * w0[0] + p0.y * w1[0];
-            const float v2 = oacc[n][2] * w0[1] + p1.x * w1[1], v3 = oacc[n][3] * w0[1] + p1.y * w1[1];
+            const float a0 = own_first ? oacc[n][0] : t0.x, a1 = own_first ? oacc[n][1] : t0.y;
+            const float a2 = own_first ? oacc[n][2] : t1.x, a3 = own_first ? oacc[n][3] : t1.y;
+            const float b0 = own_first ? t0.x : oacc[n][0], b1 = own_first ? t0.y : oacc[n][1];
+            const float b2 = own_first ? t1.x : oacc[n][2], b3 = own_first ? t1.y : oacc[n][3];
+            const float v0 = __fmaf_rn(b0, w1[0], __fmul_rn(a0, w0[0]));
+            const float v1 = __fmaf_rn(b1, w1[0], __fmul_rn(a1, w0[0]));
+            const float v2 = __fmaf_rn(b2, w1[1], __fmul_rn(a2, w0[1]));
+            const float v3 = __fmaf_rn(b3, w1[1], __fmul_rn(a3, w0[1]));
             range_ok &= fabsf(v0) <= 65000.f && fabsf(v1) <= 65000.f && fabsf(v2) <= 65000.f &&
                         fabsf(v3) <= 65000.f;
             *(__half2*)(opart + ra * ROWB + col * 2) = __floats2half2_rn(v0, v1);
             *(__half2*)(opart + rb2 * ROWB + col * 2) = __floats2half2_rn(v2, v3);
+        };
+        if (kh == 0) {
+#pragma unroll
+            for (int n = 0; n < NH; ++n) {
+                const int c = n * 8 + 2 * cq;
+                merge(n, *(const float2*)(take + ra * OS + c), *(const float2*)(take + rb2 * OS + c), true);
+            }
+        } else {
+#pragma unroll
+            for (int n = NH; n < 2 * NH; ++n) {
+                const int c = (n - NH) * 8 + 2 * cq;
+                merge(n, *(const float2*)(take + ra * OS + c), *(const float2*)(take + rb2 * OS + c), false);
+            }
         }
         if (!range_ok) atomicCAS(a.err, 0, (int)DEV_FP16_RANGE);
     }
@@ -382,11 +413,12 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         const int R = row0 + r;
         if (R >= nrows || !got) continue;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        // All 16 slots are loaded together (slots past the last split read this CTA's own row
+        // with a zero coefficient), then summed in split order.
 #pragma unroll
         for (int s = 0; s < AT_MAX_SPLITS; ++s) {
-            if (s >= ns) break;
-            const float c = coef[(r - r_lo) * AT_MAX_SPLITS + s];
-            const uint2 hv = *(const uint2*)(srow(s, r) + 2 * d);
+            const float c = s < ns ? coef[(r - r_lo) * AT_MAX_SPLITS + s] : 0.f;
+            const uint2 hv = *(const uint2*)(srow(s < ns ? s : rank, r) + 2 * d);
             const float2 v01 = __half22float2(*reinterpret_cast<const __half2*>(&hv.x));
             const float2 v23 = __half22float2(*reinterpret_cast<const __half2*>(&hv.y));
             acc.x = fmaf(c, v01.x, acc.x);
