@@ -276,22 +276,35 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
             }
             if (!ok) continue;
             const int f1 = tile * TILE_ROWS + p, f2 = f1 + 64;
+            // QKV: head section and index of this pair; request b and position i of the item's
+            // first token, advanced token by token (no division per token).
+            int sec = 0, d = 0, qb = 0, qi = 0;
+            if (KIND == G_QKV) {
+                const int hd = a.D >> 1, pair = tile * 64 + p;
+                sec = pair / hd;
+                d = pair - sec * hd;
+                qb = (tok0 + t0) / a.S;
+                qi = tok0 + t0 - qb * a.S;
+            }
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int tok = tok0 + t0 + e;
+                const int b = qb, i = qi;   // request and position of token tok (QKV)
+                if (KIND == G_QKV && ++qi == a.S) {
+                    qi = 0;
+                    ++qb;
+                }
                 if (t0 + e >= TT || tok >= a.Mt) continue;
                 const float u1 = f4get(y1, e) + b1, u2 = f4get(y2, e) + b2;
                 if (KIND == G_QKV) {
-                    const int hd = a.D >> 1, pair = tile * 64 + p;
-                    const int sec = pair / hd, d = pair - sec * hd;
-                    const int b = tok / a.S, pos = a.P + (tok - b * a.S);
+                    const int hd = a.D >> 1;
                     float r1 = u1, r2 = u2;
                     if (sec <= a.H) {
                         r1 = u1 * cs[e].x - u2 * cs[e].y;
                         r2 = u2 * cs[e].x + u1 * cs[e].y;
                     }
                     __nv_bfloat16* dst = (sec < a.H) ? a.q + ((size_t)tok * a.H + sec) * a.D
-                                                     : (sec == a.H ? a.kst : a.vst) + ((size_t)b * a.kv_rows + pos) * a.D;
+                                                     : (sec == a.H ? a.kst : a.vst) + ((size_t)b * a.kv_rows + a.P + i) * a.D;
                     dst[d] = __float2bfloat16_rn(r1);
                     dst[d + hd] = __float2bfloat16_rn(r2);
                 } else if (KIND == G_GU) {
