@@ -147,8 +147,8 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     }
     __syncthreads();
     // Receive barriers are initialised cluster-wide before anyone pushes: arrive now, wait
-    // before the first push.
-    ptx::cluster_arrive();
+    // before the first push (published by fence.mbarrier_init, so the arrival is relaxed).
+    ptx::cluster_arrive_relaxed();
 
     // Prefix keys/values were written before this graph ran: the first block's prefix rows are
     // fetched before the dependency wait; the suffix rows (written by the QKV kernel) after it.

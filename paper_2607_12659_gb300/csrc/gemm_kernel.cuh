@@ -117,7 +117,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
     if (tid < nitems) prefetch(tid, 0);
     // Every CTA's receive barrier is initialised before any CTA pushes into it: arrive now, wait
     // before the first push (the round trip overlaps the previous kernel and this one's loads).
-    ptx::cluster_arrive();
+    // The initialisation is published by fence.mbarrier_init, so the arrival itself is relaxed
+    // (a release arrival would also wait for the weight copies in flight).
+    ptx::cluster_arrive_relaxed();
     ptx::grid_dep_wait();
 
     const int ntt = (a.Mt + TT - 1) / TT;
