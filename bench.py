@@ -58,6 +58,18 @@ def algorithmic_bytes(cfg, B, P, C, N):
     return N * per_step + time_w + kv + io
 
 
+def algorithmic_flops(cfg, B, P, C, N):
+    """Multiply-adds x 2 of a denoise: the layer projections at M = B (C + 1) tokens, the
+    attention of the S H query rows over P + S keys, and the per-call modulation GEMV."""
+    W, H, D, F, L = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim, cfg.n_layers
+    S = C + 1
+    Mt = B * S
+    proj = L * (H * D * W + 2 * D * W + H * D * W + 3 * F * W)
+    attn = L * B * S * H * (P + S) * D * 2
+    per_step = 2 * (Mt * proj + attn + Mt * (cfg.state_dim + cfg.action_dim) * W + B * C * W * cfg.action_dim)
+    return N * per_step + 2 * (6 * L + 2) * W * W * N
+
+
 def op_bytes(cfg, op, B, P, C):
     """Algorithmic bytes of one launch of a layer op (weights + activation reads/writes)."""
     W, H, D, F = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim
@@ -226,6 +238,8 @@ def our_arm(args):
     jpi.load()
 
     B, P, C, N = (WORKLOAD[k] for k in ("batch", "prefix", "chunk", "steps"))
+    B, P = args.batch or B, args.prefix or P
+    default_workload = (B, P) == (WORKLOAD["batch"], WORKLOAD["prefix"])
     cfg = PI05
     w = make_weights(cfg, 2000)
     ex = jpi.Expert(cfg, w, max_batch=B, max_prefix=P, max_chunk=C, max_steps=N)
@@ -317,15 +331,21 @@ def our_arm(args):
     n_kernels = jpi.jpi_graph_kernel_count(ex.handle, B, C, N)
     alg = algorithmic_bytes(cfg, B, P, C, N)
     path_bw = alg / (ms_per_step * 1e-3) / 1e9
+    flops = algorithmic_flops(cfg, B, P, C, N)
+    path_tf = flops / (ms_per_step * 1e-3) / 1e12
 
     if rank == 0:
-        cpu = run_cpu_baseline(os.cpu_count() or 1) if world == 1 and not args.no_cpu_baseline else None
+        cpu = (run_cpu_baseline(os.cpu_count() or 1)
+               if world == 1 and default_workload and not args.no_cpu_baseline else None)
         clocks = clk.summary()
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "metric": METRIC if default_workload else METRIC.replace("batch 1", f"batch {B}"),
+            "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": WORKLOAD_NAME, **WORKLOAD,
+            "config": {"workload": WORKLOAD_NAME if default_workload else
+                       WORKLOAD_NAME.replace("batch 1, prefix 816", f"batch {B}, prefix {P}"),
+                       **WORKLOAD, "batch": B, "prefix": P,
                        "l2": "no flush: each call streams 6.2 GB of weights (> 129 MB L2)",
                        "parallelism": f"replicas x{world}"},
             "us_per_denoise": {"median": statistics.median(per) * 1e3,
@@ -333,7 +353,9 @@ def our_arm(args):
                                "p90": sorted(per)[min(len(per) - 1, int(0.9 * len(per)))] * 1e3},
             "path_roofline": {"bound": "hbm", "algorithmic_bytes": alg, "achieved_gbs": path_bw,
                               "peak_gbs": hbm_peak, "frac": path_bw / hbm_peak,
-                              "roofline_us": alg / hbm_peak / 1e3},
+                              "roofline_us": alg / hbm_peak / 1e3,
+                              "algorithmic_flops": flops, "achieved_tflops": path_tf,
+                              "tensor_peak_tflops": tc_peak, "tensor_frac": path_tf / tc_peak if tc_peak else None},
             "roofline": {"bound": "hbm", "kernel": OP_NAMES[dom], "achieved": achieved,
                          "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                          "traffic": traffic, "peak_source": peak_src,
@@ -387,6 +409,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="requests per denoise (default: the batch-1 workload); for documentation runs")
+    ap.add_argument("--prefix", type=int, default=0, help="prefix tokens per request (default 816)")
     ap.add_argument("--cpu-baseline-child", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
     if args.cpu_baseline_child:

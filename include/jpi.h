@@ -13,7 +13,7 @@
  *     with the action tokens; flow matching refines the noise over a fixed number of steps.
  *   - Tab. "Model architecture parameters of pi series VLA models": 18 layers, width 1024,
  *     8 heads x 256, 10 denoising steps.
- *   - Sec. 3.3 "System Design": fixed token length (so one captured CUDA graph is reused),
+ *   - Sec. 4.3 "System Design": fixed token length (so one captured CUDA graph is reused),
  *     fixed GPU-resident buffers between components, and all denoising iterations unrolled
  *     into one graph.
  *
@@ -123,14 +123,14 @@ JPI_API jpi_status jpi_expert_destroy(jpi_handle* h);
 
 /*
  * Copy the VLM prefix KV cache into the handle's GPU-resident KV store (App. A: per-layer
- * KV handoff from the LLM to the expert; Sec. 3.3: GPU-resident intermediate buffer).
+ * KV handoff from the LLM to the expert; Sec. 4.3: GPU-resident intermediate buffer).
  *   k_layers[l], v_layers[l]: device pointers, l < n_layers, each [batch][prefix_len][D]
  *                             row-major, fp32 if kv_is_fp32 else bf16 (uint16 bit patterns).
  *   batch <= max_batch, 1 <= prefix_len <= max_prefix. Keys are used as given (already
  *   position-encoded by their producer).
  * Asynchronous on `stream`: the caller keeps its buffers alive until the stream reaches this
  * point. In JPI_BF16 mode fp32 input is rounded to bf16; bf16 input in JPI_FP32 mode is widened.
- * The prefix length fixes the graph shape of later jpi_denoise calls (Sec. 3.3, fixed length).
+ * The prefix length fixes the graph shape of later jpi_denoise calls (Sec. 4.3, fixed length).
  */
 JPI_API jpi_status jpi_set_prefix_kv(jpi_handle* h, const void* const* k_layers,
                                      const void* const* v_layers, int batch, int prefix_len,
@@ -156,7 +156,7 @@ JPI_API jpi_status jpi_commit_prefix(jpi_handle* h, int batch, int prefix_len);
  *   batch must equal the batch of the last jpi_set_prefix_kv/jpi_commit_prefix;
  *   1 <= chunk <= max_chunk; 1 <= num_steps <= max_steps.
  * The first call for a (batch, chunk, num_steps, prefix_len) shape captures the whole
- * unrolled N-step loop as one CUDA graph (Sec. 3.3: graph reuse and flow unrolling) and every
+ * unrolled N-step loop as one CUDA graph (Sec. 4.3: graph reuse and flow unrolling) and every
  * later call with that shape replays it. Asynchronous on `stream`; inputs are read and the
  * output written in stream order. Errors: INVALID_ARG, SHAPE, NOT_READY, CUDA.
  */

@@ -6,7 +6,7 @@ bench's CPU-baseline leg may import it; the library never does, and it shares no
 the CUDA path (the seeded input generator in ``synth`` is the only common module).
 
 What the paper fixes (App. A "Model Architecture of pi series Models", Tab. "Model
-architecture parameters of pi series VLA models", Sec. 3.3 "System Design"):
+architecture parameters of pi series VLA models", Sec. 4.3 "System Design"):
   * the action expert is a DiT whose queries come from the action-noise tokens and whose keys
     and values are the matching LLM layer's KV cache concatenated with those tokens;
   * 18 layers, width 1024, 8 attention heads of dimension 256;

@@ -1,7 +1,7 @@
 // C-ABI entry points: argument checks, the handle's persistent buffers, weight packing, the
 // GPU-resident prefix-KV store and the captured, unrolled N-step denoise graph.
 //
-// Sec. 3.3 of the paper ("System Design") motivates the runtime shape: the token length is
+// Sec. 4.3 of the paper ("System Design") motivates the runtime shape: the token length is
 // fixed for a given prefix, so the denoise of one chunk is captured once as a CUDA graph with
 // every Euler step unrolled into it and replayed afterwards; every intermediate lives in a
 // fixed device buffer allocated once at create time.

@@ -57,7 +57,8 @@ constexpr int MAX_SPLIT_K = 16;
 // Operand of the RMSNorm-fed projections on the tensor-core path: xs = bf16((1 + sigma) * h) for
 // the next norm's scale sigma, in tiles of 64 rows: 63 token rows, then one row holding the
 // norm's shift beta. The projection of a tile then carries W * beta in its last column, and the
-// per-token 1 / rms(h) is applied to the product (Sec. 4 norm folded into the matmul).
+// per-token 1 / rms(h) is applied to the product: W u = rinv * (W xs) + W beta for the adaptive
+// RMSNorm u = h * rinv * (1 + sigma) + beta of App. A's expert layers.
 constexpr int XS_TOKENS = 63;
 __host__ __device__ inline int xs_row(int t) { return (t / XS_TOKENS) * 64 + t % XS_TOKENS; }
 __host__ __device__ inline int xs_tiles(int Mt) { return (Mt + XS_TOKENS - 1) / XS_TOKENS; }
