@@ -13,8 +13,10 @@
 //      the whole cluster has seen at kernel start); the owner sums the slices in rank order from
 //      its own shared memory. The receive buffer is used by nothing else.
 //   4. Epilogue on the owned rows. A CTA arrives on the cluster barrier as soon as everything
-//      addressed to it has landed and waits on it only before it exits (or, with several token
-//      tiles, before the next tile reuses the buffers), so the barrier is off the critical path.
+//      addressed to it has landed and waits on it only before it exits, so the barrier is off
+//      the critical path.
+// Token tiles are the grid's y dimension: every (weight tile, token tile) pair is its own
+// cluster, and all of them run concurrently (repeated weight tiles come from L2).
 //
 // Partial rows are 64 fp16 columns (128 bytes) with their 16-byte chunks XOR-swizzled by the row
 // index mod 8, which keeps both the TMEM write-out (one row per lane) and the reduction reads
@@ -80,8 +82,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
     // thread only). For the first token tile they are read before the dependency wait: the rotary
     // table is constant, the modulation vectors come from kernels that finished long before, and
     // the residual stream h was last written two projections back (the previous norm-fed kernel
-    // passed its own dependency wait, so that writer has completed). Later tiles issue them after
-    // the TMEM read-out, which global loads in flight slow down.
+    // passed its own dependency wait, so that writer has completed). Global loads still in flight
+    // at the TMEM read-out would slow it down.
     float hv1[4] = {0.f, 0.f, 0.f, 0.f}, hv2[4] = {0.f, 0.f, 0.f, 0.f}, g1 = 0.f, g2 = 0.f;
     float sn1 = 0.f, sn2 = 0.f;
     float2 cs[4] = {make_float2(1.f, 0.f), make_float2(1.f, 0.f), make_float2(1.f, 0.f), make_float2(1.f, 0.f)};
@@ -114,7 +116,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
             }
         }
     };
-    if (tid < nitems) prefetch(tid, 0);
+    if (tid < nitems) prefetch(tid, (int)blockIdx.y * TT);
     // Every CTA's receive barrier is initialised before any CTA pushes into it: arrive now, wait
     // before the first push (the round trip overlaps the previous kernel and this one's loads).
     // The initialisation is published by fence.mbarrier_init, so the arrival itself is relaxed
@@ -122,10 +124,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
     ptx::cluster_arrive_relaxed();
     ptx::grid_dep_wait();
 
-    const int ntt = (a.Mt + TT - 1) / TT;
-    for (int tt = 0; tt < ntt; ++tt) {
+    {
+        const int tt = blockIdx.y;   // token tile
         const int tok0 = tt * TT;
-        const bool last = tt == ntt - 1;
         // ---- 1. B operand (64 rows from row tt * 64 of the operand buffer) ----
         if (tid == 0) {
             const uint64_t pol = ptx::l2_policy_evict_first();
@@ -138,8 +139,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
 
         // ---- 2. MMA: D[128 rows][64 columns] over this CTA's K blocks ----
         if (tid == 0 && *flag == 0) {
-            bool ok_in = ptx::mbar_wait_bounded(&bars[1], tt & 1, WAIT_LIMIT_NS);
-            if (ok_in && tt == 0) ok_in = ptx::mbar_wait_bounded(&bars[0], 0, WAIT_LIMIT_NS);
+            bool ok_in = ptx::mbar_wait_bounded(&bars[1], 0, WAIT_LIMIT_NS);
+            if (ok_in) ok_in = ptx::mbar_wait_bounded(&bars[0], 0, WAIT_LIMIT_NS);
             if (!ok_in) {
                 *flag = DEV_TIMEOUT_WEIGHTS;
             } else {
@@ -183,7 +184,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
                 rinv_s[c] = r;
             }
         }
-        if (!ptx::mbar_wait_bounded(&bars[2], tt & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
+        if (!ptx::mbar_wait_bounded(&bars[2], 0, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
         __syncthreads();
         const bool ok = *flag == 0;
         ptx::tc_fence_after();
@@ -221,11 +222,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         }
         ptx::tc_fence_before();
         ptx::fence_proxy_async_smem();
-        if (tt > 0 && tid < nitems) prefetch(tid, tok0);
         __syncthreads();
 
         // ---- 3b. push each other rank's rows (pairs r*npairs.. and +64) to that rank ----
-        if (tt == 0) ptx::cluster_wait();   // receive barriers initialised everywhere
+        ptx::cluster_wait();   // receive barriers initialised everywhere
         if (tid == 0) {
             const uint32_t chunk = (uint32_t)(npairs * 128);
             const uint32_t bar_u = ptx::smem_u32(&bars[3]);
@@ -238,14 +238,14 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
                 ptx::bulk_copy_to_cluster(dst + chunk, part + (size_t)(r * npairs + 64) * 64, chunk, rbar);
             }
         }
-        if (!ptx::mbar_wait_bounded(&bars[3], tt & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
+        if (!ptx::mbar_wait_bounded(&bars[3], 0, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
         // Everything addressed to this CTA has landed (seen through its own mbarrier); once all
         // ranks arrive, every copy out of this CTA's partial has completed as well. Nothing else
         // is published through this barrier, so the arrival is relaxed.
-        if (last) ptx::cluster_arrive_relaxed();
+        ptx::cluster_arrive_relaxed();
         // The next kernel may start now: its weight prefetch would otherwise compete with this
         // kernel's operand loads, MMAs and exchange for memory and shared-memory bandwidth.
-        if (tt == 0) ptx::grid_dep_launch();
+        ptx::grid_dep_launch();
 
         // ---- 4. rank-ordered sum of the slices (own rows read in place) + epilogue ----
         float ssq[4] = {0.f, 0.f, 0.f, 0.f};
@@ -356,12 +356,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
                 a.ss_out[(size_t)(tile * a.splits + rank) * a.ss_ld + tok0 + tid] = s;
             }
         }
-        // Several token tiles: the next tile's pushes and loads reuse every buffer, so all ranks
-        // must be done reading them.
-        if (!last) ptx::cluster_sync_all();
     }
-    // Pairs the last arrival: after the final tile's receive wait, or (no tokens) the one made
-    // before the dependency wait.
+    // Pairs the arrival after the receive wait.
     ptx::cluster_wait();
 
     if (tid == 0 && *flag != 0) set_device_error(a.err, *flag);

@@ -251,8 +251,10 @@ jpi_status pack(const float* tmp, __nv_bfloat16* dst, const int* dmap, int rows,
 template <int KIND>
 jpi_status launch_gemm(jpi_handle* h, const GemmPlan& pl, const CUtensorMap& wmap,
                        const CUtensorMap& xmap, const GemmArgs& a, cudaStream_t st) {
+    // One grid row per token tile (63 tokens + the beta row for the norm-fed kinds, else 64).
+    constexpr int TT = (KIND == G_QKV || KIND == G_GU) ? XS_TOKENS : NT;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(pl.ctas);
+    cfg.gridDim = dim3(pl.ctas, (unsigned)std::max(1, (a.Mt + TT - 1) / TT));
     cfg.blockDim = dim3(GEMM_THREADS);
     cfg.dynamicSmemBytes = pl.smem;
     cfg.stream = st;
