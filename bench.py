@@ -35,14 +35,21 @@ OP_NAMES = {2: "norm+qkv+rope", 3: "attention", 4: "o_proj+residual", 5: "norm+g
 
 # DRAM bytes per launch from an ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
 # valid only while the kernel sources hash to `source_sha256`.
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {
+    # profiles/layer_kernels_pi05_forward.md (layer 1 of one eager forward, batch 1, P 816).
+    "norm+qkv+rope": {"bytes": 5488896, "source_sha256": "4c094ba21c472595"},
+    "attention": {"bytes": 1148160, "source_sha256": "4c094ba21c472595"},
+    "o_proj+residual": {"bytes": 4663552, "source_sha256": "4c094ba21c472595"},
+    "norm+gate_up+geglu": {"bytes": 16959744, "source_sha256": "4c094ba21c472595"},
+    "down_proj+residual": {"bytes": 9067008, "source_sha256": "4c094ba21c472595"},
+}
 
 
 def source_sha() -> str:
     d = os.path.join(ROOT, "paper_2607_12659_gb300", "csrc")
     h = hashlib.sha256()
     for f in sorted(os.listdir(d)):
-        if f.endswith((".cu", ".h")):
+        if f.endswith((".cu", ".cuh", ".h")):
             h.update(open(os.path.join(d, f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -326,7 +333,7 @@ def our_arm(args):
     achieved = dom_bytes / (op_ms[dom] * 1e-3) / 1e9
     sha = source_sha()
     tr = NCU_TRAFFIC.get(OP_NAMES[dom])
-    traffic = tr["bytes"] if tr and tr.get("source_sha256") == sha else None
+    traffic = tr["bytes"] if tr and tr.get("source_sha256") == sha and default_workload else None
 
     n_kernels = jpi.jpi_graph_kernel_count(ex.handle, B, C, N)
     alg = algorithmic_bytes(cfg, B, P, C, N)
