@@ -60,6 +60,13 @@ __device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
+// 2^x by the hardware approximation (PTX ex2.approx.ftz.f32, relative error ~2^-22); the
+// arguments here are <= 0 (differences to a running maximum).
+__device__ __forceinline__ float fast_exp2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&v);
@@ -241,7 +248,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
             bmax[hh] = fmaxf(bmax[hh], __shfl_xor_sync(0xffffffffu, bmax[hh], 1));
             bmax[hh] = fmaxf(bmax[hh], __shfl_xor_sync(0xffffffffu, bmax[hh], 2));
             mnew[hh] = fmaxf(m_run[hh], bmax[hh]);
-            alpha[hh] = (mnew[hh] == -INFINITY) ? 1.f : exp2f(m_run[hh] - mnew[hh]);
+            alpha[hh] = (mnew[hh] == -INFINITY) ? 1.f : fast_exp2(m_run[hh] - mnew[hh]);
         }
         float psum[2] = {0.f, 0.f};
 #pragma unroll
@@ -249,7 +256,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int hh = e >> 1;
-                const float p = (sacc[nt][e] == -INFINITY) ? 0.f : exp2f(sacc[nt][e] - mnew[hh]);
+                const float p = (sacc[nt][e] == -INFINITY) ? 0.f : fast_exp2(sacc[nt][e] - mnew[hh]);
                 sacc[nt][e] = p;
                 psum[hh] += p;
             }
@@ -323,8 +330,8 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
             const int r = hh ? rb2 : ra;
             const float2 h0 = mls[r], h1 = mls[AT_ROWS + r];
             const float m = fmaxf(h0.x, h1.x);
-            w0[hh] = (h0.x == -INFINITY) ? 0.f : exp2f(h0.x - m);
-            w1[hh] = (h1.x == -INFINITY) ? 0.f : exp2f(h1.x - m);
+            w0[hh] = (h0.x == -INFINITY) ? 0.f : fast_exp2(h0.x - m);
+            w1[hh] = (h1.x == -INFINITY) ? 0.f : fast_exp2(h1.x - m);
             const float l = __fmaf_rn(h1.y, w1[hh], __fmul_rn(h0.y, w0[hh]));
             if (kh == 0 && cq == 0) *(float2*)(opart + r * ROWB + 2 * D) = make_float2(m, l);
         }
@@ -401,7 +408,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         float mx = ml.x;
 #pragma unroll
         for (int o = 1; o < AT_MAX_SPLITS; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        const float w = (ml.x == -INFINITY) ? 0.f : exp2f(ml.x - mx);
+        const float w = (ml.x == -INFINITY) ? 0.f : fast_exp2(ml.x - mx);
         float L = w * ml.y;
 #pragma unroll
         for (int o = 1; o < AT_MAX_SPLITS; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
