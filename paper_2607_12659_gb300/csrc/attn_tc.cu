@@ -415,28 +415,31 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         if (idx < nrow_here * AT_MAX_SPLITS) coef[(r - r_lo) * AT_MAX_SPLITS + s] = L > 0.f ? w / L : 0.f;
     }
     __syncthreads();
-    for (int idx = tid; idx < nrow_here * (D / 4); idx += AT_THREADS) {
-        const int r = r_lo + idx / (D / 4), d = (idx % (D / 4)) * 4;
+    // One item = 8 output dimensions of one owned row (a 16-byte load per split).
+    for (int idx = tid; idx < nrow_here * (D / 8); idx += AT_THREADS) {
+        const int r = r_lo + idx / (D / 8), d = (idx % (D / 8)) * 8;
         const int R = row0 + r;
         if (R >= nrows || !got) continue;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         // All 16 slots are loaded together (slots past the last split read this CTA's own row
         // with a zero coefficient), then summed in split order.
 #pragma unroll
         for (int s = 0; s < AT_MAX_SPLITS; ++s) {
             const float c = s < ns ? coef[(r - r_lo) * AT_MAX_SPLITS + s] : 0.f;
-            const uint2 hv = *(const uint2*)(srow(s < ns ? s : rank, r) + 2 * d);
-            const float2 v01 = __half22float2(*reinterpret_cast<const __half2*>(&hv.x));
-            const float2 v23 = __half22float2(*reinterpret_cast<const __half2*>(&hv.y));
-            acc.x = fmaf(c, v01.x, acc.x);
-            acc.y = fmaf(c, v01.y, acc.y);
-            acc.z = fmaf(c, v23.x, acc.z);
-            acc.w = fmaf(c, v23.y, acc.w);
+            const uint4 hv = *(const uint4*)(srow(s < ns ? s : rank, r) + 2 * d);
+            const uint32_t w4[4] = {hv.x, hv.y, hv.z, hv.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 v = __half22float2(*reinterpret_cast<const __half2*>(&w4[k]));
+                acc[2 * k] = fmaf(c, v.x, acc[2 * k]);
+                acc[2 * k + 1] = fmaf(c, v.y, acc[2 * k + 1]);
+            }
         }
         const int i = R / a.H, head = R - i * a.H;
         const size_t tok = (size_t)b * a.S + i;
-        uint2 packed = make_uint2(pack_bf16x2(acc.x, acc.y), pack_bf16x2(acc.z, acc.w));
-        *(uint2*)(a.o + (tok * a.H + head) * D + d) = packed;
+        *(uint4*)(a.o + (tok * a.H + head) * D + d) =
+            make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
+                       pack_bf16x2(acc[6], acc[7]));
     }
     if (tid == 0 && !got) atomicCAS(a.err, 0, (int)DEV_TIMEOUT_MMA);
     // No split exits while a copy out of its shared memory may still be in flight.

@@ -258,6 +258,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
             const int off63 = ((7 ^ (p & 7)) << 3) + 7;
             float4 y1 = make_float4(0.f, 0.f, 0.f, 0.f), y2 = y1;
             float b1 = 0.f, b2 = 0.f;
+#pragma unroll 4
             for (int r = 0; r < a.splits; ++r) {
                 const __half* s1;
                 const __half* s2;
