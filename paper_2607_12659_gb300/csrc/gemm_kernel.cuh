@@ -123,6 +123,13 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
     // (a release arrival would also wait for the weight copies in flight).
     ptx::cluster_arrive_relaxed();
     ptx::grid_dep_wait();
+    // When the next kernel may start: right away after the output projection, because the next
+    // one (gate/up) streams the largest weight set of the layer (2F x W, four times the output
+    // projection's) and needs the whole of this kernel to prefetch it; otherwise after the
+    // split-K receive (below), so that the next kernel's weight prefetch does not compete with
+    // this kernel's operand loads, MMAs and exchange.
+    constexpr bool EARLY_TRIGGER = (KIND == G_O);
+    if (EARLY_TRIGGER) ptx::grid_dep_launch();
 
     {
         const int tt = blockIdx.y;   // token tile
@@ -243,9 +250,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         // ranks arrive, every copy out of this CTA's partial has completed as well. Nothing else
         // is published through this barrier, so the arrival is relaxed.
         ptx::cluster_arrive_relaxed();
-        // The next kernel may start now: its weight prefetch would otherwise compete with this
-        // kernel's operand loads, MMAs and exchange for memory and shared-memory bandwidth.
-        ptx::grid_dep_launch();
+        if (!EARLY_TRIGGER) ptx::grid_dep_launch();
 
         // ---- 4. rank-ordered sum of the slices (own rows read in place) + epilogue ----
         float ssq[4] = {0.f, 0.f, 0.f, 0.f};
