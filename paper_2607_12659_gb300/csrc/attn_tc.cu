@@ -455,10 +455,13 @@ template <int D>
 jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     const int S = C + 1, nrows = S * h->H, nk = h->cur_prefix + S;
     const int rblocks = (nrows + AT_ROWS - 1) / AT_ROWS;
-    // Enough key splits for one request to put about two CTAs on every SM, at most 16 (one
-    // cluster). The split depends on the request's sizes only, never on the batch, so a request
-    // gives bitwise the same output alone or inside any batch.
-    int want = (2 * h->num_sms + rblocks - 1) / rblocks;
+    // Enough key splits for the launch to put about two CTAs on every SM, at most 16 (one
+    // cluster): 14 splits for one pi0.5-shaped request, one when many requests fill the GPU by
+    // themselves (then each CTA runs an online softmax over all keys and nothing is exchanged).
+    // The split follows the launch's sizes, so a request's low-order bits depend on the batch
+    // size it runs with; they never depend on timing.
+    const int blocks = rblocks * B;
+    int want = (2 * h->num_sms + blocks - 1) / blocks;
     want = want < 1 ? 1 : (want > h->attn_max_splits ? h->attn_max_splits : want);
     int chunk = (nk + want - 1) / want;
     chunk = (chunk + 15) / 16 * 16;

@@ -132,11 +132,12 @@ def test_pi05_batches_sampled_requests(pi05, B):
     got = gpu_denoise(ex, PI05, r, 10)
     sample = sorted({0, B // 2, B - 1})
     assert_close(got[sample], oracle_denoise(PI05, w, r, 10, sample), PI05, f"batch {B}")
-    # Batch independence: request b alone gives the same actions as inside the batch.
+    # Batch independence: request b alone gives the same actions as inside the batch, up to the
+    # low-order bits that the attention's batch-dependent key split moves.
     b = B - 1
     r1 = make_requests(PI05, 4000 + B, 1, 816, 50, first_request=b)
     one = gpu_denoise(ex, PI05, r1, 10)
-    assert np.abs(one[0] - got[b]).max() <= 1e-5
+    assert_close(got[b:b + 1], one, PI05, f"batch {B} vs alone")
 
 
 def test_pi05_high_gain_forward():
