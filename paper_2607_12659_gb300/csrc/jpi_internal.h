@@ -159,6 +159,7 @@ struct jpi_handle {
     // Tensor-core path: one plan per projection (QKV, O, gate/up, down) and tensor maps
     // (4 per layer, same order).
     jpi::GemmPlan plans[4];
+    int big_min_tokens = 512;   // launches with at least this many tokens use the large-M GEMMs
     std::vector<CUtensorMap> tmaps;
     CUtensorMap xmaps[3];       // B operands: hx, o, z
 

@@ -21,6 +21,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <type_traits>
 #include <cmath>
 #include <cstdlib>
 #include <vector>
@@ -125,6 +126,7 @@ __host__ __device__ __forceinline__ GemmSmem gemm_layout(int kpb, int splits, bo
 }
 
 #include "gemm_kernel.cuh"
+#include "gemm_big.cuh"
 
 // ---------------------------------------------------------------------------------------------
 // Host side: packing, plans, tensor maps, launches.
@@ -280,6 +282,29 @@ jpi_status launch_gemm(jpi_handle* h, const GemmPlan& pl, const CUtensorMap& wma
     return JPI_OK;
 }
 
+// Large-M variant: grid (weight tiles, 128-row operand tiles), no cluster, full K per CTA.
+template <int KIND>
+jpi_status launch_gemm_big(jpi_handle* h, const GemmPlan& pl, const CUtensorMap& wmap,
+                           const CUtensorMap& xmap, const GemmArgs& a, cudaStream_t st) {
+    constexpr int TT = (KIND == G_QKV || KIND == G_GU) ? 2 * XS_TOKENS : BIG_NT;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(pl.ntiles, (unsigned)std::max(1, (a.Mt + TT - 1) / TT));
+    cfg.blockDim = dim3(BIG_THREADS);
+    cfg.dynamicSmemBytes = 1024 + big_smem_bytes();
+    cfg.stream = st;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = h->pdl ? 1 : 0;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_big<KIND>, wmap, xmap, a);
+    if (e != cudaSuccess) {
+        set_error("tensor-core GEMM launch failed: %s", cudaGetErrorString(e));
+        return JPI_ERR_CUDA;
+    }
+    return JPI_OK;
+}
+
 GemmArgs base_args(jpi_handle* h, int B, int C, const GemmPlan& pl) {
     GemmArgs a = {};
     a.Mt = B * (C + 1);
@@ -373,6 +398,12 @@ jpi_status tc_prepare(jpi_handle* h) {
         }
         JPI_CUDA_TRY(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024));
     }
+    auto big_kernels = {k_tc_gemm_big<G_QKV>, k_tc_gemm_big<G_O>, k_tc_gemm_big<G_GU>, k_tc_gemm_big<G_DOWN>};
+    for (auto k : big_kernels)
+        JPI_CUDA_TRY(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes()));
+    // Launches with at least this many tokens use the large-M kernels (full K per CTA).
+    const char* big_env = std::getenv("JPI_BIG_GEMM_MIN_TOKENS");
+    h->big_min_tokens = big_env ? std::atoi(big_env) : 512;
     const int rows[4] = {h->QKV, h->W, 2 * h->F, h->W};
     const int ks[4] = {h->W, h->HD, h->W, h->F};
     // The K split (and so the summation order) is chosen once per projection, for every batch
@@ -434,18 +465,31 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * W + (size_t)6 * l * W;
     const size_t kv_layer = (size_t)l * h->maxB * h->kv_rows * h->D;
     const jpi::GemmPlan* plans = h->plans;
+    const int Mt = B * (C + 1);
+    // Batched launches with many tokens: one CTA per (weight tile, 128-row operand tile) over
+    // the whole K range. Residual kinds then leave one sum-of-squares slot per weight tile.
+    const bool big = h->big_min_tokens > 0 && Mt >= h->big_min_tokens;
+    auto run = [&](auto kind_tag, const GemmPlan& pl, const CUtensorMap& wm, const CUtensorMap& xm,
+                   const GemmArgs& a) -> jpi_status {
+        constexpr int KIND = decltype(kind_tag)::value;
+        return big ? launch_gemm_big<KIND>(h, pl, wm, xm, a, st) : launch_gemm<KIND>(h, pl, wm, xm, a, st);
+    };
+    using KQ = std::integral_constant<int, G_QKV>;
+    using KO = std::integral_constant<int, G_O>;
+    using KG = std::integral_constant<int, G_GU>;
+    using KD = std::integral_constant<int, G_DOWN>;
     switch (op) {
         case 2: {
             const GemmPlan& pl = plans[G_QKV];
             GemmArgs a = base_args(h, B, C, pl);
             // Sums of squares left by the embedding (one per 128 features) or the previous
             // layer's down projection (one per CTA).
-            if (l > 0) a.nslot = plans[G_DOWN].ntiles * plans[G_DOWN].splits;
+            if (l > 0) a.nslot = big ? plans[G_DOWN].ntiles : plans[G_DOWN].ntiles * plans[G_DOWN].splits;
             a.q = (__nv_bfloat16*)h->q;
             a.kst = (__nv_bfloat16*)h->kv_k + kv_layer;
             a.vst = (__nv_bfloat16*)h->kv_v + kv_layer;
             a.rope = h->rope_tab;
-            return launch_gemm<G_QKV>(h, pl, h->tmaps[4 * l + G_QKV], h->xmaps[0], a, st);
+            return run(KQ{}, pl, h->tmaps[4 * l + G_QKV], h->xmaps[0], a);
         }
         case 3:
             return attn_tc_supported(h) ? launch_attn_tc(h, l, B, C, st)
@@ -459,14 +503,14 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
             a.beta_next = ms + 4 * W;
             a.gamma = ms + 2 * W;
             a.ss_out = h->ss;
-            return launch_gemm<G_O>(h, pl, h->tmaps[4 * l + G_O], h->xmaps[1], a, st);
+            return run(KO{}, pl, h->tmaps[4 * l + G_O], h->xmaps[1], a);
         }
         case 5: {
             const GemmPlan& pl = plans[G_GU];
             GemmArgs a = base_args(h, B, C, pl);
-            a.nslot = plans[G_O].ntiles * plans[G_O].splits;   // left by the output projection
+            a.nslot = big ? plans[G_O].ntiles : plans[G_O].ntiles * plans[G_O].splits;   // left by O
             a.z = (__nv_bfloat16*)h->z;
-            return launch_gemm<G_GU>(h, pl, h->tmaps[4 * l + G_GU], h->xmaps[0], a, st);
+            return run(KG{}, pl, h->tmaps[4 * l + G_GU], h->xmaps[0], a);
         }
         case 6: {
             const GemmPlan& pl = plans[G_DOWN];
@@ -479,7 +523,7 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
             }
             a.gamma = ms + 5 * W;
             a.ss_out = h->ss;
-            return launch_gemm<G_DOWN>(h, pl, h->tmaps[4 * l + G_DOWN], h->xmaps[2], a, st);
+            return run(KD{}, pl, h->tmaps[4 * l + G_DOWN], h->xmaps[2], a);
         }
         default:
             set_error("unknown layer op %d", op);
