@@ -39,6 +39,11 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool v
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
                  : "memory");
 }
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
 __device__ __forceinline__ void cp_async_wait_all() {
     asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
 }
@@ -101,12 +106,13 @@ template <int D>
 __host__ __device__ constexpr int attn_ofp_stride() {
     return D / 2 + 8;
 }
-// Shared-memory layout (bytes from the 128-aligned base): q/k/v, reused after the key loop for
-// each key half's hand-over columns (fp32) and (m, l), then this split's partial rows; the receive
-// buffer; the combine coefficients; the receive barrier.
-template <int D>
+// Shared-memory layout (bytes from the 128-aligned base): q and NBUF k/v buffers, reused after
+// the key loop for each key half's hand-over columns (fp32) and (m, l), then this split's partial
+// rows; the receive buffer; the combine coefficients; the receive barrier.
+template <int D, int NBUF>
 struct AttnSmem {
-    static constexpr int QKV = (AT_ROWS + 2 * AT_KEYS) * D * 2;
+    static constexpr int KB = NBUF == 2 ? AT_KEYS / 2 : AT_KEYS;   // keys per block
+    static constexpr int QKV = (AT_ROWS + 2 * KB * NBUF) * D * 2;
     static constexpr int OFP = 2 * AT_ROWS * attn_ofp_stride<D>() * 4;   // [2 halves][32][OS]
     static constexpr int ML = OFP;                               // [2 halves][32] float2
     static constexpr int OPART = ML + 2 * AT_ROWS * 8;           // [32][row bytes]
@@ -118,14 +124,19 @@ struct AttnSmem {
     static constexpr int TOTAL = BAR + 16;
 };
 
-template <int D>
+// NBUF = 2 when a split spans several key blocks: blocks of 32 keys, double-buffered (the next
+// block's K/V loads are issued before the current block is processed) in the same shared memory
+// as one 64-key block, so two CTAs still fit on an SM.
+template <int D, int NBUF>
 __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ AttnArgs a) {
-    using L = AttnSmem<D>;
+    using L = AttnSmem<D, NBUF>;
+    constexpr int KB = L::KB;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((128u - (ptx::smem_u32(smem_raw) & 127u)) & 127u);
     uint8_t* qs = smem;                                  // [32][D] bf16
-    uint8_t* ks = qs + AT_ROWS * D * 2;                  // [64][D] bf16
-    uint8_t* vs = ks + AT_KEYS * D * 2;                  // [64][D] bf16
+    uint8_t* ks = qs + AT_ROWS * D * 2;                  // [NBUF][k [64][D], v [64][D]] bf16
+    uint8_t* vs = ks + KB * D * 2;
+    constexpr uint32_t KV_BUF = 2 * KB * D * 2;     // bytes of one k/v buffer pair
     constexpr int ROWB = attn_row_bytes<D>();
     constexpr int OS = attn_ofp_stride<D>();
     float* ofp = (float*)smem;                           // [2][32][OS] columns handed over
@@ -162,18 +173,19 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     const __nv_bfloat16* kb_ = a.kst + (size_t)b * a.kv_rows * D;
     const __nv_bfloat16* vb_ = a.vst + (size_t)b * a.kv_rows * D;
     const uint32_t qs_u = ptx::smem_u32(qs), ks_u = ptx::smem_u32(ks), vs_u = ptx::smem_u32(vs);
-    auto load_kv = [&](int key0, int r_from, int r_to) {
-        for (int idx = tid; idx < AT_KEYS * DC; idx += AT_THREADS) {
+    auto load_kv = [&](int key0, int r_from, int r_to, int buf) {
+        const uint32_t kd = ks_u + buf * KV_BUF, vd = vs_u + buf * KV_BUF;
+        for (int idx = tid; idx < KB * DC; idx += AT_THREADS) {
             const int r = idx / DC, c = idx % DC;
             if (r < r_from || r >= r_to) continue;
             const bool ok = key0 + r < k_end;
             const size_t off = (size_t)(ok ? key0 + r : 0) * D + c * 8;
-            cp_async16(ks_u + sw_off<D>(r, c), kb_ + off, ok);
-            cp_async16(vs_u + sw_off<D>(r, c), vb_ + off, ok);
+            cp_async16(kd + sw_off<D>(r, c), kb_ + off, ok);
+            cp_async16(vd + sw_off<D>(r, c), vb_ + off, ok);
         }
     };
-    const int first_suffix_row = min(AT_KEYS, max(0, a.P - k_begin));
-    load_kv(k_begin, 0, first_suffix_row);
+    const int first_suffix_row = min(KB, max(0, a.P - k_begin));
+    load_kv(k_begin, 0, first_suffix_row, 0);
 
     ptx::grid_dep_wait();
 
@@ -184,7 +196,8 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         const bool ok = row0 + r < nrows;
         cp_async16(qs_u + sw_off<D>(r, c), qb + (size_t)(ok ? row0 + r : 0) * D + c * 8, ok);
     }
-    load_kv(k_begin, first_suffix_row, AT_KEYS);
+    load_kv(k_begin, first_suffix_row, KB, 0);
+    if (NBUF == 2) cp_async_commit();   // group: q and the first block
 
     // Per-thread rows g and g + 8 of this warp's 16; their visible key count.
     const int g = lane >> 2, cq = lane & 3;
@@ -200,13 +213,26 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
 #pragma unroll
     for (int n = 0; n < D / 8; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.f;
     float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-    constexpr int HK = AT_KEYS / 2;                      // keys per half
+    constexpr int HK = KB / 2;                      // keys per half
 
-    for (int key0 = k_begin; key0 < k_end; key0 += AT_KEYS) {
+    int buf = 0;
+    for (int key0 = k_begin; key0 < k_end; key0 += KB) {
+        __syncthreads();   // every warp is done with the buffer refilled below
+        if (NBUF == 2) {
+            if (key0 + KB < k_end) {
+                load_kv(key0 + KB, 0, KB, buf ^ 1);
+                cp_async_commit();
+                cp_async_wait_group<1>();   // this block's group has landed
+            } else {
+                cp_async_wait_group<0>();
+            }
+        } else {
+            if (key0 != k_begin) load_kv(key0, 0, KB, 0);
+            cp_async_wait_all();
+        }
         __syncthreads();
-        if (key0 != k_begin) load_kv(key0, 0, AT_KEYS);
-        cp_async_wait_all();
-        __syncthreads();
+        const uint32_t kbuf_u = ks_u + buf * KV_BUF, vbuf_u = vs_u + buf * KV_BUF;
+        if (NBUF == 2) buf ^= 1;
 
         // S = Q K^T for this warp's 16 rows x 32 keys.
         float sacc[HK / 8][4];
@@ -225,7 +251,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
                 uint32_t b0, b1, b2, b3;
                 const int r = kh * HK + (nt + (lane >> 4)) * 8 + (lane & 7);
                 const int c = kc * 2 + ((lane >> 3) & 1);
-                ldsm_x4(ks_u + sw_off<D>(r, c), b0, b1, b2, b3);
+                ldsm_x4(kbuf_u + sw_off<D>(r, c), b0, b1, b2, b3);
                 mma16816(sacc[nt], a0, a1, a2, a3, b0, b1);
                 mma16816(sacc[nt + 1], a0, a1, a2, a3, b2, b3);
             }
@@ -286,7 +312,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
                 uint32_t b0, b1, b2, b3;
                 const int r = kh * HK + j * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                 const int c = dt + (lane >> 4);
-                ldsm_x4_t(vs_u + sw_off<D>(r, c), b0, b1, b2, b3);
+                ldsm_x4_t(vbuf_u + sw_off<D>(r, c), b0, b1, b2, b3);
                 mma16816(oacc[dt], a0, a1, a2, a3, b0, b1);
                 mma16816(oacc[dt + 1], a0, a1, a2, a3, b2, b3);
             }
@@ -446,9 +472,9 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     ptx::cluster_wait();
 }
 
-template <int D>
+template <int D, int NBUF>
 size_t attn_smem() {
-    return 128 + (size_t)AttnSmem<D>::TOTAL;
+    return 128 + (size_t)AttnSmem<D, NBUF>::TOTAL;
 }
 
 template <int D>
@@ -483,7 +509,11 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(rblocks, ns, B);
     cfg.blockDim = dim3(AT_THREADS);
-    cfg.dynamicSmemBytes = attn_smem<D>();
+    // Splits of 2..8 key blocks: 32-key blocks, double-buffered (measured faster there); longer
+    // splits keep 64-key blocks, where the per-block rescale of the output accumulators would
+    // otherwise double.
+    const bool two = chunk > AT_KEYS && chunk <= 8 * AT_KEYS;
+    cfg.dynamicSmemBytes = two ? attn_smem<D, 2>() : attn_smem<D, 1>();
     cfg.stream = st;
     cudaLaunchAttribute attrs[2];
     int n = 0;
@@ -499,7 +529,7 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     }
     cfg.attrs = attrs;
     cfg.numAttrs = n;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_tc<D>, a);
+    cudaError_t e = two ? cudaLaunchKernelEx(&cfg, k_attn_tc<D, 2>, a) : cudaLaunchKernelEx(&cfg, k_attn_tc<D, 1>, a);
     if (e != cudaSuccess) {
         set_error("attention launch failed: %s", cudaGetErrorString(e));
         return JPI_ERR_CUDA;
@@ -509,9 +539,12 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
 
 template <int D>
 jpi_status prepare_d(jpi_handle* h) {
-    JPI_CUDA_TRY(cudaFuncSetAttribute(k_attn_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      (int)attn_smem<D>()));
-    if (cudaFuncSetAttribute(k_attn_tc<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_attn_tc<D, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)attn_smem<D, 1>()));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_attn_tc<D, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)attn_smem<D, 2>()));
+    if (cudaFuncSetAttribute(k_attn_tc<D, 1>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
+        cudaFuncSetAttribute(k_attn_tc<D, 2>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
         cudaGetLastError();
         h->attn_max_splits = 8;
     } else {
