@@ -171,3 +171,33 @@ def test_pi05_batch64_prefix2048_sampled():
         assert_close(got[sample], oracle_denoise(PI05, w, r, 10, sample), PI05, "batch 64 P2048")
     finally:
         ex.close()
+
+
+@pytest.fixture
+def large_m_everywhere(monkeypatch):
+    """Handles created under this fixture run every projection through the large-M kernel."""
+    monkeypatch.setenv("JPI_BIG_GEMM_MIN_TOKENS", "1")
+
+
+@pytest.mark.parametrize("B,P,C,N", [(1, 100, 13, 2), (3, 257, 50, 1), (2, 64, 70, 3)])
+def test_small_bf16_large_m_projection_path(large_m_everywhere, B, P, C, N):
+    w = make_weights(SMALL_BF16, 2200)
+    ex = make_expert(SMALL_BF16, w, max_batch=3, max_prefix=300, max_chunk=70, max_steps=3)
+    try:
+        r = make_requests(SMALL_BF16, 2201 + B, B, P, C)
+        got = gpu_denoise(ex, SMALL_BF16, r, N)
+        assert_close(got, oracle_denoise(SMALL_BF16, oracle.to_f64(w), r, N), SMALL_BF16,
+                     f"small bf16 large-M B{B} P{P} C{C} N{N}")
+    finally:
+        ex.close()
+
+
+def test_pi05_large_m_projection_path(large_m_everywhere):
+    w = make_weights(PI05, 2000)
+    ex = make_expert(PI05, w, max_batch=3, max_prefix=816, max_chunk=50, max_steps=10)
+    try:
+        r = make_requests(PI05, 2300, 3, 816, 50)
+        got = gpu_denoise(ex, PI05, r, 10)
+        assert_close(got[[0, 2]], oracle_denoise(PI05, w, r, 10, [0, 2]), PI05, "pi0.5 large-M B3")
+    finally:
+        ex.close()
