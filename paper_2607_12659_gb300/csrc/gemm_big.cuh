@@ -10,9 +10,10 @@
 //   warps 2-5  the epilogue: one TMEM lane (weight row) per thread, then the same per-kind
 //           epilogues as the split-K kernel (rotary + scatter, GeGLU, gated residual with the
 //           next norm's operand and sums of squares). Row pairs (p, p + 64) meet through a
-//           shared fp32 staging tile that reuses the stage ring once the MMAs are done. While
-//           the MMAs run, the epilogue threads stage their residual rows (or rotary factors)
-//           from global memory into shared memory, so no global load is left after them.
+//           shared fp32 staging tile that reuses the stage ring once the MMAs are done. The
+//           accumulator is read and the residual rows / rotary factors are loaded in chunks of
+//           16-32 columns (each chunk's loads issued together). Two CTAs share an SM, so one
+//           CTA's epilogue overlaps the other's mainloop.
 // The next kernel is released once the accumulator is complete. All waits are bounded.
 
 constexpr int BIG_NT = 128;                       // operand rows per tile
@@ -22,17 +23,14 @@ constexpr int BIG_XBYTES = BIG_NT * KBLK * 2;     // 16 KB operand block
 constexpr int BIG_STAGE_BYTES = TILE_BYTES + BIG_XBYTES;
 constexpr int BIG_YS = BIG_NT + 1;                // fp32 staging row stride: conflict-free rows and columns
 
-constexpr int BIG_PRE_OFF = BIG_STAGES * BIG_STAGE_BYTES;   // residual rows / rotary factors
-constexpr int BIG_PRE_BYTES = BIG_NT * BIG_YS * 4;
 __host__ __device__ constexpr int big_smem_bytes() {
-    // stages | pre-staged epilogue inputs | rinv[128] | bars (full, empty, acc) + TMEM slot + flag
-    return BIG_PRE_OFF + BIG_PRE_BYTES + BIG_NT * 4 + 128;
+    // stages | rinv[128] | bars (full, empty, acc) + TMEM slot + flag
+    return BIG_STAGES * BIG_STAGE_BYTES + BIG_NT * 4 + 128;
 }
-static_assert(BIG_NT * XS_TOKENS * 8 <= BIG_PRE_BYTES, "rotary factors fit in the pre-stage region");
 static_assert(BIG_NT * BIG_YS * 4 <= BIG_STAGES * BIG_STAGE_BYTES, "staging tile fits in the stage ring");
 
 template <int KIND>
-__global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_constant__ CUtensorMap wmap,
+__global__ void __launch_bounds__(BIG_THREADS, 2) k_tc_gemm_big(const __grid_constant__ CUtensorMap wmap,
                                                              const __grid_constant__ CUtensorMap xmap,
                                                              const __grid_constant__ GemmArgs a) {
     constexpr bool NORM_IN = (KIND == G_QKV || KIND == G_GU);
@@ -44,8 +42,7 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
     uint8_t* smem = smem_raw + ((1024u - (ptx::smem_u32(smem_raw) & 1023u)) & 1023u);
     uint8_t* stages = smem;                                        // [stage][W 16 KB | X 16 KB]
     float* ystage = (float*)smem;                                  // [128][BIG_YS] after the MMAs
-    float* pre = (float*)(smem + BIG_PRE_OFF);                     // [128][BIG_YS] h, or [128][63] float2
-    float* rinv_s = pre + BIG_NT * BIG_YS;                         // [128]
+    float* rinv_s = (float*)(smem + BIG_STAGES * BIG_STAGE_BYTES); // [128]
     uint64_t* full = (uint64_t*)(rinv_s + BIG_NT);
     uint64_t* empty = full + BIG_STAGES;
     uint64_t* accb = empty + BIG_STAGES;
@@ -132,27 +129,6 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
             sec = pair / hd;
             d = pair - sec * hd;
         }
-        if (RESID) {
-            // This thread's residual row for the tile's tokens (coalesced across the warp).
-            const int f = tile * TILE_ROWS + row;
-#pragma unroll 16
-            for (int c = 0; c < BIG_NT; ++c) {
-                const int t = tok0 + c;
-                pre[row * BIG_YS + c] = t < a.Mt ? a.hres[(size_t)t * a.W + f] : 0.f;
-            }
-        }
-        if (KIND == G_QKV && a.rope && sec <= a.H) {
-            // Rotary factors of this pair for its 63 tokens.
-            const int hd = a.D >> 1;
-            float2* rs = (float2*)pre + et * XS_TOKENS;
-            const int tfirst = tok0 + h * XS_TOKENS;
-            int qi = tfirst % a.S;
-#pragma unroll 8
-            for (int j = 0; j < XS_TOKENS; ++j) {
-                rs[j] = tfirst + j < a.Mt ? __ldg(a.rope + (size_t)(a.P + qi) * hd + d) : make_float2(1.f, 0.f);
-                if (++qi == a.S) qi = 0;
-            }
-        }
         if (NORM_IN) {
             // Column scale: rinv of the column's token (sums of squares in slot order), 1 for
             // the beta columns 63 and 127.
@@ -176,68 +152,121 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
         ptx::grid_dep_launch();
         const bool ok = *flag == 0;
 
-        float v[BIG_NT];
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-#pragma unroll
-        for (int c0 = 0; c0 < BIG_NT; c0 += 16) {
-            uint32_t r[16];
-            ptx::tmem_ld_x16(lane_base + (uint32_t)c0, r);
-            ptx::tmem_ld_wait();
-#pragma unroll
-            for (int i = 0; i < 16; ++i) v[c0 + i] = __uint_as_float(r[i]);
-        }
-
         if (NORM_IN) {
-            const float beta0 = v[63], beta1 = v[127];
+            // y = rinv * acc + (W beta of the column's 64-group), staged as fp32 rows.
+            float beta0, beta1;
+            {
+                uint32_t r[16];
+                ptx::tmem_ld_x16(lane_base + 48u, r);
+                ptx::tmem_ld_wait();
+                beta0 = __uint_as_float(r[15]);
+                ptx::tmem_ld_x16(lane_base + 112u, r);
+                ptx::tmem_ld_wait();
+                beta1 = __uint_as_float(r[15]);
+            }
 #pragma unroll
-            for (int c = 0; c < BIG_NT; ++c)
-                ystage[row * BIG_YS + c] = (c & 63) == 63 ? 0.f : rinv_s[c] * v[c] + (c < 64 ? beta0 : beta1);
+            for (int c0 = 0; c0 < BIG_NT; c0 += 16) {
+                uint32_t r[16];
+                ptx::tmem_ld_x16(lane_base + (uint32_t)c0, r);
+                ptx::tmem_ld_wait();
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int c = c0 + i;
+                    ystage[row * BIG_YS + c] =
+                        (c & 63) == 63 ? 0.f : rinv_s[c] * __uint_as_float(r[i]) + (c < 64 ? beta0 : beta1);
+                }
+            }
             ptx::named_bar_sync(1, 128);
-            // Thread (pair p, column half h): rows p and p + 64 of this tile for 63 tokens.
-            const float2* rs = (const float2*)pre + et * XS_TOKENS;
+            // Thread (pair p, column half h): rows p and p + 64 of this tile for 63 tokens, in
+            // chunks of 16 tokens whose rotary factors are loaded together.
             const int tfirst = tok0 + h * XS_TOKENS;
             int qb = tfirst / a.S, qi = tfirst - qb * a.S;   // request and position of the token
-            for (int j = 0; j < XS_TOKENS; ++j) {
-                const int t = tfirst + j;
-                const int b = qb, i = qi;
-                if (++qi == a.S) {
-                    qi = 0;
-                    ++qb;
-                }
-                if (t >= a.Mt || !ok) break;
-                const int c = h * 64 + j;
-                const float u1 = ystage[p * BIG_YS + c], u2 = ystage[(p + 64) * BIG_YS + c];
-                if (KIND == G_QKV) {
+            const bool rot = KIND == G_QKV && a.rope && sec <= a.H;
+            for (int j0 = 0; j0 < XS_TOKENS; j0 += 16) {
+                float2 cs[16];
+                if (rot) {
                     const int hd = a.D >> 1;
-                    float r1 = u1, r2 = u2;
-                    if (sec <= a.H && a.rope) {
-                        const float2 cs = rs[j];
-                        r1 = u1 * cs.x - u2 * cs.y;
-                        r2 = u2 * cs.x + u1 * cs.y;
+                    int ql = qi;
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const bool in = j0 + i < XS_TOKENS && tfirst + j0 + i < a.Mt;
+                        cs[i] = in ? __ldg(a.rope + (size_t)(a.P + ql) * hd + d) : make_float2(1.f, 0.f);
+                        if (++ql == a.S) ql = 0;
                     }
-                    __nv_bfloat16* dst = (sec < a.H) ? a.q + ((size_t)t * a.H + sec) * a.D
-                                                     : (sec == a.H ? a.kst : a.vst) + ((size_t)b * a.kv_rows + a.P + i) * a.D;
-                    dst[d] = __float2bfloat16_rn(r1);
-                    dst[d + hd] = __float2bfloat16_rn(r2);
-                } else {
-                    a.z[(size_t)t * a.F + pair] = __float2bfloat16_rn(gelu_tanh(u1) * u2);
+                }
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int j = j0 + i;
+                    if (j >= XS_TOKENS) break;
+                    const int t = tfirst + j;
+                    const int b = qb, ii = qi;
+                    if (++qi == a.S) {
+                        qi = 0;
+                        ++qb;
+                    }
+                    if (t >= a.Mt || !ok) continue;
+                    const int c = h * 64 + j;
+                    const float u1 = ystage[p * BIG_YS + c], u2 = ystage[(p + 64) * BIG_YS + c];
+                    if (KIND == G_QKV) {
+                        const int hd = a.D >> 1;
+                        float r1 = u1, r2 = u2;
+                        if (rot) {
+                            r1 = u1 * cs[i].x - u2 * cs[i].y;
+                            r2 = u2 * cs[i].x + u1 * cs[i].y;
+                        }
+                        __nv_bfloat16* dst = (sec < a.H) ? a.q + ((size_t)t * a.H + sec) * a.D
+                                                         : (sec == a.H ? a.kst : a.vst) + ((size_t)b * a.kv_rows + a.P + ii) * a.D;
+                        dst[d] = __float2bfloat16_rn(r1);
+                        dst[d + hd] = __float2bfloat16_rn(r2);
+                    } else {
+                        a.z[(size_t)t * a.F + pair] = __float2bfloat16_rn(gelu_tanh(u1) * u2);
+                    }
                 }
             }
         } else {
             const int f = tile * TILE_ROWS + row;
             const float g = a.gamma[f];
             const float sn = a.xs ? a.sigma_next[f] : 0.f;
+            // 16 columns at a time; the next chunk's residual values are loaded (together) before
+            // this chunk is updated, so their latency overlaps the updates.
+            float hv[16];
+            auto load_h = [&](int c0, float (&dst)[16]) {
 #pragma unroll
-            for (int c = 0; c < BIG_NT; ++c) {
-                const int t = tok0 + c;
-                float sq = 0.f;
-                if (t < a.Mt && ok) {
-                    const float n = pre[row * BIG_YS + c] + g * v[c];
-                    a.hres[(size_t)t * a.W + f] = n;
-                    if (a.xs) a.xs[(size_t)xs_row(t) * a.W + f] = __float2bfloat16_rn((1.f + sn) * n);
-                    sq = n * n;
+                for (int i = 0; i < 16; ++i) {
+                    const int t = tok0 + c0 + i;
+                    dst[i] = t < a.Mt ? a.hres[(size_t)t * a.W + f] : 0.f;
                 }
-                ystage[row * BIG_YS + c] = sq;
+            };
+            // The accumulator goes to this thread's staging row first, so no global load is in
+            // flight while TMEM is read.
+#pragma unroll
+            for (int c0 = 0; c0 < BIG_NT; c0 += 16) {
+                uint32_t r[16];
+                ptx::tmem_ld_x16(lane_base + (uint32_t)c0, r);
+                ptx::tmem_ld_wait();
+#pragma unroll
+                for (int i = 0; i < 16; ++i) ystage[row * BIG_YS + c0 + i] = __uint_as_float(r[i]);
+            }
+            load_h(0, hv);
+#pragma unroll 1
+            for (int c0 = 0; c0 < BIG_NT; c0 += 16) {
+                float hn[16];
+                if (c0 + 16 < BIG_NT) load_h(c0 + 16, hn);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int c = c0 + i, t = tok0 + c;
+                    float sq = 0.f;
+                    if (t < a.Mt && ok) {
+                        const float n = hv[i] + g * ystage[row * BIG_YS + c];
+                        a.hres[(size_t)t * a.W + f] = n;
+                        if (a.xs) a.xs[(size_t)xs_row(t) * a.W + f] = __float2bfloat16_rn((1.f + sn) * n);
+                        sq = n * n;
+                    }
+                    ystage[row * BIG_YS + c] = sq;
+                }
+#pragma unroll
+                for (int i = 0; i < 16; ++i) hv[i] = hn[i];
             }
             // The next norm's shift in the last row of each of its token tiles (this tile's rows).
             if (a.xs && xt == 0 && ok) {
