@@ -183,18 +183,22 @@ __global__ void __launch_bounds__(BIG_THREADS, 2) k_tc_gemm_big(const __grid_con
             const int tfirst = tok0 + h * XS_TOKENS;
             int qb = tfirst / a.S, qi = tfirst - qb * a.S;   // request and position of the token
             const bool rot = KIND == G_QKV && a.rope && sec <= a.H;
-            for (int j0 = 0; j0 < XS_TOKENS; j0 += 16) {
-                float2 cs[16];
-                if (rot) {
-                    const int hd = a.D >> 1;
-                    int ql = qi;
+            // Rotary factors of tokens j0..j0+15, loaded together; position ql advances with j.
+            int ql = qi;
+            auto load_cs = [&](int j0, float2 (&dst)[16]) {
+                const int hd = a.D >> 1;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const bool in = j0 + i < XS_TOKENS && tfirst + j0 + i < a.Mt;
-                        cs[i] = in ? __ldg(a.rope + (size_t)(a.P + ql) * hd + d) : make_float2(1.f, 0.f);
-                        if (++ql == a.S) ql = 0;
-                    }
+                for (int i = 0; i < 16; ++i) {
+                    const bool in = rot && j0 + i < XS_TOKENS && tfirst + j0 + i < a.Mt;
+                    dst[i] = in ? __ldg(a.rope + (size_t)(a.P + ql) * hd + d) : make_float2(1.f, 0.f);
+                    if (++ql == a.S) ql = 0;
                 }
+            };
+            float2 cs[16];
+            load_cs(0, cs);
+            for (int j0 = 0; j0 < XS_TOKENS; j0 += 16) {
+                float2 cn[16];
+                if (j0 + 16 < XS_TOKENS) load_cs(j0 + 16, cn);   // the next chunk's factors in flight
 #pragma unroll
                 for (int i = 0; i < 16; ++i) {
                     const int j = j0 + i;
@@ -223,6 +227,8 @@ __global__ void __launch_bounds__(BIG_THREADS, 2) k_tc_gemm_big(const __grid_con
                         a.z[(size_t)t * a.F + pair] = __float2bfloat16_rn(gelu_tanh(u1) * u2);
                     }
                 }
+#pragma unroll
+                for (int i = 0; i < 16; ++i) cs[i] = cn[i];
             }
         } else {
             const int f = tile * TILE_ROWS + row;
