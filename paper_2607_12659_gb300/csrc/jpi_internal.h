@@ -160,6 +160,9 @@ struct jpi_handle {
     // (4 per layer, same order).
     jpi::GemmPlan plans[4];
     int big_min_tokens = 512;   // launches with at least this many tokens use the large-M GEMMs
+    int attn_t5_min_batch = 4;  // batches of at least this many requests use the unsplit attention
+    bool attn_t5 = false;       // its tensor maps and attributes are ready
+    CUtensorMap amaps[3];       // attention operands: q, prefix/suffix K, V (all layers)
     std::vector<CUtensorMap> tmaps;
     CUtensorMap xmaps[3];       // B operands: hx, o, z
 

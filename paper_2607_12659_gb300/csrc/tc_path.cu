@@ -330,6 +330,10 @@ GemmArgs base_args(jpi_handle* h, int B, int C, const GemmPlan& pl) {
 
 }  // namespace
 
+jpi_status tc_make_tmap(const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows, CUtensorMap* map) {
+    return make_tmap(base, rows, cols, box_rows, map);
+}
+
 bool tc_supported(const jpi_handle* h) {
     return h->W % TILE_ROWS == 0 && h->D % TILE_ROWS == 0 && h->F % 64 == 0 && h->HD % KBLK == 0 &&
            h->W / TILE_ROWS <= 64;
@@ -386,6 +390,7 @@ jpi_status tc_prepare(jpi_handle* h) {
     JPI_CUDA_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     h->num_sms = sms;
     if (attn_tc_supported(h)) JPI_TRY(attn_tc_prepare(h));
+    JPI_TRY(attn_t5_prepare(h));
     const char* pdl_env = std::getenv("JPI_PDL");
     h->pdl = !(pdl_env && pdl_env[0] == '0');
 
@@ -492,6 +497,10 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
             return run(KQ{}, pl, h->tmaps[4 * l + G_QKV], h->xmaps[0], a);
         }
         case 3:
+            // Batched launches: one CTA per 128 query rows over all keys (tcgen05, no split);
+            // otherwise the split-KV kernel that spreads one request over the whole GPU.
+            if (h->attn_t5 && h->attn_t5_min_batch > 0 && B >= h->attn_t5_min_batch)
+                return launch_attn_t5(h, l, B, C, st);
             return attn_tc_supported(h) ? launch_attn_tc(h, l, B, C, st)
                                         : launch_op_simt(h, 3, l, step, B, C, st);
         case 4: {

@@ -20,6 +20,12 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int layer, int step, int batch, i
 bool attn_tc_supported(const jpi_handle* h);
 jpi_status attn_tc_prepare(jpi_handle* h);
 jpi_status launch_attn_tc(jpi_handle* h, int layer, int batch, int chunk, cudaStream_t st);
+// Tensor-core attention without key splits for batched launches (attn_t5.cu).
+bool attn_t5_supported(const jpi_handle* h);
+jpi_status attn_t5_prepare(jpi_handle* h);
+jpi_status launch_attn_t5(jpi_handle* h, int layer, int batch, int chunk, cudaStream_t st);
+// 2D bf16 tensor map over [rows][cols] row-major, 128-byte swizzle, box {64 cols, box_rows}.
+jpi_status tc_make_tmap(const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows, CUtensorMap* map);
 // Frees what tc_prepare created outside the handle's allocation list.
 void tc_release(jpi_handle* h);
 
