@@ -9,9 +9,11 @@
 // (row = i * H + head). The state row (i = 0) sees the prefix and itself only.
 //
 // Grid: (32-row query blocks, key splits, requests). The key splits of one query block form a
-// thread-block cluster. Inside a CTA, warp w takes query rows 16 (w mod 2) .. + 15 and key half
-// w / 2 of every 64-key block (staged in shared memory with cp.async), with its own online
-// softmax; the two key halves of a row group are merged in shared memory, and the cluster then
+// thread-block cluster. Inside a CTA, warp w takes query rows 16 (w mod 2) .. + 15 of every key
+// block (staged in shared memory with cp.async): it computes the scores of key half w / 2, the
+// two warps of a row group exchange their block maxima and write the probabilities P (bf16) to
+// shared memory, and each then accumulates output columns half w / 2 over all keys of the block
+// (one online softmax per row group, nothing left to merge). The cluster then
 // combines the per-split (max, sum, output) triples through distributed shared memory in split
 // order, so the result does not depend on timing. Each split pushes the rows owned by every other
 // split into that split's dedicated receive buffer as soon as its own rows are final; the only
@@ -99,12 +101,11 @@ template <int D>
 __host__ __device__ constexpr int attn_row_bytes() {
     return 2 * D + 16;
 }
-// Row stride (floats) of the fp32 staging of one key half's output columns that the other key
-// half merges (D / 2 columns): 8 floats of padding put the 4 rows a half-warp writes at one column
-// (8-byte accesses) on disjoint banks.
-template <int D>
-__host__ __device__ constexpr int attn_ofp_stride() {
-    return D / 2 + 8;
+// Row stride (bytes) of the bf16 probability tile P [32][KB]: 16 bytes of padding put the 8 rows
+// of an ldmatrix phase, and the 8 rows a warp's 4-byte stores hit, on disjoint banks.
+template <int KB>
+__host__ __device__ constexpr int AT_PSTRIDE() {
+    return KB * 2 + 16;
 }
 // Shared-memory layout (bytes from the 128-aligned base): q and NBUF k/v buffers, reused after
 // the key loop for each key half's hand-over columns (fp32) and (m, l), then this split's partial
@@ -113,14 +114,15 @@ template <int D, int NBUF>
 struct AttnSmem {
     static constexpr int KB = NBUF == 2 ? AT_KEYS / 2 : AT_KEYS;   // keys per block
     static constexpr int QKV = (AT_ROWS + 2 * KB * NBUF) * D * 2;
-    static constexpr int OFP = 2 * AT_ROWS * attn_ofp_stride<D>() * 4;   // [2 halves][32][OS]
-    static constexpr int ML = OFP;                               // [2 halves][32] float2
-    static constexpr int OPART = ML + 2 * AT_ROWS * 8;           // [32][row bytes]
+    static constexpr int OPART = 0;                              // [32][row bytes], after the keys
     static constexpr int REGION_USED = OPART + AT_ROWS * attn_row_bytes<D>();
     static constexpr int REGION = QKV > REGION_USED ? QKV : REGION_USED;
     static constexpr int RECV = REGION;                          // [AT_MAX_RECV_ROWS][row bytes]
     static constexpr int COEF = RECV + AT_MAX_RECV_ROWS * attn_row_bytes<D>();   // [32][16] floats
-    static constexpr int BAR = COEF + AT_ROWS * AT_MAX_SPLITS * 4;
+    static constexpr int PB = COEF + AT_ROWS * AT_MAX_SPLITS * 4;   // [32][KB] bf16 P, padded rows
+    static constexpr int XM = PB + AT_ROWS * AT_PSTRIDE<KB>();     // [2 halves][32] block maxima
+    static constexpr int LS = XM + 2 * AT_ROWS * 4;                // [2 halves][32] l shares
+    static constexpr int BAR = LS + 2 * AT_ROWS * 4;
     static constexpr int TOTAL = BAR + 16;
 };
 
@@ -138,16 +140,16 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     uint8_t* vs = ks + KB * D * 2;
     constexpr uint32_t KV_BUF = 2 * KB * D * 2;     // bytes of one k/v buffer pair
     constexpr int ROWB = attn_row_bytes<D>();
-    constexpr int OS = attn_ofp_stride<D>();
-    float* ofp = (float*)smem;                           // [2][32][OS] columns handed over
-    float2* mls = (float2*)(smem + L::ML);               // [2][32] (m, l) of each key half
     uint8_t* opart = smem + L::OPART;                    // [32][ROWB] this split's partial rows
+    uint8_t* pbuf = smem + L::PB;                        // [32][KB] bf16 probabilities
+    float* xmax = (float*)(smem + L::XM);                // [2][32] block maxima of each key half
+    float* lsum = (float*)(smem + L::LS);                // [2][32] l of each key half
     uint8_t* recv = smem + L::RECV;                      // [(splits - 1) x rows_per][ROWB]
     float* coef = (float*)(smem + L::COEF);              // [32][AT_MAX_SPLITS]
     uint64_t* rbar = (uint64_t*)(smem + L::BAR);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int rg = warp & 1, kh = warp >> 1;             // row group, key half
+    const int rg = warp & 1, kh = warp >> 1;             // row group, key half / column half
     const int rb = blockIdx.x, b = blockIdx.z;
     const int nrows = a.S * a.H, nk = a.P + a.S;
     const int row0 = rb * AT_ROWS;
@@ -209,15 +211,20 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         nvis[hh] = (R < nrows && i == 0) ? a.P + 1 : nk;
     }
 
-    float oacc[D / 8][4];
+    // This warp's output columns: half kh of the D dimensions, for all keys of a block.
+    constexpr int NOT = D / 16;                          // n-tiles of 8 columns per half
+    float oacc[NOT][4];
 #pragma unroll
-    for (int n = 0; n < D / 8; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.f;
+    for (int n = 0; n < NOT; ++n) oacc[n][0] = oacc[n][1] = oacc[n][2] = oacc[n][3] = 0.f;
+    // Both warps of a row group share one running maximum; l is this warp's key-half share.
     float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
     constexpr int HK = KB / 2;                      // keys per half
+    const int ra = rg * 16 + g, rb2 = ra + 8;             // this thread's two rows
+    const uint32_t pb_u = ptx::smem_u32(pbuf);
 
     int buf = 0;
     for (int key0 = k_begin; key0 < k_end; key0 += KB) {
-        __syncthreads();   // every warp is done with the buffer refilled below
+        __syncthreads();   // every warp is done with the buffer refilled below (and with P)
         if (NBUF == 2) {
             if (key0 + KB < k_end) {
                 load_kv(key0 + KB, 0, KB, buf ^ 1);
@@ -234,7 +241,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         const uint32_t kbuf_u = ks_u + buf * KV_BUF, vbuf_u = vs_u + buf * KV_BUF;
         if (NBUF == 2) buf ^= 1;
 
-        // S = Q K^T for this warp's 16 rows x 32 keys.
+        // S = Q K^T for this warp's 16 rows x its key half.
         float sacc[HK / 8][4];
 #pragma unroll
         for (int n = 0; n < HK / 8; ++n) sacc[n][0] = sacc[n][1] = sacc[n][2] = sacc[n][3] = 0.f;
@@ -256,7 +263,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
                 mma16816(sacc[nt + 1], a0, a1, a2, a3, b2, b3);
             }
         }
-        // Scale to log2 units, mask, online softmax.
+        // Scale to log2 units, mask; the block maximum of each row over both key halves.
         float bmax[2] = {-INFINITY, -INFINITY};
 #pragma unroll
         for (int nt = 0; nt < HK / 8; ++nt)
@@ -268,17 +275,28 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
                 sacc[nt][e] = s;
                 bmax[hh] = fmaxf(bmax[hh], s);
             }
-        float alpha[2], mnew[2];
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
             bmax[hh] = fmaxf(bmax[hh], __shfl_xor_sync(0xffffffffu, bmax[hh], 1));
             bmax[hh] = fmaxf(bmax[hh], __shfl_xor_sync(0xffffffffu, bmax[hh], 2));
+        }
+        if (cq == 0) {
+            xmax[kh * AT_ROWS + ra] = bmax[0];
+            xmax[kh * AT_ROWS + rb2] = bmax[1];
+        }
+        ptx::named_bar_sync(1 + rg, 64);   // the two warps of this row group
+        bmax[0] = fmaxf(bmax[0], xmax[(1 - kh) * AT_ROWS + ra]);
+        bmax[1] = fmaxf(bmax[1], xmax[(1 - kh) * AT_ROWS + rb2]);
+        float alpha[2], mnew[2];
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
             mnew[hh] = fmaxf(m_run[hh], bmax[hh]);
             alpha[hh] = (mnew[hh] == -INFINITY) ? 1.f : fast_exp2(m_run[hh] - mnew[hh]);
         }
+        // P = 2^(s - m) for this warp's keys: summed into l, stored as bf16 for both warps' P V.
         float psum[2] = {0.f, 0.f};
 #pragma unroll
-        for (int nt = 0; nt < HK / 8; ++nt)
+        for (int nt = 0; nt < HK / 8; ++nt) {
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int hh = e >> 1;
@@ -286,6 +304,10 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
                 sacc[nt][e] = p;
                 psum[hh] += p;
             }
+            const uint32_t col_b = (uint32_t)(kh * HK + nt * 8 + 2 * cq) * 2;
+            *(uint32_t*)(pbuf + ra * AT_PSTRIDE<KB>() + col_b) = pack_bf16x2(sacc[nt][0], sacc[nt][1]);
+            *(uint32_t*)(pbuf + rb2 * AT_PSTRIDE<KB>() + col_b) = pack_bf16x2(sacc[nt][2], sacc[nt][3]);
+        }
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
             psum[hh] += __shfl_xor_sync(0xffffffffu, psum[hh], 1);
@@ -294,24 +316,27 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
             m_run[hh] = mnew[hh];
         }
 #pragma unroll
-        for (int n = 0; n < D / 8; ++n) {
+        for (int n = 0; n < NOT; ++n) {
             oacc[n][0] *= alpha[0];
             oacc[n][1] *= alpha[0];
             oacc[n][2] *= alpha[1];
             oacc[n][3] *= alpha[1];
         }
-        // O += P V: the S accumulators of key tiles (2j, 2j+1) are the A operand of k-step j.
+        ptx::named_bar_sync(1 + rg, 64);   // both halves of P are in shared memory
+        // O[:, half kh] += P V over all KB keys of the block.
 #pragma unroll
-        for (int j = 0; j < HK / 16; ++j) {
-            const uint32_t a0 = pack_bf16x2(sacc[2 * j][0], sacc[2 * j][1]);
-            const uint32_t a1 = pack_bf16x2(sacc[2 * j][2], sacc[2 * j][3]);
-            const uint32_t a2 = pack_bf16x2(sacc[2 * j + 1][0], sacc[2 * j + 1][1]);
-            const uint32_t a3 = pack_bf16x2(sacc[2 * j + 1][2], sacc[2 * j + 1][3]);
+        for (int j = 0; j < KB / 16; ++j) {
+            uint32_t a0, a1, a2, a3;
+            {
+                const int r = rg * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int c = j * 2 + (lane >> 4);
+                ldsm_x4(pb_u + (uint32_t)(r * AT_PSTRIDE<KB>() + c * 16), a0, a1, a2, a3);
+            }
 #pragma unroll
-            for (int dt = 0; dt < D / 8; dt += 2) {
+            for (int dt = 0; dt < NOT; dt += 2) {
                 uint32_t b0, b1, b2, b3;
-                const int r = kh * HK + j * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-                const int c = dt + (lane >> 4);
+                const int r = j * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int c = kh * NOT + dt + (lane >> 4);
                 ldsm_x4_t(vbuf_u + sw_off<D>(r, c), b0, b1, b2, b3);
                 mma16816(oacc[dt], a0, a1, a2, a3, b0, b1);
                 mma16816(oacc[dt + 1], a0, a1, a2, a3, b2, b3);
@@ -319,77 +344,27 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         }
     }
 
-    // ---- merge the two key halves of each row group (q/k/v are dead past this barrier) ----
-    // Key half kh merges output columns [kh D/2, (kh + 1) D/2): it hands the other half of its
-    // columns over in fp32, then combines its own with the ones handed to it.
-    __syncthreads();
-    const int ra = rg * 16 + g, rb2 = ra + 8;             // this thread's two rows
-    constexpr int NH = D / 16;                           // n-tiles per column half
-    float* give = ofp + (size_t)kh * AT_ROWS * OS;       // this half's hand-over rows
-    const float* take = ofp + (size_t)(1 - kh) * AT_ROWS * OS;
-    if (kh == 0) {
-#pragma unroll
-        for (int n = NH; n < 2 * NH; ++n) {
-            const int col = (n - NH) * 8 + 2 * cq;
-            *(float2*)(give + ra * OS + col) = make_float2(oacc[n][0], oacc[n][1]);
-            *(float2*)(give + rb2 * OS + col) = make_float2(oacc[n][2], oacc[n][3]);
-        }
-    } else {
-#pragma unroll
-        for (int n = 0; n < NH; ++n) {
-            const int col = n * 8 + 2 * cq;
-            *(float2*)(give + ra * OS + col) = make_float2(oacc[n][0], oacc[n][1]);
-            *(float2*)(give + rb2 * OS + col) = make_float2(oacc[n][2], oacc[n][3]);
-        }
-    }
+    // ---- this split's partial rows (q/k/v are dead past this barrier) ----
     if (cq == 0) {
-        mls[kh * AT_ROWS + ra] = make_float2(m_run[0], l_run[0]);
-        mls[kh * AT_ROWS + rb2] = make_float2(m_run[1], l_run[1]);
+        lsum[kh * AT_ROWS + ra] = l_run[0];
+        lsum[kh * AT_ROWS + rb2] = l_run[1];
     }
     __syncthreads();
     {
-        // Partial rows of this split: O unnormalised in fp16 (a value beyond the fp16 range
-        // raises a device error), then m and l in fp32. o = o_half0 w0 + o_half1 w1.
-        float w0[2], w1[2];
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            const int r = hh ? rb2 : ra;
-            const float2 h0 = mls[r], h1 = mls[AT_ROWS + r];
-            const float m = fmaxf(h0.x, h1.x);
-            w0[hh] = (h0.x == -INFINITY) ? 0.f : fast_exp2(h0.x - m);
-            w1[hh] = (h1.x == -INFINITY) ? 0.f : fast_exp2(h1.x - m);
-            const float l = __fmaf_rn(h1.y, w1[hh], __fmul_rn(h0.y, w0[hh]));
-            if (kh == 0 && cq == 0) *(float2*)(opart + r * ROWB + 2 * D) = make_float2(m, l);
+        // O unnormalised in fp16 (a value beyond the fp16 range raises a device error), then
+        // m and l in fp32; each warp writes its half of the columns.
+        if (kh == 0 && cq == 0) {
+            *(float2*)(opart + ra * ROWB + 2 * D) = make_float2(m_run[0], lsum[ra] + lsum[AT_ROWS + ra]);
+            *(float2*)(opart + rb2 * ROWB + 2 * D) = make_float2(m_run[1], lsum[rb2] + lsum[AT_ROWS + rb2]);
         }
         bool range_ok = true;
-        auto merge = [&](int n, float2 t0, float2 t1, bool own_first) {
-            // own_first: this warp is key half 0 (its values carry w0).
-            const int col = n * 8 + 2 * cq;
-            const float a0 = own_first ? oacc[n][0] : t0.x, a1 = own_first ? oacc[n][1] : t0.y;
-            const float a2 = own_first ? oacc[n][2] : t1.x, a3 = own_first ? oacc[n][3] : t1.y;
-            const float b0 = own_first ? t0.x : oacc[n][0], b1 = own_first ? t0.y : oacc[n][1];
-            const float b2 = own_first ? t1.x : oacc[n][2], b3 = own_first ? t1.y : oacc[n][3];
-            const float v0 = __fmaf_rn(b0, w1[0], __fmul_rn(a0, w0[0]));
-            const float v1 = __fmaf_rn(b1, w1[0], __fmul_rn(a1, w0[0]));
-            const float v2 = __fmaf_rn(b2, w1[1], __fmul_rn(a2, w0[1]));
-            const float v3 = __fmaf_rn(b3, w1[1], __fmul_rn(a3, w0[1]));
-            range_ok &= fabsf(v0) <= 65000.f && fabsf(v1) <= 65000.f && fabsf(v2) <= 65000.f &&
-                        fabsf(v3) <= 65000.f;
-            *(__half2*)(opart + ra * ROWB + col * 2) = __floats2half2_rn(v0, v1);
-            *(__half2*)(opart + rb2 * ROWB + col * 2) = __floats2half2_rn(v2, v3);
-        };
-        if (kh == 0) {
 #pragma unroll
-            for (int n = 0; n < NH; ++n) {
-                const int c = n * 8 + 2 * cq;
-                merge(n, *(const float2*)(take + ra * OS + c), *(const float2*)(take + rb2 * OS + c), true);
-            }
-        } else {
-#pragma unroll
-            for (int n = NH; n < 2 * NH; ++n) {
-                const int c = (n - NH) * 8 + 2 * cq;
-                merge(n, *(const float2*)(take + ra * OS + c), *(const float2*)(take + rb2 * OS + c), false);
-            }
+        for (int n = 0; n < NOT; ++n) {
+            const int col = kh * (D / 2) + n * 8 + 2 * cq;
+            range_ok &= fabsf(oacc[n][0]) <= 65000.f && fabsf(oacc[n][1]) <= 65000.f &&
+                        fabsf(oacc[n][2]) <= 65000.f && fabsf(oacc[n][3]) <= 65000.f;
+            *(__half2*)(opart + ra * ROWB + col * 2) = __floats2half2_rn(oacc[n][0], oacc[n][1]);
+            *(__half2*)(opart + rb2 * ROWB + col * 2) = __floats2half2_rn(oacc[n][2], oacc[n][3]);
         }
         if (!range_ok) atomicCAS(a.err, 0, (int)DEV_FP16_RANGE);
     }
