@@ -159,7 +159,7 @@ struct jpi_handle {
     // Tensor-core path: one plan per projection (QKV, O, gate/up, down) and tensor maps
     // (4 per layer, same order).
     jpi::GemmPlan plans[4];
-    int big_min_tokens = 512;   // launches with at least this many tokens use the large-M GEMMs
+    int big_min_tokens[4] = {512, 512, 128, 512};   // per projection kind: from this many tokens the large-M GEMM
     int attn_t5_min_batch = 4;  // batches of at least this many requests use the unsplit attention
     bool attn_t5 = false;       // its tensor maps and attributes are ready
     CUtensorMap amaps[3];       // attention operands: q, prefix/suffix K, V (all layers)

@@ -406,9 +406,13 @@ jpi_status tc_prepare(jpi_handle* h) {
     auto big_kernels = {k_tc_gemm_big<G_QKV>, k_tc_gemm_big<G_O>, k_tc_gemm_big<G_GU>, k_tc_gemm_big<G_DOWN>};
     for (auto k : big_kernels)
         JPI_CUDA_TRY(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes()));
-    // Launches with at least this many tokens use the large-M kernels (full K per CTA).
+    // Launches with at least this many tokens use the large-M kernels (full K per CTA). The
+    // gate/up projection (64 weight tiles at pi0.5 sizes) fills the GPU with them from 128 tokens;
+    // the narrower ones (8-20 weight tiles) keep the K-split kernel up to 512 tokens (measured).
+    // JPI_BIG_GEMM_MIN_TOKENS sets one threshold for all four.
     const char* big_env = std::getenv("JPI_BIG_GEMM_MIN_TOKENS");
-    h->big_min_tokens = big_env ? std::atoi(big_env) : 512;
+    if (big_env)
+        for (int k = 0; k < 4; ++k) h->big_min_tokens[k] = std::atoi(big_env);
     const int rows[4] = {h->QKV, h->W, 2 * h->F, h->W};
     const int ks[4] = {h->W, h->HD, h->W, h->F};
     // The K split (and so the summation order) is chosen once per projection, for every batch
@@ -472,12 +476,14 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
     const jpi::GemmPlan* plans = h->plans;
     const int Mt = B * (C + 1);
     // Batched launches with many tokens: one CTA per (weight tile, 128-row operand tile) over
-    // the whole K range. Residual kinds then leave one sum-of-squares slot per weight tile.
-    const bool big = h->big_min_tokens > 0 && Mt >= h->big_min_tokens;
+    // the whole K range. Residual kinds then leave one sum-of-squares slot per weight tile, and
+    // the norm-fed kind after them reads as many slots as its producer left.
+    auto big = [&](int kind) { return h->big_min_tokens[kind] > 0 && Mt >= h->big_min_tokens[kind]; };
+    auto slots_left = [&](int kind) { return big(kind) ? plans[kind].ntiles : plans[kind].ntiles * plans[kind].splits; };
     auto run = [&](auto kind_tag, const GemmPlan& pl, const CUtensorMap& wm, const CUtensorMap& xm,
                    const GemmArgs& a) -> jpi_status {
         constexpr int KIND = decltype(kind_tag)::value;
-        return big ? launch_gemm_big<KIND>(h, pl, wm, xm, a, st) : launch_gemm<KIND>(h, pl, wm, xm, a, st);
+        return big(KIND) ? launch_gemm_big<KIND>(h, pl, wm, xm, a, st) : launch_gemm<KIND>(h, pl, wm, xm, a, st);
     };
     using KQ = std::integral_constant<int, G_QKV>;
     using KO = std::integral_constant<int, G_O>;
@@ -489,7 +495,7 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
             GemmArgs a = base_args(h, B, C, pl);
             // Sums of squares left by the embedding (one per 128 features) or the previous
             // layer's down projection (one per CTA).
-            if (l > 0) a.nslot = big ? plans[G_DOWN].ntiles : plans[G_DOWN].ntiles * plans[G_DOWN].splits;
+            if (l > 0) a.nslot = slots_left(G_DOWN);
             a.q = (__nv_bfloat16*)h->q;
             a.kst = (__nv_bfloat16*)h->kv_k + kv_layer;
             a.vst = (__nv_bfloat16*)h->kv_v + kv_layer;
@@ -517,7 +523,7 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
         case 5: {
             const GemmPlan& pl = plans[G_GU];
             GemmArgs a = base_args(h, B, C, pl);
-            a.nslot = big ? plans[G_O].ntiles : plans[G_O].ntiles * plans[G_O].splits;   // left by O
+            a.nslot = slots_left(G_O);   // left by O
             a.z = (__nv_bfloat16*)h->z;
             return run(KG{}, pl, h->tmaps[4 * l + G_GU], h->xmaps[0], a);
         }
