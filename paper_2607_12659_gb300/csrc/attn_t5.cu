@@ -135,6 +135,7 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                 load_kv(pre, pre);
                 ++pre;
             }
+            ptx::prefetch_tmap(&qmap);
             ptx::grid_dep_wait();
             ptx::mbar_expect_tx(qfull, (uint32_t)L::QBYTES);
             for (int db = 0; db < NDB; ++db)

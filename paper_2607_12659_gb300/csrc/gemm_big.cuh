@@ -75,6 +75,7 @@ __global__ void __launch_bounds__(BIG_THREADS, 2) k_tc_gemm_big(const __grid_con
                 ptx::mbar_expect_tx(&full[s], (uint32_t)BIG_STAGE_BYTES);
                 ptx::tma_load_2d(stages + s * BIG_STAGE_BYTES, &wmap, &full[s], 0, (tile * nkb + kb) * TILE_ROWS, pol);
             };
+            ptx::prefetch_tmap(&xmap);
             auto load_x = [&](int kb, int s) {
                 uint8_t* xs = stages + s * BIG_STAGE_BYTES + TILE_BYTES;
                 ptx::tma_load_2d(xs, &xmap, &full[s], kb * KBLK, xt * BIG_NT, pol);

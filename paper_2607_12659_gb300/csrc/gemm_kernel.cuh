@@ -77,6 +77,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
         for (int j = 0; j < a.kpb; ++j)
             ptx::tma_load_2d(wsm + j * TILE_BYTES, &wmap, &bars[0], 0,
                              (tile * a.nkb + kb0 + j) * TILE_ROWS, pol);
+        ptx::prefetch_tmap(&xmap);   // the operand copy right after the dependency wait
     }
     // Epilogue inputs from global memory that do not depend on the product (first item of this
     // thread only). For the first token tile they are read before the dependency wait: the rotary

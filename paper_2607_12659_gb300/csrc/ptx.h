@@ -67,6 +67,11 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_
         "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
         : "memory");
 }
+// Brings a tensor map (a __grid_constant__ kernel parameter) into the descriptor cache ahead of
+// its first bulk tensor copy.
+__device__ __forceinline__ void prefetch_tmap(const void* tmap) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
+}
 // Generic-proxy writes to shared memory become visible to the async proxy (tensor cores).
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
