@@ -385,14 +385,15 @@ def our_arm(args):
 
 
 def profile_forward(args):
-    """Small case for kernel captures: the workload's expert, two eager expert passes."""
+    """Small case for kernel captures: the workload's expert, eager expert passes (batch and
+    prefix as given, else the workload's)."""
     import torch
     from paper_2607_12659_gb300 import build, jpi
     from synth import PI05, make_requests, make_weights
     build.build()
     jpi.load()
     torch.cuda.set_device(0)
-    B, P, C = WORKLOAD["batch"], WORKLOAD["prefix"], WORKLOAD["chunk"]
+    B, P, C = args.batch or WORKLOAD["batch"], args.prefix or WORKLOAD["prefix"], WORKLOAD["chunk"]
     ex = jpi.Expert(PI05, make_weights(PI05, 2000), max_batch=B, max_prefix=P, max_chunk=C,
                     max_steps=WORKLOAD["steps"])
     r = make_requests(PI05, 2001, B, P, C)

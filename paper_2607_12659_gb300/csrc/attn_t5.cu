@@ -5,12 +5,18 @@
 // is shared by all heads, so one request is a dense [S*H] x [P+S] problem (rows token-major,
 // row = i * H + head; the state row i = 0 sees the prefix and itself only).
 //
-// One CTA = 128 query rows of one request over all of its keys, in blocks of 64 keys:
-//   warp 0  one thread: bulk tensor copies of the query tile once, then (K, V) blocks through a
-//           two-stage ring (prefix blocks may be fetched before the grid-dependency wait);
+// One CTA = 128 query rows of one request over all of its keys, in blocks of 64 keys (two TMEM
+// score buffers and two shared-memory P buffers, so block i+1's softmax overlaps block i's P V):
+//   warp 0  one thread: bulk tensor copies of the query tile once, then K and V blocks through
+//           two-slot rings of their own (K of block i+2 as soon as S_i is done, V of block i+2
+//           once P_i V_i is done; prefix blocks may be fetched before the grid-dependency wait). The
+//           row blocks of one request form a cluster of up to 4 CTAs that share each stage: every
+//           CTA copies a quarter of the stage's boxes to all of them (multicast), and a stage is
+//           refilled once every CTA's P V has released it;
 //   warp 1  one thread: S_i = Q K_i^T (M = 128, N = 64, K = D) into one of two TMEM score
-//           buffers, then O += P_i V_i (M = 128, N = D, K = 64) into the TMEM output with V read
-//           as an MN-major operand straight from its bulk copy;
+//           buffers, and O += P_i V_i (M = 128, N = D, K = 64) into the TMEM output with V read
+//           as an MN-major operand straight from its bulk copy; order S_0, S_1, then P_i V_i as
+//           soon as P_i is written followed by S_{i+2}, so P V never waits for a copy;
 //   warps 2-5  one query row per thread (its TMEM lane): scale, mask, block maximum, softmax
 //           probabilities P_i written to shared memory (bf16, 128-byte swizzled K-major rows).
 //           The running maximum is only moved, and O rescaled in TMEM, when a block's maximum
@@ -36,6 +42,7 @@ constexpr float T5_RESCALE = 8.f;   // log2 units
 
 struct T5Args {
     int S, H, P, kv_rows, maxB, layer;
+    int cx;             // CTAs per cluster along the row blocks of one request (1, 2 or 4)
     float scale_log2;   // log2(e) / sqrt(D)
     __nv_bfloat16* o;   // [Mt][H][D]
     int* err;
@@ -45,11 +52,12 @@ template <int D>
 struct T5Smem {
     static constexpr int QBYTES = T5_ROWS * D * 2;        // D/64 blocks of [128 rows][128 B]
     static constexpr int KVBYTES = T5_KEYS * D * 2;       // D/64 blocks of [64 rows][128 B]
-    static constexpr int STAGE = 2 * KVBYTES;             // K then V
+    static constexpr int STAGE = 2 * KVBYTES;             // ring slot s: K then V
     static constexpr int ST_OFF = QBYTES;
-    static constexpr int P_OFF = ST_OFF + T5_STAGES * STAGE;
-    static constexpr int BAR_OFF = P_OFF + T5_ROWS * T5_KEYS * 2;
-    static constexpr int TOTAL = BAR_OFF + 128;
+    static constexpr int PBYTES = T5_ROWS * T5_KEYS * 2;      // one P buffer [128 rows][128 B]
+    static constexpr int P_OFF = ST_OFF + T5_STAGES * STAGE;   // two P buffers
+    static constexpr int BAR_OFF = P_OFF + 2 * PBYTES;
+    static constexpr int TOTAL = BAR_OFF + 256;
     static constexpr int TMEM_COLS = D == 256 ? 512 : 256;   // 2 score buffers of 64 + O (D)
 };
 
@@ -81,11 +89,15 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     uint64_t* bars = (uint64_t*)(smem + L::BAR_OFF);
     uint64_t* qfull = bars;                       // 1
     uint64_t* sfull = bars + 1;                   // 2: score buffer b ready
-    uint64_t* pfull = bars + 3;                   // 1: P written by the 128 softmax threads
-    uint64_t* odone = bars + 4;                   // 1: P V of the block done
-    uint64_t* stfull = bars + 5;                  // T5_STAGES
-    uint64_t* stempty = stfull + T5_STAGES;       // T5_STAGES
-    uint32_t* tmem_slot = (uint32_t*)(stempty + T5_STAGES);
+    uint64_t* pfull = bars + 3;                   // 2: P buffer b written by the 128 softmax threads
+    uint64_t* odone = bars + 5;                   // 2: P V of the block in P buffer b done
+    // K and V have their own rings (slot i mod 2), so K of block i+2 is fetched as soon as
+    // S_i is done and V of block i+2 once P_i V_i is done.
+    uint64_t* kfull = bars + 7;                   // T5_STAGES
+    uint64_t* vfull = kfull + T5_STAGES;
+    uint64_t* kempty = vfull + T5_STAGES;
+    uint64_t* vempty = kempty + T5_STAGES;
+    uint32_t* tmem_slot = (uint32_t*)(vempty + T5_STAGES);
     int* flag = (int*)(tmem_slot + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -93,6 +105,11 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     const int nrows = a.S * a.H, nk = a.P + a.S;
     const int row0 = rb * T5_ROWS;
     const int nb = (nk + T5_KEYS - 1) / T5_KEYS;
+    // The row blocks of one request read the same keys and values: a cluster of cx of them
+    // shares every (K, V) stage, each CTA copying 1/cx of its boxes to all of them.
+    const int cx = a.cx;
+    const int crank = cx > 1 ? (int)ptx::cluster_rank() : 0;
+    const uint16_t cmask = (uint16_t)((1u << cx) - 1u);
 
     if (warp == 1) {
         ptx::tmem_alloc(tmem_slot, L::TMEM_COLS);
@@ -102,11 +119,15 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
         ptx::mbar_init(qfull, 1);
         ptx::mbar_init(&sfull[0], 1);
         ptx::mbar_init(&sfull[1], 1);
-        ptx::mbar_init(pfull, 128);
-        ptx::mbar_init(odone, 1);
+        for (int b2 = 0; b2 < 2; ++b2) {
+            ptx::mbar_init(&pfull[b2], 128);
+            ptx::mbar_init(&odone[b2], 1);
+        }
         for (int s = 0; s < T5_STAGES; ++s) {
-            ptx::mbar_init(&stfull[s], 1);
-            ptx::mbar_init(&stempty[s], 1);
+            ptx::mbar_init(&kfull[s], 1);
+            ptx::mbar_init(&vfull[s], 1);
+            ptx::mbar_init(&kempty[s], cx);   // released by the MMA thread of every CTA in the cluster
+            ptx::mbar_init(&vempty[s], cx);
         }
         ptx::fence_mbar_init();
         *flag = 0;
@@ -115,50 +136,79 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // Every CTA's barriers are initialised before any copy or release addressed to it is issued.
+    if (cx > 1) {
+        ptx::cluster_arrive_relaxed();
+        ptx::cluster_wait();
+    }
 
     if (warp == 0) {
         if (lane == 0) {
             const uint64_t pol = ptx::l2_policy_evict_first();
             const int kv0 = (a.layer * a.maxB + b) * a.kv_rows;
-            auto load_kv = [&](int i, int s) {
-                uint8_t* st = stages + s * L::STAGE;
-                ptx::mbar_expect_tx(&stfull[s], (uint32_t)L::STAGE);
-                for (int db = 0; db < NDB; ++db) {
-                    ptx::tma_load_2d(st + db * (T5_KEYS * 128), &kmap, &stfull[s], db * 64, kv0 + i * T5_KEYS, pol);
-                    ptx::tma_load_2d(st + L::KVBYTES + db * (T5_KEYS * 128), &vmap, &stfull[s], db * 64,
-                                     kv0 + i * T5_KEYS, pol);
+            // One half-stage (K or V of block i, ring slot i mod 2): NDB column boxes; this CTA
+            // copies boxes crank, crank + cx, ... to every CTA of the cluster and expects them all.
+            auto load_half = [&](bool is_v, int i) {
+                const int sl = i % T5_STAGES;
+                uint64_t* bar = is_v ? &vfull[sl] : &kfull[sl];
+                uint8_t* base = stages + sl * L::STAGE + (is_v ? L::KVBYTES : 0);
+                const CUtensorMap* map = is_v ? &vmap : &kmap;
+                ptx::mbar_expect_tx(bar, (uint32_t)L::KVBYTES);
+                for (int db = crank; db < NDB; db += cx) {
+                    if (cx > 1)
+                        ptx::tma_load_2d_mc(base + db * (T5_KEYS * 128), map, bar, db * 64, kv0 + i * T5_KEYS, cmask, pol);
+                    else
+                        ptx::tma_load_2d(base + db * (T5_KEYS * 128), map, bar, db * 64, kv0 + i * T5_KEYS, pol);
                 }
             };
-            // Blocks made only of prefix keys were written before this graph ran.
-            int pre = 0;
-            while (pre < T5_STAGES && pre < nb && (pre + 1) * T5_KEYS <= a.P) {
-                load_kv(pre, pre);
-                ++pre;
+            // First use of both slots: blocks made only of prefix keys were written before this
+            // graph ran and are fetched before the dependency wait.
+            int first = 0;
+            while (first < T5_STAGES && first < nb && (first + 1) * T5_KEYS <= a.P) {
+                load_half(false, first);
+                load_half(true, first);
+                ++first;
             }
             ptx::prefetch_tmap(&qmap);
             ptx::grid_dep_wait();
             ptx::mbar_expect_tx(qfull, (uint32_t)L::QBYTES);
             for (int db = 0; db < NDB; ++db)
                 ptx::tma_load_2d(qs + db * (T5_ROWS * 128), &qmap, qfull, db * 64, b * nrows + row0, pol);
-            for (int i = pre; i < nb; ++i) {
-                const int s = i % T5_STAGES, n = i / T5_STAGES;
-                if (i >= T5_STAGES && !ptx::mbar_wait_bounded(&stempty[s], (n - 1) & 1, T5_WAIT_NS)) {
-                    *flag = DEV_TIMEOUT_WEIGHTS;
-                    break;
+            for (; first < T5_STAGES && first < nb; ++first) {
+                load_half(false, first);
+                load_half(true, first);
+            }
+            // Refills in the order the MMA thread frees them (S_0, S_1, P_0 V_0, S_2, P_1 V_1, ...):
+            // K of block j once S_{j-2} is done, then V of block j-1 once P_{j-3} V_{j-3} is done.
+            for (int j = T5_STAGES; j <= nb; ++j) {
+                if (j < nb) {
+                    if (!ptx::mbar_wait_bounded(&kempty[j % T5_STAGES], ((j - 2) >> 1) & 1, T5_WAIT_NS)) {
+                        *flag = DEV_TIMEOUT_WEIGHTS;
+                        break;
+                    }
+                    load_half(false, j);
                 }
-                load_kv(i, s);
+                const int jv = j - 1;
+                if (jv >= T5_STAGES && jv < nb) {
+                    if (!ptx::mbar_wait_bounded(&vempty[jv % T5_STAGES], ((jv - 2) >> 1) & 1, T5_WAIT_NS)) {
+                        *flag = DEV_TIMEOUT_WEIGHTS;
+                        break;
+                    }
+                    load_half(true, jv);
+                }
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {
             const uint32_t qb = ptx::smem_u32(qs), sb = ptx::smem_u32(stages), pb = ptx::smem_u32(ps);
             bool good = ptx::mbar_wait_bounded(qfull, 0, T5_WAIT_NS);
+            // S_i = Q K_i^T into score buffer i mod 2; K slot i mod 2 is released when it is done.
             auto issue_s = [&](int i) {
-                const int s = i % T5_STAGES;
-                if (!ptx::mbar_wait_bounded(&stfull[s], (i / T5_STAGES) & 1, T5_WAIT_NS)) good = false;
+                const int sl = i % T5_STAGES;
+                if (!ptx::mbar_wait_bounded(&kfull[sl], (i >> 1) & 1, T5_WAIT_NS)) good = false;
                 ptx::tc_fence_after();
                 if (good) {
-                    const uint32_t kb = sb + s * L::STAGE;
+                    const uint32_t kb = sb + sl * L::STAGE;
                     for (int db = 0; db < NDB; ++db)
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
@@ -168,22 +218,39 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                                           (db | kk) != 0);
                 }
                 ptx::mma_commit(&sfull[i & 1]);
+                if (i + T5_STAGES < nb) {
+                    if (cx > 1)
+                        ptx::mma_commit_mc(&kempty[sl], cmask);
+                    else
+                        ptx::mma_commit(&kempty[sl]);
+                }
             };
+            // Issue order S_0, S_1, then P_i V_i as soon as P_i is written, followed by S_{i+2}
+            // (its score buffer was read by the softmax of block i): P V never waits for a copy.
             issue_s(0);
+            if (nb > 1) issue_s(1);
             for (int i = 0; i < nb; ++i) {
-                if (i + 1 < nb) issue_s(i + 1);
-                if (!ptx::mbar_wait_bounded(pfull, i & 1, T5_WAIT_NS)) good = false;
+                const int sl = i % T5_STAGES;
+                if (!ptx::mbar_wait_bounded(&pfull[i & 1], (i >> 1) & 1, T5_WAIT_NS)) good = false;
+                if (!ptx::mbar_wait_bounded(&vfull[sl], (i >> 1) & 1, T5_WAIT_NS)) good = false;
                 ptx::tc_fence_after();
                 if (good) {
-                    const uint32_t vb = sb + (i % T5_STAGES) * L::STAGE + L::KVBYTES;
+                    const uint32_t vb = sb + sl * L::STAGE + L::KVBYTES;
+                    const uint32_t pbi = pb + (uint32_t)((i & 1) * L::PBYTES);
 #pragma unroll
                     for (int kk = 0; kk < T5_KEYS / 16; ++kk)
-                        ptx::mma_bf16(tmem + 128u, ptx::desc_sw128(pb + kk * 32),
+                        ptx::mma_bf16(tmem + 128u, ptx::desc_sw128(pbi + kk * 32),
                                       ptx::desc_sw128_mn(vb + kk * 16 * 128, T5_KEYS * 128, 1024), IDESC_PV,
                                       (i | kk) != 0);
                 }
-                if (i + T5_STAGES < nb) ptx::mma_commit(&stempty[i % T5_STAGES]);
-                ptx::mma_commit(odone);
+                if (i + T5_STAGES < nb) {
+                    if (cx > 1)
+                        ptx::mma_commit_mc(&vempty[sl], cmask);
+                    else
+                        ptx::mma_commit(&vempty[sl]);
+                }
+                ptx::mma_commit(&odone[i & 1]);
+                if (i + 2 < nb) issue_s(i + 2);
             }
             if (!good) *flag = DEV_TIMEOUT_MMA;
         }
@@ -200,38 +267,43 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
         for (int i = 0; i < nb; ++i) {
             if (!ptx::mbar_wait_bounded(&sfull[i & 1], (i >> 1) & 1, T5_WAIT_NS)) good = false;
             ptx::tc_fence_after();
-            float s[T5_KEYS];
-#pragma unroll
-            for (int c0 = 0; c0 < T5_KEYS; c0 += 16) {
-                uint32_t r[16];
-                ptx::tmem_ld_x16(lane_base + (uint32_t)(64 * (i & 1) + c0), r);
+            // The block's 64 raw scores: four loads in flight, one wait.
+            uint32_t r[4][16];
+            {
+                const uint32_t sa = lane_base + (uint32_t)(64 * (i & 1));
+                ptx::tmem_ld_x16(sa, r[0]);
+                ptx::tmem_ld_x16(sa + 16u, r[1]);
+                ptx::tmem_ld_x16(sa + 32u, r[2]);
+                ptx::tmem_ld_x16(sa + 48u, r[3]);
                 ptx::tmem_ld_wait();
-#pragma unroll
-                for (int j = 0; j < 16; ++j) s[c0 + j] = __uint_as_float(r[j]);
             }
-            const int key0 = i * T5_KEYS;
-            float mb = -INFINITY;
+            // Keys of this block the row sees: all of them except in the last block(s).
+            const int vis = nvis - i * T5_KEYS;
+            const bool full = vis >= T5_KEYS;
+            // Block maximum in log2 units (the scale is positive, so it commutes with the max);
+            // four independent chains.
+            float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-            for (int j = 0; j < T5_KEYS; ++j) {
-                s[j] = key0 + j < nvis ? s[j] * a.scale_log2 : -INFINITY;
-                mb = fmaxf(mb, s[j]);
-            }
-            // P V of the previous block is done: the P buffer is free and O is settled.
-            if (i > 0 && !ptx::mbar_wait_bounded(odone, (i - 1) & 1, T5_WAIT_NS)) good = false;
-            ptx::tc_fence_after();
+            for (int j = 0; j < 16; ++j)
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    if (full || 16 * q + j < vis) m4[q] = fmaxf(m4[q], __uint_as_float(r[q][j]));
+            const float mb = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;
             const bool move = mb > m_used + T5_RESCALE;
             const float alpha = !move ? 1.f : m_used == -INFINITY ? 0.f : ex2(m_used - mb);
             // TMEM loads and stores are warp-collective: the warp rescales together, lanes whose
-            // maximum stays put multiply by 1.
+            // maximum stays put multiply by 1. O is settled once P V of the previous block is done.
             if (__any_sync(0xffffffffu, move && i > 0 && m_used != -INFINITY)) {
+                if (!ptx::mbar_wait_bounded(&odone[(i - 1) & 1], ((i - 1) >> 1) & 1, T5_WAIT_NS)) good = false;
+                ptx::tc_fence_after();
 #pragma unroll 1
                 for (int c0 = 0; c0 < D; c0 += 16) {
-                    uint32_t r[16];
-                    ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)c0, r);
+                    uint32_t ro[16];
+                    ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)c0, ro);
                     ptx::tmem_ld_wait();
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) r[j] = __float_as_uint(__uint_as_float(r[j]) * alpha);
-                    ptx::tmem_st_x16(lane_base + 128u + (uint32_t)c0, r);
+                    for (int j = 0; j < 16; ++j) ro[j] = __float_as_uint(__uint_as_float(ro[j]) * alpha);
+                    ptx::tmem_st_x16(lane_base + 128u + (uint32_t)c0, ro);
                 }
                 ptx::tmem_st_wait();
             }
@@ -239,42 +311,65 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                 l *= alpha;
                 m_used = mb;
             }
+            // p = 2^(s * scale - m): one FMA and one exp per key; zero for hidden keys and while
+            // the row has seen no key at all. Four partial sums.
+            const bool seen = m_used != -INFINITY;
+            const float neg_m = seen ? -m_used : 0.f;
+            float l4[4] = {0.f, 0.f, 0.f, 0.f};
             uint32_t pk[T5_KEYS / 2];
 #pragma unroll
-            for (int j = 0; j < T5_KEYS; j += 2) {
-                const float p0 = s[j] == -INFINITY ? 0.f : ex2(s[j] - m_used);
-                const float p1 = s[j + 1] == -INFINITY ? 0.f : ex2(s[j + 1] - m_used);
-                l += p0 + p1;
-                pk[j / 2] = pack_bf16x2_t5(p0, p1);
-            }
+            for (int q = 0; q < 4; ++q)
+#pragma unroll
+                for (int j = 0; j < 16; j += 2) {
+                    const int k = 16 * q + j;
+                    float p0 = ex2(fmaf(__uint_as_float(r[q][j]), a.scale_log2, neg_m));
+                    float p1 = ex2(fmaf(__uint_as_float(r[q][j + 1]), a.scale_log2, neg_m));
+                    if (!full || !seen) {
+                        p0 = (seen && k < vis) ? p0 : 0.f;
+                        p1 = (seen && k + 1 < vis) ? p1 : 0.f;
+                    }
+                    l4[q] += p0 + p1;
+                    pk[k / 2] = pack_bf16x2_t5(p0, p1);
+                }
+            l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
+            // P buffer i mod 2 is free once P V of block i - 2 is done.
+            if (i >= 2 && !ptx::mbar_wait_bounded(&odone[i & 1], ((i - 2) >> 1) & 1, T5_WAIT_NS)) good = false;
+            ptx::tc_fence_after();
             // Row `row` of P: 8 chunks of 16 bytes, chunk c at position c ^ (row mod 8).
-            uint4* prow = (uint4*)(ps + row * 128);
+            uint4* prow = (uint4*)(ps + (i & 1) * L::PBYTES + row * 128);
 #pragma unroll
             for (int c = 0; c < 8; ++c)
                 prow[c ^ (row & 7)] = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
             ptx::fence_proxy_async_smem();
             ptx::tc_fence_before();
-            ptx::mbar_arrive(pfull);
+            ptx::mbar_arrive(&pfull[i & 1]);
         }
-        if (!ptx::mbar_wait_bounded(odone, (nb - 1) & 1, T5_WAIT_NS)) good = false;
+        // Every P V is done (both buffers' last commits observed, so none arrives after exit).
+        if (nb >= 2 && !ptx::mbar_wait_bounded(&odone[(nb - 2) & 1], ((nb - 2) >> 1) & 1, T5_WAIT_NS)) good = false;
+        if (!ptx::mbar_wait_bounded(&odone[(nb - 1) & 1], ((nb - 1) >> 1) & 1, T5_WAIT_NS)) good = false;
         ptx::tc_fence_after();
         ptx::grid_dep_launch();
         if (!good) *flag = DEV_TIMEOUT_MMA;
         const float inv = l > 0.f ? 1.f / l : 0.f;
         __nv_bfloat16* orow = a.o + ((size_t)b * nrows + R) * D;
 #pragma unroll 1
-        for (int c0 = 0; c0 < D; c0 += 16) {
-            uint32_t r[16];
-            ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)c0, r);
+        for (int c0 = 0; c0 < D; c0 += 32) {
+            uint32_t r[2][16];
+            ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)c0, r[0]);
+            ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)(c0 + 16), r[1]);
             ptx::tmem_ld_wait();
             if (valid && good) {
-                uint32_t w8[8];
 #pragma unroll
-                for (int j = 0; j < 8; ++j)
-                    w8[j] = pack_bf16x2_t5(__uint_as_float(r[2 * j]) * inv, __uint_as_float(r[2 * j + 1]) * inv);
-                uint4* dst = (uint4*)(orow + c0);
-                dst[0] = make_uint4(w8[0], w8[1], w8[2], w8[3]);
-                dst[1] = make_uint4(w8[4], w8[5], w8[6], w8[7]);
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t w8[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        w8[j] = pack_bf16x2_t5(__uint_as_float(r[h][2 * j]) * inv,
+                                               __uint_as_float(r[h][2 * j + 1]) * inv);
+                    uint4* dst = (uint4*)(orow + c0 + 16 * h);
+                    dst[0] = make_uint4(w8[0], w8[1], w8[2], w8[3]);
+                    dst[1] = make_uint4(w8[4], w8[5], w8[6], w8[7]);
+                }
             }
         }
     }
@@ -283,6 +378,11 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     __syncthreads();
     ptx::tc_fence_after();
     if (tid == 0 && *flag != 0) atomicCAS(a.err, 0, *flag);
+    // No CTA leaves while a peer may still address its shared memory.
+    if (cx > 1) {
+        ptx::cluster_arrive_relaxed();
+        ptx::cluster_wait();
+    }
     if (warp == 1) ptx::tmem_dealloc(tmem, L::TMEM_COLS);
 }
 
@@ -302,19 +402,30 @@ jpi_status launch_t5(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     a.kv_rows = h->kv_rows;
     a.maxB = h->maxB;
     a.layer = l;
+    const int rblocks = (a.S * a.H + T5_ROWS - 1) / T5_ROWS;
+    a.cx = rblocks % 4 == 0 ? 4 : rblocks % 2 == 0 ? 2 : 1;
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
     a.o = (__nv_bfloat16*)h->o;
     a.err = h->dev_err;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((a.S * a.H + T5_ROWS - 1) / T5_ROWS, B);
+    cfg.gridDim = dim3(rblocks, B);
     cfg.blockDim = dim3(T5_THREADS);
     cfg.dynamicSmemBytes = 1024 + T5Smem<D>::TOTAL;
     cfg.stream = st;
-    cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr.val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = &attr;
-    cfg.numAttrs = h->pdl ? 1 : 0;
+    cudaLaunchAttribute attrs[2];
+    int n = 0;
+    attrs[n].id = cudaLaunchAttributeClusterDimension;
+    attrs[n].val.clusterDim.x = a.cx;
+    attrs[n].val.clusterDim.y = 1;
+    attrs[n].val.clusterDim.z = 1;
+    ++n;
+    if (h->pdl) {
+        attrs[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attrs[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    cfg.attrs = attrs;
+    cfg.numAttrs = n;
     cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_t5<D>, h->amaps[0], h->amaps[1], h->amaps[2], a);
     if (e != cudaSuccess) {
         set_error("attention launch failed: %s", cudaGetErrorString(e));
