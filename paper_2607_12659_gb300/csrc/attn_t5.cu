@@ -9,10 +9,7 @@
 // score buffers and two shared-memory P buffers, so block i+1's softmax overlaps block i's P V):
 //   warp 0  one thread: bulk tensor copies of the query tile once, then K and V blocks through
 //           two-slot rings of their own (K of block i+2 as soon as S_i is done, V of block i+2
-//           once P_i V_i is done; prefix blocks may be fetched before the grid-dependency wait). The
-//           row blocks of one request form a cluster of up to 4 CTAs that share each stage: every
-//           CTA copies a quarter of the stage's boxes to all of them (multicast), and a stage is
-//           refilled once every CTA's P V has released it;
+//           once P_i V_i is done; prefix blocks may be fetched before the grid-dependency wait);
 //   warp 1  one thread: S_i = Q K_i^T (M = 128, N = 64, K = D) into one of two TMEM score
 //           buffers, and O += P_i V_i (M = 128, N = D, K = 64) into the TMEM output with V read
 //           as an MN-major operand straight from its bulk copy; order S_0, S_1, then P_i V_i as
@@ -42,7 +39,6 @@ constexpr float T5_RESCALE = 8.f;   // log2 units
 
 struct T5Args {
     int S, H, P, kv_rows, maxB, layer;
-    int cx;             // CTAs per cluster along the row blocks of one request (1, 2 or 4)
     float scale_log2;   // log2(e) / sqrt(D)
     __nv_bfloat16* o;   // [Mt][H][D]
     int* err;
@@ -105,11 +101,6 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     const int nrows = a.S * a.H, nk = a.P + a.S;
     const int row0 = rb * T5_ROWS;
     const int nb = (nk + T5_KEYS - 1) / T5_KEYS;
-    // The row blocks of one request read the same keys and values: a cluster of cx of them
-    // shares every (K, V) stage, each CTA copying 1/cx of its boxes to all of them.
-    const int cx = a.cx;
-    const int crank = cx > 1 ? (int)ptx::cluster_rank() : 0;
-    const uint16_t cmask = (uint16_t)((1u << cx) - 1u);
 
     if (warp == 1) {
         ptx::tmem_alloc(tmem_slot, L::TMEM_COLS);
@@ -126,8 +117,8 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
         for (int s = 0; s < T5_STAGES; ++s) {
             ptx::mbar_init(&kfull[s], 1);
             ptx::mbar_init(&vfull[s], 1);
-            ptx::mbar_init(&kempty[s], cx);   // released by the MMA thread of every CTA in the cluster
-            ptx::mbar_init(&vempty[s], cx);
+            ptx::mbar_init(&kempty[s], 1);
+            ptx::mbar_init(&vempty[s], 1);
         }
         ptx::fence_mbar_init();
         *flag = 0;
@@ -136,30 +127,20 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    // Every CTA's barriers are initialised before any copy or release addressed to it is issued.
-    if (cx > 1) {
-        ptx::cluster_arrive_relaxed();
-        ptx::cluster_wait();
-    }
 
     if (warp == 0) {
         if (lane == 0) {
             const uint64_t pol = ptx::l2_policy_evict_first();
             const int kv0 = (a.layer * a.maxB + b) * a.kv_rows;
-            // One half-stage (K or V of block i, ring slot i mod 2): NDB column boxes; this CTA
-            // copies boxes crank, crank + cx, ... to every CTA of the cluster and expects them all.
+            // One half-stage (K or V of block i, ring slot i mod 2): NDB column boxes.
             auto load_half = [&](bool is_v, int i) {
                 const int sl = i % T5_STAGES;
                 uint64_t* bar = is_v ? &vfull[sl] : &kfull[sl];
                 uint8_t* base = stages + sl * L::STAGE + (is_v ? L::KVBYTES : 0);
                 const CUtensorMap* map = is_v ? &vmap : &kmap;
                 ptx::mbar_expect_tx(bar, (uint32_t)L::KVBYTES);
-                for (int db = crank; db < NDB; db += cx) {
-                    if (cx > 1)
-                        ptx::tma_load_2d_mc(base + db * (T5_KEYS * 128), map, bar, db * 64, kv0 + i * T5_KEYS, cmask, pol);
-                    else
-                        ptx::tma_load_2d(base + db * (T5_KEYS * 128), map, bar, db * 64, kv0 + i * T5_KEYS, pol);
-                }
+                for (int db = 0; db < NDB; ++db)
+                    ptx::tma_load_2d(base + db * (T5_KEYS * 128), map, bar, db * 64, kv0 + i * T5_KEYS, pol);
             };
             // First use of both slots: blocks made only of prefix keys were written before this
             // graph ran and are fetched before the dependency wait.
@@ -218,12 +199,7 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                                           (db | kk) != 0);
                 }
                 ptx::mma_commit(&sfull[i & 1]);
-                if (i + T5_STAGES < nb) {
-                    if (cx > 1)
-                        ptx::mma_commit_mc(&kempty[sl], cmask);
-                    else
-                        ptx::mma_commit(&kempty[sl]);
-                }
+                if (i + T5_STAGES < nb) ptx::mma_commit(&kempty[sl]);
             };
             // Issue order S_0, S_1, then P_i V_i as soon as P_i is written, followed by S_{i+2}
             // (its score buffer was read by the softmax of block i): P V never waits for a copy.
@@ -243,12 +219,7 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                                       ptx::desc_sw128_mn(vb + kk * 16 * 128, T5_KEYS * 128, 1024), IDESC_PV,
                                       (i | kk) != 0);
                 }
-                if (i + T5_STAGES < nb) {
-                    if (cx > 1)
-                        ptx::mma_commit_mc(&vempty[sl], cmask);
-                    else
-                        ptx::mma_commit(&vempty[sl]);
-                }
+                if (i + T5_STAGES < nb) ptx::mma_commit(&vempty[sl]);
                 ptx::mma_commit(&odone[i & 1]);
                 if (i + 2 < nb) issue_s(i + 2);
             }
@@ -378,11 +349,6 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     __syncthreads();
     ptx::tc_fence_after();
     if (tid == 0 && *flag != 0) atomicCAS(a.err, 0, *flag);
-    // No CTA leaves while a peer may still address its shared memory.
-    if (cx > 1) {
-        ptx::cluster_arrive_relaxed();
-        ptx::cluster_wait();
-    }
     if (warp == 1) ptx::tmem_dealloc(tmem, L::TMEM_COLS);
 }
 
@@ -403,7 +369,6 @@ jpi_status launch_t5(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     a.maxB = h->maxB;
     a.layer = l;
     const int rblocks = (a.S * a.H + T5_ROWS - 1) / T5_ROWS;
-    a.cx = rblocks % 4 == 0 ? 4 : rblocks % 2 == 0 ? 2 : 1;
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
     a.o = (__nv_bfloat16*)h->o;
     a.err = h->dev_err;
@@ -412,20 +377,11 @@ jpi_status launch_t5(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     cfg.blockDim = dim3(T5_THREADS);
     cfg.dynamicSmemBytes = 1024 + T5Smem<D>::TOTAL;
     cfg.stream = st;
-    cudaLaunchAttribute attrs[2];
-    int n = 0;
-    attrs[n].id = cudaLaunchAttributeClusterDimension;
-    attrs[n].val.clusterDim.x = a.cx;
-    attrs[n].val.clusterDim.y = 1;
-    attrs[n].val.clusterDim.z = 1;
-    ++n;
-    if (h->pdl) {
-        attrs[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attrs[n].val.programmaticStreamSerializationAllowed = 1;
-        ++n;
-    }
-    cfg.attrs = attrs;
-    cfg.numAttrs = n;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = h->pdl ? 1 : 0;
     cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_t5<D>, h->amaps[0], h->amaps[1], h->amaps[2], a);
     if (e != cudaSuccess) {
         set_error("attention launch failed: %s", cudaGetErrorString(e));
