@@ -43,6 +43,7 @@ enum GemmKind { G_QKV = 0, G_O = 1, G_GU = 2, G_DOWN = 3 };
 
 struct GemmArgs {
     int Mt, K, nkb, kpb, splits;
+    int ntiles;              // weight tiles (large-M kernel: tiles walked by the persistent CTAs)
     // RMSNorm-fed projections (QKV, gate/up): W u = rinv * (W xs) + W beta, with xs = (1 + sigma) h
     // and beta packed as tiles of 63 tokens + 1 beta row by the producer of h, and rinv from the
     // per-token sums of squares it left.
@@ -287,8 +288,12 @@ template <int KIND>
 jpi_status launch_gemm_big(jpi_handle* h, const GemmPlan& pl, const CUtensorMap& wmap,
                            const CUtensorMap& xmap, const GemmArgs& a, cudaStream_t st) {
     constexpr int TT = (KIND == G_QKV || KIND == G_GU) ? 2 * XS_TOKENS : BIG_NT;
+    // Persistent: one CTA per SM (at most one per tile).
+    const int total = pl.ntiles * std::max(1, (a.Mt + TT - 1) / TT);
+    GemmArgs ab = a;
+    ab.ntiles = pl.ntiles;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(pl.ntiles, (unsigned)std::max(1, (a.Mt + TT - 1) / TT));
+    cfg.gridDim = dim3((unsigned)std::min(total, h->num_sms));
     cfg.blockDim = dim3(BIG_THREADS);
     cfg.dynamicSmemBytes = 1024 + big_smem_bytes();
     cfg.stream = st;
@@ -297,7 +302,7 @@ jpi_status launch_gemm_big(jpi_handle* h, const GemmPlan& pl, const CUtensorMap&
     attr.val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = &attr;
     cfg.numAttrs = h->pdl ? 1 : 0;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_big<KIND>, wmap, xmap, a);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_big<KIND>, wmap, xmap, ab);
     if (e != cudaSuccess) {
         set_error("tensor-core GEMM launch failed: %s", cudaGetErrorString(e));
         return JPI_ERR_CUDA;
