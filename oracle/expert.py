@@ -11,7 +11,7 @@ architecture parameters of pi series VLA models", Sec. 4.3 "System Design"):
     and values are the matching LLM layer's KV cache concatenated with those tokens;
   * 18 layers, width 1024, 8 attention heads of dimension 256;
   * flow matching refines noise into an action chunk over a fixed number of steps (10).
-Everything else is a reading, numbered R1..R14 where it is used below:
+Everything else is a reading, numbered R1..R15 where it is used below:
   R1  time runs t_k = k/N, k = 0..N-1, with step delta = 1/N and x_{k+1} = x_k + delta * v.
   R2  sinusoidal time embedding, half sin / half cos, periods geometric from t_min_period to
       t_max_period.
@@ -28,6 +28,12 @@ Everything else is a reading, numbered R1..R14 where it is used below:
   R9  velocity read from the action rows only.
   R10 requests in a batch are independent.
   R13 the Gemma projections (q, k, v, o, gate, up, down) carry no bias.
+  R15 correction items (Sec. 3 "Foresight-Aligned Asynchronous Correction", App. B): the T'
+      predicted compressed VLM states (width d_AE, the expert's width) given to the action
+      expert enter it as context tokens right after the state token, taken as the residual
+      stream's input row unchanged (no projection, d_AE = width). The state and context rows
+      see the prefix and each other, action rows see every key, and the velocity is read from
+      the action rows. With T' = 0 this is the plain expert.
 """
 
 from __future__ import annotations
@@ -80,10 +86,11 @@ def rope(x: np.ndarray, positions: np.ndarray, base: float) -> np.ndarray:
     return np.concatenate([a * cos - b * sin, b * cos + a * sin], axis=-1)
 
 
-def suffix_mask(prefix_len: int, suffix_len: int) -> np.ndarray:
-    """R7: visible[i][n] for suffix row i (0 = state, 1.. = actions) and key n in [prefix; suffix]."""
+def suffix_mask(prefix_len: int, suffix_len: int, n_ctx: int = 1) -> np.ndarray:
+    """R7, R15: visible[i][n] for suffix row i and key n in [prefix; suffix]. Rows 0..n_ctx-1
+    (the state token and the context tokens) see the prefix and each other; action rows see all."""
     vis = np.ones((suffix_len, prefix_len + suffix_len), dtype=bool)
-    vis[0, prefix_len + 1:] = False
+    vis[:n_ctx, prefix_len + n_ctx:] = False
     return vis
 
 
@@ -115,21 +122,27 @@ def layer_mods(c: np.ndarray, w: dict, layer: int, W: int):
 
 
 def expert_forward(x: np.ndarray, s: np.ndarray, t: float, prefix_k: np.ndarray,
-                   prefix_v: np.ndarray, w: dict, cfg, return_hidden: bool = False):
+                   prefix_v: np.ndarray, w: dict, cfg, return_hidden: bool = False,
+                   corr: np.ndarray | None = None):
     """Velocity v [C][A] of one request at flow time t (App. A, one DiT pass).
 
-    x [C][A] noisy actions, s [S_d] state, prefix_k / prefix_v [L][P][D] the per-layer LLM KV.
+    x [C][A] noisy actions, s [S_d] state, prefix_k / prefix_v [L][P][D] the per-layer LLM KV,
+    corr [T'][W] the correction items (R15; None or T' = 0: none).
     With return_hidden, also returns the residual stream h [S][W] after the last layer.
     """
     W, H, D = cfg.width, cfg.n_heads, cfg.head_dim
     L, P, C = cfg.n_layers, prefix_k.shape[1], x.shape[0]
-    S = C + 1
+    T = 0 if corr is None else corr.shape[0]
+    n_ctx = 1 + T
+    S = C + n_ctx
     c = time_conditioning(t, w, cfg)
-    # R4: row 0 is the state token, rows 1..C the action tokens.
+    # R4, R15: row 0 is the state token, rows 1..T' the correction items, then the C action tokens.
     h = np.empty((S, W), dtype=F64)
     h[0] = w["state_in_w"] @ s + w["state_in_b"]
-    h[1:] = x @ w["action_in_w"].T + w["action_in_b"]
-    visible = suffix_mask(P, S)
+    if T:
+        h[1:n_ctx] = corr
+    h[n_ctx:] = x @ w["action_in_w"].T + w["action_in_b"]
+    visible = suffix_mask(P, S, n_ctx)
     pos = P + np.arange(S)
     for l in range(L):
         sa, ba, ga, sm, bm, gm = layer_mods(c, w, l, W)
@@ -148,7 +161,7 @@ def expert_forward(x: np.ndarray, s: np.ndarray, t: float, prefix_k: np.ndarray,
         h = h + gm * (z @ w["w_down"][l].T)
     fm = w["final_mod_w"] @ c + w["final_mod_b"]
     u = rms_modulate(h, fm[:W], fm[W:], cfg.rms_eps)
-    vel = u[1:] @ w["action_out_w"].T + w["action_out_b"]          # R9
+    vel = u[n_ctx:] @ w["action_out_w"].T + w["action_out_b"]      # R9
     return (vel, h) if return_hidden else vel
 
 
@@ -158,12 +171,12 @@ def flow_times(num_steps: int) -> np.ndarray:
 
 
 def denoise(noise: np.ndarray, s: np.ndarray, num_steps: int, prefix_k: np.ndarray,
-            prefix_v: np.ndarray, w: dict, cfg) -> np.ndarray:
+            prefix_v: np.ndarray, w: dict, cfg, corr: np.ndarray | None = None) -> np.ndarray:
     """Flow-matching denoise of one request: N Euler steps x <- x + delta v (R1, App. A)."""
     delta = 1.0 / num_steps
     x = noise.astype(F64)
     for t in flow_times(num_steps):
-        x = x + delta * expert_forward(x, s, t, prefix_k, prefix_v, w, cfg)
+        x = x + delta * expert_forward(x, s, t, prefix_k, prefix_v, w, cfg, corr=corr)
     return x
 
 
@@ -180,25 +193,27 @@ def to_f64(w: dict) -> dict:
 
 
 def denoise_batch(noise: np.ndarray, state: np.ndarray, num_steps: int, prefix_k: np.ndarray,
-                  prefix_v: np.ndarray, w: dict, cfg) -> np.ndarray:
-    """R10: each request b runs independently. prefix_k/v [L][B][P][D] -> actions [B][C][A]."""
+                  prefix_v: np.ndarray, w: dict, cfg, corr: np.ndarray | None = None) -> np.ndarray:
+    """R10: each request b runs independently. prefix_k/v [L][B][P][D], corr [B][T'][W] or
+    None -> actions [B][C][A]."""
     w64 = to_f64(w)
     return np.stack([
         denoise(noise[b], state[b].astype(F64), num_steps,
-                prefix_k[:, b].astype(F64), prefix_v[:, b].astype(F64), w64, cfg)
+                prefix_k[:, b].astype(F64), prefix_v[:, b].astype(F64), w64, cfg,
+                corr=None if corr is None else corr[b].astype(F64))
         for b in range(noise.shape[0])
     ])
 
 
 def forward_batch(x: np.ndarray, state: np.ndarray, t: float, prefix_k: np.ndarray,
-                  prefix_v: np.ndarray, w: dict, cfg):
+                  prefix_v: np.ndarray, w: dict, cfg, corr: np.ndarray | None = None):
     """One expert pass per request: returns (v [B][C][A], h [B][S][W])."""
     w64 = to_f64(w)
     vs, hs = [], []
     for b in range(x.shape[0]):
         v, h = expert_forward(x[b].astype(F64), state[b].astype(F64), t,
                               prefix_k[:, b].astype(F64), prefix_v[:, b].astype(F64), w64, cfg,
-                              return_hidden=True)
+                              return_hidden=True, corr=None if corr is None else corr[b].astype(F64))
         vs.append(v)
         hs.append(h)
     return np.stack(vs), np.stack(hs)

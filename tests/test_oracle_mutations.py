@@ -19,7 +19,10 @@ SRC = os.path.join(os.path.dirname(os.path.dirname(__file__)), "oracle", "expert
 MUTATIONS = [
     ("r * (1.0 + sigma) + beta", "r * sigma + beta"),
     ("/ np.sqrt(F64(D))", ""),
-    ("vis[0, prefix_len + 1:] = False", "vis[0, prefix_len:] = False"),
+    ("vis[:n_ctx, prefix_len + n_ctx:] = False", "vis[:n_ctx, prefix_len:] = False"),
+    ("vis[:n_ctx, prefix_len + n_ctx:] = False", "vis[:1, prefix_len + 1:] = False"),
+    ("        h[1:n_ctx] = corr", "        h[1:n_ctx] = 0.5 * corr"),
+    ("    n_ctx = 1 + T", "    n_ctx = 1"),
     ("[a * cos - b * sin, b * cos + a * sin]", "[a * cos + b * sin, b * cos - a * sin]"),
     ("/ (half - 1)", "/ half"),
     ("[np.sin(theta), np.cos(theta)]", "[np.cos(theta), np.sin(theta)]"),
@@ -32,8 +35,8 @@ MUTATIONS = [
     ('w["time_mlp_out_w"] @ c1', 'w["time_mlp_out_w"].T @ c1'),
     ("pos = P + np.arange(S)", "pos = np.arange(S)"),
     ("K = np.concatenate([prefix_k[l], k], axis=0)", "K = np.concatenate([k, prefix_k[l]], axis=0)"),
-    ('h[1:] = x @ w["action_in_w"].T + w["action_in_b"]', 'h[1:] = x @ w["action_in_w"].T'),
-    ("vel = u[1:] @", "vel = u[:-1] @"),
+    ('h[n_ctx:] = x @ w["action_in_w"].T + w["action_in_b"]', 'h[n_ctx:] = x @ w["action_in_w"].T'),
+    ("vel = u[n_ctx:] @", "vel = u[:-1] @"),
     ("return ma[:W], ma[W:2 * W], ma[2 * W:], mm[:W]", "return ma[W:2 * W], ma[:W], ma[2 * W:], mm[:W]"),
     ("z = gelu_tanh(u @ w[\"w_gate\"][l].T) * (u @ w[\"w_up\"][l].T)",
      "z = gelu_tanh(u @ w[\"w_up\"][l].T) * (u @ w[\"w_gate\"][l].T)"),

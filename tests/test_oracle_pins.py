@@ -349,3 +349,78 @@ def test_velocity_of_action_j_comes_from_token_j():
         x2[j] += 0.5
         d = np.abs(oracle.expert_forward(x2, s, 0.3, *args) - v0).max(axis=1)
         assert d[j] > 1e-6 and np.all(np.delete(d, j) == 0.0)
+
+
+# ---------------------------------------------------------------- correction items (R15)
+
+def _corr(T, W, seed=31):
+    return np.random.default_rng(seed).normal(0.0, 1.0, (T, W))
+
+
+def _identity_layers(w, cfg):
+    """Both sublayer gates zero: every layer is the identity on the residual stream."""
+    W = cfg.width
+    for l in range(cfg.n_layers):
+        for mw, mb in (("attn_mod_w", "attn_mod_b"), ("mlp_mod_w", "mlp_mod_b")):
+            w[mw][l][2 * W:] = 0.0
+            w[mb][l][2 * W:] = 0.0
+    return w
+
+
+def test_no_correction_items_is_the_plain_expert():
+    w, r = micro_setup(mod_bias_std=1.0)
+    args = (r["prefix_k"][:, 0].astype(float), r["prefix_v"][:, 0].astype(float), w, MICRO)
+    x, s = r["noise"][0].astype(float), r["state"][0].astype(float)
+    v0, h0 = oracle.expert_forward(x, s, 0.4, *args, return_hidden=True)
+    v1, h1 = oracle.expert_forward(x, s, 0.4, *args, return_hidden=True,
+                                   corr=np.zeros((0, MICRO.width)))
+    np.testing.assert_array_equal(v0, v1)
+    np.testing.assert_array_equal(h0, h1)
+
+
+def test_correction_items_enter_the_residual_stream_unchanged():
+    # With identity layers the stream after the last layer is its input: state embedding,
+    # the items as given, the action embeddings; the velocity is the plain expert's.
+    w, r = micro_setup()
+    w = _identity_layers(w, MICRO)
+    args = (r["prefix_k"][:, 0].astype(float), r["prefix_v"][:, 0].astype(float), w, MICRO)
+    x, s = r["noise"][0].astype(float), r["state"][0].astype(float)
+    corr = _corr(3, MICRO.width)
+    v, h = oracle.expert_forward(x, s, 0.3, *args, return_hidden=True, corr=corr)
+    assert h.shape == (1 + 3 + x.shape[0], MICRO.width)
+    np.testing.assert_allclose(h[0], w["state_in_w"] @ s + w["state_in_b"], rtol=1e-14)
+    np.testing.assert_array_equal(h[1:4], corr)
+    np.testing.assert_allclose(h[4:], x @ w["action_in_w"].T + w["action_in_b"], rtol=1e-14)
+    np.testing.assert_allclose(v, oracle.expert_forward(x, s, 0.3, *args), rtol=1e-14)
+
+
+def test_context_rows_do_not_see_the_actions_and_the_actions_see_every_item():
+    w, r = micro_setup(mod_bias_std=1.0)
+    args = (r["prefix_k"][:, 0].astype(float), r["prefix_v"][:, 0].astype(float), w, MICRO)
+    x, s = r["noise"][0].astype(float), r["state"][0].astype(float)
+    corr = _corr(3, MICRO.width)
+    v1, h1 = oracle.expert_forward(x, s, 0.2, *args, return_hidden=True, corr=corr)
+    v2, h2 = oracle.expert_forward(x + 1.0, s, 0.2, *args, return_hidden=True, corr=corr)
+    np.testing.assert_array_equal(h1[:4], h2[:4])          # state and context rows
+    assert np.abs(h1[4:] - h2[4:]).max() > 1e-3
+    for j in range(3):
+        c2 = corr.copy()
+        c2[j] += 0.5
+        v3, h3 = oracle.expert_forward(x, s, 0.2, *args, return_hidden=True, corr=c2)
+        assert np.abs(v3 - v1).max() > 1e-6                # every item reaches the actions
+        assert np.abs(h3[0] - h1[0]).max() > 1e-6          # and the state row sees it
+
+
+def test_correction_items_are_an_unordered_set_without_rope():
+    # Without position encoding attention does not depend on key order, so permuting the
+    # items permutes their rows of the stream and leaves the velocity unchanged.
+    cfg = MICRO.with_(rope_base=0.0)
+    w, r = micro_setup(cfg=cfg, mod_bias_std=1.0)
+    args = (r["prefix_k"][:, 0].astype(float), r["prefix_v"][:, 0].astype(float), w, cfg)
+    x, s = r["noise"][0].astype(float), r["state"][0].astype(float)
+    corr = _corr(4, cfg.width)
+    perm = np.array([2, 0, 3, 1])
+    v1, h1 = oracle.expert_forward(x, s, 0.5, *args, return_hidden=True, corr=corr)
+    v2, h2 = oracle.expert_forward(x, s, 0.5, *args, return_hidden=True, corr=corr[perm])
+    np.testing.assert_allclose(v2, v1, rtol=1e-11, atol=1e-13)
+    np.testing.assert_allclose(h2[1:5], h1[1:5][perm], rtol=1e-11, atol=1e-13)
