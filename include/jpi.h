@@ -59,6 +59,9 @@ typedef enum jpi_precision {
     JPI_FP32 = 1    /* fp32 weights and activations everywhere (verification mode, CUDA cores)   */
 } jpi_precision;
 
+/* Most correction items (context tokens, see jpi_set_correction) one request may carry. */
+#define JPI_MAX_CORRECTION 8
+
 /* Model dimensions and the handle's maxima. The expert has exactly one KV head. */
 typedef struct jpi_config {
     int n_layers;     /* L, number of expert layers (18 for pi0.5)                               */
@@ -72,7 +75,8 @@ typedef struct jpi_config {
     int time_dim;     /* d_t, sinusoidal time-embedding size (even, >= 4)                         */
     int max_batch;    /* largest batch a call may use                                             */
     int max_prefix;   /* largest prefix length (tokens) of the KV store                           */
-    int max_chunk;    /* largest action chunk C; the suffix is C + 1 tokens (state + actions)     */
+    int max_chunk;    /* largest action chunk C; the suffix is 1 + T' + C tokens (state,          */
+                      /* T' <= JPI_MAX_CORRECTION correction items, actions)                      */
     int max_steps;    /* largest number of Euler steps per call                                   */
     float rope_base;  /* rotary base for the suffix positions (10000); 0 disables rotary coding   */
     float rms_eps;    /* RMSNorm epsilon (1e-6)                                                   */
@@ -148,14 +152,36 @@ JPI_API jpi_status jpi_prefix_kv_ptr(jpi_handle* h, int layer, void** k, void** 
 JPI_API jpi_status jpi_commit_prefix(jpi_handle* h, int batch, int prefix_len);
 
 /*
+ * Correction items (Sec. 3 "Foresight-Aligned Asynchronous Correction", App. B and Alg. 1):
+ * the future correction module's prediction of the compressed VLM final-layer state at
+ * t + Delta, T' tokens of width d_AE, is given to the action expert as future environment
+ * information. The expert takes them as context tokens right after the state token: their
+ * rows of the residual stream start as the items themselves (d_AE equals the expert's
+ * width, so no projection), the state and context rows see the prefix and each other, and
+ * the action rows see every key. The paper does not spell out this wiring; this is the
+ * reading the library implements.
+ *   items:     device fp32 [batch][num_items][width]
+ *   num_items: 0 (no items: the plain expert) .. JPI_MAX_CORRECTION
+ *   batch:     1 .. max_batch; later jpi_denoise / jpi_expert_forward calls with items set
+ *              must use this batch.
+ * The items are copied into the handle on `stream` (the caller may reuse its buffer once the
+ * stream reaches this point) and stay until the next call. num_items is part of the graph
+ * shape: the first denoise after a change of num_items captures a new graph; new item values
+ * with the same count reuse it. Errors: INVALID_ARG, SHAPE, CUDA.
+ */
+JPI_API jpi_status jpi_set_correction(jpi_handle* h, const float* items, int batch, int num_items,
+                                      void* stream);
+
+/*
  * Flow-matching denoise (App. A): x_0 = noise; for k = 0..N-1, t_k = k/N,
  * x_{k+1} = x_k + (1/N) * v(x_k, state, t_k; prefix KV); out_actions = x_N.
  *   state:       device fp32 [batch][S_d]
  *   noise:       device fp32 [batch][chunk][A]
  *   out_actions: device fp32 [batch][chunk][A] (may alias noise)
- *   batch must equal the batch of the last jpi_set_prefix_kv/jpi_commit_prefix;
- *   1 <= chunk <= max_chunk; 1 <= num_steps <= max_steps.
- * The first call for a (batch, chunk, num_steps, prefix_len) shape captures the whole
+ *   batch must equal the batch of the last jpi_set_prefix_kv/jpi_commit_prefix (and of the
+ *   last jpi_set_correction while items are set); 1 <= chunk <= max_chunk;
+ *   1 <= num_steps <= max_steps.
+ * The first call for a (batch, chunk, num_steps, prefix_len, num_items) shape captures the whole
  * unrolled N-step loop as one CUDA graph (Sec. 4.3: graph reuse and flow unrolling) and every
  * later call with that shape replays it. Asynchronous on `stream`; inputs are read and the
  * output written in stream order. Errors: INVALID_ARG, SHAPE, NOT_READY, CUDA.
@@ -177,7 +203,8 @@ JPI_API jpi_status jpi_denoise_host(jpi_handle* h, const float* state, const flo
  * One expert evaluation (one Euler step's velocity) at flow time t, for testing:
  *   x_t [batch][chunk][A] device fp32 in; out_v [batch][chunk][A] device fp32 out;
  *   out_h, if not NULL, receives the residual stream after the last layer,
- *   [batch][chunk + 1][W] fp32 (row 0 of each request is the state token).
+ *   [batch][1 + T' + chunk][W] fp32 (row 0 of each request is the state token, rows 1..T'
+ *   the correction items' context tokens).
  * Not captured in a graph. Asynchronous on `stream`.
  */
 JPI_API jpi_status jpi_expert_forward(jpi_handle* h, const float* state, const float* x_t,

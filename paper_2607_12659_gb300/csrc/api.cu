@@ -117,7 +117,7 @@ jpi_status check_config(const jpi_config* c) {
     if (!(c->rms_eps >= 0.f) || !(c->rope_base >= 0.f) || !(c->t_min_period > 0.f) ||
         !(c->t_max_period > 0.f))
         return fail(JPI_ERR_INVALID_ARG, "rms_eps/rope_base must be >= 0 and periods > 0");
-    const long long mt = (long long)c->max_batch * (c->max_chunk + 1);
+    const long long mt = (long long)c->max_batch * (c->max_chunk + 1 + JPI_MAX_CORRECTION);
     if (mt > (1 << 20) || (long long)c->max_prefix > (1 << 20))
         return fail(JPI_ERR_SHAPE, "maxima too large");
     return JPI_OK;
@@ -206,6 +206,7 @@ jpi_status alloc_buffers(jpi_handle* h) {
     JPI_TRY(dev_alloc(h, &h->h, Mt * W));
     JPI_TRY(dev_alloc(h, &h->x, (size_t)h->maxB * h->maxC * h->A));
     JPI_TRY(dev_alloc(h, &h->state, (size_t)h->maxB * h->Sd));
+    JPI_TRY(dev_alloc(h, &h->corr, (size_t)h->maxB * JPI_MAX_CORRECTION * h->W));
     JPI_TRY(dev_alloc(h, &h->out, (size_t)h->maxB * h->maxC * h->A));
     JPI_TRY(dev_alloc(h, &h->temb, (size_t)h->maxN * h->dt));
     JPI_TRY(dev_alloc(h, &h->c1, (size_t)h->maxN * W));
@@ -217,6 +218,11 @@ jpi_status alloc_buffers(jpi_handle* h) {
     JPI_TRY(dev_alloc(h, (char**)&h->q, Mt * h->HD * ts));
     JPI_TRY(dev_alloc(h, (char**)&h->o, Mt * h->HD * ts));
     JPI_TRY(dev_alloc(h, (char**)&h->z, Mt * h->F * ts));
+    // Operand rows past a launch's last token are read by the tiled copies: start them at zero.
+    JPI_CUDA_TRY(cudaMemset(h->act, 0, Mt * actw * ts));
+    JPI_CUDA_TRY(cudaMemset(h->q, 0, Mt * h->HD * ts));
+    JPI_CUDA_TRY(cudaMemset(h->o, 0, Mt * h->HD * ts));
+    JPI_CUDA_TRY(cudaMemset(h->z, 0, Mt * h->F * ts));
     const size_t kv = (size_t)h->L * h->maxB * h->kv_rows * h->D;
     JPI_TRY(dev_alloc(h, (char**)&h->kv_k, kv * ts));
     JPI_TRY(dev_alloc(h, (char**)&h->kv_v, kv * ts));
@@ -283,7 +289,7 @@ jpi_status enqueue_denoise(jpi_handle* h, int B, int C, int N, cudaStream_t st) 
 }
 
 jpi_status get_graph(jpi_handle* h, int B, int C, int N, cudaGraphExec_t* out) {
-    const GraphKey key{B, C, N, h->cur_prefix};
+    const GraphKey key{B, C, N, h->cur_prefix, h->n_corr};
     auto it = h->graphs.find(key);
     if (it != h->graphs.end()) {
         *out = it->second;
@@ -330,6 +336,8 @@ jpi_status check_call(jpi_handle* h, int B, int C, int N) {
     if (!h->prefix_ready) return fail(JPI_ERR_NOT_READY, "no prefix KV has been set");
     if (B != h->cur_batch)
         return fail(JPI_ERR_SHAPE, "batch %d differs from the prefix KV's batch %d", B, h->cur_batch);
+    if (h->n_corr > 0 && B != h->corr_batch)
+        return fail(JPI_ERR_SHAPE, "batch %d differs from the correction items' batch %d", B, h->corr_batch);
     return JPI_OK;
 }
 
@@ -356,7 +364,7 @@ JPI_API jpi_status jpi_expert_create(const jpi_config* cfg, const jpi_weights* w
     h->F = cfg->mlp_dim; h->A = cfg->action_dim; h->Sd = cfg->state_dim; h->dt = cfg->time_dim;
     h->HD = h->H * h->D; h->QKV = (h->H + 2) * h->D;
     h->maxB = cfg->max_batch; h->maxP = cfg->max_prefix; h->maxC = cfg->max_chunk;
-    h->maxS = cfg->max_chunk + 1; h->maxN = cfg->max_steps;
+    h->maxS = cfg->max_chunk + 1 + JPI_MAX_CORRECTION; h->maxN = cfg->max_steps;
     h->maxMt = h->maxB * h->maxS;
     h->kv_rows = h->maxP + h->maxS;
     jpi_status s = JPI_OK;
@@ -435,6 +443,23 @@ JPI_API jpi_status jpi_commit_prefix(jpi_handle* h, int batch, int prefix_len) {
     return JPI_OK;
 }
 
+JPI_API jpi_status jpi_set_correction(jpi_handle* h, const float* items, int batch, int num_items,
+                                      void* stream) {
+    clear_error();
+    if (!h) return fail(JPI_ERR_INVALID_ARG, "handle is NULL");
+    if (num_items < 0 || batch < 1) return fail(JPI_ERR_INVALID_ARG, "num_items must be >= 0 and batch >= 1");
+    if (num_items > JPI_MAX_CORRECTION || batch > h->maxB)
+        return fail(JPI_ERR_SHAPE, "num_items %d / batch %d exceed the maxima %d / %d", num_items, batch,
+                    JPI_MAX_CORRECTION, h->maxB);
+    if (num_items > 0 && !items) return fail(JPI_ERR_INVALID_ARG, "items are NULL");
+    if (num_items > 0)
+        JPI_CUDA_TRY(cudaMemcpyAsync(h->corr, items, (size_t)batch * num_items * h->W * sizeof(float),
+                                     cudaMemcpyDeviceToDevice, (cudaStream_t)stream));
+    h->n_corr = num_items;
+    h->corr_batch = batch;
+    return JPI_OK;
+}
+
 JPI_API jpi_status jpi_denoise(jpi_handle* h, const float* state, const float* noise, int batch,
                                int chunk, int num_steps, float* out_actions, void* stream) {
     clear_error();
@@ -487,7 +512,7 @@ JPI_API jpi_status jpi_expert_forward(jpi_handle* h, const float* state, const f
     JPI_TRY(launch_time_conditioning(h, 1, st));
     JPI_TRY(enqueue_step(h, 0, batch, chunk, 0.f, out_v, st));
     if (out_h)
-        JPI_CUDA_TRY(cudaMemcpyAsync(out_h, h->h, (size_t)batch * (chunk + 1) * h->W * sizeof(float),
+        JPI_CUDA_TRY(cudaMemcpyAsync(out_h, h->h, (size_t)batch * (chunk + h->n_ctx()) * h->W * sizeof(float),
                                      cudaMemcpyDeviceToDevice, st));
     return JPI_OK;
 }
@@ -512,7 +537,7 @@ JPI_API jpi_status jpi_graph_kernel_count(jpi_handle* h, int batch, int chunk, i
     if (!count) return fail(JPI_ERR_INVALID_ARG, "count is NULL");
     cudaGraphExec_t ex = nullptr;
     JPI_TRY(get_graph(h, batch, chunk, num_steps, &ex));
-    *count = h->graph_kernels[GraphKey{batch, chunk, num_steps, h->cur_prefix}];
+    *count = h->graph_kernels[GraphKey{batch, chunk, num_steps, h->cur_prefix, h->n_corr}];
     return JPI_OK;
 }
 

@@ -3,7 +3,8 @@
 // App. A of the paper: the expert's queries (state token + C action tokens, all H heads) attend
 // over the matching LLM layer's KV cache followed by the suffix's own keys/values; one KV head
 // is shared by all heads, so one request is a dense [S*H] x [P+S] problem (rows token-major,
-// row = i * H + head; the state row i = 0 sees the prefix and itself only).
+// row = i * H + head; the state row i = 0 and the correction items' context rows i < nctx see
+// the prefix and each other only).
 //
 // One CTA = 128 query rows of one request over all of its keys, in blocks of 64 keys (two TMEM
 // score buffers and two shared-memory P buffers, so block i+1's softmax overlaps block i's P V):
@@ -39,6 +40,7 @@ constexpr float T5_RESCALE = 8.f;   // log2 units
 
 struct T5Args {
     int S, H, P, kv_rows, maxB, layer;
+    int nctx;           // suffix rows 0..nctx-1 (state, context tokens) see P + nctx keys
     float scale_log2;   // log2(e) / sqrt(D)
     __nv_bfloat16* o;   // [Mt][H][D]
     int* err;
@@ -230,8 +232,8 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
         const int row = (warp & 3) * 32 + lane;
         const int R = row0 + row;
         const bool valid = R < nrows;
-        // Visible keys: the state row sees the prefix and itself; padding rows see none.
-        const int nvis = !valid ? 0 : R / a.H == 0 ? a.P + 1 : nk;
+        // Visible keys: state and context rows see the prefix and each other; padding rows none.
+        const int nvis = !valid ? 0 : R / a.H < a.nctx ? a.P + a.nctx : nk;
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         float m_used = -INFINITY, l = 0.f;
         bool good = true;
@@ -362,7 +364,8 @@ jpi_status prepare_t5(jpi_handle* h) {
 template <int D>
 jpi_status launch_t5(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     T5Args a;
-    a.S = C + 1;
+    a.S = C + h->n_ctx();
+    a.nctx = h->n_ctx();
     a.H = h->H;
     a.P = h->cur_prefix;
     a.kv_rows = h->kv_rows;

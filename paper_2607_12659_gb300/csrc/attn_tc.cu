@@ -6,7 +6,8 @@
 // layer's KV cache concatenated with the suffix tokens' own keys/values. With a single KV head
 // every query head of every suffix token attends to the same K/V rows, so one request's
 // S x H query rows form one dense [S*H][D] x [D][P+S] problem; rows are ordered token-major
-// (row = i * H + head). The state row (i = 0) sees the prefix and itself only.
+// (row = i * H + head). The state row (i = 0) and the correction items' context rows
+// (i < nctx) see the prefix and each other only.
 //
 // Grid: (32-row query blocks, key splits, requests). The key splits of one query block form a
 // thread-block cluster. Inside a CTA, warp w takes query rows 16 (w mod 2) .. + 15 of every key
@@ -92,6 +93,7 @@ struct AttnArgs {
     const __nv_bfloat16* vst;
     __nv_bfloat16* o;           // [Mt][H * D]
     int S, H, P, kv_rows, chunk, nsplit;
+    int nctx;                   // suffix rows 0..nctx-1 (state, context tokens) see P + nctx keys
     float scale_log2;           // log2(e) / sqrt(D)
     int* err;
 };
@@ -208,7 +210,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     for (int hh = 0; hh < 2; ++hh) {
         const int R = row0 + rg * 16 + g + hh * 8;
         const int i = R / a.H;
-        nvis[hh] = (R < nrows && i == 0) ? a.P + 1 : nk;
+        nvis[hh] = (R < nrows && i < a.nctx) ? a.P + a.nctx : nk;
     }
 
     // This warp's output columns: half kh of the D dimensions, for all keys of a block.
@@ -454,7 +456,7 @@ size_t attn_smem() {
 
 template <int D>
 jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
-    const int S = C + 1, nrows = S * h->H, nk = h->cur_prefix + S;
+    const int S = C + h->n_ctx(), nrows = S * h->H, nk = h->cur_prefix + S;
     const int rblocks = (nrows + AT_ROWS - 1) / AT_ROWS;
     // Enough key splits for the launch to put about two CTAs on every SM, at most 16 (one
     // cluster): 14 splits for one pi0.5-shaped request, one when many requests fill the GPU by
@@ -474,6 +476,7 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     a.vst = (const __nv_bfloat16*)h->kv_v + kv_layer;
     a.o = (__nv_bfloat16*)h->o;
     a.S = S;
+    a.nctx = h->n_ctx();
     a.H = h->H;
     a.P = h->cur_prefix;
     a.kv_rows = h->kv_rows;

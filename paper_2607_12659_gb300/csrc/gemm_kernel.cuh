@@ -217,7 +217,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
                         v0 *= rinv_s[cbase + c0 + 2 * i];
                         v1 *= rinv_s[cbase + c0 + 2 * i + 1];
                     }
-                    range_ok &= fabsf(v0) <= 65000.f && fabsf(v1) <= 65000.f;
+                    // Only live columns count: tokens of this launch (and the beta column);
+                    // columns past the last token hold products of padding rows.
+                    const int col = cbase + c0 + 2 * i, tok = (int)blockIdx.y * TT + col;
+                    if (col >= TT || tok < a.Mt) range_ok &= fabsf(v0) <= 65000.f;
+                    if (col + 1 >= TT || tok + 1 < a.Mt) range_ok &= fabsf(v1) <= 65000.f;
                     __half2 hv = __floats2half2_rn(v0, v1);
                     hp[i] = *reinterpret_cast<uint32_t*>(&hv);
                 }

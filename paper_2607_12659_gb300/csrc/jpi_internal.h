@@ -92,9 +92,9 @@ struct GemmPlan {
 };
 
 struct GraphKey {
-    int batch, chunk, steps, prefix;
+    int batch, chunk, steps, prefix, items;
     bool operator<(const GraphKey& o) const {
-        return std::tie(batch, chunk, steps, prefix) < std::tie(o.batch, o.chunk, o.steps, o.prefix);
+        return std::tie(batch, chunk, steps, prefix, items) < std::tie(o.batch, o.chunk, o.steps, o.prefix, o.items);
     }
 };
 
@@ -169,6 +169,12 @@ struct jpi_handle {
     // State.
     int cur_batch = 0, cur_prefix = 0;
     bool prefix_ready = false;
+    // Correction items (context tokens after the state token): [maxB][JPI_MAX_CORRECTION][W] fp32,
+    // n_corr of them per request for corr_batch requests. Suffix rows 0 .. n_ctx() - 1 are the
+    // state and context tokens, then the actions.
+    float* corr = nullptr;
+    int n_corr = 0, corr_batch = 0;
+    int n_ctx() const { return 1 + n_corr; }
     cudaStream_t cap_stream = nullptr;
     std::map<jpi::GraphKey, cudaGraphExec_t> graphs;
     std::map<jpi::GraphKey, int> graph_kernels;

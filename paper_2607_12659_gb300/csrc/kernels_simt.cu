@@ -183,7 +183,8 @@ __global__ void __launch_bounds__(256) k_mod_gemv(const TW* __restrict__ Wm, con
 }
 
 // ---------------------------------------------------------------------------------------------
-// Token embedding: row 0 of each request is the state token, rows 1..C the action tokens.
+// Token embedding: row 0 of each request is the state token, rows 1..nctx-1 the correction
+// items (context tokens, taken as given), then the C action tokens.
 // Block = 128 features of one token. For the tensor-core path it also writes the operand of
 // the first layer's norm-fed projection (xs = bf16((1 + sigma) * h) at row xs_row(m), and beta in
 // the last row of tile m while m < xs_tiles) and that slice's sum of squares (ss[slice][m]).
@@ -192,25 +193,30 @@ __global__ void __launch_bounds__(128) k_embed(
     const float* __restrict__ beta, float* __restrict__ ss, int ss_ld,
     const float* __restrict__ state,
     const float* __restrict__ x, const float* __restrict__ Ws, const float* __restrict__ bs,
-    const float* __restrict__ Wa, const float* __restrict__ ba, int S, int C, int W, int Sd, int A) {
+    const float* __restrict__ Wa, const float* __restrict__ ba, const float* __restrict__ corr, int nctx,
+    int S, int C, int W, int Sd, int A) {
     __shared__ float scratch[32];
     const int m = blockIdx.y;
     const int b = m / S, i = m % S;
-    const float* in;
-    const float* Wm;
-    const float* bias;
-    int K;
+    const float* in = nullptr;
+    const float* Wm = nullptr;
+    const float* bias = nullptr;
+    int K = 0;
     if (i == 0) {
         in = state + (size_t)b * Sd; Wm = Ws; bias = bs; K = Sd;
-    } else {
-        in = x + ((size_t)b * C + (i - 1)) * A; Wm = Wa; bias = ba; K = A;
+    } else if (i >= nctx) {
+        in = x + ((size_t)b * C + (i - nctx)) * A; Wm = Wa; bias = ba; K = A;
     }
     const int n = blockIdx.x * 128 + threadIdx.x;
     float v = 0.f;
     if (n < W) {
-        float acc = 0.f;
-        for (int k = 0; k < K; ++k) acc = fmaf(Wm[(size_t)n * K + k], in[k], acc);
-        v = acc + bias[n];
+        if (i > 0 && i < nctx) {
+            v = corr[((size_t)b * (nctx - 1) + (i - 1)) * W + n];
+        } else {
+            float acc = 0.f;
+            for (int k = 0; k < K; ++k) acc = fmaf(Wm[(size_t)n * K + k], in[k], acc);
+            v = acc + bias[n];
+        }
         hres[(size_t)m * W + n] = v;
         if (xs) {
             xs[(size_t)xs_row(m) * W + n] = __float2bfloat16_rn((1.f + sigma[n]) * v);
@@ -344,21 +350,22 @@ __global__ void k_qkv_post(const float* __restrict__ qkv, TQ* __restrict__ q,
 
 // ---------------------------------------------------------------------------------------------
 // Attention of one suffix token (all H heads, one warp each) over [prefix ; suffix] keys of
-// the single KV head. The state row (i = 0) sees the prefix and itself; action rows see all.
+// the single KV head. The state and context rows (i < nctx) see the prefix and each other;
+// action rows see all.
 // Online softmax over chunks of 32 keys staged in shared memory.
 constexpr int ATT_MAXD = 256;
 
 template <typename TQ, typename TKV, typename TO>
 __global__ void k_attn_simt(const TQ* __restrict__ q, const TKV* __restrict__ kst,
                             const TKV* __restrict__ vst, TO* __restrict__ o, int S, int H, int D,
-                            int P, int kv_rows, float scale) {
+                            int P, int kv_rows, int nctx, float scale) {
     extern __shared__ float sm[];
     float* qs = sm;                      // [H][D]
     float* ks = qs + H * D;              // [32][D + 1]
     float* vs = ks + 32 * (D + 1);       // [32][D]
     const int m = blockIdx.x;
     const int b = m / S, i = m % S;
-    const int nvis = (i == 0) ? P + 1 : P + S;
+    const int nvis = (i < nctx) ? P + nctx : P + S;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int idx = threadIdx.x; idx < H * D; idx += blockDim.x)
         qs[idx] = ldf(q + (size_t)m * H * D + idx);
@@ -412,13 +419,13 @@ __global__ void k_attn_simt(const TQ* __restrict__ q, const TKV* __restrict__ ks
 __global__ void k_final(const float* __restrict__ hres, const float* __restrict__ sigma,
                         const float* __restrict__ beta, const float* __restrict__ Wout,
                         const float* __restrict__ bout, float* __restrict__ x,
-                        float* __restrict__ vout, float* __restrict__ outcopy, int S, int C,
+                        float* __restrict__ vout, float* __restrict__ outcopy, int S, int nctx, int C,
                         int W, int A, float eps, float delta) {
     extern __shared__ float us[];        // [W]
     __shared__ float scratch[32];
     const int bj = blockIdx.x;           // request b, action j
     const int b = bj / C, j = bj % C;
-    const float* hr = hres + ((size_t)b * S + 1 + j) * W;
+    const float* hr = hres + ((size_t)b * S + nctx + j) * W;
     float ss = 0.f;
     for (int k = threadIdx.x; k < W; k += blockDim.x) ss = fmaf(hr[k], hr[k], ss);
     ss = block_sum(ss, scratch);
@@ -473,7 +480,7 @@ inline int grid_for(long long n, int block, int cap = 4096) {
 // 5 norm + gate/up + GeGLU, 6 down-proj + residual.
 template <typename T>
 jpi_status op_simt(jpi_handle* h, int op, int l, int step, int B, int C, cudaStream_t st) {
-    const int S = C + 1, Mt = B * S, W = h->W, F = h->F, HD = h->HD, D = h->D;
+    const int S = C + h->n_ctx(), Mt = B * S, W = h->W, F = h->F, HD = h->HD, D = h->D;
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * W + (size_t)6 * l * W;
     const LayerPlain* lwp = (size_t)l < h->plain.size() ? &h->plain[l] : nullptr;
     T* act = (T*)h->act;
@@ -498,7 +505,7 @@ jpi_status op_simt(jpi_handle* h, int op, int l, int step, int B, int C, cudaStr
         case 3: {
             const size_t att_smem = sizeof(float) * ((size_t)h->H * D + 32 * (D + 1) + 32 * D);
             k_attn_simt<T, T, T><<<Mt, 32 * h->H, att_smem, st>>>(
-                (const T*)h->q, kst, vst, (T*)h->o, S, h->H, D, h->cur_prefix, h->kv_rows,
+                (const T*)h->q, kst, vst, (T*)h->o, S, h->H, D, h->cur_prefix, h->kv_rows, h->n_ctx(),
                 1.f / sqrtf((float)D));
             break;
         }
@@ -645,14 +652,14 @@ jpi_status launch_time_conditioning_into(jpi_handle* h, double t, float* temb, f
 }
 
 jpi_status launch_embed(jpi_handle* h, int step, int B, int C, const float* x, cudaStream_t st) {
-    const int S = C + 1;
+    const int S = C + h->n_ctx();
     // Scale and shift of layer 0's attention norm at this step.
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * h->W;
     k_embed<<<dim3((h->W + 127) / 128, B * S), 128, 0, st>>>(
         h->h, h->tc ? (__nv_bfloat16*)h->hx : nullptr, ms, ms + h->W, h->tc ? h->ss : nullptr, h->maxMt,
         h->state,
         x, h->state_in_w, h->state_in_b,
-        h->action_in_w, h->action_in_b, S, C, h->W, h->Sd, h->A);
+        h->action_in_w, h->action_in_b, h->corr, h->n_ctx(), S, C, h->W, h->Sd, h->A);
     return check_launch("embed");
 }
 
@@ -673,7 +680,7 @@ jpi_status launch_final(jpi_handle* h, int step, int B, int C, float delta, floa
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * W + (size_t)6 * h->L * W;
     k_final<<<B * C, 256, sizeof(float) * W, st>>>(h->h, ms, ms + W, h->action_out_w,
                                                    h->action_out_b, x_inout, v_out, out_copy,
-                                                   C + 1, C, W, h->A, h->cfg.rms_eps, delta);
+                                                   C + h->n_ctx(), h->n_ctx(), C, W, h->A, h->cfg.rms_eps, delta);
     return check_launch("final norm + Euler");
 }
 

@@ -71,7 +71,7 @@ extern "C" JPI_API jpi_status jpi_expert_forward_noalloc(jpi_handle* h, const fl
     }
     JPI_TRY(jpi::launch_final(h, 0, batch, chunk, 0.f, nullptr, out_v, nullptr, st));
     if (out_h)
-        JPI_CUDA_TRY(cudaMemcpyAsync(out_h, h->h, (size_t)batch * (chunk + 1) * h->W * sizeof(float),
+        JPI_CUDA_TRY(cudaMemcpyAsync(out_h, h->h, (size_t)batch * (chunk + h->n_ctx()) * h->W * sizeof(float),
                                      cudaMemcpyDeviceToDevice, st));
     return JPI_OK;
 }

@@ -312,7 +312,7 @@ jpi_status launch_gemm_big(jpi_handle* h, const GemmPlan& pl, const CUtensorMap&
 
 GemmArgs base_args(jpi_handle* h, int B, int C, const GemmPlan& pl) {
     GemmArgs a = {};
-    a.Mt = B * (C + 1);
+    a.Mt = B * (C + h->n_ctx());
     a.K = pl.K;
     a.nkb = pl.nkb;
     a.kpb = pl.kpb;
@@ -323,7 +323,7 @@ GemmArgs base_args(jpi_handle* h, int B, int C, const GemmPlan& pl) {
     a.eps = h->cfg.rms_eps;
     a.inv_w = 1.f / (float)h->W;
     a.W = h->W;
-    a.S = C + 1;
+    a.S = C + h->n_ctx();
     a.H = h->H;
     a.D = h->D;
     a.P = h->cur_prefix;
@@ -479,7 +479,7 @@ jpi_status tc_launch_op(jpi_handle* h, int op, int l, int step, int B, int C, cu
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * W + (size_t)6 * l * W;
     const size_t kv_layer = (size_t)l * h->maxB * h->kv_rows * h->D;
     const jpi::GemmPlan* plans = h->plans;
-    const int Mt = B * (C + 1);
+    const int Mt = B * (C + h->n_ctx());
     // Batched launches with many tokens: one CTA per (weight tile, 128-row operand tile) over
     // the whole K range. Residual kinds then leave one sum-of-squares slot per weight tile, and
     // the norm-fed kind after them reads as many slots as its producer left.

@@ -62,6 +62,7 @@ _SIGS = {
     "jpi_set_prefix_kv": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p],
     "jpi_prefix_kv_ptr": [c_void_p, c_int, POINTER(c_void_p), POINTER(c_void_p), POINTER(c_longlong)],
     "jpi_commit_prefix": [c_void_p, c_int, c_int],
+    "jpi_set_correction": [c_void_p, c_void_p, c_int, c_int, c_void_p],
     "jpi_denoise": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p],
     "jpi_denoise_host": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p],
     "jpi_expert_forward": [c_void_p, c_void_p, c_void_p, c_float, c_int, c_int, c_void_p,
@@ -151,6 +152,11 @@ def jpi_prefix_kv_ptr(h, layer):
 
 def jpi_commit_prefix(h, batch, prefix_len):
     _check(load().jpi_commit_prefix(h, batch, prefix_len), "jpi_commit_prefix")
+
+
+def jpi_set_correction(h, items, batch, num_items, stream=None):
+    _check(load().jpi_set_correction(h, _ptr(items), batch, num_items, _stream(stream)),
+           "jpi_set_correction")
 
 
 def jpi_denoise(h, state, noise, batch, chunk, num_steps, out_actions, stream=None):
@@ -263,6 +269,20 @@ class Expert:
                           fp32, stream)
         self._kv_keepalive = (k, v)
 
+    def set_correction(self, items, stream=None):
+        """items: CUDA float32 tensor [B][T'][width] (T' = 0 clears them), or None to clear."""
+        if items is None or items.shape[1] == 0:
+            jpi_set_correction(self.handle, None, 1, 0, stream)
+            self._corr = None
+            self.n_corr = 0
+            return
+        assert items.is_cuda and items.dim() == 3 and items.shape[2] == self.dims.width
+        items = items.contiguous().float()
+        B, T, _ = items.shape
+        jpi_set_correction(self.handle, items, B, T, stream)
+        self._corr = (items,)
+        self.n_corr = T
+
     def denoise(self, state, noise, num_steps, out=None, stream=None):
         import torch
         B, C, _ = noise.shape
@@ -283,7 +303,8 @@ class Expert:
         import torch
         B, C, A = x_t.shape
         v = torch.empty_like(x_t)
-        hres = torch.empty((B, C + 1, self.dims.width), dtype=torch.float32, device=x_t.device)
+        hres = torch.empty((B, 1 + getattr(self, "n_corr", 0) + C, self.dims.width), dtype=torch.float32,
+                           device=x_t.device)
         jpi_expert_forward(self.handle, state, x_t, t, B, C, v, hres, stream)
         return v, hres
 

@@ -1,6 +1,6 @@
 """Seeded synthetic inputs for the action-expert denoise.
 
-This package draws weights, prefix KV caches, robot states and action noise from a seeded
+This package draws weights, prefix KV caches, robot states, action noise and correction items from a seeded
 numpy PCG64 generator. It is shared by the CPU oracle and by the CUDA path's tests and bench,
 and it holds none of the method's arithmetic: only shapes, draws and the bf16 rounding of the
 drawn values (input preparation, so that both sides consume bit-identical numbers).
@@ -15,5 +15,6 @@ from .inputs import (  # noqa: F401
     round_to_bf16,
     make_weights,
     make_requests,
+    make_correction,
     weight_shapes,
 )

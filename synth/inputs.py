@@ -167,3 +167,14 @@ def make_requests(cfg: ExpertConfig, seed: int, batch: int, prefix_len: int, chu
         K = round_to_bf16(K)
         V = round_to_bf16(V)
     return {"prefix_k": K, "prefix_v": V, "state": state, "noise": noise}
+
+
+def make_correction(cfg: ExpertConfig, seed: int, batch: int, num_items: int,
+                    first_request: int = 0, std: float = 1.0) -> np.ndarray:
+    """Correction items [B][T'][width] fp32 (the compressed future VLM state given to the
+    expert), request ``b`` from its own generator, separate from ``make_requests``' streams."""
+    out = np.empty((batch, num_items, cfg.width), np.float32)
+    for b in range(batch):
+        rng = np.random.Generator(np.random.PCG64([seed, 7919, first_request + b]))
+        out[b] = _draw(rng, (num_items, cfg.width), std)
+    return out
