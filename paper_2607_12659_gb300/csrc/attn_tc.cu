@@ -23,6 +23,7 @@
 
 #include "jpi_internal.h"
 #include "ptx.h"
+#include "tc_path.h"
 
 #include <cooperative_groups.h>
 
@@ -80,6 +81,11 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Byte offset of 16-byte chunk `c` of row `r` of the query tile as its bulk tensor copies land
+// it: D/64 column blocks of [32 rows][128 B], 16-byte chunks XOR-swizzled by (r mod 8).
+__device__ __forceinline__ uint32_t q_off(int r, int c) {
+    return (uint32_t)((c >> 3) * (AT_ROWS * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+}
 // Byte offset of 16-byte chunk `c` of row `r` in a [rows][D] bf16 tile whose chunks are
 // XOR-swizzled by (r mod 8), so 8 rows read at one logical column hit 8 distinct bank groups.
 template <int D>
@@ -110,8 +116,8 @@ __host__ __device__ constexpr int AT_PSTRIDE() {
     return KB * 2 + 16;
 }
 // Shared-memory layout (bytes from the 128-aligned base): q and NBUF k/v buffers, reused after
-// the key loop for each key half's hand-over columns (fp32) and (m, l), then this split's partial
-// rows; the receive buffer; the combine coefficients; the receive barrier.
+// the key loop for this split's partial rows; the receive buffer; the P tile, block maxima and
+// l shares; the receive barrier.
 template <int D, int NBUF>
 struct AttnSmem {
     static constexpr int KB = NBUF == 2 ? AT_KEYS / 2 : AT_KEYS;   // keys per block
@@ -120,8 +126,7 @@ struct AttnSmem {
     static constexpr int REGION_USED = OPART + AT_ROWS * attn_row_bytes<D>();
     static constexpr int REGION = QKV > REGION_USED ? QKV : REGION_USED;
     static constexpr int RECV = REGION;                          // [AT_MAX_RECV_ROWS][row bytes]
-    static constexpr int COEF = RECV + AT_MAX_RECV_ROWS * attn_row_bytes<D>();   // [32][16] floats
-    static constexpr int PB = COEF + AT_ROWS * AT_MAX_SPLITS * 4;   // [32][KB] bf16 P, padded rows
+    static constexpr int PB = RECV + AT_MAX_RECV_ROWS * attn_row_bytes<D>();   // [32][KB] bf16 P, padded rows
     static constexpr int XM = PB + AT_ROWS * AT_PSTRIDE<KB>();     // [2 halves][32] block maxima
     static constexpr int LS = XM + 2 * AT_ROWS * 4;                // [2 halves][32] l shares
     static constexpr int BAR = LS + 2 * AT_ROWS * 4;
@@ -132,11 +137,12 @@ struct AttnSmem {
 // block's K/V loads are issued before the current block is processed) in the same shared memory
 // as one 64-key block, so two CTAs still fit on an SM.
 template <int D, int NBUF>
-__global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ AttnArgs a) {
+__global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ CUtensorMap qmap,
+                                                        const __grid_constant__ AttnArgs a) {
     using L = AttnSmem<D, NBUF>;
     constexpr int KB = L::KB;
     extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = smem_raw + ((128u - (ptx::smem_u32(smem_raw) & 127u)) & 127u);
+    uint8_t* smem = smem_raw + ((1024u - (ptx::smem_u32(smem_raw) & 1023u)) & 1023u);
     uint8_t* qs = smem;                                  // [32][D] bf16
     uint8_t* ks = qs + AT_ROWS * D * 2;                  // [NBUF][k [64][D], v [64][D]] bf16
     uint8_t* vs = ks + KB * D * 2;
@@ -147,8 +153,8 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     float* xmax = (float*)(smem + L::XM);                // [2][32] block maxima of each key half
     float* lsum = (float*)(smem + L::LS);                // [2][32] l of each key half
     uint8_t* recv = smem + L::RECV;                      // [(splits - 1) x rows_per][ROWB]
-    float* coef = (float*)(smem + L::COEF);              // [32][AT_MAX_SPLITS]
     uint64_t* rbar = (uint64_t*)(smem + L::BAR);
+    uint64_t* qbar = rbar + 1;                           // the query tile's bulk copies
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int rg = warp & 1, kh = warp >> 1;             // row group, key half / column half
@@ -164,6 +170,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     constexpr int DC = D / 8;                            // 16-byte chunks per row
     if (tid == 0) {
         ptx::mbar_init(rbar, 1);
+        ptx::mbar_init(qbar, 1);
         ptx::fence_mbar_init();
         ptx::mbar_expect_tx(rbar, (uint32_t)((ns - 1) * (r_hi - r_lo) * ROWB));
     }
@@ -190,18 +197,20 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     };
     const int first_suffix_row = min(KB, max(0, a.P - k_begin));
     load_kv(k_begin, 0, first_suffix_row, 0);
+    if (tid == 0) ptx::prefetch_tmap(&qmap);
 
     ptx::grid_dep_wait();
 
-    // Query block (rows beyond this request's S*H rows are zero).
-    const __nv_bfloat16* qb = a.q + (size_t)b * nrows * D;
-    for (int idx = tid; idx < AT_ROWS * DC; idx += AT_THREADS) {
-        const int r = idx / DC, c = idx % DC;
-        const bool ok = row0 + r < nrows;
-        cp_async16(qs_u + sw_off<D>(r, c), qb + (size_t)(ok ? row0 + r : 0) * D + c * 8, ok);
+    // Query block: D/64 bulk tensor copies of 32 rows (rows past this request's S*H rows are
+    // the next request's or zero fill; their results are never stored).
+    if (tid == 0) {
+        const uint64_t pol = ptx::l2_policy_evict_first();
+        ptx::mbar_expect_tx(qbar, (uint32_t)(AT_ROWS * D * 2));
+        for (int db = 0; db < D / 64; ++db)
+            ptx::tma_load_2d(qs + db * (AT_ROWS * 128), &qmap, qbar, db * 64, b * nrows + row0, pol);
     }
     load_kv(k_begin, first_suffix_row, KB, 0);
-    if (NBUF == 2) cp_async_commit();   // group: q and the first block
+    if (NBUF == 2) cp_async_commit();   // group: the first block
 
     // Per-thread rows g and g + 8 of this warp's 16; their visible key count.
     const int g = lane >> 2, cq = lane & 3;
@@ -240,6 +249,8 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
             cp_async_wait_all();
         }
         __syncthreads();
+        if (key0 == k_begin && !ptx::mbar_wait_bounded(qbar, 0, 200ull * 1000 * 1000) && tid == 0)
+            atomicCAS(a.err, 0, (int)DEV_TIMEOUT_WEIGHTS);
         const uint32_t kbuf_u = ks_u + buf * KV_BUF, vbuf_u = vs_u + buf * KV_BUF;
         if (NBUF == 2) buf ^= 1;
 
@@ -253,7 +264,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
             {
                 const int r = rg * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                 const int c = kc * 2 + (lane >> 4);
-                ldsm_x4(qs_u + sw_off<D>(r, c), a0, a1, a2, a3);
+                ldsm_x4(qs_u + q_off(r, c), a0, a1, a2, a3);
             }
 #pragma unroll
             for (int nt = 0; nt < HK / 8; nt += 2) {
@@ -401,13 +412,14 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     };
 
     // ---- combine the splits for the owned rows, in split order ----
-    // Coefficients: 16 lanes per row (lane s = split s), max and sum by butterflies.
+    // One warp per owned row: lane s (and s + 16) turns split s's (m, l) into its coefficient
+    // w_s / L by butterflies over the 16 splits; each lane then sums 8 output dimensions over the
+    // splits in split order, taking the coefficients by shuffles.
     const int nrow_here = r_hi - r_lo;
-    for (int base = 0; base < nrow_here * AT_MAX_SPLITS; base += AT_THREADS) {
-        const int idx = base + tid;
-        const int r = r_lo + idx / AT_MAX_SPLITS, s = idx % AT_MAX_SPLITS;
-        const bool valid = idx < nrow_here * AT_MAX_SPLITS && s < ns;
-        const float2 ml = valid ? *(const float2*)(srow(s, r) + 2 * D) : make_float2(-INFINITY, 0.f);
+    for (int rr = warp; rr < nrow_here; rr += AT_THREADS / 32) {
+        const int r = r_lo + rr;
+        const int sl = lane & (AT_MAX_SPLITS - 1);
+        const float2 ml = sl < ns ? *(const float2*)(srow(sl, r) + 2 * D) : make_float2(-INFINITY, 0.f);
         float mx = ml.x;
 #pragma unroll
         for (int o = 1; o < AT_MAX_SPLITS; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
@@ -415,34 +427,32 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
         float L = w * ml.y;
 #pragma unroll
         for (int o = 1; o < AT_MAX_SPLITS; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-        if (idx < nrow_here * AT_MAX_SPLITS) coef[(r - r_lo) * AT_MAX_SPLITS + s] = L > 0.f ? w / L : 0.f;
-    }
-    __syncthreads();
-    // One item = 8 output dimensions of one owned row (a 16-byte load per split).
-    for (int idx = tid; idx < nrow_here * (D / 8); idx += AT_THREADS) {
-        const int r = r_lo + idx / (D / 8), d = (idx % (D / 8)) * 8;
-        const int R = row0 + r;
-        if (R >= nrows || !got) continue;
+        const float cf = L > 0.f ? w / L : 0.f;   // 0 for lanes past the last split
+        const int R = row0 + r, d = lane * 8;
         float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         // All 16 slots are loaded together (slots past the last split read this CTA's own row
         // with a zero coefficient), then summed in split order.
 #pragma unroll
         for (int s = 0; s < AT_MAX_SPLITS; ++s) {
-            const float c = s < ns ? coef[(r - r_lo) * AT_MAX_SPLITS + s] : 0.f;
-            const uint4 hv = *(const uint4*)(srow(s < ns ? s : rank, r) + 2 * d);
-            const uint32_t w4[4] = {hv.x, hv.y, hv.z, hv.w};
+            const float c = __shfl_sync(0xffffffffu, cf, s);
+            if (d < D) {
+                const uint4 hv = *(const uint4*)(srow(s < ns ? s : rank, r) + 2 * d);
+                const uint32_t w4[4] = {hv.x, hv.y, hv.z, hv.w};
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const float2 v = __half22float2(*reinterpret_cast<const __half2*>(&w4[k]));
-                acc[2 * k] = fmaf(c, v.x, acc[2 * k]);
-                acc[2 * k + 1] = fmaf(c, v.y, acc[2 * k + 1]);
+                for (int k = 0; k < 4; ++k) {
+                    const float2 v = __half22float2(*reinterpret_cast<const __half2*>(&w4[k]));
+                    acc[2 * k] = fmaf(c, v.x, acc[2 * k]);
+                    acc[2 * k + 1] = fmaf(c, v.y, acc[2 * k + 1]);
+                }
             }
         }
-        const int i = R / a.H, head = R - i * a.H;
-        const size_t tok = (size_t)b * a.S + i;
-        *(uint4*)(a.o + (tok * a.H + head) * D + d) =
-            make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
-                       pack_bf16x2(acc[6], acc[7]));
+        if (d < D && R < nrows && got) {
+            const int i = R / a.H, head = R - i * a.H;
+            const size_t tok = (size_t)b * a.S + i;
+            *(uint4*)(a.o + (tok * a.H + head) * D + d) =
+                make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
+                           pack_bf16x2(acc[6], acc[7]));
+        }
     }
     if (tid == 0 && !got) atomicCAS(a.err, 0, (int)DEV_TIMEOUT_MMA);
     // No split exits while a copy out of its shared memory may still be in flight.
@@ -451,7 +461,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
 
 template <int D, int NBUF>
 size_t attn_smem() {
-    return 128 + (size_t)AttnSmem<D, NBUF>::TOTAL;
+    return 1024 + (size_t)AttnSmem<D, NBUF>::TOTAL;
 }
 
 template <int D>
@@ -507,7 +517,8 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     }
     cfg.attrs = attrs;
     cfg.numAttrs = n;
-    cudaError_t e = two ? cudaLaunchKernelEx(&cfg, k_attn_tc<D, 2>, a) : cudaLaunchKernelEx(&cfg, k_attn_tc<D, 1>, a);
+    cudaError_t e = two ? cudaLaunchKernelEx(&cfg, k_attn_tc<D, 2>, h->qmap_at, a)
+                        : cudaLaunchKernelEx(&cfg, k_attn_tc<D, 1>, h->qmap_at, a);
     if (e != cudaSuccess) {
         set_error("attention launch failed: %s", cudaGetErrorString(e));
         return JPI_ERR_CUDA;
@@ -538,6 +549,8 @@ bool attn_tc_supported(const jpi_handle* h) {
 }
 
 jpi_status attn_tc_prepare(jpi_handle* h) {
+    // The query tile as 32-row boxes of 64 columns (128-byte swizzle) over q [maxMt * H][D].
+    JPI_TRY(tc_make_tmap(h->q, (uint64_t)h->maxMt * h->H, h->D, AT_ROWS, &h->qmap_at));
     switch (h->D) {
         case 64: return prepare_d<64>(h);
         case 128: return prepare_d<128>(h);

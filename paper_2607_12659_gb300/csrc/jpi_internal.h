@@ -163,6 +163,7 @@ struct jpi_handle {
     int attn_t5_min_batch = 4;  // batches of at least this many requests use the unsplit attention
     bool attn_t5 = false;       // its tensor maps and attributes are ready
     CUtensorMap amaps[3];       // attention operands: q, prefix/suffix K, V (all layers)
+    CUtensorMap qmap_at;        // q as 32-row boxes for the split-KV attention
     std::vector<CUtensorMap> tmaps;
     CUtensorMap xmaps[3];       // B operands: hx, o, z
 
