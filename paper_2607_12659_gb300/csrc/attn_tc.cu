@@ -11,7 +11,7 @@
 //
 // Grid: (32-row query blocks, key splits, requests). The key splits of one query block form a
 // thread-block cluster. Inside a CTA, warp w takes query rows 16 (w mod 2) .. + 15 of every key
-// block (staged in shared memory with cp.async): it computes the scores of key half w / 2, the
+// block (staged in shared memory by bulk tensor copies): it computes the scores of key half w / 2, the
 // two warps of a row group exchange their block maxima and write the probabilities P (bf16) to
 // shared memory, and each then accumulates output columns half w / 2 over all keys of the block
 // (one online softmax per row group, nothing left to merge). The cluster then
@@ -39,18 +39,6 @@ constexpr int AT_MAX_SPLITS = 16;
 // Most rows one split receives: (splits - 1) x ceil(32 / splits), largest at 15 splits.
 constexpr int AT_MAX_RECV_ROWS = 42;
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
-                 : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait_group() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void cp_async_wait_all() {
-    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
-}
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
                  : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
@@ -86,17 +74,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 __device__ __forceinline__ uint32_t q_off(int r, int c) {
     return (uint32_t)((c >> 3) * (AT_ROWS * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4));
 }
-// Byte offset of 16-byte chunk `c` of row `r` in a [rows][D] bf16 tile whose chunks are
-// XOR-swizzled by (r mod 8), so 8 rows read at one logical column hit 8 distinct bank groups.
-template <int D>
-__device__ __forceinline__ uint32_t sw_off(int r, int c) {
-    return (uint32_t)(r * (D * 2) + ((c ^ (r & 7)) << 4));
+// The same for a K or V block of KB rows (D/64 column blocks of [KB rows][128 B]).
+template <int KB>
+__device__ __forceinline__ uint32_t kv_off(int r, int c) {
+    return (uint32_t)((c >> 3) * (KB * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4));
 }
-
 struct AttnArgs {
     const __nv_bfloat16* q;     // [Mt][H][D]
-    const __nv_bfloat16* kst;   // [maxB][kv_rows][D] (this layer)
-    const __nv_bfloat16* vst;
+    int kv_row0;                // this layer's first row in the K/V tensor maps (all layers)
     __nv_bfloat16* o;           // [Mt][H * D]
     int S, H, P, kv_rows, chunk, nsplit;
     int nctx;                   // suffix rows 0..nctx-1 (state, context tokens) see P + nctx keys
@@ -130,7 +115,7 @@ struct AttnSmem {
     static constexpr int XM = PB + AT_ROWS * AT_PSTRIDE<KB>();     // [2 halves][32] block maxima
     static constexpr int LS = XM + 2 * AT_ROWS * 4;                // [2 halves][32] l shares
     static constexpr int BAR = LS + 2 * AT_ROWS * 4;
-    static constexpr int TOTAL = BAR + 16;
+    static constexpr int TOTAL = BAR + 32;   // receive, query, and NBUF K/V barriers
 };
 
 // NBUF = 2 when a split spans several key blocks: blocks of 32 keys, double-buffered (the next
@@ -138,6 +123,8 @@ struct AttnSmem {
 // as one 64-key block, so two CTAs still fit on an SM.
 template <int D, int NBUF>
 __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ CUtensorMap qmap,
+                                                        const __grid_constant__ CUtensorMap kmap,
+                                                        const __grid_constant__ CUtensorMap vmap,
                                                         const __grid_constant__ AttnArgs a) {
     using L = AttnSmem<D, NBUF>;
     constexpr int KB = L::KB;
@@ -155,6 +142,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     uint8_t* recv = smem + L::RECV;                      // [(splits - 1) x rows_per][ROWB]
     uint64_t* rbar = (uint64_t*)(smem + L::BAR);
     uint64_t* qbar = rbar + 1;                           // the query tile's bulk copies
+    uint64_t* kvbar = rbar + 2;                          // [NBUF] each K/V buffer's bulk copies
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int rg = warp & 1, kh = warp >> 1;             // row group, key half / column half
@@ -167,10 +155,10 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     // Rows [s * rows_per, ...) of the 32 belong to split s, which combines them.
     const int rows_per = (AT_ROWS + ns - 1) / ns;
     const int r_lo = min(AT_ROWS, rank * rows_per), r_hi = min(AT_ROWS, r_lo + rows_per);
-    constexpr int DC = D / 8;                            // 16-byte chunks per row
     if (tid == 0) {
         ptx::mbar_init(rbar, 1);
         ptx::mbar_init(qbar, 1);
+        for (int i = 0; i < NBUF; ++i) ptx::mbar_init(&kvbar[i], 1);
         ptx::fence_mbar_init();
         ptx::mbar_expect_tx(rbar, (uint32_t)((ns - 1) * (r_hi - r_lo) * ROWB));
     }
@@ -179,38 +167,42 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     // before the first push (published by fence.mbarrier_init, so the arrival is relaxed).
     ptx::cluster_arrive_relaxed();
 
-    // Prefix keys/values were written before this graph ran: the first block's prefix rows are
-    // fetched before the dependency wait; the suffix rows (written by the QKV kernel) after it.
-    const __nv_bfloat16* kb_ = a.kst + (size_t)b * a.kv_rows * D;
-    const __nv_bfloat16* vb_ = a.vst + (size_t)b * a.kv_rows * D;
+    // K and V blocks by bulk tensor copies (one thread): D/64 column blocks x KB/32 boxes of 32
+    // rows each. Rows past the split's last key are whatever the store holds there (finite:
+    // zero-initialised, or other requests' and layers' keys); their scores are masked.
     const uint32_t qs_u = ptx::smem_u32(qs), ks_u = ptx::smem_u32(ks), vs_u = ptx::smem_u32(vs);
-    auto load_kv = [&](int key0, int r_from, int r_to, int buf) {
-        const uint32_t kd = ks_u + buf * KV_BUF, vd = vs_u + buf * KV_BUF;
-        for (int idx = tid; idx < KB * DC; idx += AT_THREADS) {
-            const int r = idx / DC, c = idx % DC;
-            if (r < r_from || r >= r_to) continue;
-            const bool ok = key0 + r < k_end;
-            const size_t off = (size_t)(ok ? key0 + r : 0) * D + c * 8;
-            cp_async16(kd + sw_off<D>(r, c), kb_ + off, ok);
-            cp_async16(vd + sw_off<D>(r, c), vb_ + off, ok);
-        }
+    const int kv_row_b = a.kv_row0 + b * a.kv_rows;      // this request's key 0 in the maps
+    const uint64_t pol = ptx::l2_policy_evict_first();
+    auto load_block = [&](int key0, int buf) {
+        uint8_t* kd = ks + buf * KV_BUF;
+        uint8_t* vd = vs + buf * KV_BUF;
+        ptx::mbar_expect_tx(&kvbar[buf], KV_BUF);
+        for (int db = 0; db < D / 64; ++db)
+            for (int hb = 0; hb < KB / 32; ++hb) {
+                const uint32_t off = (uint32_t)(db * (KB * 128) + hb * (32 * 128));
+                const int y = kv_row_b + key0 + hb * 32;
+                ptx::tma_load_2d(kd + off, &kmap, &kvbar[buf], db * 64, y, pol);
+                ptx::tma_load_2d(vd + off, &vmap, &kvbar[buf], db * 64, y, pol);
+            }
     };
-    const int first_suffix_row = min(KB, max(0, a.P - k_begin));
-    load_kv(k_begin, 0, first_suffix_row, 0);
-    if (tid == 0) ptx::prefetch_tmap(&qmap);
+    // A first block made only of prefix keys (written before this graph ran) is fetched before
+    // the dependency wait; one holding suffix keys (written by the QKV kernel) after it.
+    const bool early = min(k_end, k_begin + KB) <= a.P;
+    if (tid == 0) {
+        ptx::prefetch_tmap(&qmap);
+        if (early) load_block(k_begin, 0);
+    }
 
     ptx::grid_dep_wait();
 
     // Query block: D/64 bulk tensor copies of 32 rows (rows past this request's S*H rows are
     // the next request's or zero fill; their results are never stored).
     if (tid == 0) {
-        const uint64_t pol = ptx::l2_policy_evict_first();
         ptx::mbar_expect_tx(qbar, (uint32_t)(AT_ROWS * D * 2));
         for (int db = 0; db < D / 64; ++db)
             ptx::tma_load_2d(qs + db * (AT_ROWS * 128), &qmap, qbar, db * 64, b * nrows + row0, pol);
+        if (!early) load_block(k_begin, 0);
     }
-    load_kv(k_begin, first_suffix_row, KB, 0);
-    if (NBUF == 2) cp_async_commit();   // group: the first block
 
     // Per-thread rows g and g + 8 of this warp's 16; their visible key count.
     const int g = lane >> 2, cq = lane & 3;
@@ -233,26 +225,21 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
     const int ra = rg * 16 + g, rb2 = ra + 8;             // this thread's two rows
     const uint32_t pb_u = ptx::smem_u32(pbuf);
 
-    int buf = 0;
-    for (int key0 = k_begin; key0 < k_end; key0 += KB) {
+    int jb = 0;   // block index within the split
+    for (int key0 = k_begin; key0 < k_end; key0 += KB, ++jb) {
         __syncthreads();   // every warp is done with the buffer refilled below (and with P)
-        if (NBUF == 2) {
-            if (key0 + KB < k_end) {
-                load_kv(key0 + KB, 0, KB, buf ^ 1);
-                cp_async_commit();
-                cp_async_wait_group<1>();   // this block's group has landed
-            } else {
-                cp_async_wait_group<0>();
-            }
-        } else {
-            if (key0 != k_begin) load_kv(key0, 0, KB, 0);
-            cp_async_wait_all();
+        // Block jb sits in buffer jb mod NBUF (its (jb / NBUF)-th use); with two buffers the next
+        // block is fetched into the other one while this one is processed.
+        const int bi = NBUF == 2 ? (jb & 1) : 0;
+        if (tid == 0) {
+            if (NBUF == 2 && key0 + KB < k_end) load_block(key0 + KB, bi ^ 1);
+            if (NBUF == 1 && key0 != k_begin) load_block(key0, 0);
         }
-        __syncthreads();
-        if (key0 == k_begin && !ptx::mbar_wait_bounded(qbar, 0, 200ull * 1000 * 1000) && tid == 0)
-            atomicCAS(a.err, 0, (int)DEV_TIMEOUT_WEIGHTS);
-        const uint32_t kbuf_u = ks_u + buf * KV_BUF, vbuf_u = vs_u + buf * KV_BUF;
-        if (NBUF == 2) buf ^= 1;
+        const uint32_t par = NBUF == 2 ? ((jb >> 1) & 1) : (jb & 1);
+        bool landed = ptx::mbar_wait_bounded(&kvbar[bi], par, 200ull * 1000 * 1000);
+        if (key0 == k_begin) landed = ptx::mbar_wait_bounded(qbar, 0, 200ull * 1000 * 1000) && landed;
+        if (!landed && tid == 0) atomicCAS(a.err, 0, (int)DEV_TIMEOUT_WEIGHTS);
+        const uint32_t kbuf_u = ks_u + bi * KV_BUF, vbuf_u = vs_u + bi * KV_BUF;
 
         // S = Q K^T for this warp's 16 rows x its key half.
         float sacc[HK / 8][4];
@@ -271,7 +258,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
                 uint32_t b0, b1, b2, b3;
                 const int r = kh * HK + (nt + (lane >> 4)) * 8 + (lane & 7);
                 const int c = kc * 2 + ((lane >> 3) & 1);
-                ldsm_x4(kbuf_u + sw_off<D>(r, c), b0, b1, b2, b3);
+                ldsm_x4(kbuf_u + kv_off<KB>(r, c), b0, b1, b2, b3);
                 mma16816(sacc[nt], a0, a1, a2, a3, b0, b1);
                 mma16816(sacc[nt + 1], a0, a1, a2, a3, b2, b3);
             }
@@ -350,7 +337,7 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
                 uint32_t b0, b1, b2, b3;
                 const int r = j * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                 const int c = kh * NOT + dt + (lane >> 4);
-                ldsm_x4_t(vbuf_u + sw_off<D>(r, c), b0, b1, b2, b3);
+                ldsm_x4_t(vbuf_u + kv_off<KB>(r, c), b0, b1, b2, b3);
                 mma16816(oacc[dt], a0, a1, a2, a3, b0, b1);
                 mma16816(oacc[dt + 1], a0, a1, a2, a3, b2, b3);
             }
@@ -480,10 +467,8 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     chunk = (chunk + 15) / 16 * 16;
     const int ns = (nk + chunk - 1) / chunk;
     AttnArgs a;
-    const size_t kv_layer = (size_t)l * h->maxB * h->kv_rows * h->D;
     a.q = (const __nv_bfloat16*)h->q;
-    a.kst = (const __nv_bfloat16*)h->kv_k + kv_layer;
-    a.vst = (const __nv_bfloat16*)h->kv_v + kv_layer;
+    a.kv_row0 = l * h->maxB * h->kv_rows;
     a.o = (__nv_bfloat16*)h->o;
     a.S = S;
     a.nctx = h->n_ctx();
@@ -517,8 +502,8 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     }
     cfg.attrs = attrs;
     cfg.numAttrs = n;
-    cudaError_t e = two ? cudaLaunchKernelEx(&cfg, k_attn_tc<D, 2>, h->qmap_at, a)
-                        : cudaLaunchKernelEx(&cfg, k_attn_tc<D, 1>, h->qmap_at, a);
+    cudaError_t e = two ? cudaLaunchKernelEx(&cfg, k_attn_tc<D, 2>, h->qmap_at, h->kmap_at, h->vmap_at, a)
+                        : cudaLaunchKernelEx(&cfg, k_attn_tc<D, 1>, h->qmap_at, h->kmap_at, h->vmap_at, a);
     if (e != cudaSuccess) {
         set_error("attention launch failed: %s", cudaGetErrorString(e));
         return JPI_ERR_CUDA;
@@ -551,6 +536,10 @@ bool attn_tc_supported(const jpi_handle* h) {
 jpi_status attn_tc_prepare(jpi_handle* h) {
     // The query tile as 32-row boxes of 64 columns (128-byte swizzle) over q [maxMt * H][D].
     JPI_TRY(tc_make_tmap(h->q, (uint64_t)h->maxMt * h->H, h->D, AT_ROWS, &h->qmap_at));
+    // K and V of all layers [L * maxB * kv_rows][D] as 32-row boxes.
+    const uint64_t kv_rows_all = (uint64_t)h->L * h->maxB * h->kv_rows;
+    JPI_TRY(tc_make_tmap(h->kv_k, kv_rows_all, h->D, 32, &h->kmap_at));
+    JPI_TRY(tc_make_tmap(h->kv_v, kv_rows_all, h->D, 32, &h->vmap_at));
     switch (h->D) {
         case 64: return prepare_d<64>(h);
         case 128: return prepare_d<128>(h);

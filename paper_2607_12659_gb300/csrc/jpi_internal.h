@@ -164,6 +164,7 @@ struct jpi_handle {
     bool attn_t5 = false;       // its tensor maps and attributes are ready
     CUtensorMap amaps[3];       // attention operands: q, prefix/suffix K, V (all layers)
     CUtensorMap qmap_at;        // q as 32-row boxes for the split-KV attention
+    CUtensorMap kmap_at, vmap_at;   // K, V of all layers as 32-row boxes for it
     std::vector<CUtensorMap> tmaps;
     CUtensorMap xmaps[3];       // B operands: hx, o, z
 
