@@ -37,11 +37,11 @@ OP_NAMES = {2: "norm+qkv+rope", 3: "attention", 4: "o_proj+residual", 5: "norm+g
 # valid only while the kernel sources hash to `source_sha256`.
 NCU_TRAFFIC = {
     # profiles/layer_kernels_pi05_forward.md (layer 1 of one eager forward, batch 1, P 816).
-    "norm+qkv+rope": {"bytes": 5492224, "source_sha256": "e8fd1625c91b9a11"},
-    "attention": {"bytes": 1137920, "source_sha256": "e8fd1625c91b9a11"},
-    "o_proj+residual": {"bytes": 4697344, "source_sha256": "e8fd1625c91b9a11"},
-    "norm+gate_up+geglu": {"bytes": 16963072, "source_sha256": "e8fd1625c91b9a11"},
-    "down_proj+residual": {"bytes": 9133312, "source_sha256": "e8fd1625c91b9a11"},
+    "norm+qkv+rope": {"bytes": 5491968, "source_sha256": "00defca3bf368457"},
+    "attention": {"bytes": 1181696, "source_sha256": "00defca3bf368457"},
+    "o_proj+residual": {"bytes": 4697600, "source_sha256": "00defca3bf368457"},
+    "norm+gate_up+geglu": {"bytes": 16963072, "source_sha256": "00defca3bf368457"},
+    "down_proj+residual": {"bytes": 9133312, "source_sha256": "00defca3bf368457"},
 }
 
 
