@@ -37,11 +37,11 @@ OP_NAMES = {2: "norm+qkv+rope", 3: "attention", 4: "o_proj+residual", 5: "norm+g
 # valid only while the kernel sources hash to `source_sha256`.
 NCU_TRAFFIC = {
     # profiles/layer_kernels_pi05_forward.md (layer 1 of one eager forward, batch 1, P 816).
-    "norm+qkv+rope": {"bytes": 5491968, "source_sha256": "00defca3bf368457"},
-    "attention": {"bytes": 1181696, "source_sha256": "00defca3bf368457"},
-    "o_proj+residual": {"bytes": 4697600, "source_sha256": "00defca3bf368457"},
-    "norm+gate_up+geglu": {"bytes": 16963072, "source_sha256": "00defca3bf368457"},
-    "down_proj+residual": {"bytes": 9133312, "source_sha256": "00defca3bf368457"},
+    "norm+qkv+rope": {"bytes": 5492224, "source_sha256": "be9ab526ee05a084"},
+    "attention": {"bytes": 1181696, "source_sha256": "be9ab526ee05a084"},
+    "o_proj+residual": {"bytes": 4697344, "source_sha256": "be9ab526ee05a084"},
+    "norm+gate_up+geglu": {"bytes": 16962816, "source_sha256": "be9ab526ee05a084"},
+    "down_proj+residual": {"bytes": 9133312, "source_sha256": "be9ab526ee05a084"},
 }
 
 
@@ -103,7 +103,8 @@ def measured_peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clock/throttle samples every 200 ms while the timed region runs."""
+    """nvidia-smi clock/throttle samples every 50 ms while the timed region runs. The region
+    starts only after the first sample has arrived, so the samples cover all of it."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -112,27 +113,44 @@ class ClockSampler:
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
         self.proc = None
+        self.lines = []
+
+    def _read(self):
+        for line in self.proc.stdout:
+            if line.strip():
+                self.lines.append(line)
+                self.first.set()
+        self.first.set()
 
     def __enter__(self):
+        import threading
+        self.lines = []
+        self.first = threading.Event()
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
+            return self
+        self.reader = threading.Thread(target=self._read, daemon=True)
+        self.reader.start()
+        self.first.wait(timeout=5.0)
+        self.n_before = len(self.lines)
         return self
 
     def __exit__(self, *exc):
-        self.lines = []
         if self.proc:
             self.proc.terminate()
             try:
-                out, _ = self.proc.communicate(timeout=5)
+                self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
-                out, _ = self.proc.communicate()
-            self.lines = [l for l in out.splitlines() if l.strip()]
+                self.proc.wait()
+            self.reader.join(timeout=5)
+            # Samples taken during the region (the one that opened it included).
+            self.lines = self.lines[max(self.n_before - 1, 0):]
 
     def summary(self):
         sm, mx, reasons = [], None, set()

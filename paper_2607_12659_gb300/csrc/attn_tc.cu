@@ -79,8 +79,8 @@ template <int KB>
 __device__ __forceinline__ uint32_t kv_off(int r, int c) {
     return (uint32_t)((c >> 3) * (KB * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4));
 }
+
 struct AttnArgs {
-    const __nv_bfloat16* q;     // [Mt][H][D]
     int kv_row0;                // this layer's first row in the K/V tensor maps (all layers)
     __nv_bfloat16* o;           // [Mt][H * D]
     int S, H, P, kv_rows, chunk, nsplit;
@@ -467,7 +467,6 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     chunk = (chunk + 15) / 16 * 16;
     const int ns = (nk + chunk - 1) / chunk;
     AttnArgs a;
-    a.q = (const __nv_bfloat16*)h->q;
     a.kv_row0 = l * h->maxB * h->kv_rows;
     a.o = (__nv_bfloat16*)h->o;
     a.S = S;
