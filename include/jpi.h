@@ -152,7 +152,7 @@ JPI_API jpi_status jpi_prefix_kv_ptr(jpi_handle* h, int layer, void** k, void** 
 JPI_API jpi_status jpi_commit_prefix(jpi_handle* h, int batch, int prefix_len);
 
 /*
- * Correction items (Sec. 3 "Foresight-Aligned Asynchronous Correction", App. B and Alg. 1):
+ * Correction items (Sec. 4.1 "Foresight-Aligned Asynchronous Correction", App. B, App. C Alg. 1):
  * the future correction module's prediction of the compressed VLM final-layer state at
  * t + Delta, T' tokens of width d_AE, is given to the action expert as future environment
  * information. The expert takes them as context tokens right after the state token: their

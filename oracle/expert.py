@@ -28,7 +28,7 @@ Everything else is a reading, numbered R1..R15 where it is used below:
   R9  velocity read from the action rows only.
   R10 requests in a batch are independent.
   R13 the Gemma projections (q, k, v, o, gate, up, down) carry no bias.
-  R15 correction items (Sec. 3 "Foresight-Aligned Asynchronous Correction", App. B): the T'
+  R15 correction items (Sec. 4.1 "Foresight-Aligned Asynchronous Correction", App. B): the T'
       predicted compressed VLM states (width d_AE, the expert's width) given to the action
       expert enter it as context tokens right after the state token, taken as the residual
       stream's input row unchanged (no projection, d_AE = width). The state and context rows
