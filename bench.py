@@ -67,14 +67,18 @@ def algorithmic_bytes(cfg, B, P, C, N):
 
 def algorithmic_flops(cfg, B, P, C, N):
     """Multiply-adds x 2 of a denoise: the layer projections at M = B (C + 1) tokens, the
-    attention of the S H query rows over P + S keys, and the per-call modulation GEMV."""
+    attention of the S H query rows over all P + S keys (QK^T and PV), the state/action
+    embeddings and the action-out projection, and per step time the time MLP and the
+    modulation GEMV."""
     W, H, D, F, L = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim, cfg.n_layers
+    Sd, A = cfg.state_dim, cfg.action_dim
     S = C + 1
     Mt = B * S
     proj = L * (H * D * W + 2 * D * W + H * D * W + 3 * F * W)
     attn = L * B * S * H * (P + S) * D * 2
-    per_step = 2 * (Mt * proj + attn + Mt * (cfg.state_dim + cfg.action_dim) * W + B * C * W * cfg.action_dim)
-    return N * per_step + 2 * (6 * L + 2) * W * W * N
+    per_step = 2 * (Mt * proj + attn + B * Sd * W + B * C * A * W + B * C * W * A)
+    per_time = 2 * (W * cfg.time_dim + W * W + (6 * L + 2) * W * W)
+    return N * (per_step + per_time)
 
 
 def op_bytes(cfg, op, B, P, C):

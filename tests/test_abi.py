@@ -41,6 +41,7 @@ def test_null_arguments_are_rejected_on_the_host(lib):
     assert lib.jpi_expert_create(None, None, None) == -1
     assert lib.jpi_denoise(None, None, None, 1, 1, 1, None, None) == -1
     assert lib.jpi_set_prefix_kv(None, None, None, 1, 1, 0, None) == -1
+    assert lib.jpi_set_correction(None, None, 1, 0, None) == -1
     assert lib.jpi_expert_destroy(None) == 0
     b = ctypes.c_longlong()
     assert lib.jpi_memory_usage(None, ctypes.byref(b)) == -1

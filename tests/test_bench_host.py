@@ -1,0 +1,98 @@
+"""Host logic of bench.py: the roofline byte and FLOP counts against an independent count from
+the weight shapes, the per-launch byte split, the clock-record parsing and the JSON contract of
+the reference arm. No GPU is used."""
+
+import json
+import os
+import subprocess
+import sys
+
+import numpy as np
+import pytest
+
+import bench
+from synth import PI05, TINY, weight_shapes
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+LAYER_PROJ = ("wq", "wk", "wv", "wo", "w_gate", "w_up", "w_down")
+
+
+def _size(shape):
+    return int(np.prod(shape))
+
+
+@pytest.mark.parametrize("cfg", [PI05, TINY], ids=["pi05", "tiny"])
+@pytest.mark.parametrize("B,P,C,N", [(1, 816, 50, 10), (4, 300, 10, 3)])
+def test_algorithmic_bytes_from_the_weight_shapes(cfg, B, P, C, N):
+    ws = weight_shapes(cfg)
+    L = cfg.n_layers
+    step = 2 * (L * sum(_size(ws[k]) for k in LAYER_PROJ)
+                + _size(ws["state_in_w"]) + _size(ws["action_in_w"]) + _size(ws["action_out_w"]))
+    time_w = 2 * (_size(ws["time_mlp_in_w"]) + _size(ws["time_mlp_out_w"])
+                  + L * (_size(ws["attn_mod_w"]) + _size(ws["mlp_mod_w"])) + _size(ws["final_mod_w"]))
+    kv = B * L * P * cfg.head_dim * 2 * 2
+    io = B * (cfg.state_dim + 2 * C * cfg.action_dim) * 4
+    assert bench.algorithmic_bytes(cfg, B, P, C, N) == N * step + time_w + kv + io
+
+
+def test_pi05_step_weights_are_the_paper_sized_expert():
+    # 18 layers x 17,301,504 projection parameters + in/out projections, bf16: 623.05 MB.
+    ws = weight_shapes(PI05)
+    assert sum(_size(ws[k]) for k in LAYER_PROJ) == 17_301_504
+    assert bench.algorithmic_bytes(PI05, 1, 816, 50, 10) == 6_480_441_984
+
+
+@pytest.mark.parametrize("B,P,C,N", [(1, 816, 50, 10), (64, 2048, 50, 10), (3, 17, 8, 2)])
+def test_algorithmic_flops_from_the_weight_shapes(B, P, C, N):
+    cfg = PI05
+    ws = weight_shapes(cfg)
+    L, H, D, W = cfg.n_layers, cfg.n_heads, cfg.head_dim, cfg.width
+    S = C + 1
+    macs_step = (B * S * L * sum(_size(ws[k]) for k in LAYER_PROJ)
+                 + L * B * 2 * (S * H) * (P + S) * D                       # QK^T and PV
+                 + B * _size(ws["state_in_w"]) + B * C * _size(ws["action_in_w"])
+                 + B * C * _size(ws["action_out_w"]))
+    macs_time = (_size(ws["time_mlp_in_w"]) + _size(ws["time_mlp_out_w"])
+                 + L * (_size(ws["attn_mod_w"]) + _size(ws["mlp_mod_w"])) + _size(ws["final_mod_w"]))
+    assert bench.algorithmic_flops(cfg, B, P, C, N) == 2 * N * (macs_step + macs_time)
+
+
+def test_layer_op_bytes_cover_each_layer_weight_once():
+    cfg, B, P, C = PI05, 2, 816, 50
+    ws = weight_shapes(cfg)
+    Mt = B * (C + 1)
+    W, F, HD, D = cfg.width, cfg.mlp_dim, cfg.n_heads * cfg.head_dim, cfg.head_dim
+    acts = {2: Mt * W * 4 + Mt * (HD + 2 * D) * 2,       # h in, q/k/v out
+            3: B * (P + C + 1) * D * 2 * 2 + Mt * HD * 2 * 2,
+            4: Mt * HD * 2 + Mt * W * 4 * 2,
+            5: Mt * W * 4 + Mt * F * 2,
+            6: Mt * F * 2 + Mt * W * 4 * 2}
+    weights = sum(bench.op_bytes(cfg, op, B, P, C) - acts[op] for op in range(2, 7))
+    assert weights == 2 * sum(_size(ws[k]) for k in LAYER_PROJ)
+    assert bench.op_bytes(cfg, 3, B, P, C) == acts[3]           # attention reads no weights
+
+
+def test_clock_record_parsing():
+    c = bench.ClockSampler(0)
+    c.lines = ["0, 2070, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active",
+               "0, 1980, 2070, 1399.0, 0x4, Not Active, Not Active, Not Active, Active",
+               "0, 2070, 2070, 1200.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+               "garbage line"]
+    s = c.summary()
+    assert s == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+    c.lines = []
+    assert c.summary()["reasons"] == ["unavailable"]
+
+
+def test_reference_arm_json_line():
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                          "--steps", "1", "--warmup", "3"], capture_output=True, text=True, timeout=600,
+                         cwd=ROOT)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                "higher_is_better", "scaling", "dtype", "data", "config", "cpu_baseline", "e2e"):
+        assert key in line, key
+    assert line["impl"] == "reference" and line["value"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
