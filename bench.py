@@ -98,6 +98,34 @@ def op_bytes(cfg, op, B, P, C):
     raise ValueError(op)
 
 
+def rank_env():
+    """(world size, rank, local rank) from the launcher's environment; (1, 0, 0) when run directly."""
+    return (int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The slowest rank's value (max-over-ranks timing); x itself at world size 1."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, batch: int, steps: int, ms: float) -> float:
+    """Chunks per second of the whole job: every replica denoises `steps` batches of `batch`
+    requests in `ms` milliseconds (the slowest replica's time)."""
+    return world * batch * steps / (ms / 1e3)
+
+
+def request_seed(rank: int) -> int:
+    """Seed of a replica's requests: each rank denoises its own, independent requests."""
+    return 2001 + rank
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -211,7 +239,7 @@ def run_cpu_baseline(cores: int) -> dict:
 def reference_arm(args):
     """The fp64 CPU oracle on this host's cores; a step is one Euler step (one expert pass)
     of the batch-1 workload, and chunks/s = 1 / (10 x mean step time)."""
-    rank = int(os.environ.get("RANK", "0"))
+    _, rank, _ = rank_env()
     if rank != 0:
         return
     import numpy as np
@@ -254,9 +282,7 @@ def our_arm(args):
     from paper_2607_12659_gb300 import build, jpi
     from synth import PI05, make_requests, make_weights
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local = rank_env()
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
@@ -273,7 +299,7 @@ def our_arm(args):
     w = make_weights(cfg, 2000)
     ex = jpi.Expert(cfg, w, max_batch=B, max_prefix=P, max_chunk=C, max_steps=N)
     del w
-    r = make_requests(cfg, 2001 + rank, B, P, C)
+    r = make_requests(cfg, request_seed(rank), B, P, C)
     ex.set_prefix_kv(torch.from_numpy(r["prefix_k"]).cuda().to(torch.bfloat16),
                      torch.from_numpy(r["prefix_v"]).cuda().to(torch.bfloat16))
     state = torch.from_numpy(r["state"]).cuda()
@@ -306,13 +332,9 @@ def our_arm(args):
     per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
     total_ms = evs[0].elapsed_time(evs[-1])
     ex.device_status()
-    t_max = total_ms
-    if world > 1:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        t_max = float(t.item())
+    t_max = max_over_ranks(total_ms, world, "cuda")
     ms_per_step = t_max / args.steps
-    value = world * B * args.steps / (t_max / 1e3)
+    value = whole_job_rate(world, B, args.steps, t_max)
 
     # ---- end to end through the host-buffer entry point (pinned host memory) ----
     hs = torch.from_numpy(r["state"]).pin_memory()
@@ -330,12 +352,8 @@ def our_arm(args):
         ex.denoise_host(hs_np, hn_np, N, ho_np)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e_value = world * B * args.steps / (e2e_ms / 1e3)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, "cuda")
+    e2e_value = whole_job_rate(world, B, args.steps, e2e_ms)
     same = bool(np.array_equal(ho_np, out.cpu().numpy()))
 
     # ---- per-op durations (each op alone, back to back, events on the launching stream) ----
