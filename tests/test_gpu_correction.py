@@ -115,3 +115,40 @@ def test_pi05_items_change_the_actions_and_clearing_restores_the_plain_expert(pi
     again = gpu_denoise(ex, PI05, r, 5)
     np.testing.assert_array_equal(again, plain)          # same graph, same arithmetic
     assert errors(with_items, plain)[0] > 1e-3
+
+
+def test_scheduler_drives_the_expert_with_predicted_states():
+    """App. C Alg. 1 over the library: each chunk the scheduler stores is the expert's denoise
+    for the state the (scripted) VLM or correction module produced, with the current KV."""
+    from paper_2607_12659_gb300.scheduler import ConfidenceScheduler, expert_act
+    w = make_weights(TINY, 0)
+    ex = make_expert(TINY, w, max_batch=1, max_prefix=64, max_chunk=8, max_steps=4)
+    try:
+        r = make_requests(TINY, 51, 1, 40, 6)
+        kv = to_dev_kv(r, TINY)
+        h0 = torch.from_numpy(make_correction(TINY, 52, 1, 2)).cuda()
+        h1 = torch.from_numpy(make_correction(TINY, 53, 1, 2)).cuda()
+        state = torch.from_numpy(r["state"]).cuda()
+        noise = torch.from_numpy(r["noise"]).cuda()
+        act = expert_act(ex, lambda: state, lambda: noise, 3)
+        sch = ConfidenceScheduler(vlm=lambda obs: (h0, kv), corr=lambda h, a: (h1, 0.5), act=act,
+                                  observe=lambda: "obs", theta=-0.2, delta=4, delta_ae=2)
+        sch.start()
+        sch.iterate()                                # correction branch: predicted state h1
+        torch.cuda.synchronize()
+        ex.device_status()
+
+        def direct(h):
+            ex.set_prefix_kv(*kv)
+            ex.set_correction(h)
+            out = ex.denoise(state, noise, 3)
+            torch.cuda.synchronize()
+            return out.cpu().numpy()[0]
+
+        first, second = direct(h0), direct(h1)
+        got = sch.buffer.committed(2 + 6)
+        np.testing.assert_array_equal(np.stack(got[:2]), first[:2])
+        np.testing.assert_array_equal(np.stack(got[2:]), second)
+        assert np.abs(first - second).max() > 1e-6
+    finally:
+        ex.close()
