@@ -1,6 +1,7 @@
 """CPU oracle (test infrastructure only).
 
-Plain fp64 numpy restatement of the action expert's flow-matching denoise. It is imported
+Plain fp64 numpy restatement of the action expert's flow-matching denoise (`expert`) and of
+the VLM's LLM prefill that produces the KV cache it attends over (`prefill`). It is imported
 only by the tests, by the smoke check and by the bench's CPU-baseline leg; the library and
 its CUDA kernels never import it and share no code with it.
 """

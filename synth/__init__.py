@@ -18,3 +18,11 @@ from .inputs import (  # noqa: F401
     make_correction,
     weight_shapes,
 )
+from .llm import (  # noqa: F401
+    GEMMA2B,
+    LLM_LAYER_WEIGHTS,
+    LLMConfig,
+    llm_weight_shapes,
+    make_llm_weights,
+    make_prefix_embeddings,
+)
