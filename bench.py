@@ -382,8 +382,11 @@ def our_arm(args):
     path_tf = flops / (ms_per_step * 1e-3) / 1e12
 
     if rank == 0:
-        cpu = (run_cpu_baseline(os.cpu_count() or 1)
-               if world == 1 and default_workload and not args.no_cpu_baseline else None)
+        cpu = None
+        if world == 1 and default_workload and not args.no_cpu_baseline:
+            cpu = run_cpu_baseline(os.cpu_count() or 1)
+            one = run_cpu_baseline(1)          # the same oracle on one thread
+            cpu["single_thread"] = {"value": one["value"], "cores": 1, "sample": one["sample"]}
         clocks = clk.summary()
         line = {
             "metric": METRIC if default_workload else METRIC.replace("batch 1", f"batch {B}"),
