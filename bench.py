@@ -45,12 +45,18 @@ NCU_TRAFFIC = {
 }
 
 
+# The sources the expert's kernels and their launches are built from. The correction module
+# (CORRECTION_SOURCES) is compiled into the same library but none of the measured kernels uses it.
+EXPERT_SOURCES = ("api.cu", "attn_t5.cu", "attn_tc.cu", "gemm_big.cuh", "gemm_kernel.cuh",
+                  "jpi_internal.h", "kernels_simt.cu", "noalloc.cu", "ptx.h", "tc_path.cu", "tc_path.h")
+CORRECTION_SOURCES = ("corr.cu",)
+
+
 def source_sha() -> str:
     d = os.path.join(ROOT, "paper_2607_12659_gb300", "csrc")
     h = hashlib.sha256()
-    for f in sorted(os.listdir(d)):
-        if f.endswith((".cu", ".cuh", ".h")):
-            h.update(open(os.path.join(d, f), "rb").read())
+    for f in sorted(EXPERT_SOURCES):
+        h.update(open(os.path.join(d, f), "rb").read())
     return h.hexdigest()[:16]
 
 

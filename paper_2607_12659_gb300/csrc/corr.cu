@@ -1,0 +1,929 @@
+// The future correction module and its Q-Former state compressor on the GPU (Sec. 4.1, App. B
+// and its figure, Eq. 2, App. C Alg. 1).
+//
+// Every token count here is small (T' = 4 compressed tokens, at most 64 committed actions per
+// request), so apart from the compressor's pass over the VLM tokens the module is a chain of
+// matrix-vector products that stream its ~44M weights once per call: at batch 1 that is HBM
+// work (88 MB in bf16), not a dense contraction, and it runs on CUDA cores with every weight
+// row read once by one warp (16-byte loads) and the few activation rows served from L1.
+//
+// The compressor's cross-attention is reassociated. Its queries come from the learned query
+// tokens through the query self-attention alone, so they are fixed by the weights; with
+// q_hi the scaled query of head h, item i, and W_k,h / W_v,h the head's rows of the key and
+// value projections:
+//   score_hij = q_hi . (W_k,h v_j + b_k,h) = (W_k,h^T q_hi) . v_j + const_hi,
+//   out_hi    = sum_j p_hij (W_v,h v_j + b_v,h) = W_v,h (sum_j p_hij v_j) + b_v,h   (sum_j p = 1).
+// The key bias only shifts every score of a query alike, which softmax cancels. So create time
+// computes a_hi = W_k,h^T q_hi once ([H T'][d_vlm]); a call scores the raw VLM tokens against
+// them, takes the softmax-weighted sum of the raw tokens, and applies W_v,h to that sum: about
+// 2 H T' T d_vlm * 2 FLOPs per request instead of the 4 T d_vlm d of projecting every token.
+
+#include "jpi_internal.h"
+#include "jpi_corr.h"
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <new>
+
+namespace {
+
+constexpr int CORR_MAX_M = 64;          // n_heads * n_items: rows of the reassociated queries
+constexpr int LIN_ROWS = 8;             // activation rows one warp carries per weight-row pass
+
+jpi_status cfail(jpi_status s, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    jpi::set_error("%s", buf);
+    return s;
+}
+
+__device__ __forceinline__ float gelu_tanh_f(float y) {
+    // 0.5 y (1 + tanh(sqrt(2/pi) (y + 0.044715 y^3))), the tanh form of GELU.
+    return 0.5f * y * (1.f + tanhf(0.7978845608028654f * (y + 0.044715f * y * y * y)));
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) v += __shfl_xor_sync(0xffffffffu, v, s);
+    return v;
+}
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+__device__ __forceinline__ float4 load4(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
+__device__ __forceinline__ float4 load4(const __nv_bfloat16* p) {
+    const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+    return make_float4(a.x, a.y, b.x, b.y);
+}
+__device__ __forceinline__ float load1(const float* p) { return __ldg(p); }
+__device__ __forceinline__ float load1(const __nv_bfloat16* p) { return __bfloat162float(p[0]); }
+
+// y[r][o] = act(sum_i x(r, o)[i] w[o][i] + bias[o]) + res[r][o] for r < rows, o < out.
+// x(r, o) is row r of x (stride ldx), or in head-select mode row
+// ((r / hs_items) * hs_heads + o / hs_dh) * hs_items + r % hs_items: the reassociated
+// cross-attention keeps one weighted token sum per (request, head, item).
+// One warp per output feature at a time; LIN_ROWS rows per pass over the weight row. y must not
+// overlap x; it may be res (each element is read and written by the same lane).
+struct LinArgs {
+    const float* x;
+    int ldx;
+    const void* w;
+    const float* bias;
+    const float* res;
+    int ldr;
+    float* y;
+    int ldy;
+    int rows, in, out, gelu;
+    int hs_items, hs_heads, hs_dh;   // head-select mode when hs_items > 0
+};
+
+template <typename TW, bool VEC>
+__global__ void __launch_bounds__(256) k_corr_linear(const LinArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int nwarps = (gridDim.x * blockDim.x) >> 5;
+    const TW* W = static_cast<const TW*>(a.w);
+    for (int o = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); o < a.out; o += nwarps) {
+        const TW* wr = W + (size_t)o * a.in;
+        const float bo = a.bias ? a.bias[o] : 0.f;
+        for (int r0 = 0; r0 < a.rows; r0 += LIN_ROWS) {
+            const float* xr[LIN_ROWS];
+#pragma unroll
+            for (int k = 0; k < LIN_ROWS; ++k) {
+                const int r = r0 + k < a.rows ? r0 + k : a.rows - 1;   // clamped; result unused
+                long long row = r;
+                if (a.hs_items > 0)
+                    row = ((long long)(r / a.hs_items) * a.hs_heads + o / a.hs_dh) * a.hs_items + r % a.hs_items;
+                xr[k] = a.x + row * a.ldx;
+            }
+            float acc[LIN_ROWS];
+#pragma unroll
+            for (int k = 0; k < LIN_ROWS; ++k) acc[k] = 0.f;
+            if (VEC) {
+                for (int i = lane * 4; i < a.in; i += 128) {
+                    const float4 w4 = load4(wr + i);
+#pragma unroll
+                    for (int k = 0; k < LIN_ROWS; ++k) {
+                        const float4 x4 = *reinterpret_cast<const float4*>(xr[k] + i);
+                        acc[k] = fmaf(w4.x, x4.x, fmaf(w4.y, x4.y, fmaf(w4.z, x4.z, fmaf(w4.w, x4.w, acc[k]))));
+                    }
+                }
+            } else {
+                for (int i = lane; i < a.in; i += 32) {
+                    const float w1 = load1(wr + i);
+#pragma unroll
+                    for (int k = 0; k < LIN_ROWS; ++k) acc[k] = fmaf(w1, xr[k][i], acc[k]);
+                }
+            }
+            float mine = 0.f;   // lane k keeps row r0 + k
+#pragma unroll
+            for (int k = 0; k < LIN_ROWS; ++k) {
+                const float v = warp_sum(acc[k]);
+                if (lane == k) mine = v;
+            }
+            const int r = r0 + lane;
+            if (lane < LIN_ROWS && r < a.rows) {
+                float v = mine + bo;
+                if (a.gelu) v = gelu_tanh_f(v);
+                if (a.res) v += a.res[(size_t)r * a.ldr + o];
+                a.y[(size_t)r * a.ldy + o] = v;
+            }
+        }
+    }
+}
+
+// Row-wise LayerNorm with the biased variance; one warp per row (grid-stride over rows).
+__global__ void __launch_bounds__(256) k_corr_layernorm(const float* __restrict__ x, int ldx,
+                                                        const float* __restrict__ g,
+                                                        const float* __restrict__ b,
+                                                        float* __restrict__ y, int ldy, int rows,
+                                                        int d, float eps) {
+    const int lane = threadIdx.x & 31, nwarps = (int)((gridDim.x * blockDim.x) >> 5);
+    for (int r = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); r < rows; r += nwarps) {
+        const float* xr = x + (size_t)r * ldx;
+        float s = 0.f;
+        for (int i = lane; i < d; i += 32) s += xr[i];
+        const float mean = warp_sum(s) / (float)d;
+        float v = 0.f;
+        for (int i = lane; i < d; i += 32) {
+            const float t = xr[i] - mean;
+            v = fmaf(t, t, v);
+        }
+        const float rstd = 1.f / sqrtf(warp_sum(v) / (float)d + eps);
+        float* yr = y + (size_t)r * ldy;
+        for (int i = lane; i < d; i += 32) yr[i] = (xr[i] - mean) * rstd * g[i] + b[i];
+    }
+}
+
+// Multi-head attention over few keys: query row (b, i) of head h against key rows (b, j),
+// j < nk, every key visible. One warp per (b, h, i); head_dim <= 256, nk <= 64.
+struct AttnSmallArgs {
+    const float* q;
+    int ldq;
+    const float* k;
+    int ldk;
+    const float* v;
+    int ldv;
+    float* o;
+    int ldo;
+    int B, nq, nk, H, Dh;
+    float scale;
+};
+
+__global__ void __launch_bounds__(256) k_corr_attn(const AttnSmallArgs a) {
+    __shared__ float sp[8][JPI_CORR_MAX_DELTA];
+    const int wib = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int gw = blockIdx.x * 8 + wib;
+    if (gw >= a.B * a.H * a.nq) return;   // whole warps leave; no block barrier follows
+    const int i = gw % a.nq, h = (gw / a.nq) % a.H, b = gw / (a.nq * a.H);
+    const float* qr = a.q + (size_t)(b * a.nq + i) * a.ldq + h * a.Dh;
+    float qf[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+        const int d = lane + 32 * t;
+        qf[t] = d < a.Dh ? qr[d] : 0.f;
+    }
+    float mx = -INFINITY;
+    for (int j = 0; j < a.nk; ++j) {
+        const float* kr = a.k + (size_t)(b * a.nk + j) * a.ldk + h * a.Dh;
+        float s = 0.f;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            const int d = lane + 32 * t;
+            if (d < a.Dh) s = fmaf(qf[t], kr[d], s);
+        }
+        s = warp_sum(s) * a.scale;
+        if (lane == 0) sp[wib][j] = s;
+        mx = fmaxf(mx, s);
+    }
+    __syncwarp();
+    float den = 0.f;
+    for (int j = lane; j < a.nk; j += 32) {
+        const float e = expf(sp[wib][j] - mx);
+        sp[wib][j] = e;
+        den += e;
+    }
+    den = warp_sum(den);
+    __syncwarp();
+    float of[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) of[t] = 0.f;
+    for (int j = 0; j < a.nk; ++j) {
+        const float p = sp[wib][j];
+        const float* vr = a.v + (size_t)(b * a.nk + j) * a.ldv + h * a.Dh;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            const int d = lane + 32 * t;
+            if (d < a.Dh) of[t] = fmaf(p, vr[d], of[t]);
+        }
+    }
+    const float inv = 1.f / den;
+    float* orow = a.o + (size_t)(b * a.nq + i) * a.ldo + h * a.Dh;
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+        const int d = lane + 32 * t;
+        if (d < a.Dh) orow[d] = of[t] * inv;
+    }
+}
+
+// Create time: a[h T' + i][c] = scale * sum_e qc[i][h Dh + e] wk[h Dh + e][c] (the cross-
+// attention's scaled queries mapped into VLM space). Grid (ceil(dv / 256), H).
+template <typename TW>
+__global__ void __launch_bounds__(256) k_corr_qk(const float* __restrict__ qc, const TW* __restrict__ wk,
+                                                 float* __restrict__ qk, int T, int Dh, int d, int dv,
+                                                 float scale) {
+    __shared__ float qs[JPI_MAX_CORRECTION][256];
+    const int h = blockIdx.y, c = blockIdx.x * 256 + threadIdx.x;
+    for (int idx = threadIdx.x; idx < T * Dh; idx += 256)
+        qs[idx / Dh][idx % Dh] = qc[(size_t)(idx / Dh) * d + h * Dh + idx % Dh];
+    __syncthreads();
+    if (c >= dv) return;
+    float acc[JPI_MAX_CORRECTION];
+#pragma unroll
+    for (int i = 0; i < JPI_MAX_CORRECTION; ++i) acc[i] = 0.f;
+    for (int e = 0; e < Dh; ++e) {
+        const float w = to_f(wk[(size_t)(h * Dh + e) * dv + c]);
+#pragma unroll
+        for (int i = 0; i < JPI_MAX_CORRECTION; ++i)
+            if (i < T) acc[i] = fmaf(qs[i][e], w, acc[i]);
+    }
+#pragma unroll
+    for (int i = 0; i < JPI_MAX_CORRECTION; ++i)
+        if (i < T) qk[((size_t)h * T + i) * dv + c] = acc[i] * scale;
+}
+
+// s[b][m][j] = sum_c qk[m][c] hv[b][j][c] for m < M, j < T. Grid (ceil(T / 32), B): 32 tokens per
+// CTA, warp w holds rows w, w + 8, ..., the c range staged 32 at a time.
+template <typename THV>
+__global__ void __launch_bounds__(256) k_corr_scores(const float* __restrict__ qk, const THV* __restrict__ hv,
+                                                     float* __restrict__ s, int M, int T, int dv) {
+    __shared__ float as[CORR_MAX_M][33];
+    __shared__ float bs[32][33];
+    const int b = blockIdx.y, j0 = blockIdx.x * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    float acc[CORR_MAX_M / 8];
+#pragma unroll
+    for (int r = 0; r < CORR_MAX_M / 8; ++r) acc[r] = 0.f;
+    const THV* hb = hv + (size_t)b * T * dv;
+    for (int c0 = 0; c0 < dv; c0 += 32) {
+        for (int idx = threadIdx.x; idx < M * 32; idx += 256) {
+            const int m = idx >> 5, kk = idx & 31;
+            as[m][kk] = c0 + kk < dv ? qk[(size_t)m * dv + c0 + kk] : 0.f;
+        }
+        for (int idx = threadIdx.x; idx < 32 * 32; idx += 256) {
+            const int t = idx >> 5, kk = idx & 31, j = j0 + t;
+            bs[t][kk] = (j < T && c0 + kk < dv) ? to_f(hb[(size_t)j * dv + c0 + kk]) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int kk = 0; kk < 32; ++kk) {
+            const float bv = bs[tx][kk];
+#pragma unroll
+            for (int r = 0; r < CORR_MAX_M / 8; ++r) {
+                const int m = ty + 8 * r;
+                if (m < M) acc[r] = fmaf(as[m][kk], bv, acc[r]);
+            }
+        }
+        __syncthreads();
+    }
+    const int j = j0 + tx;
+    if (j < T)
+#pragma unroll
+        for (int r = 0; r < CORR_MAX_M / 8; ++r) {
+            const int m = ty + 8 * r;
+            if (m < M) s[((size_t)b * M + m) * T + j] = acc[r];
+        }
+}
+
+// In-place softmax of each row of length n; one warp per row (grid-stride over rows).
+__global__ void __launch_bounds__(256) k_corr_softmax(float* __restrict__ s, int rows, int n) {
+    const int lane = threadIdx.x & 31, nwarps = (int)((gridDim.x * blockDim.x) >> 5);
+    for (int r = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); r < rows; r += nwarps) {
+        float* row = s + (size_t)r * n;
+        float mx = -INFINITY;
+        for (int j = lane; j < n; j += 32) mx = fmaxf(mx, row[j]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        float den = 0.f;
+        for (int j = lane; j < n; j += 32) {
+            const float e = expf(row[j] - mx);
+            row[j] = e;
+            den += e;
+        }
+        const float inv = 1.f / warp_sum(den);
+        for (int j = lane; j < n; j += 32) row[j] *= inv;
+    }
+}
+
+// g[b][m][c] = sum_j p[b][m][j] hv[b][j][c]. Grid (ceil(dv / 256), ceil(M / 16), B): one column
+// per thread, 16 rows per CTA, the probabilities staged 64 tokens at a time.
+template <typename THV>
+__global__ void __launch_bounds__(256) k_corr_wsum(const float* __restrict__ p, const THV* __restrict__ hv,
+                                                   float* __restrict__ g, int M, int T, int dv) {
+    __shared__ float ps[16][64];
+    const int b = blockIdx.z, m0 = blockIdx.y * 16, c = blockIdx.x * 256 + threadIdx.x;
+    float acc[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r) acc[r] = 0.f;
+    const THV* hb = hv + (size_t)b * T * dv;
+    for (int j0 = 0; j0 < T; j0 += 64) {
+        for (int idx = threadIdx.x; idx < 16 * 64; idx += 256) {
+            const int r = idx >> 6, jj = idx & 63;
+            ps[r][jj] = (m0 + r < M && j0 + jj < T) ? p[((size_t)b * M + m0 + r) * T + j0 + jj] : 0.f;
+        }
+        __syncthreads();
+        if (c < dv) {
+            const int jn = T - j0 < 64 ? T - j0 : 64;
+            for (int jj = 0; jj < jn; ++jj) {
+                const float hvv = to_f(hb[(size_t)(j0 + jj) * dv + c]);
+#pragma unroll
+                for (int r = 0; r < 16; ++r) acc[r] = fmaf(ps[r][jj], hvv, acc[r]);
+            }
+        }
+        __syncthreads();
+    }
+    if (c < dv)
+#pragma unroll
+        for (int r = 0; r < 16; ++r)
+            if (m0 + r < M) g[((size_t)b * M + m0 + r) * dv + c] = acc[r];
+}
+
+// y[(b n + k)][c] += pos[k][c] for b < B, k < n, c < d.
+__global__ void k_corr_add_pos(float* __restrict__ y, const float* __restrict__ pos, int B, int n, int d) {
+    const long long total = (long long)B * n * d;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int c = (int)(idx % d);
+        const int k = (int)((idx / d) % n);
+        y[idx] += pos[(size_t)k * d + c];
+    }
+}
+
+// xj[(b T' + i)][0 .. d) = state[b][i][.], xj[(b T' + i)][d .. 2d) = summary[b][.].
+__global__ void k_corr_join(const float* __restrict__ state, const float* __restrict__ summary,
+                            float* __restrict__ xj, int B, int T, int d) {
+    const long long total = (long long)B * T * 2 * d;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int c = (int)(idx % (2 * d));
+        const long long r = idx / (2 * d);   // b T' + i
+        const int b = (int)(r / T);
+        xj[idx] = c < d ? state[r * d + c] : summary[(size_t)b * d + (c - d)];
+    }
+}
+
+// conf[b] = w . mean_i u[b T' + i] + bias; one warp per request (grid-stride over requests).
+__global__ void k_corr_confidence(const float* __restrict__ u, const float* __restrict__ w,
+                                  const float* __restrict__ bias, float* __restrict__ conf, int B,
+                                  int T, int d) {
+    const int lane = threadIdx.x & 31, nwarps = (int)((gridDim.x * blockDim.x) >> 5);
+    for (int b = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); b < B; b += nwarps) {
+        float s = 0.f;
+        for (int c = lane; c < d; c += 32) {
+            float m = 0.f;
+            for (int i = 0; i < T; ++i) m += u[((size_t)b * T + i) * d + c];
+            s = fmaf(w[c], m / (float)T, s);
+        }
+        s = warp_sum(s);
+        if (lane == 0) conf[b] = s + bias[0];
+    }
+}
+
+__global__ void k_corr_cast(const float* __restrict__ src, __nv_bfloat16* __restrict__ dst, long long n) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
+         i += (long long)gridDim.x * blockDim.x)
+        dst[i] = __float2bfloat16_rn(src[i]);
+}
+
+// dst[r n + i] = src[i] for r < reps, i < n. src may be the start of dst: the first n elements are
+// rewritten with their own values.
+__global__ void k_corr_repeat(const float* src, float* dst, long long n, int reps) {
+    const long long total = n * reps;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x)
+        dst[i] = src[i % n];
+}
+
+int grid_for(long long threads, int block = 256, int cap = 8192) {
+    long long g = (threads + block - 1) / block;
+    if (g < 1) g = 1;
+    if (g > cap) g = cap;
+    return (int)g;
+}
+
+// Device copy of one block: q/k/v rows packed as [wq; wk; wv] ([3d][d]) with [bq; bk; bv].
+struct BlockDev {
+    float *ln1_w = nullptr, *ln1_b = nullptr;
+    void* wqkv = nullptr;
+    float* bqkv = nullptr;
+    void* wo = nullptr;
+    float* bo = nullptr;
+    float *ln2_w = nullptr, *ln2_b = nullptr;
+    void* w1 = nullptr;
+    float* b1 = nullptr;
+    void* w2 = nullptr;
+    float* b2 = nullptr;
+};
+
+}  // namespace
+
+struct jpi_corr_handle {
+    jpi_corr_config cfg;
+    bool bf16 = true;
+    int d = 0, H = 0, Dh = 0, F = 0, dv = 0, Ti = 0, A = 0, Dm = 0, J = 0, B = 0, Tm = 0, M = 0;
+    std::vector<void*> allocs;
+    size_t bytes = 0;
+    float* staging = nullptr;   // fp32 device staging for host weights
+    size_t staging_elems = 0;
+
+    // Weights.
+    float* qf_query = nullptr;   // [T'][d]
+    BlockDev qf_sa;
+    float *qf_ln2_w = nullptr, *qf_ln2_b = nullptr;
+    void *qf_ca_wq = nullptr, *qf_ca_wk = nullptr, *qf_ca_wv = nullptr, *qf_ca_wo = nullptr;
+    float *qf_ca_bq = nullptr, *qf_ca_bv = nullptr, *qf_ca_bo = nullptr;
+    float *qf_ln3_w = nullptr, *qf_ln3_b = nullptr, *qf_lnf_w = nullptr, *qf_lnf_b = nullptr;
+    void *qf_w1 = nullptr, *qf_w2 = nullptr;
+    float *qf_b1 = nullptr, *qf_b2 = nullptr;
+    void *act_w1 = nullptr, *act_w2 = nullptr;
+    float *act_b1 = nullptr, *act_b2 = nullptr, *act_pos = nullptr;
+    BlockDev ab;
+    void* fuse_w = nullptr;
+    float* fuse_b = nullptr;
+    std::vector<BlockDev> jb;
+    float *head_ln_w = nullptr, *head_ln_b = nullptr;
+    void* corr_w = nullptr;
+    float *corr_b = nullptr, *conf_w = nullptr, *conf_b = nullptr;
+
+    // Weight-only values computed at create time.
+    float* x1b = nullptr;   // [B T'][d] the queries after their self-attention, per request slot
+    float* qk = nullptr;    // [H T'][dv] cross-attention queries mapped into VLM space (scaled)
+
+    // Activations (fp32).
+    float *t1 = nullptr, *xa = nullptr, *ua = nullptr, *kva = nullptr;   // [B Dm][d], kva [B Dm][2d]
+    float *ql = nullptr, *ol = nullptr, *xl = nullptr, *ul = nullptr;    // [B][d]
+    float* hidl = nullptr;                                                // [B][F]
+    float *xj = nullptr, *xf = nullptr, *u = nullptr, *qkv = nullptr, *o = nullptr;   // [B T'] rows
+    float* hid = nullptr;                                                 // [B T'][F]
+    float *sc = nullptr, *gs = nullptr;                                   // [B][M][Tm], [B][M][dv]
+    float* conf_scratch = nullptr;                                        // [B]
+};
+
+namespace {
+
+template <typename T>
+jpi_status corr_alloc(jpi_corr_handle* h, T** p, size_t count) {
+    void* q = nullptr;
+    const size_t bytes = count * sizeof(T);
+    const cudaError_t e = cudaMalloc(&q, bytes ? bytes : 16);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return cfail(JPI_ERR_OOM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+    }
+    h->allocs.push_back(q);
+    h->bytes += bytes;
+    *p = static_cast<T*>(q);
+    return JPI_OK;
+}
+
+// Copies an fp32 tensor of n elements (host or device) to dst: fp32 as is, or rounded to bf16.
+jpi_status put(jpi_corr_handle* h, bool on_device, void* dst, bool to_bf16, const float* src, size_t n,
+               const char* name) {
+    if (!src) return cfail(JPI_ERR_INVALID_ARG, "weight tensor %s is NULL", name);
+    const float* dsrc = src;
+    if (!on_device) {
+        if (!to_bf16) {
+            JPI_CUDA_TRY(cudaMemcpy(dst, src, n * sizeof(float), cudaMemcpyHostToDevice));
+            return JPI_OK;
+        }
+        JPI_CUDA_TRY(cudaMemcpy(h->staging, src, n * sizeof(float), cudaMemcpyHostToDevice));
+        dsrc = h->staging;
+    }
+    if (to_bf16) {
+        k_corr_cast<<<grid_for((long long)n), 256>>>(dsrc, static_cast<__nv_bfloat16*>(dst), (long long)n);
+        JPI_CUDA_TRY(cudaGetLastError());
+    } else {
+        JPI_CUDA_TRY(cudaMemcpy(dst, dsrc, n * sizeof(float), cudaMemcpyDeviceToDevice));
+    }
+    return JPI_OK;
+}
+
+// A weight matrix (stored bf16 or fp32) and a vector (fp32) of the handle.
+jpi_status put_mat(jpi_corr_handle* h, bool dev, void** dst, const float* src, size_t n, const char* name) {
+    if (h->bf16) {
+        __nv_bfloat16* p = nullptr;
+        JPI_TRY(corr_alloc(h, &p, n));
+        *dst = p;
+    } else {
+        float* p = nullptr;
+        JPI_TRY(corr_alloc(h, &p, n));
+        *dst = p;
+    }
+    return put(h, dev, *dst, h->bf16, src, n, name);
+}
+
+jpi_status put_vec(jpi_corr_handle* h, bool dev, float** dst, const float* src, size_t n, const char* name) {
+    JPI_TRY(corr_alloc(h, dst, n));
+    return put(h, dev, *dst, false, src, n, name);
+}
+
+size_t tw_bytes(const jpi_corr_handle* h) { return h->bf16 ? 2 : 4; }
+const void* tw_rows(const jpi_corr_handle* h, const void* base, size_t row, size_t in) {
+    return static_cast<const char*>(base) + row * in * tw_bytes(h);
+}
+
+jpi_status put_block(jpi_corr_handle* h, bool dev, BlockDev* out, const jpi_corr_block& b, bool with_mlp,
+                     const char* name) {
+    const size_t d = (size_t)h->d, F = (size_t)h->F;
+    char nm[64];
+    auto N = [&](const char* f) {
+        snprintf(nm, sizeof(nm), "%s.%s", name, f);
+        return nm;
+    };
+    JPI_TRY(put_vec(h, dev, &out->ln1_w, b.ln1_w, d, N("ln1_w")));
+    JPI_TRY(put_vec(h, dev, &out->ln1_b, b.ln1_b, d, N("ln1_b")));
+    if (h->bf16) {
+        __nv_bfloat16* p = nullptr;
+        JPI_TRY(corr_alloc(h, &p, 3 * d * d));
+        out->wqkv = p;
+    } else {
+        float* p = nullptr;
+        JPI_TRY(corr_alloc(h, &p, 3 * d * d));
+        out->wqkv = p;
+    }
+    char* wq = static_cast<char*>(out->wqkv);
+    JPI_TRY(put(h, dev, wq, h->bf16, b.wq, d * d, N("wq")));
+    JPI_TRY(put(h, dev, wq + d * d * tw_bytes(h), h->bf16, b.wk, d * d, N("wk")));
+    JPI_TRY(put(h, dev, wq + 2 * d * d * tw_bytes(h), h->bf16, b.wv, d * d, N("wv")));
+    JPI_TRY(corr_alloc(h, &out->bqkv, 3 * d));
+    JPI_TRY(put(h, dev, out->bqkv, false, b.bq, d, N("bq")));
+    JPI_TRY(put(h, dev, out->bqkv + d, false, b.bk, d, N("bk")));
+    JPI_TRY(put(h, dev, out->bqkv + 2 * d, false, b.bv, d, N("bv")));
+    JPI_TRY(put_mat(h, dev, &out->wo, b.wo, d * d, N("wo")));
+    JPI_TRY(put_vec(h, dev, &out->bo, b.bo, d, N("bo")));
+    if (with_mlp) {
+        JPI_TRY(put_vec(h, dev, &out->ln2_w, b.ln2_w, d, N("ln2_w")));
+        JPI_TRY(put_vec(h, dev, &out->ln2_b, b.ln2_b, d, N("ln2_b")));
+        JPI_TRY(put_mat(h, dev, &out->w1, b.w1, F * d, N("w1")));
+        JPI_TRY(put_vec(h, dev, &out->b1, b.b1, F, N("b1")));
+        JPI_TRY(put_mat(h, dev, &out->w2, b.w2, d * F, N("w2")));
+        JPI_TRY(put_vec(h, dev, &out->b2, b.b2, d, N("b2")));
+    }
+    return JPI_OK;
+}
+
+// ---------------------------------------------------------------- launchers
+
+jpi_status linear(const jpi_corr_handle* h, cudaStream_t st, const float* x, int ldx, const void* w,
+                  const float* bias, const float* res, int ldr, float* y, int ldy, int rows, int in,
+                  int out, bool gelu, int hs_items = 0) {
+    if (rows <= 0 || out <= 0) return JPI_OK;
+    LinArgs a;
+    a.x = x;
+    a.ldx = ldx;
+    a.w = w;
+    a.bias = bias;
+    a.res = res;
+    a.ldr = ldr;
+    a.y = y;
+    a.ldy = ldy;
+    a.rows = rows;
+    a.in = in;
+    a.out = out;
+    a.gelu = gelu ? 1 : 0;
+    a.hs_items = hs_items;
+    a.hs_heads = h->H;
+    a.hs_dh = h->Dh;
+    const bool vec = in % 4 == 0 && ldx % 4 == 0 && ((uintptr_t)x & 15) == 0 &&
+                     ((uintptr_t)w & (h->bf16 ? 7 : 15)) == 0;
+    const int blocks = grid_for((long long)out * 32, 256, 4096);
+    if (h->bf16) {
+        if (vec) k_corr_linear<__nv_bfloat16, true><<<blocks, 256, 0, st>>>(a);
+        else k_corr_linear<__nv_bfloat16, false><<<blocks, 256, 0, st>>>(a);
+    } else {
+        if (vec) k_corr_linear<float, true><<<blocks, 256, 0, st>>>(a);
+        else k_corr_linear<float, false><<<blocks, 256, 0, st>>>(a);
+    }
+    JPI_CUDA_TRY(cudaGetLastError());
+    return JPI_OK;
+}
+
+jpi_status layernorm(const jpi_corr_handle* h, cudaStream_t st, const float* x, int ldx, const float* g,
+                     const float* b, float* y, int ldy, int rows) {
+    if (rows <= 0) return JPI_OK;
+    k_corr_layernorm<<<grid_for((long long)rows * 32), 256, 0, st>>>(x, ldx, g, b, y, ldy, rows, h->d,
+                                                                     h->cfg.ln_eps);
+    JPI_CUDA_TRY(cudaGetLastError());
+    return JPI_OK;
+}
+
+jpi_status attention(const jpi_corr_handle* h, cudaStream_t st, const float* q, int ldq, const float* k,
+                     int ldk, const float* v, int ldv, float* o, int ldo, int B, int nq, int nk) {
+    AttnSmallArgs a;
+    a.q = q;
+    a.ldq = ldq;
+    a.k = k;
+    a.ldk = ldk;
+    a.v = v;
+    a.ldv = ldv;
+    a.o = o;
+    a.ldo = ldo;
+    a.B = B;
+    a.nq = nq;
+    a.nk = nk;
+    a.H = h->H;
+    a.Dh = h->Dh;
+    a.scale = 1.f / sqrtf((float)h->Dh);
+    const long long warps = (long long)B * h->H * nq;
+    k_corr_attn<<<(int)((warps + 7) / 8), 256, 0, st>>>(a);
+    JPI_CUDA_TRY(cudaGetLastError());
+    return JPI_OK;
+}
+
+// One pre-LN block over `rows` rows of x (rows = B n, n tokens per request), in place.
+jpi_status block(const jpi_corr_handle* h, cudaStream_t st, const BlockDev& w, float* x, int B, int n) {
+    const int d = h->d, rows = B * n;
+    JPI_TRY(layernorm(h, st, x, d, w.ln1_w, w.ln1_b, h->u, d, rows));
+    JPI_TRY(linear(h, st, h->u, d, w.wqkv, w.bqkv, nullptr, 0, h->qkv, 3 * d, rows, d, 3 * d, false));
+    JPI_TRY(attention(h, st, h->qkv, 3 * d, h->qkv + d, 3 * d, h->qkv + 2 * d, 3 * d, h->o, d, B, n, n));
+    JPI_TRY(linear(h, st, h->o, d, w.wo, w.bo, x, d, x, d, rows, d, d, false));
+    JPI_TRY(layernorm(h, st, x, d, w.ln2_w, w.ln2_b, h->u, d, rows));
+    JPI_TRY(linear(h, st, h->u, d, w.w1, w.b1, nullptr, 0, h->hid, h->F, rows, d, h->F, true));
+    JPI_TRY(linear(h, st, h->hid, h->F, w.w2, w.b2, x, d, x, d, rows, h->F, d, false));
+    return JPI_OK;
+}
+
+// Weight-only part of the compressor: x1 = q0 + SA(LN1 q0) for the learned queries q0 (one copy
+// per request slot), and the cross-attention queries of LN2 x1 mapped into VLM space.
+jpi_status prepare(jpi_corr_handle* h, cudaStream_t st) {
+    const int d = h->d, T = h->Ti;
+    const BlockDev& sa = h->qf_sa;
+    JPI_TRY(layernorm(h, st, h->qf_query, d, sa.ln1_w, sa.ln1_b, h->u, d, T));
+    JPI_TRY(linear(h, st, h->u, d, sa.wqkv, sa.bqkv, nullptr, 0, h->qkv, 3 * d, T, d, 3 * d, false));
+    JPI_TRY(attention(h, st, h->qkv, 3 * d, h->qkv + d, 3 * d, h->qkv + 2 * d, 3 * d, h->o, d, 1, T, T));
+    JPI_TRY(linear(h, st, h->o, d, sa.wo, sa.bo, h->qf_query, d, h->x1b, d, T, d, d, false));
+    JPI_TRY(layernorm(h, st, h->x1b, d, h->qf_ln2_w, h->qf_ln2_b, h->u, d, T));
+    JPI_TRY(linear(h, st, h->u, d, h->qf_ca_wq, h->qf_ca_bq, nullptr, 0, h->o, d, T, d, d, false));
+    const dim3 grid((unsigned)((h->dv + 255) / 256), (unsigned)h->H);
+    const float scale = 1.f / sqrtf((float)h->Dh);
+    if (h->bf16)
+        k_corr_qk<__nv_bfloat16><<<grid, 256, 0, st>>>(h->o, static_cast<const __nv_bfloat16*>(h->qf_ca_wk),
+                                                        h->qk, T, h->Dh, d, h->dv, scale);
+    else
+        k_corr_qk<float><<<grid, 256, 0, st>>>(h->o, static_cast<const float*>(h->qf_ca_wk), h->qk, T, h->Dh,
+                                               d, h->dv, scale);
+    JPI_CUDA_TRY(cudaGetLastError());
+    const long long n = (long long)T * d;
+    k_corr_repeat<<<grid_for(n * h->B), 256, 0, st>>>(h->x1b, h->x1b, n, h->B);
+    JPI_CUDA_TRY(cudaGetLastError());
+    return JPI_OK;
+}
+
+jpi_status check_corr_config(const jpi_corr_config* c) {
+    if (c->width < 32 || c->width % 32 || c->width > 16384)
+        return cfail(JPI_ERR_INVALID_ARG, "width must be a multiple of 32 in [32, 16384]");
+    if (c->head_dim < 32 || c->head_dim % 32 || c->head_dim > 256)
+        return cfail(JPI_ERR_UNSUPPORTED, "head_dim must be a multiple of 32 and at most 256");
+    if (c->n_heads < 1 || c->n_heads * c->head_dim != c->width)
+        return cfail(JPI_ERR_INVALID_ARG, "n_heads * head_dim must equal width");
+    if (c->mlp_dim < 1 || c->d_vlm < 1 || c->action_dim < 1)
+        return cfail(JPI_ERR_INVALID_ARG, "mlp_dim, d_vlm and action_dim must be >= 1");
+    if (c->n_items < 1 || c->n_items > JPI_MAX_CORRECTION)
+        return cfail(JPI_ERR_UNSUPPORTED, "n_items must be in [1, %d]", JPI_MAX_CORRECTION);
+    if (c->n_heads * c->n_items > CORR_MAX_M)
+        return cfail(JPI_ERR_UNSUPPORTED, "n_heads * n_items must be at most %d", CORR_MAX_M);
+    if (c->max_delta < 1 || c->max_delta > JPI_CORR_MAX_DELTA)
+        return cfail(JPI_ERR_UNSUPPORTED, "max_delta must be in [1, %d]", JPI_CORR_MAX_DELTA);
+    if (c->n_joint < 0 || c->n_joint > 8) return cfail(JPI_ERR_UNSUPPORTED, "n_joint must be in [0, 8]");
+    if (c->max_batch < 1 || c->max_batch > 65535 || c->max_vlm_tokens < 1)
+        return cfail(JPI_ERR_INVALID_ARG, "max_batch must be in [1, 65535] and max_vlm_tokens >= 1");
+    if ((long long)c->max_batch * c->n_heads * c->n_items * c->max_vlm_tokens > (1ll << 31))
+        return cfail(JPI_ERR_UNSUPPORTED, "max_batch * n_heads * n_items * max_vlm_tokens is too large");
+    if (c->precision != JPI_BF16 && c->precision != JPI_FP32)
+        return cfail(JPI_ERR_INVALID_ARG, "unknown precision %d", (int)c->precision);
+    if (!(c->ln_eps >= 0.f)) return cfail(JPI_ERR_INVALID_ARG, "ln_eps must be >= 0");
+    return JPI_OK;
+}
+
+jpi_status setup(jpi_corr_handle* h, const jpi_corr_config* c, const jpi_corr_weights* w) {
+    h->cfg = *c;
+    h->bf16 = c->precision == JPI_BF16;
+    h->d = c->width;
+    h->H = c->n_heads;
+    h->Dh = c->head_dim;
+    h->F = c->mlp_dim;
+    h->dv = c->d_vlm;
+    h->Ti = c->n_items;
+    h->A = c->action_dim;
+    h->Dm = c->max_delta;
+    h->J = c->n_joint;
+    h->B = c->max_batch;
+    h->Tm = c->max_vlm_tokens;
+    h->M = h->H * h->Ti;
+    const size_t d = (size_t)h->d, F = (size_t)h->F, dv = (size_t)h->dv, T = (size_t)h->Ti;
+    const size_t B = (size_t)h->B, Dm = (size_t)h->Dm, A = (size_t)h->A, M = (size_t)h->M;
+    const bool dev = w->on_device != 0;
+    if (!dev) {
+        size_t m = d * d;
+        for (size_t v : {F * d, d * dv, Dm * d, 2 * d * d, T * d, d * A}) m = v > m ? v : m;
+        JPI_TRY(corr_alloc(h, &h->staging, m));
+        h->staging_elems = m;
+    }
+
+    // Q-Former compressor.
+    JPI_TRY(put_vec(h, dev, &h->qf_query, w->qf_query, T * d, "qf_query"));
+    JPI_TRY(put_block(h, dev, &h->qf_sa, w->qf_sa, false, "qf_sa"));
+    JPI_TRY(put_vec(h, dev, &h->qf_ln2_w, w->qf_ln2_w, d, "qf_ln2_w"));
+    JPI_TRY(put_vec(h, dev, &h->qf_ln2_b, w->qf_ln2_b, d, "qf_ln2_b"));
+    JPI_TRY(put_mat(h, dev, &h->qf_ca_wq, w->qf_ca_wq, d * d, "qf_ca_wq"));
+    JPI_TRY(put_vec(h, dev, &h->qf_ca_bq, w->qf_ca_bq, d, "qf_ca_bq"));
+    JPI_TRY(put_mat(h, dev, &h->qf_ca_wk, w->qf_ca_wk, d * dv, "qf_ca_wk"));
+    // qf_ca_bk adds the same amount to every score of a query; softmax cancels it.
+    JPI_TRY(put_mat(h, dev, &h->qf_ca_wv, w->qf_ca_wv, d * dv, "qf_ca_wv"));
+    JPI_TRY(put_vec(h, dev, &h->qf_ca_bv, w->qf_ca_bv, d, "qf_ca_bv"));
+    JPI_TRY(put_mat(h, dev, &h->qf_ca_wo, w->qf_ca_wo, d * d, "qf_ca_wo"));
+    JPI_TRY(put_vec(h, dev, &h->qf_ca_bo, w->qf_ca_bo, d, "qf_ca_bo"));
+    JPI_TRY(put_vec(h, dev, &h->qf_ln3_w, w->qf_ln3_w, d, "qf_ln3_w"));
+    JPI_TRY(put_vec(h, dev, &h->qf_ln3_b, w->qf_ln3_b, d, "qf_ln3_b"));
+    JPI_TRY(put_mat(h, dev, &h->qf_w1, w->qf_mlp_w1, F * d, "qf_mlp_w1"));
+    JPI_TRY(put_vec(h, dev, &h->qf_b1, w->qf_mlp_b1, F, "qf_mlp_b1"));
+    JPI_TRY(put_mat(h, dev, &h->qf_w2, w->qf_mlp_w2, d * F, "qf_mlp_w2"));
+    JPI_TRY(put_vec(h, dev, &h->qf_b2, w->qf_mlp_b2, d, "qf_mlp_b2"));
+    JPI_TRY(put_vec(h, dev, &h->qf_lnf_w, w->qf_lnf_w, d, "qf_lnf_w"));
+    JPI_TRY(put_vec(h, dev, &h->qf_lnf_b, w->qf_lnf_b, d, "qf_lnf_b"));
+    // Action branch, join, joint blocks, heads.
+    JPI_TRY(put_mat(h, dev, &h->act_w1, w->act_w1, d * A, "act_w1"));
+    JPI_TRY(put_vec(h, dev, &h->act_b1, w->act_b1, d, "act_b1"));
+    JPI_TRY(put_mat(h, dev, &h->act_w2, w->act_w2, d * d, "act_w2"));
+    JPI_TRY(put_vec(h, dev, &h->act_b2, w->act_b2, d, "act_b2"));
+    JPI_TRY(put_vec(h, dev, &h->act_pos, w->act_pos, Dm * d, "act_pos"));
+    JPI_TRY(put_block(h, dev, &h->ab, w->ab, true, "ab"));
+    JPI_TRY(put_mat(h, dev, &h->fuse_w, w->fuse_w, d * 2 * d, "fuse_w"));
+    JPI_TRY(put_vec(h, dev, &h->fuse_b, w->fuse_b, d, "fuse_b"));
+    h->jb.resize((size_t)h->J);
+    for (int i = 0; i < h->J; ++i) {
+        char nm[16];
+        snprintf(nm, sizeof(nm), "jb%d", i);
+        JPI_TRY(put_block(h, dev, &h->jb[(size_t)i], w->jb[i], true, nm));
+    }
+    JPI_TRY(put_vec(h, dev, &h->head_ln_w, w->head_ln_w, d, "head_ln_w"));
+    JPI_TRY(put_vec(h, dev, &h->head_ln_b, w->head_ln_b, d, "head_ln_b"));
+    JPI_TRY(put_mat(h, dev, &h->corr_w, w->corr_w, d * d, "corr_w"));
+    JPI_TRY(put_vec(h, dev, &h->corr_b, w->corr_b, d, "corr_b"));
+    JPI_TRY(put_vec(h, dev, &h->conf_w, w->conf_w, d, "conf_w"));
+    JPI_TRY(put_vec(h, dev, &h->conf_b, w->conf_b, 1, "conf_b"));
+
+    // Weight-only values and activations.
+    JPI_TRY(corr_alloc(h, &h->x1b, B * T * d));
+    JPI_TRY(corr_alloc(h, &h->qk, M * dv));
+    JPI_TRY(corr_alloc(h, &h->t1, B * Dm * d));
+    JPI_TRY(corr_alloc(h, &h->xa, B * Dm * d));
+    JPI_TRY(corr_alloc(h, &h->ua, B * Dm * d));
+    JPI_TRY(corr_alloc(h, &h->kva, B * Dm * 2 * d));
+    JPI_TRY(corr_alloc(h, &h->ql, B * d));
+    JPI_TRY(corr_alloc(h, &h->ol, B * d));
+    JPI_TRY(corr_alloc(h, &h->xl, B * d));
+    JPI_TRY(corr_alloc(h, &h->ul, B * d));
+    JPI_TRY(corr_alloc(h, &h->hidl, B * F));
+    JPI_TRY(corr_alloc(h, &h->xj, B * T * 2 * d));
+    JPI_TRY(corr_alloc(h, &h->xf, B * T * d));
+    JPI_TRY(corr_alloc(h, &h->u, B * T * d));
+    JPI_TRY(corr_alloc(h, &h->qkv, B * T * 3 * d));
+    JPI_TRY(corr_alloc(h, &h->o, B * T * d));
+    JPI_TRY(corr_alloc(h, &h->hid, B * T * F));
+    JPI_TRY(corr_alloc(h, &h->sc, B * M * (size_t)h->Tm));
+    JPI_TRY(corr_alloc(h, &h->gs, B * M * dv));
+    JPI_TRY(corr_alloc(h, &h->conf_scratch, B));
+
+    JPI_TRY(prepare(h, nullptr));
+    JPI_CUDA_TRY(cudaStreamSynchronize(nullptr));
+    return JPI_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+JPI_API jpi_status jpi_corr_create(const jpi_corr_config* cfg, const jpi_corr_weights* w,
+                                   jpi_corr_handle** out) {
+    jpi::clear_error();
+    if (!out) return cfail(JPI_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (!cfg || !w) return cfail(JPI_ERR_INVALID_ARG, "config or weights is NULL");
+    JPI_TRY(check_corr_config(cfg));
+    if (cfg->n_joint > 0 && !w->jb) return cfail(JPI_ERR_INVALID_ARG, "joint blocks (jb) are NULL");
+    jpi_corr_handle* h = new (std::nothrow) jpi_corr_handle();
+    if (!h) return cfail(JPI_ERR_OOM, "host allocation failed");
+    const jpi_status s = setup(h, cfg, w);
+    if (s != JPI_OK) {
+        cudaStreamSynchronize(nullptr);   // let any conversion in flight finish before its buffers go
+        cudaGetLastError();
+        for (void* p : h->allocs) cudaFree(p);
+        delete h;
+        return s;
+    }
+    *out = h;
+    return JPI_OK;
+}
+
+JPI_API jpi_status jpi_corr_destroy(jpi_corr_handle* h) {
+    jpi::clear_error();
+    if (!h) return JPI_OK;
+    for (void* p : h->allocs) cudaFree(p);
+    delete h;
+    return JPI_OK;
+}
+
+JPI_API jpi_status jpi_corr_compress(jpi_corr_handle* h, const void* h_vlm, int vlm_is_fp32, int batch,
+                                     int n_tokens, float* out_state, void* stream) {
+    jpi::clear_error();
+    if (!h) return cfail(JPI_ERR_INVALID_ARG, "handle is NULL");
+    if (!h_vlm || !out_state) return cfail(JPI_ERR_INVALID_ARG, "NULL input or output");
+    if (batch < 1 || n_tokens < 1) return cfail(JPI_ERR_INVALID_ARG, "batch and n_tokens must be >= 1");
+    if (batch > h->B || n_tokens > h->Tm)
+        return cfail(JPI_ERR_SHAPE, "batch %d / n_tokens %d exceed the maxima %d / %d", batch, n_tokens, h->B,
+                     h->Tm);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int d = h->d, T = h->Ti, M = h->M, dv = h->dv, rows = batch * T;
+    const dim3 gs((unsigned)((n_tokens + 31) / 32), (unsigned)batch);
+    const dim3 gw((unsigned)((dv + 255) / 256), (unsigned)((M + 15) / 16), (unsigned)batch);
+    if (vlm_is_fp32) {
+        const float* hv = static_cast<const float*>(h_vlm);
+        k_corr_scores<float><<<gs, 256, 0, st>>>(h->qk, hv, h->sc, M, n_tokens, dv);
+        k_corr_softmax<<<grid_for((long long)batch * M * 32), 256, 0, st>>>(h->sc, batch * M, n_tokens);
+        k_corr_wsum<float><<<gw, 256, 0, st>>>(h->sc, hv, h->gs, M, n_tokens, dv);
+    } else {
+        const __nv_bfloat16* hv = static_cast<const __nv_bfloat16*>(h_vlm);
+        k_corr_scores<__nv_bfloat16><<<gs, 256, 0, st>>>(h->qk, hv, h->sc, M, n_tokens, dv);
+        k_corr_softmax<<<grid_for((long long)batch * M * 32), 256, 0, st>>>(h->sc, batch * M, n_tokens);
+        k_corr_wsum<__nv_bfloat16><<<gw, 256, 0, st>>>(h->sc, hv, h->gs, M, n_tokens, dv);
+    }
+    JPI_CUDA_TRY(cudaGetLastError());
+    // out_hi = W_v,h g_hi + b_v (head-select rows of gs), then the output projection onto the
+    // queries' residual, the MLP, and the output LayerNorm.
+    JPI_TRY(linear(h, st, h->gs, dv, h->qf_ca_wv, h->qf_ca_bv, nullptr, 0, h->o, d, rows, dv, d, false, T));
+    JPI_TRY(linear(h, st, h->o, d, h->qf_ca_wo, h->qf_ca_bo, h->x1b, d, h->xf, d, rows, d, d, false));
+    JPI_TRY(layernorm(h, st, h->xf, d, h->qf_ln3_w, h->qf_ln3_b, h->u, d, rows));
+    JPI_TRY(linear(h, st, h->u, d, h->qf_w1, h->qf_b1, nullptr, 0, h->hid, h->F, rows, d, h->F, true));
+    JPI_TRY(linear(h, st, h->hid, h->F, h->qf_w2, h->qf_b2, h->xf, d, h->xf, d, rows, h->F, d, false));
+    JPI_TRY(layernorm(h, st, h->xf, d, h->qf_lnf_w, h->qf_lnf_b, out_state, d, rows));
+    return JPI_OK;
+}
+
+JPI_API jpi_status jpi_corr_predict(jpi_corr_handle* h, const float* state, const float* actions, int batch,
+                                    int delta, float* out_state, float* out_confidence, void* stream) {
+    jpi::clear_error();
+    if (!h) return cfail(JPI_ERR_INVALID_ARG, "handle is NULL");
+    if (!state || !actions || !out_state) return cfail(JPI_ERR_INVALID_ARG, "NULL input or output");
+    if (batch < 1 || delta < 1) return cfail(JPI_ERR_INVALID_ARG, "batch and delta must be >= 1");
+    if (batch > h->B || delta > h->Dm)
+        return cfail(JPI_ERR_SHAPE, "batch %d / delta %d exceed the maxima %d / %d", batch, delta, h->B, h->Dm);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int d = h->d, T = h->Ti, F = h->F, ra = batch * delta, rows = batch * T;
+    const BlockDev& ab = h->ab;
+    // Action tokens: MLP, plus the position row of each action.
+    JPI_TRY(linear(h, st, actions, h->A, h->act_w1, h->act_b1, nullptr, 0, h->t1, d, ra, h->A, d, true));
+    JPI_TRY(linear(h, st, h->t1, d, h->act_w2, h->act_b2, nullptr, 0, h->xa, d, ra, d, d, false));
+    k_corr_add_pos<<<grid_for((long long)ra * d), 256, 0, st>>>(h->xa, h->act_pos, batch, delta, d);
+    JPI_CUDA_TRY(cudaGetLastError());
+    // Block ab, kept at the last action of each request only: keys and values of every action,
+    // the query, attention output, residual and MLP of the last.
+    JPI_TRY(layernorm(h, st, h->xa, d, ab.ln1_w, ab.ln1_b, h->ua, d, ra));
+    JPI_TRY(linear(h, st, h->ua, d, tw_rows(h, ab.wqkv, (size_t)d, (size_t)d), ab.bqkv + d, nullptr, 0, h->kva,
+                   2 * d, ra, d, 2 * d, false));
+    const size_t last = (size_t)(delta - 1) * d;
+    JPI_TRY(linear(h, st, h->ua + last, delta * d, ab.wqkv, ab.bqkv, nullptr, 0, h->ql, d, batch, d, d, false));
+    JPI_TRY(attention(h, st, h->ql, d, h->kva, 2 * d, h->kva + d, 2 * d, h->ol, d, batch, 1, delta));
+    JPI_TRY(linear(h, st, h->ol, d, ab.wo, ab.bo, h->xa + last, delta * d, h->xl, d, batch, d, d, false));
+    JPI_TRY(layernorm(h, st, h->xl, d, ab.ln2_w, ab.ln2_b, h->ul, d, batch));
+    JPI_TRY(linear(h, st, h->ul, d, ab.w1, ab.b1, nullptr, 0, h->hidl, F, batch, d, F, true));
+    JPI_TRY(linear(h, st, h->hidl, F, ab.w2, ab.b2, h->xl, d, h->xl, d, batch, F, d, false));
+    // Join: [compressed token ; action summary] projected back to the module width.
+    k_corr_join<<<grid_for((long long)rows * 2 * d), 256, 0, st>>>(state, h->xl, h->xj, batch, T, d);
+    JPI_CUDA_TRY(cudaGetLastError());
+    JPI_TRY(linear(h, st, h->xj, 2 * d, h->fuse_w, h->fuse_b, nullptr, 0, h->xf, d, rows, 2 * d, d, false));
+    for (int i = 0; i < h->J; ++i) JPI_TRY(block(h, st, h->jb[(size_t)i], h->xf, batch, T));
+    // Heads.
+    JPI_TRY(layernorm(h, st, h->xf, d, h->head_ln_w, h->head_ln_b, h->u, d, rows));
+    JPI_TRY(linear(h, st, h->u, d, h->corr_w, h->corr_b, nullptr, 0, out_state, d, rows, d, d, false));
+    float* conf = out_confidence ? out_confidence : h->conf_scratch;
+    k_corr_confidence<<<grid_for((long long)batch * 32), 256, 0, st>>>(h->u, h->conf_w, h->conf_b, conf, batch,
+                                                                       T, d);
+    JPI_CUDA_TRY(cudaGetLastError());
+    return JPI_OK;
+}
+
+JPI_API jpi_status jpi_corr_memory_usage(const jpi_corr_handle* h, long long* bytes) {
+    jpi::clear_error();
+    if (!h || !bytes) return cfail(JPI_ERR_INVALID_ARG, "handle or bytes is NULL");
+    *bytes = (long long)h->bytes;
+    return JPI_OK;
+}
+
+}  // extern "C"

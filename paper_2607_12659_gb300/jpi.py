@@ -79,9 +79,14 @@ _lib = None
 
 
 def header_symbols() -> list[str]:
-    """Names of every entry point declared in include/jpi.h."""
-    text = open(HEADER).read()
-    return re.findall(r"JPI_API\s+[\w\s\*]+?\b(jpi_\w+)\s*\(", text)
+    """Names of every entry point declared in the headers under include/ (jpi.h, jpi_corr.h)."""
+    inc = os.path.dirname(HEADER)
+    names = []
+    for f in sorted(os.listdir(inc)):
+        if f.endswith(".h"):
+            text = open(os.path.join(inc, f)).read()
+            names += re.findall(r"JPI_API\s+[\w\s\*]+?\b(jpi_\w+)\s*\(", text)
+    return names
 
 
 def load():

@@ -60,3 +60,32 @@ def test_bad_configs_are_rejected_before_any_device_call(lib):
         st = lib.jpi_expert_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h))
         assert st in (-1, -7, -2), (kw, st)
         assert h.value is None
+
+
+def test_correction_module_arguments_are_checked_on_the_host(lib):
+    from paper_2607_12659_gb300 import corr
+    from synth import PI05_CORRECTION
+    lib = corr.load()
+    h = ctypes.c_void_p()
+    assert lib.jpi_corr_create(None, None, ctypes.byref(h)) == -1
+    assert lib.jpi_corr_create(None, None, None) == -1
+    assert lib.jpi_corr_destroy(None) == 0
+    assert lib.jpi_corr_compress(None, None, 1, 1, 1, None, None) == -1
+    assert lib.jpi_corr_predict(None, None, None, 1, 1, None, None, None) == -1
+    b = ctypes.c_longlong()
+    assert lib.jpi_corr_memory_usage(None, ctypes.byref(b)) == -1
+    w = corr.jpi_corr_weights()
+    bad = [dict(width=1000), dict(head_dim=48), dict(n_heads=3), dict(n_items=0), dict(n_items=9),
+           dict(max_delta=0), dict(max_delta=65), dict(n_joint=9), dict(max_batch=0), dict(precision=5),
+           dict(n_heads=16, head_dim=64, n_items=8), dict(max_vlm_tokens=0), dict(d_vlm=0)]
+    for kw in bad:
+        cfg = corr.make_corr_config(PI05_CORRECTION, 1, 816)
+        for k, v in kw.items():
+            setattr(cfg, k, v)
+        st = lib.jpi_corr_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h))
+        assert st in (-1, -7), (kw, st)
+        assert h.value is None
+    # A valid shape whose joint blocks are missing is refused before any device call.
+    cfg = corr.make_corr_config(PI05_CORRECTION, 1, 816)
+    assert lib.jpi_corr_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h)) == -1
+    assert b"jb" in lib.jpi_last_error()

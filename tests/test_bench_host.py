@@ -96,3 +96,12 @@ def test_reference_arm_json_line():
     assert line["impl"] == "reference" and line["value"] > 0
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
+
+
+def test_every_kernel_source_is_accounted_for_by_the_traffic_hash():
+    # A source the measured kernels are built from must change `source_sha` (and so null the
+    # recorded DRAM traffic) when it changes; only the correction module's files stay outside.
+    d = os.path.join(bench.ROOT, "paper_2607_12659_gb300", "csrc")
+    files = {f for f in os.listdir(d) if f.endswith((".cu", ".cuh", ".h"))}
+    assert files == set(bench.EXPERT_SOURCES) | set(bench.CORRECTION_SOURCES)
+    assert not set(bench.EXPERT_SOURCES) & set(bench.CORRECTION_SOURCES)
