@@ -3,7 +3,9 @@
 Host control logic around the action expert. The VLM, the future correction module and the
 observation source are callables supplied by the caller (they are outside this library); the
 action expert is usually `expert_act(...)`, which runs the expert's flow-matching denoise on the
-GPU with the predicted compressed VLM state as correction items.
+GPU with the predicted compressed VLM state as correction items; `corrector_corr` and
+`corrector_vlm` build f_corr and the compressing side of f_vlm from the library's correction
+module (`corr.Corrector`).
 
 One iteration, after the start-up pass (VLM on the first observation, expert on its output):
   * confidence c > theta (theta < 0): skip the VLM. Take the next delta_ae actions of the
@@ -25,6 +27,8 @@ from __future__ import annotations
 import threading
 from dataclasses import dataclass, field
 from typing import Any, Callable, Sequence
+
+import numpy as np
 
 
 class ActionBuffer:
@@ -170,3 +174,27 @@ def expert_act(expert, state_fn: Callable[[], Any], noise_fn: Callable[[], Any],
         out = expert.denoise(state_fn(), noise_fn(), num_steps)
         return out.cpu().numpy()[0]
     return act
+
+
+def corrector_corr(corrector):
+    """f_corr over the library's correction module: the state buffer holds a compressed state
+    ([1][T'][width] CUDA tensor) and the committed actions are the executor's action rows; returns
+    the predicted state (on the device) and its confidence (one host float, read back because the
+    scheduler branches on it)."""
+    import torch
+
+    def corr(h, actions):
+        a = torch.as_tensor(np.stack([np.asarray(x, np.float32) for x in actions])[None],
+                            device=h.device)
+        h_future, conf = corrector.predict(h, a)
+        return h_future, float(conf[0].item())
+    return corr
+
+
+def corrector_vlm(vlm_forward, corrector):
+    """f_vlm followed by the compressor (Alg. 1's state buffer holds compressed states):
+    vlm_forward(obs) -> (final-layer output [1][T][d_VLM] CUDA tensor, kv)."""
+    def vlm(obs):
+        out, kv = vlm_forward(obs)
+        return corrector.compress(out), kv
+    return vlm

@@ -157,3 +157,39 @@ def test_predicted_items_drive_the_expert_on_the_device():
     assert np.abs(out.cpu().numpy() - want).max() <= 1e-4
     ex.close()
     mod.close()
+
+
+def test_alg1_on_the_gpu_components():
+    # Alg. 1 with f_corr and the compressor from the library and the expert as f_act: each chunk
+    # is the expert's denoise for the state the module predicted from the compressed VLM output.
+    import torch
+    from paper_2607_12659_gb300.scheduler import (ConfidenceScheduler, corrector_corr, corrector_vlm,
+                                                  expert_act)
+    from tests.gpu_util import make_expert
+    ecfg = TINY
+    cfg = SMALL.with_(width=ecfg.width, n_heads=4, head_dim=64, action_dim=ecfg.action_dim, precision="fp32")
+    mod, w, inp, dev = _setup(cfg, 71, 1, 24, 4, max_batch=1)
+    we = make_weights(ecfg, 72)
+    P, C, N = 16, 8, 3
+    r = make_requests(ecfg, 73, 1, P, C)
+    ex = make_expert(ecfg, we, max_batch=1, max_prefix=P, max_chunk=C, max_steps=N)
+    kv = (torch.from_numpy(r["prefix_k"]).cuda(), torch.from_numpy(r["prefix_v"]).cuda())
+    state = torch.from_numpy(r["state"]).cuda()
+    noise = torch.from_numpy(r["noise"]).cuda()
+    sch = ConfidenceScheduler(vlm=corrector_vlm(lambda obs: (dev["h_vlm"], kv), mod), corr=corrector_corr(mod),
+                              act=expert_act(ex, lambda: state, lambda: noise, N), observe=lambda: "obs",
+                              theta=-1e30, delta=4, delta_ae=2)
+    sch.start()
+    first = np.stack(sch.buffer.committed(C))
+    sch.iterate()
+    torch.cuda.synchronize()
+    w64 = oc.to_f64_corr(w)
+    h0 = oc.qformer_compress(inp["h_vlm"][0].astype(np.float64), w64, cfg)
+    h1, c1 = oc.future_correction(h0, first[:2].astype(np.float64), w64, cfg)
+    assert abs(sch.confidence - c1) <= MAX_ABS
+    want = oracle.denoise_batch(r["noise"], r["state"], N, r["prefix_k"], r["prefix_v"], we, ecfg,
+                                corr=h1[None])
+    got = np.stack(sch.buffer.committed(2 + C))[2:]
+    assert np.abs(got - want[0]).max() <= 1e-3
+    ex.close()
+    mod.close()
