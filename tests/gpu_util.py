@@ -6,7 +6,7 @@ import os
 import numpy as np
 
 import oracle
-from synth import ExpertConfig, PI05, TINY, make_requests, make_weights
+from synth import ExpertConfig
 
 # Tolerances: bf16 weights and tensor-core inputs with fp32 accumulation, and the fp32
 # verification mode, against the fp64 oracle on the same (bf16-rounded) inputs.

@@ -3,7 +3,6 @@ exports every entry point include/jpi.h declares, and rejects bad arguments befo
 the device."""
 
 import ctypes
-import os
 import subprocess
 
 import pytest

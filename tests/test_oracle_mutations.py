@@ -5,7 +5,6 @@ operand). The mutated source is loaded as a separate module on the CPU and the p
 ``test_oracle_pins`` are run against it; the real oracle is untouched.
 """
 
-import importlib.util
 import inspect
 import os
 import types

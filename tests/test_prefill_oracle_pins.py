@@ -7,7 +7,6 @@ import math
 import os
 
 import numpy as np
-import pytest
 
 import oracle.prefill as pf
 from synth import GEMMA2B, llm_weight_shapes, make_llm_weights, make_prefix_embeddings
