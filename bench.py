@@ -433,6 +433,78 @@ def our_arm(args):
         dist.destroy_process_group()
 
 
+# Correction-module tensors used only at create time (the compressor's query self-attention and
+# the cross-attention queries mapped through the key projection): not streamed per call.
+CORR_CREATE_ONLY = ("qf_query", "qf_ln1_w", "qf_ln1_b", "qf_ln2_w", "qf_ln2_b", "qf_ca_wq", "qf_ca_bq",
+                    "qf_ca_wk", "qf_ca_bk")
+
+
+def correction_bytes(cfg, B, T, delta):
+    """Bytes one compress + predict call must move: every per-call weight once (projection
+    matrices in bf16; vectors, the position table and the confidence row in fp32, as the library
+    stores them), the bf16 VLM output, the actions, the state in and out, the confidences."""
+    import numpy as np
+    from synth.correction import correction_weight_shapes
+    wb = 0
+    for name, shp in correction_weight_shapes(cfg).items():
+        if name in CORR_CREATE_ONLY or name.startswith("qf_sa_"):
+            continue
+        mat = len(shp) == 2 and name not in ("act_pos", "conf_w")
+        wb += int(np.prod(shp)) * (2 if mat and cfg.precision == "bf16" else 4)
+    io = B * T * cfg.d_vlm * 2 + B * delta * cfg.action_dim * 4 + 3 * B * cfg.n_items * cfg.width * 4 + B * 4
+    return wb + io
+
+
+def correction_arm(args):
+    """The future correction module (compress + predict, pi0.5 sizes, bf16 weights) timed alone."""
+    import torch
+    from paper_2607_12659_gb300 import build, corr
+    from synth.correction import PI05_CORRECTION, make_correction_inputs, make_correction_weights
+    build.build()
+    torch.cuda.set_device(0)
+    cfg = PI05_CORRECTION
+    B, T, delta = args.batch or 1, args.prefix or WORKLOAD["prefix"], 9
+    mod = corr.Corrector(cfg, make_correction_weights(cfg, 3000), max_batch=B, max_vlm_tokens=T)
+    inp = make_correction_inputs(cfg, 3001, B, T, delta)
+    hv = torch.from_numpy(inp["h_vlm"]).cuda().to(torch.bfloat16)
+    acts = torch.from_numpy(inp["actions"]).cuda()
+    state = torch.empty((B, cfg.n_items, cfg.width), dtype=torch.float32, device="cuda")
+    hf, conf = torch.empty_like(state), torch.empty((B,), dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        mod.compress(hv, out=state)
+        mod.predict(state, acts, out=hf, confidence=conf)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3 * args.steps)]
+    with ClockSampler(0) as clk:
+        for i in range(args.steps):
+            ev[3 * i].record(stream)
+            mod.compress(hv, out=state)
+            ev[3 * i + 1].record(stream)
+            mod.predict(state, acts, out=hf, confidence=conf)
+            ev[3 * i + 2].record(stream)
+        torch.cuda.synchronize()
+    comp = [ev[3 * i].elapsed_time(ev[3 * i + 1]) for i in range(args.steps)]
+    pred = [ev[3 * i + 1].elapsed_time(ev[3 * i + 2]) for i in range(args.steps)]
+    call_ms = statistics.median([a + b for a, b in zip(comp, pred)])
+    hbm_peak, _, peak_src = measured_peaks()
+    alg = correction_bytes(cfg, B, T, delta)
+    achieved = alg / (call_ms * 1e-3) / 1e9
+    print(json.dumps({
+        "metric": f"future correction module calls/s (compress + predict), batch {B}",
+        "value": B / (call_ms * 1e-3), "unit": "calls/s", "steps": args.steps, "warmup": args.warmup,
+        "config": {"workload": f"pi0.5-sized correction module (d_AE 1024, d_VLM 2048, T' 4), "
+                               f"{T} VLM tokens, Delta {delta}", "batch": B},
+        "us": {"compress": statistics.median(comp) * 1e3, "predict": statistics.median(pred) * 1e3,
+               "call": call_ms * 1e3},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "traffic": None, "peak_source": peak_src,
+                     "bytes_per_call": alg},
+        "dtype": "bf16 weights, fp32 activations", "data": "synthetic", "clocks": clk.summary(),
+    }), flush=True)
+    mod.close()
+
+
 def profile_forward(args):
     """Small case for kernel captures: the workload's expert, eager expert passes (batch and
     prefix as given, else the workload's)."""
@@ -461,6 +533,8 @@ def main():
     ap.add_argument("--profile-forward", action="store_true",
                     help="run eager expert passes of the workload (small case for ncu captures)")
     ap.add_argument("--forward-passes", type=int, default=2)
+    ap.add_argument("--correction", action="store_true",
+                    help="time the future correction module alone (compress + predict)")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
@@ -479,7 +553,9 @@ def main():
         return
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    if args.impl == "reference":
+    if args.correction:
+        correction_arm(args)
+    elif args.impl == "reference":
         reference_arm(args)
     else:
         our_arm(args)

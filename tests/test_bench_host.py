@@ -105,3 +105,22 @@ def test_every_kernel_source_is_accounted_for_by_the_traffic_hash():
     files = {f for f in os.listdir(d) if f.endswith((".cu", ".cuh", ".h"))}
     assert files == set(bench.EXPERT_SOURCES) | set(bench.CORRECTION_SOURCES)
     assert not set(bench.EXPERT_SOURCES) & set(bench.CORRECTION_SOURCES)
+
+
+def test_correction_bytes_from_the_weight_shapes():
+    # Per-call weights: everything but the compressor's query-side tensors, which create time
+    # folds into the queries mapped into VLM space; plus the bf16 VLM output and the small I/O.
+    from synth.correction import PI05_CORRECTION as c
+    d, F, dv, A = c.width, c.mlp_dim, c.d_vlm, c.action_dim
+    block_mats = 4 * d * d + 2 * d * F
+    block_vecs = 4 * d + 4 * d + F + d           # ln1, ln2 (w, b), q/k/v/o biases, b1, b2
+    mats = (d * dv + d * d + 2 * d * F          # compressor: value, output, MLP
+            + d * A + d * d + c.max_delta * d    # action MLP, position table
+            + block_mats * (1 + c.n_joint) + 2 * d * d + d * d + d)   # blocks, fuse, corr, conf
+    vecs = (3 * d + F + 2 * d + 2 * d            # compressor: b_v, b_o, b2; b1; ln3; lnf
+            + 2 * d                              # action biases
+            + block_vecs * (1 + c.n_joint) + d + 2 * d + d + 1)   # fuse b, head ln, corr b, conf b
+    want_w = 2 * (mats - c.max_delta * d - d) + 4 * (c.max_delta * d + d) + 4 * vecs
+    B, T, delta = 1, 816, 9
+    io = B * T * dv * 2 + B * delta * A * 4 + 3 * B * c.n_items * d * 4 + B * 4
+    assert bench.correction_bytes(c, B, T, delta) == want_w + io
