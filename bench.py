@@ -505,6 +505,59 @@ def correction_arm(args):
     mod.close()
 
 
+def prefill_flops(cfg, B, P):
+    """FLOPs of one prefill: 2 per multiply-add of every projection (Q/K/V, output, gate/up, down)
+    over B P tokens, plus the scores and the probability-weighted values (H P^2 D each) per
+    request and layer."""
+    W, H, D, F = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim
+    proj = W * (H + 2) * D + H * D * W + 2 * F * W + F * W
+    return cfg.n_layers * (2 * B * P * proj + 2 * 2 * B * H * P * P * D)
+
+
+def prefill_arm(args):
+    """The Gemma-2B-shaped prefill (18 layers, bf16 weights) timed alone, into KV tensors."""
+    import torch
+    from paper_2607_12659_gb300 import build, prefill
+    from synth import GEMMA2B, make_llm_weights, make_prefix_embeddings
+    build.build()
+    torch.cuda.set_device(0)
+    cfg = GEMMA2B
+    B, P = args.batch or 1, args.prefix or WORKLOAD["prefix"]
+    pre = prefill.Prefill(cfg, make_llm_weights(cfg, 4000), max_batch=B, max_prefix=P)
+    x = torch.from_numpy(make_prefix_embeddings(cfg, 4001, B, P)).cuda().to(torch.bfloat16)
+    L, D = cfg.n_layers, cfg.head_dim
+    K = torch.empty((L, B, P, D), dtype=torch.bfloat16, device="cuda")
+    V = torch.empty_like(K)
+    kp, vp = [K[l].data_ptr() for l in range(L)], [V[l].data_ptr() for l in range(L)]
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        pre.run(x, kp, vp, P * D, final=False)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    with ClockSampler(0) as clk:
+        ev[0].record(stream)
+        for i in range(args.steps):
+            pre.run(x, kp, vp, P * D, final=False)
+            ev[i + 1].record(stream)
+        torch.cuda.synchronize()
+    ms = statistics.median([ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)])
+    _, tc_peak, peak_src = measured_peaks()
+    flops = prefill_flops(cfg, B, P)
+    tf = flops / (ms * 1e-3) / 1e12
+    print(json.dumps({
+        "metric": f"Gemma-2B prefix prefill, {P} tokens x batch {B}, ms per prefill",
+        "value": ms, "unit": "ms", "higher_is_better": False, "steps": args.steps, "warmup": args.warmup,
+        "config": {"workload": f"Gemma-2B-shaped LLM (18 x W2048, 8x256 heads, 1 KV head, GeGLU 16384), "
+                               f"batch {B}, prefix {P}"},
+        "roofline": {"bound": "tensor", "achieved": tf, "peak": tc_peak, "unit": "TFLOP/s",
+                     "frac": tf / tc_peak if tc_peak else None, "traffic": None, "peak_source": peak_src,
+                     "flops_per_call": flops},
+        "dtype": "bf16 GEMM operands, fp32 accumulation and residual stream", "data": "synthetic",
+        "clocks": clk.summary(),
+    }), flush=True)
+    pre.close()
+
+
 def profile_forward(args):
     """Small case for kernel captures: the workload's expert, eager expert passes (batch and
     prefix as given, else the workload's)."""
@@ -535,6 +588,7 @@ def main():
     ap.add_argument("--forward-passes", type=int, default=2)
     ap.add_argument("--correction", action="store_true",
                     help="time the future correction module alone (compress + predict)")
+    ap.add_argument("--prefill", action="store_true", help="time the Gemma-2B-shaped prefix prefill alone")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
@@ -555,6 +609,8 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.correction:
         correction_arm(args)
+    elif args.prefill:
+        prefill_arm(args)
     elif args.impl == "reference":
         reference_arm(args)
     else:

@@ -1,8 +1,14 @@
-"""Builds the library ``libjpi.so`` in-tree for sm_103a with nvcc (no cmake, no torch build).
+"""Builds the libraries in-tree for sm_103a with nvcc (no cmake, no torch build).
 
-Each CUDA translation unit compiles in parallel; the objects link into one shared library
+``libjpi.so``: the action expert and the future correction module (every .cu directly under
+csrc/). Each translation unit compiles in parallel; the objects link into one shared library
 with the CUDA runtime linked statically, so the library needs no libcuda at load time (the
 driver entry points are resolved at run time).
+
+``libjpi_prefill.so``: the LLM prefill (csrc/prefill/), linked against the toolkit's cuBLASLt
+(found next to nvcc, recorded as the library's run path). It is separate so that the expert's
+library depends on nothing but the C and C++ runtimes; a toolkit without cuBLASLt leaves only
+the prefill unbuilt (reported on stderr and by ``PREFILL_BUILD_ERROR``).
 """
 
 from __future__ import annotations
@@ -18,6 +24,9 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libjpi.so")
+PREFILL_SRC = os.path.join(CSRC, "prefill")
+PREFILL_LIB = os.path.join(PKG, "libjpi_prefill.so")
+PREFILL_BUILD_ERROR = None
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + [
@@ -47,8 +56,45 @@ def _stale(obj: str, src: str) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
+def cuda_lib_dir(cc: str) -> str:
+    return os.path.realpath(os.path.join(os.path.dirname(os.path.realpath(cc)), "..", "lib64"))
+
+
+def build_prefill(verbose: bool = False, force: bool = False) -> str:
+    """Compile csrc/prefill/*.cu and link libjpi_prefill.so against cuBLASLt."""
+    cc = nvcc()
+    out = os.path.join(BUILD, "prefill")
+    os.makedirs(out, exist_ok=True)
+    srcs = sorted(os.path.join(PREFILL_SRC, f) for f in os.listdir(PREFILL_SRC) if f.endswith(".cu"))
+    headers = [os.path.join(ROOT, "include", f) for f in ("jpi.h", "jpi_prefill.h")]
+    objs = []
+    for src in srcs:
+        obj = os.path.join(out, os.path.basename(src)[:-3] + ".o")
+        objs.append(obj)
+        if not force and os.path.exists(obj) and all(
+                os.path.getmtime(d) <= os.path.getmtime(obj) for d in [src] + headers):
+            continue
+        r = subprocess.run([cc] + NVCC_FLAGS + ["-c", src, "-o", obj], capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed for {os.path.basename(src)}:\n{r.stderr}")
+        if verbose and r.stderr:
+            print(r.stderr, file=sys.stderr)
+    if force or not os.path.exists(PREFILL_LIB) or any(
+            os.path.getmtime(o) > os.path.getmtime(PREFILL_LIB) for o in objs):
+        libdir = cuda_lib_dir(cc)
+        tmp = PREFILL_LIB + ".tmp"
+        cmd = [cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs + [
+            "-L", libdir, "-lcublasLt", "-Xlinker", f"-rpath={libdir}"]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"link of libjpi_prefill.so failed:\n{r.stderr}")
+        os.replace(tmp, PREFILL_LIB)
+    return PREFILL_LIB
+
+
 def build(verbose: bool = False, force: bool = False) -> str:
-    """Compile every .cu under csrc/ and link libjpi.so; returns the library path."""
+    """Compile every .cu directly under csrc/ and link libjpi.so, then the prefill library;
+    returns libjpi.so's path."""
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
     srcs = sources()
@@ -77,6 +123,13 @@ def build(verbose: bool = False, force: bool = False) -> str:
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stderr}")
         os.replace(tmp, LIB)
+    global PREFILL_BUILD_ERROR
+    try:
+        build_prefill(verbose, force)
+        PREFILL_BUILD_ERROR = None
+    except (RuntimeError, OSError) as e:
+        PREFILL_BUILD_ERROR = str(e)
+        print(f"warning: libjpi_prefill.so not built: {e}", file=sys.stderr)
     return LIB
 
 

@@ -78,11 +78,14 @@ _SIGS = {
 _lib = None
 
 
-def header_symbols() -> list[str]:
-    """Names of every entry point declared in the headers under include/ (jpi.h, jpi_corr.h)."""
+LIB_HEADERS = ("jpi.h", "jpi_corr.h")   # the entry points libjpi.so exports
+
+
+def header_symbols(headers=LIB_HEADERS) -> list[str]:
+    """Names of every entry point declared in the given headers under include/."""
     inc = os.path.dirname(HEADER)
     names = []
-    for f in sorted(os.listdir(inc)):
+    for f in headers:
         if f.endswith(".h"):
             text = open(os.path.join(inc, f)).read()
             names += re.findall(r"JPI_API\s+[\w\s\*]+?\b(jpi_\w+)\s*\(", text)

@@ -1,8 +1,9 @@
-"""Host-side checks of the C-ABI library that need no GPU: it builds, loads without a driver,
-exports every entry point include/jpi.h declares, and rejects bad arguments before touching
-the device."""
+"""Host-side checks of the C-ABI libraries that need no GPU: they build, load without a driver,
+export every entry point their headers declare (libjpi.so: include/jpi.h and jpi_corr.h;
+libjpi_prefill.so: jpi_prefill.h), and reject bad arguments before touching the device."""
 
 import ctypes
+import os
 import subprocess
 
 import pytest
@@ -88,3 +89,43 @@ def test_correction_module_arguments_are_checked_on_the_host(lib):
     cfg = corr.make_corr_config(PI05_CORRECTION, 1, 816)
     assert lib.jpi_corr_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h)) == -1
     assert b"jb" in lib.jpi_last_error()
+
+
+def test_every_header_belongs_to_a_library():
+    from paper_2607_12659_gb300 import prefill
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    headers = {f for f in os.listdir(inc) if f.endswith(".h")}
+    assert headers == set(jpi.LIB_HEADERS) | {"jpi_prefill.h"}
+    assert len(prefill.header_symbols()) == 5
+
+
+def test_prefill_library_exports_its_entry_points_and_checks_arguments(lib):
+    from paper_2607_12659_gb300 import build as b, prefill
+    from synth import GEMMA2B
+    assert b.PREFILL_BUILD_ERROR is None, b.PREFILL_BUILD_ERROR
+    plib = prefill.load()
+    out = subprocess.run(["nm", "-D", "--defined-only", prefill.LIB_PATH], capture_output=True, text=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    assert exported == set(prefill.header_symbols())
+    ldd = subprocess.run(["ldd", prefill.LIB_PATH], capture_output=True, text=True).stdout
+    assert "libcublasLt" in ldd and "libcuda.so" not in ldd and "libtorch" not in ldd
+    h = ctypes.c_void_p()
+    assert plib.jpi_prefill_create(None, None, ctypes.byref(h)) == -1
+    assert b"NULL" in plib.jpi_prefill_last_error()
+    assert plib.jpi_prefill_destroy(None) == 0
+    assert plib.jpi_prefill_run(None, None, 1, 1, 1, None, None, 256, None, None) == -1
+    n = ctypes.c_longlong()
+    assert plib.jpi_prefill_memory_usage(None, ctypes.byref(n)) == -1
+    w = prefill.jpi_prefill_weights()
+    bad = [dict(n_layers=0), dict(width=2044), dict(head_dim=250), dict(head_dim=1024), dict(mlp_dim=12),
+           dict(max_batch=0), dict(max_prefix=0), dict(rms_eps=-1.0), dict(max_prefix=70000)]
+    for kw in bad:
+        cfg = prefill.make_prefill_config(GEMMA2B, 1, 816)
+        for k, v in kw.items():
+            setattr(cfg, k, v)
+        st = plib.jpi_prefill_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h))
+        assert st in (-1, -7), (kw, st)
+        assert h.value is None
+    cfg = prefill.make_prefill_config(GEMMA2B, 1, 816)
+    assert plib.jpi_prefill_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h)) == -1   # NULL weights
+    assert b"NULL" in plib.jpi_prefill_last_error()

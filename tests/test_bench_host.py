@@ -124,3 +124,23 @@ def test_correction_bytes_from_the_weight_shapes():
     B, T, delta = 1, 816, 9
     io = B * T * dv * 2 + B * delta * A * 4 + 3 * B * c.n_items * d * 4 + B * 4
     assert bench.correction_bytes(c, B, T, delta) == want_w + io
+
+
+def test_prefill_flops_by_brute_count():
+    # Count multiply-adds product by product for a tiny model and compare.
+    from synth import GEMMA2B
+    cfg = GEMMA2B.with_(n_layers=2, width=8, n_heads=2, head_dim=4, mlp_dim=12)
+    B, P = 3, 5
+    W, H, D, F = 8, 2, 4, 12
+    macs = 0
+    for _ in range(cfg.n_layers):
+        macs += B * P * W * (H * D + D + D)      # q, k, v
+        macs += B * H * P * P * D                # scores
+        macs += B * H * P * P * D                # probabilities x V
+        macs += B * P * (H * D) * W              # output projection
+        macs += B * P * W * F * 2                # gate and up
+        macs += B * P * F * W                    # down
+    assert bench.prefill_flops(cfg, B, P) == 2 * macs
+    # Gemma-2B at 816 tokens: the ~2B projection parameters dominate (3.2 TFLOP per request).
+    f = bench.prefill_flops(GEMMA2B, 1, 816)
+    assert 3.1e12 < f < 3.4e12
