@@ -183,11 +183,20 @@ struct LayerW {
 
 struct GemmKey {
     int opw, M, N, K, ldx, ldw, ldy, tx, tw, ty, acc;
+    unsigned alx, alw, aly;   // byte alignment of each operand's address (at most 256)
     bool operator<(const GemmKey& o) const {
-        return std::tie(opw, M, N, K, ldx, ldw, ldy, tx, tw, ty, acc) <
-               std::tie(o.opw, o.M, o.N, o.K, o.ldx, o.ldw, o.ldy, o.tx, o.tw, o.ty, o.acc);
+        return std::tie(opw, M, N, K, ldx, ldw, ldy, tx, tw, ty, acc, alx, alw, aly) <
+               std::tie(o.opw, o.M, o.N, o.K, o.ldx, o.ldw, o.ldy, o.tx, o.tw, o.ty, o.acc, o.alx, o.alw, o.aly);
     }
 };
+
+// Largest power of two up to 256 that divides the address.
+unsigned alignment_of(const void* p) {
+    const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+    unsigned r = 256;
+    while (r > 1 && (a % r) != 0) r >>= 1;
+    return r;
+}
 
 struct GemmPlan {
     cublasLtMatmulDesc_t desc = nullptr;
@@ -235,18 +244,62 @@ jpi_status pf_alloc(jpi_prefill_handle* h, T** p, size_t count) {
     return JPI_OK;
 }
 
+void destroy_plan(GemmPlan& pl) {
+    if (pl.desc) cublasLtMatmulDescDestroy(pl.desc);
+    if (pl.a) cublasLtMatrixLayoutDestroy(pl.a);
+    if (pl.b) cublasLtMatrixLayoutDestroy(pl.b);
+    if (pl.c) cublasLtMatrixLayoutDestroy(pl.c);
+    pl = GemmPlan();
+}
+
 void release(jpi_prefill_handle* h) {
-    for (auto& kv : h->plans) {
-        if (kv.second.desc) cublasLtMatmulDescDestroy(kv.second.desc);
-        if (kv.second.a) cublasLtMatrixLayoutDestroy(kv.second.a);
-        if (kv.second.b) cublasLtMatrixLayoutDestroy(kv.second.b);
-        if (kv.second.c) cublasLtMatrixLayoutDestroy(kv.second.c);
-    }
+    for (auto& kv : h->plans) destroy_plan(kv.second);
     h->plans.clear();
     if (h->lt) cublasLtDestroy(h->lt);
     h->lt = nullptr;
     for (void* p : h->allocs) cudaFree(p);
     h->allocs.clear();
+}
+
+// Descriptors, layouts and the heuristic's algorithm for one product shape; the algorithm is
+// chosen for the operands' actual address alignment (cuBLASLt otherwise assumes 256 bytes).
+cublasStatus_t make_plan(jpi_prefill_handle* h, const GemmKey& k, GemmPlan* pl) {
+    cublasStatus_t s = cublasLtMatmulDescCreate(&pl->desc, CUBLAS_COMPUTE_32F, CUDA_R_32F);
+    const cublasOperation_t opa = k.opw ? CUBLAS_OP_T : CUBLAS_OP_N, opb = CUBLAS_OP_N;
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatmulDescSetAttribute(pl->desc, CUBLASLT_MATMUL_DESC_TRANSA, &opa, sizeof(opa));
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatmulDescSetAttribute(pl->desc, CUBLASLT_MATMUL_DESC_TRANSB, &opb, sizeof(opb));
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = k.opw ? cublasLtMatrixLayoutCreate(&pl->a, (cudaDataType)k.tw, (uint64_t)k.K, (uint64_t)k.N, (int64_t)k.ldw)
+                  : cublasLtMatrixLayoutCreate(&pl->a, (cudaDataType)k.tw, (uint64_t)k.N, (uint64_t)k.K, (int64_t)k.ldw);
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatrixLayoutCreate(&pl->b, (cudaDataType)k.tx, (uint64_t)k.K, (uint64_t)k.M, (int64_t)k.ldx);
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatrixLayoutCreate(&pl->c, (cudaDataType)k.ty, (uint64_t)k.N, (uint64_t)k.M, (int64_t)k.ldy);
+    if (s != CUBLAS_STATUS_SUCCESS) return s;
+    cublasLtMatmulPreference_t pref = nullptr;
+    s = cublasLtMatmulPreferenceCreate(&pref);
+    if (s != CUBLAS_STATUS_SUCCESS) return s;
+    const uint64_t wsb = WORKSPACE_BYTES;
+    const uint32_t al[4] = {k.alw, k.alx, k.aly, k.aly};   // A = W, B = X, C = D = Y
+    s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES, &wsb, sizeof(wsb));
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_A_BYTES, &al[0], sizeof(al[0]));
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_B_BYTES, &al[1], sizeof(al[1]));
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_C_BYTES, &al[2], sizeof(al[2]));
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_D_BYTES, &al[3], sizeof(al[3]));
+    cublasLtMatmulHeuristicResult_t res;
+    int nres = 0;
+    if (s == CUBLAS_STATUS_SUCCESS)
+        s = cublasLtMatmulAlgoGetHeuristic(h->lt, pl->desc, pl->a, pl->b, pl->c, pl->c, pref, 1, &res, &nres);
+    cublasLtMatmulPreferenceDestroy(pref);
+    if (s == CUBLAS_STATUS_SUCCESS && nres < 1) s = CUBLAS_STATUS_NOT_SUPPORTED;
+    if (s == CUBLAS_STATUS_SUCCESS) pl->algo = res.algo;
+    return s;
 }
 
 // Y [M][N] (row-major, leading dimension ldy) = alpha X [M][K] op(W) + beta Y, where op(W) = W^T
@@ -256,37 +309,17 @@ void release(jpi_prefill_handle* h) {
 jpi_status row_gemm(jpi_prefill_handle* h, cudaStream_t st, const void* X, cudaDataType tx, int ldx,
                     const void* Wm, cudaDataType tw, int ldw, bool w_nk, void* Y, cudaDataType ty, int ldy,
                     int M, int N, int K, float alpha, float beta) {
-    const GemmKey key{w_nk ? 1 : 0, M, N, K, ldx, ldw, ldy, (int)tx, (int)tw, (int)ty, beta != 0.f ? 1 : 0};
+    const GemmKey key{w_nk ? 1 : 0, M, N, K, ldx, ldw, ldy, (int)tx, (int)tw, (int)ty, beta != 0.f ? 1 : 0,
+                      alignment_of(X), alignment_of(Wm), alignment_of(Y)};
     auto it = h->plans.find(key);
     if (it == h->plans.end()) {
         GemmPlan pl;
-        PF_LT(cublasLtMatmulDescCreate(&pl.desc, CUBLAS_COMPUTE_32F, CUDA_R_32F));
-        const cublasOperation_t opa = w_nk ? CUBLAS_OP_T : CUBLAS_OP_N, opb = CUBLAS_OP_N;
-        PF_LT(cublasLtMatmulDescSetAttribute(pl.desc, CUBLASLT_MATMUL_DESC_TRANSA, &opa, sizeof(opa)));
-        PF_LT(cublasLtMatmulDescSetAttribute(pl.desc, CUBLASLT_MATMUL_DESC_TRANSB, &opb, sizeof(opb)));
-        if (w_nk) PF_LT(cublasLtMatrixLayoutCreate(&pl.a, tw, (uint64_t)K, (uint64_t)N, (int64_t)ldw));
-        else PF_LT(cublasLtMatrixLayoutCreate(&pl.a, tw, (uint64_t)N, (uint64_t)K, (int64_t)ldw));
-        PF_LT(cublasLtMatrixLayoutCreate(&pl.b, tx, (uint64_t)K, (uint64_t)M, (int64_t)ldx));
-        PF_LT(cublasLtMatrixLayoutCreate(&pl.c, ty, (uint64_t)N, (uint64_t)M, (int64_t)ldy));
-        cublasLtMatmulPreference_t pref = nullptr;
-        PF_LT(cublasLtMatmulPreferenceCreate(&pref));
-        const uint64_t wsb = WORKSPACE_BYTES;
-        cublasStatus_t s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES,
-                                                                &wsb, sizeof(wsb));
-        cublasLtMatmulHeuristicResult_t res;
-        int nres = 0;
-        if (s == CUBLAS_STATUS_SUCCESS)
-            s = cublasLtMatmulAlgoGetHeuristic(h->lt, pl.desc, pl.a, pl.b, pl.c, pl.c, pref, 1, &res, &nres);
-        cublasLtMatmulPreferenceDestroy(pref);
-        if (s != CUBLAS_STATUS_SUCCESS || nres < 1) {
-            cublasLtMatmulDescDestroy(pl.desc);
-            cublasLtMatrixLayoutDestroy(pl.a);
-            cublasLtMatrixLayoutDestroy(pl.b);
-            cublasLtMatrixLayoutDestroy(pl.c);
+        const cublasStatus_t s = make_plan(h, key, &pl);
+        if (s != CUBLAS_STATUS_SUCCESS) {
+            destroy_plan(pl);
             return pfail(JPI_ERR_UNSUPPORTED, "no cuBLASLt algorithm for a %d x %d x %d product (%s)", M, N, K,
                          cublasLtGetStatusString(s));
         }
-        pl.algo = res.algo;
         it = h->plans.emplace(key, pl).first;
     }
     const GemmPlan& pl = it->second;
