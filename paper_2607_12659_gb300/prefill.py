@@ -164,7 +164,9 @@ class Prefill:
         return K, V, out
 
     def into_expert(self, x, expert, final=True, stream=None):
-        """Writes the KV of every layer into a (bf16) Expert's store and commits it."""
+        """Writes the KV of every layer into a bf16 Expert's store and commits it."""
+        if getattr(expert.dims, "precision", "bf16") != "bf16":
+            raise ValueError("the prefill writes bf16 keys and values: the expert must use JPI_BF16")
         B, P, _ = x.shape
         ptrs = [jpi.jpi_prefix_kv_ptr(expert.handle, l) for l in range(self.dims.n_layers)]
         stride = ptrs[0][2]

@@ -198,3 +198,18 @@ def corrector_vlm(vlm_forward, corrector):
         out, kv = vlm_forward(obs)
         return corrector.compress(out), kv
     return vlm
+
+
+def prefill_vlm(prefill, expert, embed: Callable[[Any], Any]):
+    """f_vlm's language-model part over the library: embed(obs) gives the prefix token
+    embeddings [1][P][W] (CUDA); the prefill writes every layer's keys and values straight into
+    the expert's store and commits it, and returns the final-layer output. The KV handle it
+    returns is a fresh token, so pair it with expert_act(..., set_kv=lambda *kv: None): the store
+    is already current."""
+    count = [0]
+
+    def vlm(obs):
+        out = prefill.into_expert(embed(obs), expert)
+        count[0] += 1
+        return out, (count[0],)
+    return vlm

@@ -193,3 +193,46 @@ def test_alg1_on_the_gpu_components():
     assert np.abs(got - want[0]).max() <= 1e-3
     ex.close()
     mod.close()
+
+
+@pytest.mark.skipif(os.environ.get("JPI_PREFILL_GPU_TESTS") != "1",
+                    reason="prefill kernels not yet run on a GB300 (JPI_PREFILL_GPU_TESTS=1)")
+def test_alg1_with_every_component_on_the_gpu():
+    # Prefill (KV straight into the expert's store) -> compressor -> expert at start-up, then
+    # f_corr -> expert: the first chunk against the oracles' chain.
+    import torch
+    import oracle.prefill as pf
+    from paper_2607_12659_gb300 import prefill
+    from paper_2607_12659_gb300.scheduler import (ConfidenceScheduler, corrector_corr, corrector_vlm,
+                                                  expert_act, prefill_vlm)
+    from synth import GEMMA2B, PI05, make_llm_weights, make_prefix_embeddings
+    from tests.gpu_util import make_expert
+    ecfg = PI05.with_(n_layers=2, width=256, n_heads=2, head_dim=128, mlp_dim=512, time_dim=64)   # bf16 store
+    lcfg = GEMMA2B.with_(n_layers=2, width=192, n_heads=2, head_dim=128, mlp_dim=384, precision="fp32")
+    cfg = SMALL.with_(width=256, n_heads=4, head_dim=64, d_vlm=192, action_dim=ecfg.action_dim)
+    P, C, N = 24, 8, 3
+    wl = make_llm_weights(lcfg, 91, std=0.05)
+    wc = make_correction_weights(cfg, 92, std=0.1, bias_std=0.1)
+    we = make_weights(ecfg, 93)
+    x = make_prefix_embeddings(lcfg, 94, 1, P)
+    r = make_requests(ecfg, 95, 1, 1, C)
+    pre = prefill.Prefill(lcfg, wl, max_batch=1, max_prefix=P)
+    mod = _lib().Corrector(cfg, wc, max_batch=1, max_vlm_tokens=P)
+    ex = make_expert(ecfg, we, max_batch=1, max_prefix=P, max_chunk=C, max_steps=N)
+    state, noise = torch.from_numpy(r["state"]).cuda(), torch.from_numpy(r["noise"]).cuda()
+    vlm = corrector_vlm(prefill_vlm(pre, ex, lambda obs: torch.from_numpy(x).cuda()), mod)
+    sch = ConfidenceScheduler(vlm=vlm, corr=corrector_corr(mod),
+                              act=expert_act(ex, lambda: state, lambda: noise, N, set_kv=lambda *kv: None),
+                              observe=lambda: "obs", theta=-1e30, delta=4, delta_ae=2)
+    sch.start()
+    torch.cuda.synchronize()
+    first = np.stack(sch.buffer.committed(C))
+    K, V, out = pf.prefill_batch(x, wl, lcfg)
+    h0 = oc.compress_batch(out.astype(np.float32), wc, cfg)
+    want = oracle.denoise_batch(r["noise"], r["state"], N, K.astype(np.float32), V.astype(np.float32), we, ecfg,
+                                corr=h0)
+    # bf16 GEMM operands in the prefill, then the bf16 expert on the KV it wrote.
+    assert np.abs(first - want[0]).max() <= 5e-2
+    ex.close()
+    mod.close()
+    pre.close()
