@@ -168,6 +168,11 @@ class Prefill:
         if getattr(expert.dims, "precision", "bf16") != "bf16":
             raise ValueError("the prefill writes bf16 keys and values: the expert must use JPI_BF16")
         B, P, _ = x.shape
+        if B > expert.cfg.max_batch or P > expert.cfg.max_prefix:
+            raise ValueError(f"batch {B} / prefix {P} exceed the expert store's maxima "
+                             f"{expert.cfg.max_batch} / {expert.cfg.max_prefix}")
+        if expert.cfg.n_layers != self.dims.n_layers or expert.cfg.head_dim != self.dims.head_dim:
+            raise ValueError("the expert's layers and head_dim must match the LLM's")
         ptrs = [jpi.jpi_prefix_kv_ptr(expert.handle, l) for l in range(self.dims.n_layers)]
         stride = ptrs[0][2]
         out = self.run(x, [p[0] for p in ptrs], [p[1] for p in ptrs], stride, final, stream)
