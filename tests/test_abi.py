@@ -129,3 +129,18 @@ def test_prefill_library_exports_its_entry_points_and_checks_arguments(lib):
     cfg = prefill.make_prefill_config(GEMMA2B, 1, 816)
     assert plib.jpi_prefill_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h)) == -1   # NULL weights
     assert b"NULL" in plib.jpi_prefill_last_error()
+
+
+def test_prefill_into_expert_refuses_stores_it_does_not_fit():
+    # The C-ABI cannot see the size of the destination store; the binding checks it first.
+    from types import SimpleNamespace as NS
+    from paper_2607_12659_gb300.prefill import Prefill
+    me = NS(dims=NS(n_layers=2, head_dim=128))
+    store = dict(max_batch=2, max_prefix=64, n_layers=2, head_dim=128)
+    for x_shape, dims, cfg in [((3, 40, 256), dict(precision="bf16"), store),
+                               ((1, 65, 256), dict(precision="bf16"), store),
+                               ((1, 40, 256), dict(precision="fp32"), store),
+                               ((1, 40, 256), dict(precision="bf16"), {**store, "n_layers": 3}),
+                               ((1, 40, 256), dict(precision="bf16"), {**store, "head_dim": 64})]:
+        with pytest.raises(ValueError):
+            Prefill.into_expert(me, NS(shape=x_shape), NS(dims=NS(**dims), cfg=NS(**cfg)))
