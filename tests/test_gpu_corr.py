@@ -9,10 +9,8 @@ roundoff 6e-8, grown about sqrt(n) over sums of up to n = 2048 terms (~3e-6 rela
 some twenty dependent stages whose LayerNorms rescale by O(1): well inside 5e-4 max-abs and
 5e-5 relative L2 on the O(1) outputs. The confidence is held to the same 5e-4.
 
-These kernels have not yet run on a GB300: the tests run when JPI_CORR_GPU_TESTS=1 is set.
+These kernels have not yet run on a GB300: the tests run when JPI_NEW_GPU_TESTS=1 is set.
 """
-
-import os
 
 import numpy as np
 import pytest
@@ -22,11 +20,9 @@ import oracle.correction as oc
 from synth import (PI05_CORRECTION, TINY, make_correction_inputs, make_correction_weights,
                    make_requests, make_weights)
 
-pytestmark = [
-    pytest.mark.gpu,
-    pytest.mark.skipif(os.environ.get("JPI_CORR_GPU_TESTS") != "1",
-                       reason="correction-module kernels not yet run on a GB300 (JPI_CORR_GPU_TESTS=1)"),
-]
+from tests.gpu_util import not_yet_run
+
+pytestmark = [pytest.mark.gpu, not_yet_run]
 
 MAX_ABS, REL_L2 = 5e-4, 5e-5
 
@@ -195,8 +191,6 @@ def test_alg1_on_the_gpu_components():
     mod.close()
 
 
-@pytest.mark.skipif(os.environ.get("JPI_PREFILL_GPU_TESTS") != "1",
-                    reason="prefill kernels not yet run on a GB300 (JPI_PREFILL_GPU_TESTS=1)")
 def test_alg1_with_every_component_on_the_gpu():
     # Prefill (KV straight into the expert's store) -> compressor -> expert at start-up, then
     # f_corr -> expert: the first chunk against the oracles' chain.

@@ -9,10 +9,8 @@ element, with fp32 sums and an fp32 residual stream; the K and V written are bf1
 After a few layers that is about 1% in relative L2, so the tests allow 2e-2 relative L2 and a
 max-abs of 5e-2 times the largest reference magnitude.
 
-These kernels have not yet run on a GB300: the tests run when JPI_PREFILL_GPU_TESTS=1 is set.
+These kernels have not yet run on a GB300: the tests run when JPI_NEW_GPU_TESTS=1 is set.
 """
-
-import os
 
 import numpy as np
 import pytest
@@ -20,11 +18,9 @@ import pytest
 import oracle.prefill as pf
 from synth import GEMMA2B, PI05, make_llm_weights, make_prefix_embeddings, make_requests, make_weights
 
-pytestmark = [
-    pytest.mark.gpu,
-    pytest.mark.skipif(os.environ.get("JPI_PREFILL_GPU_TESTS") != "1",
-                       reason="prefill kernels not yet run on a GB300 (JPI_PREFILL_GPU_TESTS=1)"),
-]
+from tests.gpu_util import not_yet_run
+
+pytestmark = [pytest.mark.gpu, not_yet_run]
 
 REL_L2, MAX_ABS_FRAC = 2e-2, 5e-2
 SMALL = GEMMA2B.with_(n_layers=3, width=256, n_heads=4, head_dim=64, mlp_dim=512, precision="bf16")

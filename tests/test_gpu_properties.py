@@ -5,7 +5,7 @@ import numpy as np
 import pytest
 
 from synth import TINY, make_requests, make_weights
-from tests.gpu_util import SMALL_BF16, gpu_denoise, lib, make_expert, to_dev_kv
+from tests.gpu_util import SMALL_BF16, gpu_denoise, lib, make_expert, not_yet_run, to_dev_kv
 
 pytestmark = pytest.mark.gpu
 torch = pytest.importorskip("torch")
@@ -161,3 +161,20 @@ def test_errors_are_status_codes():
         assert np.isfinite(gpu_denoise(ex, cfg, r, 2)).all()
     finally:
         ex.close()
+
+
+@not_yet_run
+def test_out_of_memory_is_a_status_and_frees_everything():
+    # Maxima the shape checks accept but whose KV store cannot fit (about 56 TB): create fails with
+    # JPI_ERR_OOM after about 14 GB of other buffers, and gives every one of them back.
+    jpi = lib()
+    cfg = TINY
+    w = make_weights(cfg, 36)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    with pytest.raises(jpi.JpiError) as e:
+        jpi.Expert(cfg, w, max_batch=(1 << 20) // 10, max_prefix=1 << 20, max_chunk=1, max_steps=1)
+    assert e.value.status == -3, e.value
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert abs(free1 - free0) < (64 << 20)
