@@ -60,25 +60,26 @@ def source_sha() -> str:
     return h.hexdigest()[:16]
 
 
-def algorithmic_bytes(cfg, B, P, C, N):
+def algorithmic_bytes(cfg, B, P, C, N, items=0):
     """Bytes an ideal denoise must move: weights once per step (bf16), the time/modulation
-    weights once per call, the prefix KV once, inputs and outputs."""
+    weights once per call, the prefix KV once, inputs (with `items` fp32 correction items per
+    request) and outputs."""
     W, H, D, F, L, A = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim, cfg.n_layers, cfg.action_dim
     per_step = (L * (H * D * W * 2 + 2 * D * W + 3 * F * W) + (cfg.state_dim + 2 * A) * W) * 2
     time_w = (W * cfg.time_dim + W * W + (6 * L + 2) * W * W) * 2
     kv = B * L * P * D * 2 * 2
-    io = B * (cfg.state_dim + 2 * C * A) * 4
+    io = B * (cfg.state_dim + 2 * C * A + items * W) * 4
     return N * per_step + time_w + kv + io
 
 
-def algorithmic_flops(cfg, B, P, C, N):
-    """Multiply-adds x 2 of a denoise: the layer projections at M = B (C + 1) tokens, the
+def algorithmic_flops(cfg, B, P, C, N, items=0):
+    """Multiply-adds x 2 of a denoise: the layer projections at M = B (C + 1 + items) tokens, the
     attention of the S H query rows over all P + S keys (QK^T and PV), the state/action
     embeddings and the action-out projection, and per step time the time MLP and the
     modulation GEMV."""
     W, H, D, F, L = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim, cfg.n_layers
     Sd, A = cfg.state_dim, cfg.action_dim
-    S = C + 1
+    S = C + 1 + items
     Mt = B * S
     proj = L * (H * D * W + 2 * D * W + H * D * W + 3 * F * W)
     attn = L * B * S * H * (P + S) * D * 2
@@ -87,14 +88,14 @@ def algorithmic_flops(cfg, B, P, C, N):
     return N * (per_step + per_time)
 
 
-def op_bytes(cfg, op, B, P, C):
+def op_bytes(cfg, op, B, P, C, items=0):
     """Algorithmic bytes of one launch of a layer op (weights + activation reads/writes)."""
     W, H, D, F = cfg.width, cfg.n_heads, cfg.head_dim, cfg.mlp_dim
-    Mt = B * (C + 1)
+    Mt = B * (C + 1 + items)
     if op == 2:
         return (H + 2) * D * W * 2 + Mt * W * 4 + Mt * (H + 2) * D * 2
     if op == 3:
-        return B * (P + C + 1) * D * 2 * 2 + Mt * H * D * 2 * 2
+        return B * (P + C + 1 + items) * D * 2 * 2 + Mt * H * D * 2 * 2
     if op == 4:
         return W * H * D * 2 + Mt * H * D * 2 + Mt * W * 4 * 2
     if op == 5:
@@ -286,7 +287,7 @@ def our_arm(args):
     import torch.distributed as dist
 
     from paper_2607_12659_gb300 import build, jpi
-    from synth import PI05, make_requests, make_weights
+    from synth import PI05, make_correction, make_requests, make_weights
 
     world, rank, local = rank_env()
     torch.cuda.set_device(local)
@@ -300,7 +301,7 @@ def our_arm(args):
 
     B, P, C, N = (WORKLOAD[k] for k in ("batch", "prefix", "chunk", "steps"))
     B, P = args.batch or B, args.prefix or P
-    default_workload = (B, P) == (WORKLOAD["batch"], WORKLOAD["prefix"])
+    default_workload = (B, P) == (WORKLOAD["batch"], WORKLOAD["prefix"]) and not args.items
     cfg = PI05
     w = make_weights(cfg, 2000)
     ex = jpi.Expert(cfg, w, max_batch=B, max_prefix=P, max_chunk=C, max_steps=N)
@@ -308,6 +309,9 @@ def our_arm(args):
     r = make_requests(cfg, request_seed(rank), B, P, C)
     ex.set_prefix_kv(torch.from_numpy(r["prefix_k"]).cuda().to(torch.bfloat16),
                      torch.from_numpy(r["prefix_v"]).cuda().to(torch.bfloat16))
+    if args.items:
+        # The correction items of Sec. 4.1 as context tokens (T' = 4 in App. B).
+        ex.set_correction(torch.from_numpy(make_correction(cfg, request_seed(rank) + 1, B, args.items)).cuda())
     state = torch.from_numpy(r["state"]).cuda()
     noise = torch.from_numpy(r["noise"]).cuda()
     out = torch.empty_like(noise)
@@ -375,16 +379,16 @@ def our_arm(args):
         op_ms[op] = a.elapsed_time(b) / reps
     dom = max(op_ms, key=op_ms.get)
     hbm_peak, tc_peak, peak_src = measured_peaks()
-    dom_bytes = op_bytes(cfg, dom, B, P, C)
+    dom_bytes = op_bytes(cfg, dom, B, P, C, args.items)
     achieved = dom_bytes / (op_ms[dom] * 1e-3) / 1e9
     sha = source_sha()
     tr = NCU_TRAFFIC.get(OP_NAMES[dom])
     traffic = tr["bytes"] if tr and tr.get("source_sha256") == sha and default_workload else None
 
     n_kernels = jpi.jpi_graph_kernel_count(ex.handle, B, C, N)
-    alg = algorithmic_bytes(cfg, B, P, C, N)
+    alg = algorithmic_bytes(cfg, B, P, C, N, args.items)
     path_bw = alg / (ms_per_step * 1e-3) / 1e9
-    flops = algorithmic_flops(cfg, B, P, C, N)
+    flops = algorithmic_flops(cfg, B, P, C, N, args.items)
     path_tf = flops / (ms_per_step * 1e-3) / 1e12
 
     if rank == 0:
@@ -400,8 +404,9 @@ def our_arm(args):
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": WORKLOAD_NAME if default_workload else
-                       WORKLOAD_NAME.replace("batch 1, prefix 816", f"batch {B}, prefix {P}"),
-                       **WORKLOAD, "batch": B, "prefix": P,
+                       WORKLOAD_NAME.replace("batch 1, prefix 816", f"batch {B}, prefix {P}")
+                       + (f", {args.items} correction items" if args.items else ""),
+                       **WORKLOAD, "batch": B, "prefix": P, "correction_items": args.items,
                        "l2": "no flush: each call streams 6.2 GB of weights (> 129 MB L2)",
                        "parallelism": f"replicas x{world}"},
             "us_per_denoise": {"median": statistics.median(per) * 1e3,
@@ -597,6 +602,8 @@ def main():
     ap.add_argument("--batch", type=int, default=0,
                     help="requests per denoise (default: the batch-1 workload); for documentation runs")
     ap.add_argument("--prefix", type=int, default=0, help="prefix tokens per request (default 816)")
+    ap.add_argument("--items", type=int, default=0,
+                    help="correction items (context tokens) per request, 0..8; for documentation runs")
     ap.add_argument("--cpu-baseline-child", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
     if args.cpu_baseline_child:

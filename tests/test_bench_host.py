@@ -42,19 +42,20 @@ def test_pi05_step_weights_are_the_paper_sized_expert():
     assert bench.algorithmic_bytes(PI05, 1, 816, 50, 10) == 6_480_441_984
 
 
-@pytest.mark.parametrize("B,P,C,N", [(1, 816, 50, 10), (64, 2048, 50, 10), (3, 17, 8, 2)])
-def test_algorithmic_flops_from_the_weight_shapes(B, P, C, N):
+@pytest.mark.parametrize("B,P,C,N,T", [(1, 816, 50, 10, 0), (64, 2048, 50, 10, 0), (3, 17, 8, 2, 0),
+                                       (1, 816, 50, 10, 4)])
+def test_algorithmic_flops_from_the_weight_shapes(B, P, C, N, T):
     cfg = PI05
     ws = weight_shapes(cfg)
     L, H, D, W = cfg.n_layers, cfg.n_heads, cfg.head_dim, cfg.width
-    S = C + 1
+    S = C + 1 + T                                  # state token, T correction items, C actions
     macs_step = (B * S * L * sum(_size(ws[k]) for k in LAYER_PROJ)
                  + L * B * 2 * (S * H) * (P + S) * D                       # QK^T and PV
                  + B * _size(ws["state_in_w"]) + B * C * _size(ws["action_in_w"])
                  + B * C * _size(ws["action_out_w"]))
     macs_time = (_size(ws["time_mlp_in_w"]) + _size(ws["time_mlp_out_w"])
                  + L * (_size(ws["attn_mod_w"]) + _size(ws["mlp_mod_w"])) + _size(ws["final_mod_w"]))
-    assert bench.algorithmic_flops(cfg, B, P, C, N) == 2 * N * (macs_step + macs_time)
+    assert bench.algorithmic_flops(cfg, B, P, C, N, T) == 2 * N * (macs_step + macs_time)
 
 
 def test_layer_op_bytes_cover_each_layer_weight_once():
