@@ -22,6 +22,14 @@ MUTATIONS = [
     ("(gelu_tanh(u @ w[\"w_gate\"][l].T) * (u @ w[\"w_up\"][l].T))", "(gelu_tanh(u @ w[\"w_up\"][l].T) * (u @ w[\"w_gate\"][l].T))"),
     ("        return K, V, rms_modulate(h, w[\"final_norm\"], 0.0, cfg.rms_eps)", "        return K, V, h"),
     ("        h = h + o @ w[\"wo\"][l].T", "        h = o @ w[\"wo\"][l].T"),
+    ("        o = attention(q, k, v, visible).reshape(P, H * D)", "        o = attention(q, k, k, visible).reshape(P, H * D)"),
+    ("        q = rope(q, pos, cfg.rope_base)                            # R18", "        q = q"),
+    ("        K[l], V[l] = k, v                                          # R20", "        K[l], V[l] = v, k"),
+    ("h = h + (gelu_tanh(u @ w[\"w_gate\"][l].T) * (u @ w[\"w_up\"][l].T)) @ w[\"w_down\"][l].T",
+     "h = (gelu_tanh(u @ w[\"w_gate\"][l].T) * (u @ w[\"w_up\"][l].T)) @ w[\"w_down\"][l].T"),
+    ("        return K, V, rms_modulate(h, w[\"final_norm\"], 0.0, cfg.rms_eps)",
+     "        return K, V, rms_modulate(h, w[\"final_norm\"] - 1.0, 0.0, cfg.rms_eps)"),
+    ("        q = (u @ w[\"wq\"][l].T).reshape(P, H, D)", "        q = (u @ w[\"wq\"][l].T).reshape(H, P, D).transpose(1, 0, 2)"),
 ]
 
 
