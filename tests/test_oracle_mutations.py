@@ -43,6 +43,14 @@ MUTATIONS = [
     ("base ** (-2.0 * np.arange(half, dtype=F64) / D)", "base ** (-1.0 * np.arange(half, dtype=F64) / D)"),
     ("scores = scores - scores.max(axis=-1, keepdims=True)", "scores = scores - scores.min(axis=-1, keepdims=True)"),
     ("return z / (1.0 + np.exp(-z))", "return z / (1.0 + np.exp(z))"),
+    ("x = x + delta * expert_forward", "x = x - delta * expert_forward"),
+    ("u = rms_modulate(h, fm[:W], fm[W:], cfg.rms_eps)", "u = rms_modulate(h, fm[W:], fm[:W], cfg.rms_eps)"),
+    ("mm[:W], mm[W:2 * W], mm[2 * W:]", "mm[W:2 * W], mm[:W], mm[2 * W:]"),
+    ("u = rms_modulate(h, sm, bm, cfg.rms_eps)", "u = rms_modulate(h, sa, ba, cfg.rms_eps)"),
+    ('h[0] = w["state_in_w"] @ s + w["state_in_b"]', 'h[0] = w["state_in_w"] @ s'),
+    ('vel = u[n_ctx:] @ w["action_out_w"].T + w["action_out_b"]', 'vel = u[n_ctx:] @ w["action_out_w"].T'),
+    ("        k = rope(k, pos, cfg.rope_base)\n", "        k = rope(k, pos, cfg.rope_base)\n        v = rope(v, pos, cfg.rope_base)\n"),
+    ("V = np.concatenate([prefix_v[l], v], axis=0)", "V = np.concatenate([prefix_k[l], v], axis=0)"),
 ]
 
 

@@ -242,6 +242,30 @@ def test_zero_gates_make_every_layer_the_identity():
     np.testing.assert_allclose(h[1:], x @ w["action_in_w"].T + w["action_in_b"], rtol=1e-14)
 
 
+def test_velocity_through_identity_layers_by_scalar_loops():
+    # With both gates zero every layer is the identity, so the velocity of action j is the final
+    # norm of its embedding: u = e / rms(e) * (1 + sigma_f) + beta_f with (sigma_f, beta_f) the
+    # first and second halves of M_f c + m_f (R5), then v = W_out u + b_out. Rebuilt by loops.
+    w, r = micro_setup(mod_bias_std=0.7)
+    W, A = MICRO.width, MICRO.action_dim
+    for l in range(MICRO.n_layers):
+        for mw, mb in (("attn_mod_w", "attn_mod_b"), ("mlp_mod_w", "mlp_mod_b")):
+            w[mw][l][2 * W:] = 0.0
+            w[mb][l][2 * W:] = 0.0
+    t = 0.3
+    x, s = r["noise"][0].astype(float), r["state"][0].astype(float)
+    v = oracle.expert_forward(x, s, t, r["prefix_k"][:, 0].astype(float), r["prefix_v"][:, 0].astype(float),
+                              w, MICRO)
+    c = oracle.time_conditioning(t, w, MICRO)
+    fm = [sum(w["final_mod_w"][i][k] * c[k] for k in range(W)) + w["final_mod_b"][i] for i in range(2 * W)]
+    for j in range(x.shape[0]):
+        e = [sum(w["action_in_w"][i][a] * x[j][a] for a in range(A)) + w["action_in_b"][i] for i in range(W)]
+        rms = math.sqrt(sum(q * q for q in e) / W + MICRO.rms_eps)
+        u = [e[i] / rms * (1.0 + fm[i]) + fm[W + i] for i in range(W)]
+        want = [sum(w["action_out_w"][a][i] * u[i] for i in range(W)) + w["action_out_b"][a] for a in range(A)]
+        np.testing.assert_allclose(v[j], want, rtol=1e-12, atol=1e-13)
+
+
 def test_state_row_does_not_see_the_actions():
     w, r = micro_setup(mod_bias_std=1.0)
     args = (r["prefix_k"][:, 0].astype(float), r["prefix_v"][:, 0].astype(float), w, MICRO)
