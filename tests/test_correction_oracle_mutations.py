@@ -51,6 +51,14 @@ MUTATIONS = [
      "confidence = float(w[\"conf_w\"][0] @ x.mean(axis=0) + w[\"conf_b\"][0])"),
     ("    return future_correction(qformer_compress(h_vlm, w, cfg), actions, w, cfg)",
      "    return future_correction(h_vlm[:cfg.n_items, :cfg.width], actions, w, cfg)"),
+    ("    x = x + w[\"act_pos\"][:n]", "    x = x"),
+    ("return (x - mu) / np.sqrt(var + eps) * w + b", "return (x - mu) / np.sqrt(var) * w + b"),
+    ("    for i in range(cfg.n_joint):", "    for i in reversed(range(cfg.n_joint)):"),
+    ("confidence = float(w[\"conf_w\"][0] @ u.mean(axis=0) + w[\"conf_b\"][0])",
+     "confidence = float(w[\"conf_w\"][0] @ u.mean(axis=0))"),
+    ("    x = x + mlp(u, w, \"qf_mlp_\")", "    x = mlp(u, w, \"qf_mlp_\")"),
+    ("x = gelu_tanh(actions @ w[\"act_w1\"].T + w[\"act_b1\"]) @ w[\"act_w2\"].T + w[\"act_b2\"]",
+     "x = (actions @ w[\"act_w1\"].T + w[\"act_b1\"]) @ w[\"act_w2\"].T + w[\"act_b2\"]"),
 ]
 
 
