@@ -180,10 +180,19 @@ def corrector_corr(corrector):
     """f_corr over the library's correction module: the state buffer holds a compressed state
     ([1][T'][width] CUDA tensor) and the committed actions are the executor's action rows; returns
     the predicted state (on the device) and its confidence (one host float, read back because the
-    scheduler branches on it)."""
+    scheduler branches on it).
+
+    With no committed action (the executor ran the buffer dry) there is nothing to predict ahead:
+    the state passes through with confidence 0, the value Alg. 1 starts from. More committed
+    actions than the module's position table holds is an error."""
     import torch
 
     def corr(h, actions):
+        if len(actions) == 0:
+            return h, 0.0
+        if len(actions) > corrector.dims.max_delta:
+            raise ValueError(f"{len(actions)} committed actions exceed the correction module's "
+                             f"max_delta {corrector.dims.max_delta}")
         a = torch.as_tensor(np.stack([np.asarray(x, np.float32) for x in actions])[None],
                             device=h.device)
         h_future, conf = corrector.predict(h, a)

@@ -139,3 +139,29 @@ def test_theta_must_be_negative():
         make(Script([]), theta=0.1)
     with pytest.raises(RuntimeError):
         make(Script([])).iterate()
+
+
+def test_library_f_corr_handles_an_empty_buffer_and_too_many_actions():
+    # The glue over the correction module, with a stand-in module that records its inputs.
+    torch = pytest.importorskip("torch")
+    import numpy as np
+    from types import SimpleNamespace
+    from paper_2607_12659_gb300.scheduler import corrector_corr
+
+    seen = []
+
+    class Stub:
+        dims = SimpleNamespace(max_delta=3)
+
+        def predict(self, h, a):
+            seen.append(a.shape)
+            return h + 1.0, torch.tensor([-0.5])
+
+    corr = corrector_corr(Stub())
+    h = torch.zeros(1, 2, 4)
+    h2, c = corr(h, [])
+    assert h2 is h and c == 0.0 and not seen            # nothing to predict ahead
+    h3, c = corr(h, [np.ones(5), np.zeros(5)])
+    assert seen == [(1, 2, 5)] and c == -0.5 and float(h3[0, 0, 0]) == 1.0
+    with pytest.raises(ValueError):
+        corr(h, [np.ones(5)] * 4)
