@@ -19,7 +19,9 @@ the first iteration after start-up skips the VLM (Alg. 1 initialises it as a lar
 
 Actions are indexed by control step. `ActionBuffer` is what an executor thread consumes
 (`pop`) while the scheduler refills it (`replace_from`); the scheduler advances t by what was
-executed meanwhile.
+executed meanwhile. The new chunk starts right after the committed actions f_corr was given:
+t + delta_ae (or t + delta) while the buffer holds that many, earlier when it holds fewer, so
+the executor, which stops at the first empty control step, always reaches it.
 """
 
 from __future__ import annotations
@@ -138,7 +140,7 @@ class ConfidenceScheduler:
             committed = self.buffer.committed(self.delta_ae)
             h_future, c = self.corr(self.h, committed)
             chunk = self.act(h_future, self.kv)
-            self.buffer.replace_from(t + self.delta_ae, chunk)
+            self.buffer.replace_from(t + len(committed), chunk)
             branch = "correction"
         else:
             obs = self.observe()
@@ -147,7 +149,7 @@ class ConfidenceScheduler:
             self.kv = kv_t
             h_future, c = self.corr(h_t, committed)
             chunk = self.act(h_future, self.kv)
-            self.buffer.replace_from(t + self.delta, chunk)
+            self.buffer.replace_from(t + len(committed), chunk)
             branch = "vlm"
         self.h = h_future
         self.confidence = float(c)

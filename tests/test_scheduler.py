@@ -165,3 +165,19 @@ def test_library_f_corr_handles_an_empty_buffer_and_too_many_actions():
     assert seen == [(1, 2, 5)] and c == -0.5 and float(h3[0, 0, 0]) == 1.0
     with pytest.raises(ValueError):
         corr(h, [np.ones(5)] * 4)
+
+
+def test_a_short_buffer_puts_the_new_chunk_right_after_what_is_committed():
+    # Only one action is left when delta_ae = 3 would be committed: the prediction covers that
+    # one action and the new chunk starts right after it, so the executor never stalls on an
+    # empty control step.
+    s = Script([0.5, 0.5], C=4)
+    sch = make(s, delta=6, delta_ae=3)
+    sch.start()
+    for _ in range(3):
+        sch.buffer.pop()                              # steps 0..2 executed, step 3 left
+    assert sch.iterate() == "correction"
+    assert s.calls[-2] == ("corr", ("h", 1), [("a", 1, 3)])
+    assert sch.buffer.committed(5) == [("a", 1, 3), ("a", 2, 0), ("a", 2, 1), ("a", 2, 2), ("a", 2, 3)]
+    popped = [sch.buffer.pop() for _ in range(5)]
+    assert popped[-1] == ("a", 2, 3) and sch.buffer.next_step == 8
