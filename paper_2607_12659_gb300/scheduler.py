@@ -48,12 +48,15 @@ class ActionBuffer:
             return self._next
 
     def replace_from(self, step: int, chunk: Sequence[Any]) -> None:
-        """Drop every action at or after `step` and store `chunk[k]` at step + k."""
+        """Drop every action at or after `step` and store `chunk[k]` at step + k. Steps the
+        executor has already passed (it kept running while the chunk was computed) are not
+        stored: their time is gone."""
         with self._lock:
             for s in [s for s in self._actions if s >= step]:
                 del self._actions[s]
             for k, a in enumerate(chunk):
-                self._actions[step + k] = a
+                if step + k >= self._next:
+                    self._actions[step + k] = a
 
     def committed(self, n: int) -> list:
         """The next n actions to be executed (those the robot runs while inference is in

@@ -181,3 +181,14 @@ def test_a_short_buffer_puts_the_new_chunk_right_after_what_is_committed():
     assert sch.buffer.committed(5) == [("a", 1, 3), ("a", 2, 0), ("a", 2, 1), ("a", 2, 2), ("a", 2, 3)]
     popped = [sch.buffer.pop() for _ in range(5)]
     assert popped[-1] == ("a", 2, 3) and sch.buffer.next_step == 8
+
+
+def test_a_chunk_that_arrives_late_keeps_only_its_future_steps():
+    b = ActionBuffer()
+    b.replace_from(0, [1, 2, 3, 4, 5])
+    for _ in range(3):
+        b.pop()                                       # steps 0..2 ran while the chunk was computed
+    b.replace_from(1, [20, 30, 40, 50])               # meant for steps 1..4
+    assert b.committed(3) == [40, 50] and len(b) == 2
+    assert b.pop() == 40 and b.pop() == 50 and b.pop() is None
+    assert len(b._actions) == 0                       # nothing stale left behind
