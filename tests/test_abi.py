@@ -144,3 +144,31 @@ def test_prefill_into_expert_refuses_stores_it_does_not_fit():
                                ((1, 40, 256), dict(precision="bf16"), {**store, "head_dim": 64})]:
         with pytest.raises(ValueError):
             Prefill.into_expert(me, NS(shape=x_shape), NS(dims=NS(**dims), cfg=NS(**cfg)))
+
+
+def _c_layout(struct, fields, tmp_path):
+    """sizeof and offsetof of a C struct from the public headers, by compiling a probe with gcc."""
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    src = tmp_path / f"{struct}.c"
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "jpi.h"', '#include "jpi_corr.h"',
+             '#include "jpi_prefill.h"', "int main(void) {", f'  printf("%zu\\n", sizeof({struct}));']
+    lines += [f'  printf("%zu\\n", offsetof({struct}, {f}));' for f in fields]
+    lines += ["  return 0;", "}"]
+    src.write_text("\n".join(lines))
+    exe = tmp_path / struct
+    subprocess.run(["gcc", "-I", inc, str(src), "-o", str(exe)], check=True, capture_output=True)
+    out = [int(x) for x in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    return out[0], out[1:]
+
+
+@pytest.mark.parametrize("mod,name", [("jpi", "jpi_config"), ("jpi", "jpi_weights"), ("corr", "jpi_corr_config"),
+                                      ("corr", "jpi_corr_block"), ("corr", "jpi_corr_weights"),
+                                      ("prefill", "jpi_prefill_config"), ("prefill", "jpi_prefill_weights")])
+def test_binding_structs_match_the_c_layout(mod, name, tmp_path):
+    import importlib
+    m = importlib.import_module(f"paper_2607_12659_gb300.{mod}")
+    st = getattr(m, name)
+    fields = [f[0] for f in st._fields_]
+    size, offsets = _c_layout(name, fields, tmp_path)
+    assert ctypes.sizeof(st) == size, (name, ctypes.sizeof(st), size)
+    assert [getattr(st, f).offset for f in fields] == offsets, name
