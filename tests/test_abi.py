@@ -172,3 +172,25 @@ def test_binding_structs_match_the_c_layout(mod, name, tmp_path):
     size, offsets = _c_layout(name, fields, tmp_path)
     assert ctypes.sizeof(st) == size, (name, ctypes.sizeof(st), size)
     assert [getattr(st, f).offset for f in fields] == offsets, name
+
+
+def _header_arities():
+    """Number of parameters of every JPI_API function in include/*.h."""
+    import re
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    arity = {}
+    for f in os.listdir(inc):
+        text = re.sub(r"/\*.*?\*/", "", open(os.path.join(inc, f)).read(), flags=re.S)
+        for m in re.finditer(r"JPI_API\s+[\w\s\*]+?\b(jpi_\w+)\s*\(([^;]*?)\)\s*;", text, flags=re.S):
+            params = m.group(2).strip()
+            arity[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
+    return arity
+
+
+def test_binding_signatures_have_the_c_arity():
+    from paper_2607_12659_gb300 import corr, prefill
+    arity = _header_arities()
+    sigs = {**jpi._SIGS, **corr._SIGS, **prefill._SIGS}
+    assert set(sigs) | {"jpi_last_error", "jpi_prefill_last_error"} == set(arity)
+    for name, args in sigs.items():
+        assert len(args) == arity[name], (name, len(args), arity[name])
