@@ -174,23 +174,41 @@ def test_binding_structs_match_the_c_layout(mod, name, tmp_path):
     assert [getattr(st, f).offset for f in fields] == offsets, name
 
 
-def _header_arities():
-    """Number of parameters of every JPI_API function in include/*.h."""
+def _header_params():
+    """Parameter kinds ('ptr', 'int', 'float', 'longlong') of every JPI_API function in include/*.h."""
     import re
     inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
-    arity = {}
+    sig = {}
     for f in os.listdir(inc):
         text = re.sub(r"/\*.*?\*/", "", open(os.path.join(inc, f)).read(), flags=re.S)
         for m in re.finditer(r"JPI_API\s+[\w\s\*]+?\b(jpi_\w+)\s*\(([^;]*?)\)\s*;", text, flags=re.S):
             params = m.group(2).strip()
-            arity[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
-    return arity
+            kinds = []
+            for p in ([] if params in ("", "void") else params.split(",")):
+                p = " ".join(p.split())
+                if "*" in p:
+                    kinds.append("ptr")
+                elif p.startswith("long long"):
+                    kinds.append("longlong")
+                elif p.startswith("float"):
+                    kinds.append("float")
+                else:
+                    assert p.startswith("int "), p
+                    kinds.append("int")
+            sig[m.group(1)] = kinds
+    return sig
 
 
-def test_binding_signatures_have_the_c_arity():
+def test_binding_signatures_match_the_c_prototypes():
     from paper_2607_12659_gb300 import corr, prefill
-    arity = _header_arities()
+    want = _header_params()
     sigs = {**jpi._SIGS, **corr._SIGS, **prefill._SIGS}
-    assert set(sigs) | {"jpi_last_error", "jpi_prefill_last_error"} == set(arity)
+    assert set(sigs) | {"jpi_last_error", "jpi_prefill_last_error"} == set(want)
+
+    def kind(t):
+        if t is ctypes.c_void_p or hasattr(t, "_type_") and isinstance(t, type(ctypes.POINTER(ctypes.c_int))):
+            return "ptr"
+        return {ctypes.c_int: "int", ctypes.c_float: "float", ctypes.c_longlong: "longlong"}[t]
+
     for name, args in sigs.items():
-        assert len(args) == arity[name], (name, len(args), arity[name])
+        assert [kind(a) for a in args] == want[name], (name, [kind(a) for a in args], want[name])
