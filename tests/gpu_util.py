@@ -21,11 +21,6 @@ SMALL_BF16 = ExpertConfig(n_layers=2, width=256, n_heads=2, head_dim=128, mlp_di
 
 _built = False
 
-# Tests written while no GPU time was left: they run once JPI_NEW_GPU_TESTS=1 is set, until their
-# first GB300 run has passed and the mark is removed.
-not_yet_run = pytest.mark.skipif(os.environ.get("JPI_NEW_GPU_TESTS") != "1",
-                                 reason="written without GPU time; not yet run on a GB300 (JPI_NEW_GPU_TESTS=1)")
-
 
 def lib():
     global _built

@@ -8,8 +8,6 @@ oracle's (bf16-representable in bf16 precision), so the differences are fp32 rou
 roundoff 6e-8, grown about sqrt(n) over sums of up to n = 2048 terms (~3e-6 relative) and over
 some twenty dependent stages whose LayerNorms rescale by O(1): well inside 5e-4 max-abs and
 5e-5 relative L2 on the O(1) outputs. The confidence is held to the same 5e-4.
-
-These kernels have not yet run on a GB300: the tests run when JPI_NEW_GPU_TESTS=1 is set.
 """
 
 import numpy as np
@@ -20,9 +18,8 @@ import oracle.correction as oc
 from synth import (PI05_CORRECTION, TINY, make_correction_inputs, make_correction_weights,
                    make_requests, make_weights)
 
-from tests.gpu_util import not_yet_run
 
-pytestmark = [pytest.mark.gpu, not_yet_run]
+pytestmark = pytest.mark.gpu
 
 MAX_ABS, REL_L2 = 5e-4, 5e-5
 
@@ -56,13 +53,12 @@ def _setup(cfg, seed, B, T, delta, std=0.1, max_batch=4, max_tokens=64):
     return mod, w, inp, dev
 
 
-@pytest.mark.parametrize("precision", ["fp32", "bf16"])
-@pytest.mark.parametrize("vlm_dtype", ["float32", "bfloat16"])
+# bf16 VLM states are drawn in bf16 precision only, so that pairing has no fp32 case.
+@pytest.mark.parametrize("precision,vlm_dtype",
+                         [("fp32", "float32"), ("bf16", "float32"), ("bf16", "bfloat16")])
 def test_compressor_matches_the_oracle(precision, vlm_dtype):
     import torch
     cfg = SMALL.with_(precision=precision)
-    if vlm_dtype == "bfloat16" and precision == "fp32":
-        pytest.skip("bf16 VLM states are drawn in bf16 precision only")
     mod, w, inp, dev = _setup(cfg, 11, 3, 45, 5)
     hv = dev["h_vlm"].to(getattr(torch, vlm_dtype))
     got = mod.compress(hv)

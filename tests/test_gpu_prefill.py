@@ -8,8 +8,6 @@ coding, V, the probabilities, the attention output, the GeGLU output), each a re
 element, with fp32 sums and an fp32 residual stream; the K and V written are bf16 themselves.
 After a few layers that is about 1% in relative L2, so the tests allow 2e-2 relative L2 and a
 max-abs of 5e-2 times the largest reference magnitude.
-
-These kernels have not yet run on a GB300: the tests run when JPI_NEW_GPU_TESTS=1 is set.
 """
 
 import numpy as np
@@ -18,9 +16,8 @@ import pytest
 import oracle.prefill as pf
 from synth import GEMMA2B, PI05, make_llm_weights, make_prefix_embeddings, make_requests, make_weights
 
-from tests.gpu_util import not_yet_run
 
-pytestmark = [pytest.mark.gpu, not_yet_run]
+pytestmark = pytest.mark.gpu
 
 REL_L2, MAX_ABS_FRAC = 2e-2, 5e-2
 SMALL = GEMMA2B.with_(n_layers=3, width=256, n_heads=4, head_dim=64, mlp_dim=512, precision="bf16")

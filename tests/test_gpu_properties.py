@@ -5,7 +5,7 @@ import numpy as np
 import pytest
 
 from synth import TINY, make_requests, make_weights
-from tests.gpu_util import SMALL_BF16, gpu_denoise, lib, make_expert, not_yet_run, to_dev_kv
+from tests.gpu_util import SMALL_BF16, gpu_denoise, lib, make_expert, to_dev_kv
 
 pytestmark = pytest.mark.gpu
 torch = pytest.importorskip("torch")
@@ -163,7 +163,6 @@ def test_errors_are_status_codes():
         ex.close()
 
 
-@not_yet_run
 def test_out_of_memory_is_a_status_and_frees_everything():
     # Maxima the shape checks accept but whose KV store cannot fit (about 56 TB): create fails with
     # JPI_ERR_OOM after about 14 GB of other buffers, and gives every one of them back.
