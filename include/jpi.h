@@ -222,8 +222,12 @@ JPI_API jpi_status jpi_expert_forward(jpi_handle* h, const float* state, const f
  *     library holds until the process exits. width and time_dim above 8192 return
  *     JPI_ERR_SHAPE. The rest of the evaluation uses the handle's buffers, as
  *     jpi_expert_forward does.
- *   - The first call on a device resolves the array's device address (cudaGetSymbolAddress);
- *     make that first call before any stream capture on that device.
+ *   - The calling thread's current device must be the handle's device (else
+ *     JPI_ERR_INVALID_ARG). The first call in a CUDA context of a device resolves the array's
+ *     device address there (cudaGetSymbolAddress) and keeps it for that context; a new context
+ *     on the device (after cudaDeviceReset) resolves it again. Make the first call on a device,
+ *     and the first after a reset, before any stream capture on that device. The lookup is
+ *     safe to make from several host threads at once.
  *   - Every call shares the one array and overwrites it in full: calls that overlap on the GPU
  *     (on different streams, or with different handles) race on it.
  */

@@ -266,19 +266,6 @@ void free_handle(jpi_handle* h) {
     delete h;
 }
 
-// One Euler step (or one forward): token embedding, L layers, final norm + projection.
-jpi_status enqueue_step(jpi_handle* h, int step, int B, int C, float delta, float* v_out,
-                        cudaStream_t st) {
-    JPI_TRY(launch_embed(h, step, B, C, h->x, st));
-    for (int l = 0; l < h->L; ++l) {
-        if (h->tc)
-            JPI_TRY(tc_launch_layer(h, l, step, B, C, st));
-        else
-            JPI_TRY(launch_layer_simt(h, l, step, B, C, st));
-    }
-    return launch_final(h, step, B, C, delta, v_out ? nullptr : h->x, v_out, nullptr, st);
-}
-
 // The whole unrolled denoise: time conditioning for every step time, then N Euler steps.
 jpi_status enqueue_denoise(jpi_handle* h, int B, int C, int N, cudaStream_t st) {
     JPI_TRY(launch_time_embed(h, N, -1.0, st));
@@ -327,6 +314,21 @@ jpi_status get_graph(jpi_handle* h, int B, int C, int N, cudaGraphExec_t* out) {
     return JPI_OK;
 }
 
+}  // namespace
+
+// One Euler step (or one forward): token embedding, L layers, final norm + projection.
+jpi_status enqueue_step(jpi_handle* h, int step, int B, int C, float delta, float* v_out,
+                        cudaStream_t st) {
+    JPI_TRY(launch_embed(h, step, B, C, h->x, st));
+    for (int l = 0; l < h->L; ++l) {
+        if (h->tc)
+            JPI_TRY(tc_launch_layer(h, l, step, B, C, st));
+        else
+            JPI_TRY(launch_layer_simt(h, l, step, B, C, st));
+    }
+    return launch_final(h, step, B, C, delta, v_out ? nullptr : h->x, v_out, nullptr, st);
+}
+
 jpi_status check_call(jpi_handle* h, int B, int C, int N) {
     if (!h) return fail(JPI_ERR_INVALID_ARG, "handle is NULL");
     if (B < 1 || C < 1 || N < 1) return fail(JPI_ERR_INVALID_ARG, "batch, chunk and num_steps must be >= 1");
@@ -341,7 +343,6 @@ jpi_status check_call(jpi_handle* h, int B, int C, int N) {
     return JPI_OK;
 }
 
-}  // namespace
 }  // namespace jpi
 
 using namespace jpi;

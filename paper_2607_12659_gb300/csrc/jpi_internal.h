@@ -108,6 +108,7 @@ struct jpi_handle {
     bool pdl = true;          // programmatic dependent launch between tensor-core kernels
     int num_sms = 0;
     int attn_max_splits = 8;  // largest key-split cluster of the attention kernel
+    int attn_force_splits = 0;  // > 0: key splits asked of the split-KV attention (JPI_ATTN_SPLITS)
 
     // Dimensions.
     int L, W, H, D, F, A, Sd, dt, HD, QKV;   // QKV = (H + 2) D
@@ -200,5 +201,14 @@ jpi_status launch_final(jpi_handle* h, int step, int batch, int chunk, float del
                         float* x_inout, float* v_out, float* out_copy, cudaStream_t st);
 jpi_status launch_convert_kv(jpi_handle* h, const void* src, int src_fp32, void* dst,
                              int batch, int prefix_len, cudaStream_t st);
+
+// Entry-point helpers (api.cu). check_call: host-side checks of a denoise or forward call of
+// `B` requests, `C` actions and `N` steps against the handle's maxima, its prefix and its
+// correction items. enqueue_step: one Euler step (or, with v_out set, one forward pass) from
+// the modulation vectors of step slot `step`: token embedding, the L layers, final norm and
+// projection.
+jpi_status check_call(jpi_handle* h, int B, int C, int N);
+jpi_status enqueue_step(jpi_handle* h, int step, int B, int C, float delta, float* v_out,
+                        cudaStream_t st);
 
 }  // namespace jpi

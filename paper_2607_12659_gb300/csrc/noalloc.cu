@@ -4,7 +4,7 @@
 #include "jpi_internal.h"
 #include "tc_path.h"
 
-#include <cstdio>
+#include <mutex>
 
 namespace {
 
@@ -17,10 +17,69 @@ constexpr int NOALLOC_MAX_DIM = 8192;
 // clearing; calls that overlap on the GPU share them and race.
 static __device__ __align__(256) float g_noalloc_tc_scratch[3 * NOALLOC_MAX_DIM];
 
-// Device address of the array, resolved once per device (host code may not use the symbol
-// itself: on the host it names a stand-in, not device memory).
+// Device address of the array per device, with the id of the CUDA context it was resolved in.
+// Host code may not use the symbol itself: on the host it names a stand-in, not device memory.
+// A new context on the device (after cudaDeviceReset, say) has a new id, and the address is
+// resolved again.
 constexpr int MAX_DEVICES = 64;
-float* g_scratch_addr[MAX_DEVICES] = {};
+struct ScratchAddr {
+    unsigned long long ctx_id = 0;
+    bool valid = false;
+    float* ptr = nullptr;
+};
+ScratchAddr g_scratch[MAX_DEVICES];
+std::mutex g_scratch_mutex;
+
+// Driver entry points for the current context's id, resolved through the runtime so that the
+// library links no driver library.
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+jpi_status current_context_id(unsigned long long* id) {
+    static CtxGetCurrentFn get_current = nullptr;
+    static CtxGetIdFn get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            get_current = (CtxGetCurrentFn)p;
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            get_id = (CtxGetIdFn)p;
+    });
+    if (!get_current || !get_id) {
+        jpi::set_error("cuCtxGetCurrent / cuCtxGetId are unavailable from the driver");
+        return JPI_ERR_CUDA;
+    }
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, id) != CUDA_SUCCESS) {
+        jpi::set_error("no current CUDA context on the calling thread");
+        return JPI_ERR_CUDA;
+    }
+    return JPI_OK;
+}
+
+// The array's device address on `dev`, which is the calling thread's current device.
+jpi_status scratch_address(int dev, float** out) {
+    // Makes the device's primary context current on this thread if no call has done so yet.
+    JPI_CUDA_TRY(cudaSetDevice(dev));
+    unsigned long long id = 0;
+    JPI_TRY(current_context_id(&id));
+    std::lock_guard<std::mutex> lock(g_scratch_mutex);
+    ScratchAddr& a = g_scratch[dev];
+    if (!a.valid || a.ctx_id != id) {
+        void* p = nullptr;
+        JPI_CUDA_TRY(cudaGetSymbolAddress(&p, g_noalloc_tc_scratch));
+        a.ptr = (float*)p;
+        a.ctx_id = id;
+        a.valid = true;
+    }
+    *out = a.ptr;
+    return JPI_OK;
+}
 
 jpi_status fail(jpi_status s, const char* msg) {
     jpi::set_error("%s", msg);
@@ -34,25 +93,19 @@ extern "C" JPI_API jpi_status jpi_expert_forward_noalloc(jpi_handle* h, const fl
                                                          int chunk, float* out_v, float* out_h,
                                                          void* stream) {
     jpi::clear_error();
-    if (!h) return fail(JPI_ERR_INVALID_ARG, "handle is NULL");
+    JPI_TRY(jpi::check_call(h, batch, chunk, 1));
     if (!state || !x_t || !out_v) return fail(JPI_ERR_INVALID_ARG, "NULL input or output");
-    if (batch < 1 || chunk < 1) return fail(JPI_ERR_INVALID_ARG, "batch and chunk must be >= 1");
     if (!(t >= 0.f)) return fail(JPI_ERR_INVALID_ARG, "t must be >= 0");
-    if (batch > h->maxB || chunk > h->maxC) return fail(JPI_ERR_SHAPE, "batch or chunk exceeds the handle's maxima");
-    if (!h->prefix_ready) return fail(JPI_ERR_NOT_READY, "no prefix KV has been set");
-    if (batch != h->cur_batch) return fail(JPI_ERR_SHAPE, "batch differs from the prefix KV's batch");
     if (h->W > NOALLOC_MAX_DIM || h->dt > NOALLOC_MAX_DIM)
         return fail(JPI_ERR_SHAPE, "width or time_dim exceeds the fixed scratch (8192)");
 
     int dev = 0;
     JPI_CUDA_TRY(cudaGetDevice(&dev));
+    if (dev != h->device)
+        return fail(JPI_ERR_INVALID_ARG, "the calling thread's current device is not the handle's device");
     if (dev < 0 || dev >= MAX_DEVICES) return fail(JPI_ERR_UNSUPPORTED, "device ordinal above 63");
-    if (!g_scratch_addr[dev]) {
-        void* p = nullptr;
-        JPI_CUDA_TRY(cudaGetSymbolAddress(&p, g_noalloc_tc_scratch));
-        g_scratch_addr[dev] = (float*)p;
-    }
-    float* temb = g_scratch_addr[dev];
+    float* temb = nullptr;
+    JPI_TRY(scratch_address(dev, &temb));
     float* c1 = temb + NOALLOC_MAX_DIM;
     float* cond = c1 + NOALLOC_MAX_DIM;
 
@@ -62,14 +115,7 @@ extern "C" JPI_API jpi_status jpi_expert_forward_noalloc(jpi_handle* h, const fl
     JPI_CUDA_TRY(cudaMemcpyAsync(h->x, x_t, (size_t)batch * chunk * h->A * sizeof(float),
                                  cudaMemcpyDeviceToDevice, st));
     JPI_TRY(jpi::launch_time_conditioning_into(h, (double)t, temb, c1, cond, st));
-    JPI_TRY(jpi::launch_embed(h, 0, batch, chunk, h->x, st));
-    for (int l = 0; l < h->L; ++l) {
-        if (h->tc)
-            JPI_TRY(jpi::tc_launch_layer(h, l, 0, batch, chunk, st));
-        else
-            JPI_TRY(jpi::launch_layer_simt(h, l, 0, batch, chunk, st));
-    }
-    JPI_TRY(jpi::launch_final(h, 0, batch, chunk, 0.f, nullptr, out_v, nullptr, st));
+    JPI_TRY(jpi::enqueue_step(h, 0, batch, chunk, 0.f, out_v, st));
     if (out_h)
         JPI_CUDA_TRY(cudaMemcpyAsync(out_h, h->h, (size_t)batch * (chunk + h->n_ctx()) * h->W * sizeof(float),
                                      cudaMemcpyDeviceToDevice, st));
