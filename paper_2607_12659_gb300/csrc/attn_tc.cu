@@ -26,6 +26,7 @@
 #include "tc_path.h"
 
 #include <cooperative_groups.h>
+#include <cstdlib>
 
 namespace cg = cooperative_groups;
 
@@ -462,6 +463,8 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     // size it runs with; they never depend on timing.
     const int blocks = rblocks * B;
     int want = (2 * h->num_sms + blocks - 1) / blocks;
+    // A split count asked through the environment at create time replaces that choice.
+    if (h->attn_force_splits > 0) want = h->attn_force_splits;
     want = want < 1 ? 1 : (want > h->attn_max_splits ? h->attn_max_splits : want);
     int chunk = (nk + want - 1) / want;
     chunk = (chunk + 15) / 16 * 16;
@@ -533,6 +536,10 @@ bool attn_tc_supported(const jpi_handle* h) {
 }
 
 jpi_status attn_tc_prepare(jpi_handle* h) {
+    // JPI_ATTN_SPLITS fixes the number of key splits (clamped to 1 .. the largest cluster),
+    // so that results can be compared across split counts; unset, the launch chooses.
+    const char* env = std::getenv("JPI_ATTN_SPLITS");
+    h->attn_force_splits = env ? std::atoi(env) : 0;
     // The query tile as 32-row boxes of 64 columns (128-byte swizzle) over q [maxMt * H][D].
     JPI_TRY(tc_make_tmap(h->q, (uint64_t)h->maxMt * h->H, h->D, AT_ROWS, &h->qmap_at));
     // K and V of all layers [L * maxB * kv_rows][D] as 32-row boxes.

@@ -167,6 +167,8 @@ struct jpi_handle {
     CUtensorMap qmap_at;        // q as 32-row boxes for the split-KV attention
     CUtensorMap kmap_at, vmap_at;   // K, V of all layers as 32-row boxes for it
     std::vector<CUtensorMap> tmaps;
+    bool mod_tc = false;        // modulation vectors on tensor cores (mod_tc.cu)
+    CUtensorMap mod_map;        // the stacked modulation matrix [(6L+2) W][W] as 128 x 64 boxes
     CUtensorMap xmaps[3];       // B operands: hx, o, z
 
     // State.

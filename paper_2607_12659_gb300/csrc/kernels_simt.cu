@@ -5,8 +5,10 @@
 // tree), so results are bitwise reproducible run to run.
 
 #include "jpi_internal.h"
+#include "tc_path.h"
 
 #include <cmath>
+#include <type_traits>
 
 namespace jpi {
 namespace {
@@ -546,8 +548,11 @@ void launch_mod_gemv(jpi_handle* h, const float* X, float* Y, int R, cudaStream_
     k_mod_gemv<T, NG><<<grid, threads, sizeof(float) * NG * W, st>>>((const T*)h->mod_w, h->mod_b, X, Y, R, W);
 }
 
+// bf16 weights with the tensor-core path: the tcgen05 kernel of mod_tc.cu; otherwise (and for
+// fp32 weights) the CUDA-core kernel above.
 template <typename T>
-void mod_gemv(jpi_handle* h, int g, const float* X, float* Y, int R, cudaStream_t st) {
+jpi_status mod_gemv(jpi_handle* h, int g, const float* X, float* Y, int R, cudaStream_t st) {
+    if (std::is_same<T, __nv_bfloat16>::value && h->mod_tc) return launch_mod_tc(h, X, Y, g, st);
     switch (g) {
 #define JPI_MOD_CASE(n) case n: launch_mod_gemv<T, n>(h, X, Y, R, st); break;
         JPI_MOD_CASE(1) JPI_MOD_CASE(2) JPI_MOD_CASE(3) JPI_MOD_CASE(4) JPI_MOD_CASE(5) JPI_MOD_CASE(6)
@@ -556,6 +561,7 @@ void mod_gemv(jpi_handle* h, int g, const float* X, float* Y, int R, cudaStream_
 #undef JPI_MOD_CASE
         default: break;
     }
+    return JPI_OK;
 }
 
 template <typename T>
@@ -583,7 +589,7 @@ jpi_status time_cond(jpi_handle* h, int N, cudaStream_t st) {
     }
     for (int n0 = 0; n0 < N; n0 += MOD_GROUP) {
         const int g = (N - n0) < MOD_GROUP ? (N - n0) : MOD_GROUP;
-        mod_gemv<T>(h, g, h->cond + (size_t)n0 * W, h->mods + (size_t)n0 * R, R, st);
+        JPI_TRY(mod_gemv<T>(h, g, h->cond + (size_t)n0 * W, h->mods + (size_t)n0 * R, R, st));
     }
     return check_launch("time conditioning");
 }
@@ -639,14 +645,14 @@ jpi_status launch_time_conditioning_into(jpi_handle* h, double t, float* temb, f
             (const T*)h->time_in_w, h->time_in_b, temb, c1, W, dt, 1);
         k_gemv_multi<T, true><<<grid_for((long long)W * 32, 256, 1024), blk, sizeof(float) * W, st>>>(
             (const T*)h->time_out_w, h->time_out_b, c1, cond, W, W, 1);
-        mod_gemv<T>(h, 1, cond, h->mods, R, st);
+        JPI_TRY(mod_gemv<T>(h, 1, cond, h->mods, R, st));
     } else {
         using T = float;
         k_gemv_multi<T, true><<<grid_for((long long)W * 32, 256, 1024), blk, sizeof(float) * dt, st>>>(
             (const T*)h->time_in_w, h->time_in_b, temb, c1, W, dt, 1);
         k_gemv_multi<T, true><<<grid_for((long long)W * 32, 256, 1024), blk, sizeof(float) * W, st>>>(
             (const T*)h->time_out_w, h->time_out_b, c1, cond, W, W, 1);
-        mod_gemv<T>(h, 1, cond, h->mods, R, st);
+        JPI_TRY(mod_gemv<T>(h, 1, cond, h->mods, R, st));
     }
     return check_launch("time conditioning (caller scratch)");
 }

@@ -471,6 +471,7 @@ jpi_status tc_prepare(jpi_handle* h) {
     JPI_TRY(make_tmap(h->hx, (uint64_t)xs_tiles(h->maxMt) * 64, h->W, NT, &h->xmaps[0]));
     JPI_TRY(make_tmap(h->o, h->maxMt, h->HD, NT, &h->xmaps[1]));
     JPI_TRY(make_tmap(h->z, h->maxMt, h->F, NT, &h->xmaps[2]));
+    JPI_TRY(mod_tc_prepare(h));
     return JPI_OK;
 }
 

@@ -24,6 +24,11 @@ jpi_status launch_attn_tc(jpi_handle* h, int layer, int batch, int chunk, cudaSt
 bool attn_t5_supported(const jpi_handle* h);
 jpi_status attn_t5_prepare(jpi_handle* h);
 jpi_status launch_attn_t5(jpi_handle* h, int layer, int batch, int chunk, cudaStream_t st);
+// Modulation vectors of N <= 16 step times on tensor cores (mod_tc.cu): Y [N][(6L+2) W] from
+// X [N][W]; used in bf16 mode when mod_tc_prepare set h->mod_tc.
+bool mod_tc_supported(const jpi_handle* h);
+jpi_status mod_tc_prepare(jpi_handle* h);
+jpi_status launch_mod_tc(jpi_handle* h, const float* X, float* Y, int N, cudaStream_t st);
 // 2D bf16 tensor map over [rows][cols] row-major, 128-byte swizzle, box {64 cols, box_rows}.
 jpi_status tc_make_tmap(const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows, CUtensorMap* map);
 // Frees what tc_prepare created outside the handle's allocation list.

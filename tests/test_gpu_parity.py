@@ -246,3 +246,57 @@ def test_pi05_unsplit_tensor_core_attention(unsplit_attention_everywhere):
             assert_close(got[[1]], oracle_denoise(PI05, w, r, 10, [1]), PI05, f"pi0.5 unsplit B2 P{P}")
     finally:
         ex.close()
+
+
+# Split-KV combine: the attention's result does not depend on how many key splits it was
+# computed in (JPI_ATTN_SPLITS fixes the count at create time; 16 asks for the largest cluster,
+# 14 splits of 64 keys at 867 keys). On the full expert every split count must match the oracle.
+# Between split counts the only differences are roundings: each split's unnormalised output is
+# rounded to fp16 (2^-11 relative) before the combine, the fp32 sums run in another order, and
+# the combined output is rounded to bf16 (2^-9). One layer carries them to its output without the
+# 18-layer growth, so there the split counts must agree to SPLIT_AGREEMENT (relative to the
+# largest output magnitude).
+SPLIT_COUNTS = (1, 2, 7, 16)
+SPLIT_AGREEMENT = 2e-3
+
+
+def _forward_with_splits(monkeypatch, cfg, w, r, t, splits):
+    monkeypatch.setenv("JPI_ATTN_SPLITS", str(splits))
+    P, C = r["prefix_k"].shape[2], r["noise"].shape[1]
+    ex = make_expert(cfg, w, max_batch=1, max_prefix=P, max_chunk=C, max_steps=1)
+    try:
+        k, v = to_dev_kv(r, cfg)
+        ex.set_prefix_kv(k, v)
+        vel, hid = ex.forward(torch.from_numpy(r["state"]).cuda(), torch.from_numpy(r["noise"]).cuda(), t)
+        torch.cuda.synchronize()
+        ex.device_status()
+        return vel.cpu().numpy(), hid.cpu().numpy()
+    finally:
+        ex.close()
+
+
+def test_pi05_every_split_count_matches_the_oracle(monkeypatch):
+    w = make_weights(PI05, 2000)
+    r = make_requests(PI05, 2600, 1, 816, 50)
+    t = 0.3
+    want, _ = oracle.forward_batch(r["noise"], r["state"], t, r["prefix_k"], r["prefix_v"], w, PI05)
+    for splits in SPLIT_COUNTS:
+        vel, _ = _forward_with_splits(monkeypatch, PI05, w, r, t, splits)
+        assert_close(vel, want, PI05, f"pi0.5 forward P816, {splits} key splits")
+
+
+def test_split_counts_agree_on_one_pi05_shaped_layer(monkeypatch):
+    cfg = PI05.with_(n_layers=1)
+    w = make_weights(cfg, 2610)
+    r = make_requests(cfg, 2611, 1, 816, 50)
+    t = 0.3
+    want_v, want_h = oracle.forward_batch(r["noise"], r["state"], t, r["prefix_k"], r["prefix_v"], w, cfg)
+    got = {s: _forward_with_splits(monkeypatch, cfg, w, r, t, s) for s in SPLIT_COUNTS}
+    scale = float(np.abs(want_h).max())
+    for s in SPLIT_COUNTS:
+        assert_close(got[s][0], want_v, cfg, f"one pi0.5 layer, {s} key splits")
+    for s in SPLIT_COUNTS[:-1]:
+        dh = float(np.abs(got[s][1] - got[16][1]).max()) / scale
+        dv = float(np.abs(got[s][0] - got[16][0]).max())
+        print(f"splits {s} vs 14: hidden {dh:.3g} (relative to max |h| {scale:.3g}), velocity {dv:.3g}")
+        assert dh <= SPLIT_AGREEMENT, f"{s} key splits: hidden state differs by {dh:.3g} of max |h|"
