@@ -17,10 +17,11 @@
  * RMSNorm(h) (1 + final_norm), the VLM state the correction module's compressor reads.
  *
  * Built as its own library (libjpi_prefill.so): its products are plain bf16 GEMMs of
- * batch * prefix rows, which it runs through cuBLASLt with fp32 accumulation; norms, rotary
- * coding, softmax and GeGLU run in its own kernels. Conventions are those of jpi.h (status codes,
- * host-side checks before anything is enqueued, row-major [out][in] matrices, one host thread
- * and one stream per handle), with its own jpi_prefill_last_error().
+ * batch * prefix rows, which run on its own tcgen05 tensor-core kernel with fp32 accumulation
+ * (no library GEMM); norms, rotary coding, softmax and GeGLU run in its own kernels. Conventions
+ * are those of jpi.h (status codes, host-side checks before anything is enqueued, row-major
+ * [out][in] matrices, one host thread and one stream per handle), with its own
+ * jpi_prefill_last_error().
  */
 #ifndef JPI_PREFILL_H
 #define JPI_PREFILL_H
@@ -82,6 +83,14 @@ JPI_API jpi_status jpi_prefill_destroy(jpi_prefill_handle* h);   /* NULL is a no
 JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_is_fp32, int batch,
                                    int prefix_len, void* const* k_layers, void* const* v_layers,
                                    long long request_stride, float* out_final, void* stream);
+
+/*
+ * Synchronises the device and reports device-side errors of earlier runs: JPI_OK, or
+ * JPI_ERR_DEVICE_TIMEOUT if a bounded wait inside a product kernel gave up (that kernel skipped
+ * its stores and returned; the outputs of that run are invalid; the word is cleared), or
+ * JPI_ERR_CUDA.
+ */
+JPI_API jpi_status jpi_prefill_device_status(jpi_prefill_handle* h);
 
 JPI_API jpi_status jpi_prefill_memory_usage(const jpi_prefill_handle* h, long long* bytes);
 JPI_API const char* jpi_prefill_last_error(void);

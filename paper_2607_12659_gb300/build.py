@@ -5,10 +5,9 @@ csrc/). Each translation unit compiles in parallel; the objects link into one sh
 with the CUDA runtime linked statically, so the library needs no libcuda at load time (the
 driver entry points are resolved at run time).
 
-``libjpi_prefill.so``: the LLM prefill (csrc/prefill/), linked against the toolkit's cuBLASLt
-(found next to nvcc, recorded as the library's run path). It is separate so that the expert's
-library depends on nothing but the C and C++ runtimes; a toolkit without cuBLASLt leaves only
-the prefill unbuilt (reported on stderr and by ``PREFILL_BUILD_ERROR``).
+``libjpi_prefill.so``: the LLM prefill (csrc/prefill/), its own tensor-core kernels, linked the
+same way. A failure to build it leaves only the prefill unbuilt (reported on stderr and by
+``PREFILL_BUILD_ERROR``).
 """
 
 from __future__ import annotations
@@ -57,17 +56,13 @@ def _stale(obj: str, src: str) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def cuda_lib_dir(cc: str) -> str:
-    return os.path.realpath(os.path.join(os.path.dirname(os.path.realpath(cc)), "..", "lib64"))
-
-
 def build_prefill(verbose: bool = False, force: bool = False) -> str:
-    """Compile csrc/prefill/*.cu and link libjpi_prefill.so against cuBLASLt."""
+    """Compile csrc/prefill/*.cu and link libjpi_prefill.so."""
     cc = nvcc()
     out = os.path.join(BUILD, "prefill")
     os.makedirs(out, exist_ok=True)
     srcs = sorted(os.path.join(PREFILL_SRC, f) for f in os.listdir(PREFILL_SRC) if f.endswith(".cu"))
-    headers = [os.path.join(ROOT, "include", f) for f in ("jpi.h", "jpi_prefill.h")]
+    headers = [os.path.join(ROOT, "include", f) for f in ("jpi.h", "jpi_prefill.h")] + [os.path.join(CSRC, "ptx.h")]
     objs = []
     for src in srcs:
         obj = os.path.join(out, os.path.basename(src)[:-3] + ".o")
@@ -82,10 +77,8 @@ def build_prefill(verbose: bool = False, force: bool = False) -> str:
             print(r.stderr, file=sys.stderr)
     if force or not os.path.exists(PREFILL_LIB) or any(
             os.path.getmtime(o) > os.path.getmtime(PREFILL_LIB) for o in objs):
-        libdir = cuda_lib_dir(cc)
         tmp = PREFILL_LIB + ".tmp"
-        cmd = [cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs + [
-            "-L", libdir, "-lcublasLt", "-Xlinker", f"-rpath={libdir}"]
+        cmd = [cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link of libjpi_prefill.so failed:\n{r.stderr}")

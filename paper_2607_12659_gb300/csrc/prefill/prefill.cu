@@ -4,17 +4,15 @@
 //
 // Every product here is a plain GEMM with batch * prefix rows (816 per request): the Q/K/V, output,
 // gate/up and down projections, and per request the scores q K^T (all heads stacked as rows,
-// since the single KV head is shared) and the probabilities times V. They run as bf16 cuBLASLt
-// matmuls with fp32 accumulation; the residual stream stays fp32, the two residual projections
-// accumulate into it in place (beta = 1). This file's own kernels do the rest: RMSNorm to a bf16
-// operand, rotary coding of q and k from a table built once in double precision (with k and v
-// scattered into the store), the row softmax, and GeGLU.
-//
-// Row-major products map onto cuBLASLt's column-major ones as Y^T = op(W) X^T: a row-major
-// [rows][cols] buffer is the column-major [cols][rows] matrix with the same leading dimension.
+// since the single KV head is shared) and the probabilities times V. They run on this file's
+// tcgen05 GEMM (bf16 operands by bulk tensor copies, fp32 accumulation in TMEM, see k_pf_gemm);
+// the residual stream stays fp32 and the two residual projections accumulate into it in place.
+// This file's other kernels do the rest: RMSNorm to a bf16 operand, rotary coding of q and k from
+// a table built once in double precision (with k and v scattered into the store), the row
+// softmax, the per-request transpose of V, and GeGLU.
 
-#include <cublasLt.h>
 #include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -22,12 +20,11 @@
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
-#include <map>
 #include <new>
-#include <tuple>
 #include <vector>
 
 #include "jpi_prefill.h"
+#include "../ptx.h"
 
 namespace {
 
@@ -49,21 +46,11 @@ jpi_status pfail(jpi_status s, const char* fmt, ...) {
                          __FILE__, __LINE__);                                                      \
     } while (0)
 
-#define PF_LT(expr)                                                                                \
-    do {                                                                                           \
-        cublasStatus_t s_ = (expr);                                                                \
-        if (s_ != CUBLAS_STATUS_SUCCESS)                                                           \
-            return pfail(JPI_ERR_CUDA, "%s failed: %s (%s:%d)", #expr, cublasLtGetStatusString(s_), \
-                         __FILE__, __LINE__);                                                      \
-    } while (0)
-
 #define PF_TRY(expr)                         \
     do {                                     \
         jpi_status s_ = (expr);              \
         if (s_ != JPI_OK) return s_;         \
     } while (0)
-
-constexpr size_t WORKSPACE_BYTES = 32u << 20;
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -181,28 +168,205 @@ struct LayerW {
     float *attn_norm = nullptr, *mlp_norm = nullptr;
 };
 
-struct GemmKey {
-    int opw, M, N, K, ldx, ldw, ldy, tx, tw, ty, acc;
-    unsigned alx, alw, aly;   // byte alignment of each operand's address (at most 256)
-    bool operator<(const GemmKey& o) const {
-        return std::tie(opw, M, N, K, ldx, ldw, ldy, tx, tw, ty, acc, alx, alw, aly) <
-               std::tie(o.opw, o.M, o.N, o.K, o.ldx, o.ldw, o.ldy, o.tx, o.tw, o.ty, o.acc, o.alx, o.alw, o.aly);
-    }
+// ---------------------------------------------------------------------------------------------
+// The products: Y[m][n] = alpha sum_k X[m][k] W[n][k] (+ Y[m][n]), X [M][K] and W [N][K] row-major
+// bf16, Y fp32 or bf16, fp32 accumulation. One output tile = 128 rows of W (the MMA's M) x 128
+// rows of X (its N) over the whole K range, in TMEM as [W row = lane][X row = column]. Persistent:
+// one CTA per SM walks the tiles u = blockIdx.x, + gridDim.x, ... (W tile fastest, so CTAs that run
+// together share X tiles through L2):
+//   warp 0  one thread streams (W block, X block) pairs of 64 K-columns by bulk tensor copies
+//           (128-byte swizzle; rows and columns past the tensors' extents arrive as zeros) into a
+//           ring of PG_STAGES stages;
+//   warp 1  one thread issues the tcgen05.mma chain (M = 128, N = 128, K = 16 each) into one of two
+//           TMEM accumulators and releases each stage through tcgen05.commit;
+//   warps 2-5  one TMEM lane (W row n) per thread: 16 columns (X rows m) at a time, scaled by alpha,
+//           added to Y when accumulating, stored (consecutive lanes write consecutive n), after
+//           which the accumulator goes back to the MMA thread.
+// Every wait is bounded; a timeout records a device error in the handle's word and the CTA returns.
+
+constexpr int PG_TILE = 128;
+constexpr int PG_KBLK = 64;
+constexpr int PG_STAGES = 6;
+constexpr int PG_BLOCK_BYTES = PG_TILE * PG_KBLK * 2;          // 16 KB
+constexpr int PG_STAGE_BYTES = 2 * PG_BLOCK_BYTES;
+constexpr int PG_THREADS = 192;
+constexpr uint64_t PG_WAIT_NS = 200ull * 1000 * 1000;
+constexpr size_t PG_SMEM = 1024 + (size_t)PG_STAGES * PG_STAGE_BYTES + 128;
+
+enum PfDeviceError { PF_DEV_OK = 0, PF_DEV_TIMEOUT_LOAD = 1, PF_DEV_TIMEOUT_MMA = 2 };
+
+struct PfGemmArgs {
+    int M, N, K;          // K: columns the maps cover (a multiple of 64 is not required)
+    float alpha;
+    int accumulate;       // Y += ... (fp32 Y only)
+    int out_bf16;
+    void* Y;
+    long long ldy;        // elements
+    int* err;
 };
 
-// Largest power of two up to 256 that divides the address.
-unsigned alignment_of(const void* p) {
-    const uintptr_t a = reinterpret_cast<uintptr_t>(p);
-    unsigned r = 256;
-    while (r > 1 && (a % r) != 0) r >>= 1;
-    return r;
+__global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant__ CUtensorMap wmap,
+                                                         const __grid_constant__ CUtensorMap xmap,
+                                                         const __grid_constant__ PfGemmArgs a) {
+    namespace ptx = jpi::ptx;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (ptx::smem_u32(smem_raw) & 1023u)) & 1023u);
+    uint8_t* stages = smem;
+    uint64_t* full = (uint64_t*)(smem + (size_t)PG_STAGES * PG_STAGE_BYTES);
+    uint64_t* empty = full + PG_STAGES;
+    uint64_t* accf = empty + PG_STAGES;
+    uint64_t* acce = accf + 2;
+    uint32_t* tmem_slot = (uint32_t*)(acce + 2);
+    int* flag = (int*)(tmem_slot + 1);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int nkb = (a.K + PG_KBLK - 1) / PG_KBLK;
+    const int ntn = (a.N + PG_TILE - 1) / PG_TILE, ntm = (a.M + PG_TILE - 1) / PG_TILE;
+    const int total = ntn * ntm;
+    const int u0 = blockIdx.x, du = gridDim.x;
+
+    if (warp == 1) {
+        ptx::tmem_alloc(tmem_slot, 2 * PG_TILE);
+        ptx::tmem_relinquish();
+    }
+    if (tid == 0) {
+        for (int i = 0; i < 2 * PG_STAGES; ++i) ptx::mbar_init(&full[i], 1);
+        ptx::mbar_init(&accf[0], 1);
+        ptx::mbar_init(&accf[1], 1);
+        ptx::mbar_init(&acce[0], 128);
+        ptx::mbar_init(&acce[1], 128);
+        ptx::fence_mbar_init();
+        *flag = 0;
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int it = 0, issued = 0;
+            bool ok = true;
+            for (int u = u0; u < total && ok; u += du) {
+                const int tn = u % ntn, tm = u / ntn;
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % PG_STAGES, n = it / PG_STAGES;
+                    if (it >= PG_STAGES && !ptx::mbar_wait_bounded(&empty[s], (n - 1) & 1, PG_WAIT_NS)) {
+                        *flag = PF_DEV_TIMEOUT_LOAD;
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* st = stages + (size_t)s * PG_STAGE_BYTES;
+                    ptx::mbar_expect_tx(&full[s], (uint32_t)PG_STAGE_BYTES);
+                    ptx::tma_load_2d_plain(st, &wmap, &full[s], kb * PG_KBLK, tn * PG_TILE);
+                    ptx::tma_load_2d_plain(st + PG_BLOCK_BYTES, &xmap, &full[s], kb * PG_KBLK, tm * PG_TILE);
+                    issued = it + 1;
+                }
+            }
+            // Nothing may land in this CTA's shared memory after it exits: wait for the last copy
+            // into every stage (complete already unless a wait above gave up).
+            for (int i = issued - PG_STAGES < 0 ? 0 : issued - PG_STAGES; i < issued; ++i)
+                if (!ptx::mbar_wait_bounded(&full[i % PG_STAGES], (i / PG_STAGES) & 1, PG_WAIT_NS))
+                    *flag = PF_DEV_TIMEOUT_LOAD;
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t IDESC = ptx::idesc_bf16_f32(PG_TILE, PG_TILE);
+            const uint32_t base = ptx::smem_u32(stages);
+            bool good = true;
+            int it = 0;
+            for (int u = u0, j = 0; u < total; u += du, ++j) {
+                const int buf = j & 1;
+                if (j >= 2 && !ptx::mbar_wait_bounded(&acce[buf], ((j - 2) >> 1) & 1, PG_WAIT_NS)) good = false;
+                ptx::tc_fence_after();
+                const uint32_t acc = tmem + (uint32_t)(buf * PG_TILE);
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % PG_STAGES, n = it / PG_STAGES;
+                    if (good && !ptx::mbar_wait_bounded(&full[s], n & 1, PG_WAIT_NS)) good = false;
+                    ptx::tc_fence_after();
+                    if (good) {
+                        const uint32_t w = base + (uint32_t)(s * PG_STAGE_BYTES), x = w + PG_BLOCK_BYTES;
+#pragma unroll
+                        for (int kk = 0; kk < PG_KBLK / 16; ++kk)
+                            ptx::mma_bf16(acc, ptx::desc_sw128(w + kk * 32), ptx::desc_sw128(x + kk * 32), IDESC,
+                                          (kb | kk) != 0);
+                    }
+                    ptx::mma_commit(&empty[s]);
+                }
+                // Committed even after a timeout so that the epilogue wakes up.
+                ptx::mma_commit(&accf[buf]);
+            }
+            if (!good) *flag = PF_DEV_TIMEOUT_MMA;
+        }
+    } else {
+        const int row = (warp & 3) * 32 + lane;   // TMEM lane: W row of the tile
+        const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+        for (int u = u0, j = 0; u < total; u += du, ++j) {
+            const int buf = j & 1;
+            const int tn = u % ntn, tm = u / ntn;
+            const bool ok = ptx::mbar_wait_bounded(&accf[buf], (j >> 1) & 1, PG_WAIT_NS) && *flag == 0;
+            ptx::tc_fence_after();
+            const int n = tn * PG_TILE + row;
+            for (int c0 = 0; c0 < PG_TILE; c0 += 16) {
+                uint32_t r[16];
+                ptx::tmem_ld_x16(lane_base + (uint32_t)(buf * PG_TILE + c0), r);
+                ptx::tmem_ld_wait();
+                if (!ok || n >= a.N) continue;
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int m = tm * PG_TILE + c0 + i;
+                    if (m >= a.M) break;
+                    const float v = a.alpha * __uint_as_float(r[i]);
+                    const size_t o = (size_t)m * a.ldy + n;
+                    if (a.out_bf16) {
+                        static_cast<__nv_bfloat16*>(a.Y)[o] = __float2bfloat16_rn(v);
+                    } else {
+                        float* y = static_cast<float*>(a.Y) + o;
+                        *y = a.accumulate ? *y + v : v;
+                    }
+                }
+            }
+            ptx::tc_fence_before();
+            ptx::mbar_arrive(&acce[buf]);
+            if (!ok && lane == 0) *flag = PF_DEV_TIMEOUT_MMA;
+        }
+    }
+
+    if (tid == 0 && *flag != 0) atomicCAS(a.err, 0, *flag);
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    if (warp == 1) ptx::tmem_dealloc(tmem, 2 * PG_TILE);
 }
 
-struct GemmPlan {
-    cublasLtMatmulDesc_t desc = nullptr;
-    cublasLtMatrixLayout_t a = nullptr, b = nullptr, c = nullptr;
-    cublasLtMatmulAlgo_t algo;
-};
+// vt[d][p] = v[p][d] for one request (p < P), so that P V runs as a product of K-major operands.
+__global__ void k_pf_transpose(const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ vt, int P, int D,
+                               int ldt) {
+    __shared__ __nv_bfloat16 t[32][33];
+    const int p0 = blockIdx.x * 32, d0 = blockIdx.y * 32;
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int p = p0 + i, d = d0 + threadIdx.x;
+        if (p < P && d < D) t[i][threadIdx.x] = v[(size_t)p * D + d];
+    }
+    __syncthreads();
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int d = d0 + i, p = p0 + threadIdx.x;
+        if (p < P && d < D) vt[(size_t)d * ldt + p] = t[threadIdx.x][i];
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        cudaDriverEntryPointQueryResult q;
+        void* p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+    }
+    return fn;
+}
 
 }  // namespace
 
@@ -222,9 +386,9 @@ struct jpi_prefill_handle {
     float* gu = nullptr;             // [Bm Pm][2 F]
     float* sc = nullptr;             // [H Pm][Pp] scores of one request
     __nv_bfloat16* pr = nullptr;     // [H Pm][Pp] probabilities of one request
-    void* ws = nullptr;
-    cublasLtHandle_t lt = nullptr;
-    std::map<GemmKey, GemmPlan> plans;
+    __nv_bfloat16* vt = nullptr;     // [D][Pp] one request's values, transposed
+    int* dev_err = nullptr;          // device error word of the GEMM's bounded waits
+    int num_sms = 0;
 };
 
 namespace {
@@ -244,87 +408,51 @@ jpi_status pf_alloc(jpi_prefill_handle* h, T** p, size_t count) {
     return JPI_OK;
 }
 
-void destroy_plan(GemmPlan& pl) {
-    if (pl.desc) cublasLtMatmulDescDestroy(pl.desc);
-    if (pl.a) cublasLtMatrixLayoutDestroy(pl.a);
-    if (pl.b) cublasLtMatrixLayoutDestroy(pl.b);
-    if (pl.c) cublasLtMatrixLayoutDestroy(pl.c);
-    pl = GemmPlan();
-}
-
 void release(jpi_prefill_handle* h) {
-    for (auto& kv : h->plans) destroy_plan(kv.second);
-    h->plans.clear();
-    if (h->lt) cublasLtDestroy(h->lt);
-    h->lt = nullptr;
     for (void* p : h->allocs) cudaFree(p);
     h->allocs.clear();
 }
 
-// Descriptors, layouts and the heuristic's algorithm for one product shape; the algorithm is
-// chosen for the operands' actual address alignment (cuBLASLt otherwise assumes 256 bytes).
-cublasStatus_t make_plan(jpi_prefill_handle* h, const GemmKey& k, GemmPlan* pl) {
-    cublasStatus_t s = cublasLtMatmulDescCreate(&pl->desc, CUBLAS_COMPUTE_32F, CUDA_R_32F);
-    const cublasOperation_t opa = k.opw ? CUBLAS_OP_T : CUBLAS_OP_N, opb = CUBLAS_OP_N;
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatmulDescSetAttribute(pl->desc, CUBLASLT_MATMUL_DESC_TRANSA, &opa, sizeof(opa));
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatmulDescSetAttribute(pl->desc, CUBLASLT_MATMUL_DESC_TRANSB, &opb, sizeof(opb));
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = k.opw ? cublasLtMatrixLayoutCreate(&pl->a, (cudaDataType)k.tw, (uint64_t)k.K, (uint64_t)k.N, (int64_t)k.ldw)
-                  : cublasLtMatrixLayoutCreate(&pl->a, (cudaDataType)k.tw, (uint64_t)k.N, (uint64_t)k.K, (int64_t)k.ldw);
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatrixLayoutCreate(&pl->b, (cudaDataType)k.tx, (uint64_t)k.K, (uint64_t)k.M, (int64_t)k.ldx);
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatrixLayoutCreate(&pl->c, (cudaDataType)k.ty, (uint64_t)k.N, (uint64_t)k.M, (int64_t)k.ldy);
-    if (s != CUBLAS_STATUS_SUCCESS) return s;
-    cublasLtMatmulPreference_t pref = nullptr;
-    s = cublasLtMatmulPreferenceCreate(&pref);
-    if (s != CUBLAS_STATUS_SUCCESS) return s;
-    const uint64_t wsb = WORKSPACE_BYTES;
-    const uint32_t al[4] = {k.alw, k.alx, k.aly, k.aly};   // A = W, B = X, C = D = Y
-    s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES, &wsb, sizeof(wsb));
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_A_BYTES, &al[0], sizeof(al[0]));
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_B_BYTES, &al[1], sizeof(al[1]));
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_C_BYTES, &al[2], sizeof(al[2]));
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MIN_ALIGNMENT_D_BYTES, &al[3], sizeof(al[3]));
-    cublasLtMatmulHeuristicResult_t res;
-    int nres = 0;
-    if (s == CUBLAS_STATUS_SUCCESS)
-        s = cublasLtMatmulAlgoGetHeuristic(h->lt, pl->desc, pl->a, pl->b, pl->c, pl->c, pref, 1, &res, &nres);
-    cublasLtMatmulPreferenceDestroy(pref);
-    if (s == CUBLAS_STATUS_SUCCESS && nres < 1) s = CUBLAS_STATUS_NOT_SUPPORTED;
-    if (s == CUBLAS_STATUS_SUCCESS) pl->algo = res.algo;
-    return s;
+// 2D bf16 tensor map over a row-major [rows][cols] matrix of leading dimension ld (elements),
+// 128-byte swizzle, boxes of 64 columns x 128 rows; reads past the extents return zeros.
+jpi_status make_map(const void* base, long long rows, long long cols, long long ld, CUtensorMap* map) {
+    auto enc = get_encode();
+    if (!enc) return pfail(JPI_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+    if ((reinterpret_cast<uintptr_t>(base) & 15) || (ld * 2) % 16)
+        return pfail(JPI_ERR_INVALID_ARG, "a GEMM operand is not 16-byte aligned (address or row stride)");
+    const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)PG_KBLK, (cuuint32_t)PG_TILE};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+                           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return pfail(JPI_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+    return JPI_OK;
 }
 
-// Y [M][N] (row-major, leading dimension ldy) = alpha X [M][K] op(W) + beta Y, where op(W) = W^T
-// for W stored [N][K] (w_nk) and W for W stored [K][N]. As a column-major product:
-// Y^T (N x M) = op_A(A) (N x K) * X^T (K x M) with A the W buffer (column-major K x N, transposed,
-// when w_nk; column-major N x K otherwise) and X^T the X buffer as column-major K x M.
-jpi_status row_gemm(jpi_prefill_handle* h, cudaStream_t st, const void* X, cudaDataType tx, int ldx,
-                    const void* Wm, cudaDataType tw, int ldw, bool w_nk, void* Y, cudaDataType ty, int ldy,
-                    int M, int N, int K, float alpha, float beta) {
-    const GemmKey key{w_nk ? 1 : 0, M, N, K, ldx, ldw, ldy, (int)tx, (int)tw, (int)ty, beta != 0.f ? 1 : 0,
-                      alignment_of(X), alignment_of(Wm), alignment_of(Y)};
-    auto it = h->plans.find(key);
-    if (it == h->plans.end()) {
-        GemmPlan pl;
-        const cublasStatus_t s = make_plan(h, key, &pl);
-        if (s != CUBLAS_STATUS_SUCCESS) {
-            destroy_plan(pl);
-            return pfail(JPI_ERR_UNSUPPORTED, "no cuBLASLt algorithm for a %d x %d x %d product (%s)", M, N, K,
-                         cublasLtGetStatusString(s));
-        }
-        it = h->plans.emplace(key, pl).first;
-    }
-    const GemmPlan& pl = it->second;
-    PF_LT(cublasLtMatmul(h->lt, pl.desc, &alpha, Wm, pl.a, X, pl.b, &beta, Y, pl.c, Y, pl.c, &pl.algo, h->ws,
-                         WORKSPACE_BYTES, st));
+// Y [M][N] (leading dimension ldy; fp32, or bf16 when y_bf16) = alpha X [M][K] W[N][K]^T, plus Y
+// when accumulating. X and W are bf16 with leading dimensions ldx and ldw.
+jpi_status row_gemm(jpi_prefill_handle* h, cudaStream_t st, const __nv_bfloat16* X, long long ldx,
+                    const __nv_bfloat16* Wm, long long ldw, void* Y, bool y_bf16, long long ldy, int M, int N,
+                    int K, float alpha, bool accumulate) {
+    CUtensorMap wmap, xmap;
+    PF_TRY(make_map(Wm, N, K, ldw, &wmap));
+    PF_TRY(make_map(X, M, K, ldx, &xmap));
+    PfGemmArgs a;
+    a.M = M;
+    a.N = N;
+    a.K = K;
+    a.alpha = alpha;
+    a.accumulate = accumulate ? 1 : 0;
+    a.out_bf16 = y_bf16 ? 1 : 0;
+    a.Y = Y;
+    a.ldy = ldy;
+    a.err = h->dev_err;
+    const long long tiles = (long long)((N + PG_TILE - 1) / PG_TILE) * ((M + PG_TILE - 1) / PG_TILE);
+    const int grid = (int)(tiles < h->num_sms ? tiles : h->num_sms);
+    k_pf_gemm<<<grid, PG_THREADS, PG_SMEM, st>>>(wmap, xmap, a);
+    PF_CUDA(cudaGetLastError());
     return JPI_OK;
 }
 
@@ -384,10 +512,12 @@ jpi_status setup(jpi_prefill_handle* h, const jpi_prefill_config* c, const jpi_p
         !w->w_down || !w->final_norm)
         return pfail(JPI_ERR_INVALID_ARG, "a weight array is NULL");
 
-    PF_LT(cublasLtCreate(&h->lt));
-    char* ws = nullptr;
-    PF_TRY(pf_alloc(h, &ws, WORKSPACE_BYTES));
-    h->ws = ws;
+    int device = 0;
+    PF_CUDA(cudaGetDevice(&device));
+    PF_CUDA(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, device));
+    PF_CUDA(cudaFuncSetAttribute(k_pf_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PG_SMEM));
+    PF_TRY(pf_alloc(h, &h->dev_err, 1));
+    PF_CUDA(cudaMemset(h->dev_err, 0, sizeof(int)));
     float* staging = nullptr;
     if (!dev) PF_TRY(pf_alloc(h, &staging, F * W));
     h->layers.resize((size_t)h->L);
@@ -431,6 +561,7 @@ jpi_status setup(jpi_prefill_handle* h, const jpi_prefill_config* c, const jpi_p
     PF_TRY(pf_alloc(h, &h->gu, Mm * 2 * F));
     PF_TRY(pf_alloc(h, &h->sc, (size_t)h->H * h->Pm * h->Pp));
     PF_TRY(pf_alloc(h, &h->pr, (size_t)h->H * h->Pm * h->Pp));
+    PF_TRY(pf_alloc(h, &h->vt, D * (size_t)h->Pp));
     return JPI_OK;
 }
 
@@ -487,7 +618,6 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
     const int W = h->W, D = h->D, H = h->H, F = h->F, P = prefix_len, Pp = (P + 7) / 8 * 8;
     const long long M = (long long)batch * P;
     const float eps = h->cfg.rms_eps, scale = 1.f / sqrtf((float)D);
-    const cudaDataType BF = CUDA_R_16BF, F32 = CUDA_R_32F;
 
     k_pf_load_x<<<grid_for(M * W), 256, 0, st>>>(x, x_is_fp32, h->h, M * W);
     PF_CUDA(cudaGetLastError());
@@ -498,7 +628,7 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
         // Attention sublayer.
         k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, lw.attn_norm, h->xn, M, W, eps);
         PF_CUDA(cudaGetLastError());
-        PF_TRY(row_gemm(h, st, h->xn, BF, W, lw.wqkv, BF, W, true, h->qkv, F32, h->QKV, (int)M, h->QKV, W, 1.f, 0.f));
+        PF_TRY(row_gemm(h, st, h->xn, W, lw.wqkv, W, h->qkv, false, h->QKV, (int)M, h->QKV, W, 1.f, false));
         k_pf_rope_scatter<<<grid_for(M * (H + 2) * (D / 2)), 256, 0, st>>>(h->qkv, h->rope, h->q, kd, vd,
                                                                              request_stride, batch, P, H, D);
         PF_CUDA(cudaGetLastError());
@@ -507,23 +637,38 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
             const __nv_bfloat16* kb = kd + (size_t)b * request_stride;  // [P][D]
             const __nv_bfloat16* vb = vd + (size_t)b * request_stride;  // [P][D]
             __nv_bfloat16* ob = h->o + (size_t)b * P * H * D;           // [(P H)][D] = [P][H D]
-            PF_TRY(row_gemm(h, st, qb, BF, D, kb, BF, D, true, h->sc, F32, Pp, P * H, P, D, scale, 0.f));
+            PF_TRY(row_gemm(h, st, qb, D, kb, D, h->sc, false, Pp, P * H, P, D, scale, false));
             k_pf_softmax<<<grid_for((long long)P * H * 32), 256, 0, st>>>(h->sc, h->pr, (long long)P * H, P, Pp);
             PF_CUDA(cudaGetLastError());
-            PF_TRY(row_gemm(h, st, h->pr, BF, Pp, vb, BF, D, false, ob, BF, D, P * H, D, P, 1.f, 0.f));
+            k_pf_transpose<<<dim3((P + 31) / 32, (D + 31) / 32), dim3(32, 8), 0, st>>>(vb, h->vt, P, D, Pp);
+            PF_CUDA(cudaGetLastError());
+            PF_TRY(row_gemm(h, st, h->pr, Pp, h->vt, Pp, ob, true, D, P * H, D, P, 1.f, false));
         }
-        PF_TRY(row_gemm(h, st, h->o, BF, H * D, lw.wo, BF, H * D, true, h->h, F32, W, (int)M, W, H * D, 1.f, 1.f));
+        PF_TRY(row_gemm(h, st, h->o, H * D, lw.wo, H * D, h->h, false, W, (int)M, W, H * D, 1.f, true));
         // MLP sublayer.
         k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, lw.mlp_norm, h->xn, M, W, eps);
         PF_CUDA(cudaGetLastError());
-        PF_TRY(row_gemm(h, st, h->xn, BF, W, lw.wgu, BF, W, true, h->gu, F32, 2 * F, (int)M, 2 * F, W, 1.f, 0.f));
+        PF_TRY(row_gemm(h, st, h->xn, W, lw.wgu, W, h->gu, false, 2 * F, (int)M, 2 * F, W, 1.f, false));
         k_pf_geglu<<<grid_for(M * F), 256, 0, st>>>(h->gu, h->xn, M, F);
         PF_CUDA(cudaGetLastError());
-        PF_TRY(row_gemm(h, st, h->xn, BF, F, lw.wd, BF, F, true, h->h, F32, W, (int)M, W, F, 1.f, 1.f));
+        PF_TRY(row_gemm(h, st, h->xn, F, lw.wd, F, h->h, false, W, (int)M, W, F, 1.f, true));
     }
     if (out_final) {
         k_pf_rmsnorm<float><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->final_norm, out_final, M, W, eps);
         PF_CUDA(cudaGetLastError());
+    }
+    return JPI_OK;
+}
+
+JPI_API jpi_status jpi_prefill_device_status(jpi_prefill_handle* h) {
+    g_err[0] = '\0';
+    if (!h) return pfail(JPI_ERR_INVALID_ARG, "handle is NULL");
+    PF_CUDA(cudaDeviceSynchronize());
+    int err = 0;
+    PF_CUDA(cudaMemcpy(&err, h->dev_err, sizeof(int), cudaMemcpyDeviceToHost));
+    if (err != PF_DEV_OK) {
+        PF_CUDA(cudaMemset(h->dev_err, 0, sizeof(int)));
+        return pfail(JPI_ERR_DEVICE_TIMEOUT, "device-side error code %d (a bounded wait in a product gave up)", err);
     }
     return JPI_OK;
 }

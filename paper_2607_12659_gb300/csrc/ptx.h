@@ -67,6 +67,14 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_
         "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
         : "memory");
 }
+// The same copy with the default L2 policy (for operands that other CTAs read again).
+__device__ __forceinline__ void tma_load_2d_plain(void* dst, const void* tmap, uint64_t* bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
 // Brings a tensor map (a __grid_constant__ kernel parameter) into the descriptor cache ahead of
 // its first bulk tensor copy.
 __device__ __forceinline__ void prefetch_tmap(const void* tmap) {

@@ -37,6 +37,7 @@ _SIGS = {
     "jpi_prefill_run": [c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p, c_longlong, c_void_p,
                         c_void_p],
     "jpi_prefill_memory_usage": [c_void_p, POINTER(c_longlong)],
+    "jpi_prefill_device_status": [c_void_p],
 }
 
 _lib = None
@@ -89,6 +90,10 @@ def jpi_prefill_run(h, x, x_is_fp32, batch, prefix_len, k_ptrs, v_ptrs, request_
     va = (c_void_p * L)(*v_ptrs)
     _check(load().jpi_prefill_run(h, _ptr(x), int(x_is_fp32), batch, prefix_len, ka, va, request_stride,
                                   _ptr(out_final), _stream(stream)), "jpi_prefill_run")
+
+
+def jpi_prefill_device_status(h):
+    _check(load().jpi_prefill_device_status(h), "jpi_prefill_device_status")
 
 
 def jpi_prefill_memory_usage(h) -> int:
@@ -179,9 +184,13 @@ class Prefill:
         jpi.jpi_commit_prefix(expert.handle, B, P)
         return out
 
+    def device_status(self):
+        jpi_prefill_device_status(self.handle)
+
     def memory_usage(self) -> int:
         return jpi_prefill_memory_usage(self.handle)
 
 
 __all__ = ["Prefill", "jpi_prefill_create", "jpi_prefill_destroy", "jpi_prefill_run", "jpi_prefill_memory_usage",
+           "jpi_prefill_device_status",
            "load", "header_symbols", "STATUS_NAMES"]

@@ -96,7 +96,7 @@ def test_every_header_belongs_to_a_library():
     inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
     headers = {f for f in os.listdir(inc) if f.endswith(".h")}
     assert headers == set(jpi.LIB_HEADERS) | {"jpi_prefill.h"}
-    assert len(prefill.header_symbols()) == 5
+    assert len(prefill.header_symbols()) == 6
 
 
 def test_prefill_library_exports_its_entry_points_and_checks_arguments(lib):
@@ -108,7 +108,8 @@ def test_prefill_library_exports_its_entry_points_and_checks_arguments(lib):
     exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
     assert exported == set(prefill.header_symbols())
     ldd = subprocess.run(["ldd", prefill.LIB_PATH], capture_output=True, text=True).stdout
-    assert "libcublasLt" in ldd and "libcuda.so" not in ldd and "libtorch" not in ldd
+    # Its products run on its own tensor-core kernel: no library GEMM, no driver or torch link.
+    assert "libcublas" not in ldd and "libcuda.so" not in ldd and "libtorch" not in ldd
     h = ctypes.c_void_p()
     assert plib.jpi_prefill_create(None, None, ctypes.byref(h)) == -1
     assert b"NULL" in plib.jpi_prefill_last_error()
@@ -116,6 +117,7 @@ def test_prefill_library_exports_its_entry_points_and_checks_arguments(lib):
     assert plib.jpi_prefill_run(None, None, 1, 1, 1, None, None, 256, None, None) == -1
     n = ctypes.c_longlong()
     assert plib.jpi_prefill_memory_usage(None, ctypes.byref(n)) == -1
+    assert plib.jpi_prefill_device_status(None) == -1
     w = prefill.jpi_prefill_weights()
     bad = [dict(n_layers=0), dict(width=2044), dict(head_dim=250), dict(head_dim=1024), dict(mlp_dim=12),
            dict(max_batch=0), dict(max_prefix=0), dict(rms_eps=-1.0), dict(max_prefix=70000)]

@@ -48,6 +48,7 @@ def test_prefill_matches_the_oracle(B, P, x_dtype):
     pre = prefill.Prefill(cfg, w, max_batch=4, max_prefix=80)
     K, V, out = pre.into_tensors(torch.from_numpy(x).cuda().to(getattr(torch, x_dtype)))
     torch.cuda.synchronize()
+    pre.device_status()
     Kw, Vw, want = pf.prefill_batch(x, w, cfg)
     for l in range(cfg.n_layers):
         _close(K[l].float().cpu().numpy(), Kw[l], f"K layer {l}")
@@ -67,6 +68,7 @@ def test_gemma2b_sized_layers():
     pre = prefill.Prefill(cfg, w, max_batch=1, max_prefix=816)
     K, V, out = pre.into_tensors(torch.from_numpy(x).cuda().to(torch.bfloat16))
     torch.cuda.synchronize()
+    pre.device_status()
     Kw, Vw, want = pf.prefill_batch(x, w, cfg)
     for l in range(cfg.n_layers):
         _close(K[l].float().cpu().numpy(), Kw[l], f"Gemma-2B K layer {l}")
@@ -98,6 +100,7 @@ def test_zero_copy_into_the_expert_store():
     b = ex.denoise(state, noise, N)
     torch.cuda.synchronize()
     ex.device_status()
+    pre.device_status()
     assert torch.equal(a, b)
     ex.close()
     pre.close()
