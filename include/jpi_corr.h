@@ -102,7 +102,11 @@ JPI_API jpi_status jpi_corr_destroy(jpi_corr_handle* h);   /* NULL is a no-op */
 /* Q-Former compressor (App. B): h_vlm [batch][n_tokens][d_vlm] device, fp32 (vlm_is_fp32 = 1)
  * or bf16 (0), the VLM's final-layer output of each request -> out_state [batch][T'][d] fp32
  * device, the compressed state. 1 <= batch <= max_batch, 1 <= n_tokens <= max_vlm_tokens.
- * Enqueued on `stream`; the inputs must stay valid until the stream reaches the call. */
+ * Enqueued on `stream`; the inputs must stay valid until the stream reaches the call.
+ * The call copies h_vlm into the handle, replays the kernel sequence as a CUDA graph captured the
+ * first time this (batch, n_tokens, input type) is asked for (on the handle's own stream, so the
+ * first call of a shape should not itself be inside a stream capture), and copies the result to
+ * out_state. */
 JPI_API jpi_status jpi_corr_compress(jpi_corr_handle* h, const void* h_vlm, int vlm_is_fp32,
                                      int batch, int n_tokens, float* out_state, void* stream);
 
@@ -111,7 +115,8 @@ JPI_API jpi_status jpi_corr_compress(jpi_corr_handle* h, const void* h_vlm, int 
  * device, the committed actions in execution order -> out_state [batch][T'][d] fp32 device, the
  * predicted compressed state at t + delta (ready to pass to jpi_set_correction), and
  * out_confidence [batch] fp32 device (may be NULL). 1 <= delta <= max_delta. out_state may be
- * the same buffer as state. Enqueued on `stream`. */
+ * the same buffer as state. Enqueued on `stream`; like jpi_corr_compress it copies its inputs in,
+ * replays a graph captured once per (batch, delta) and copies its outputs out. */
 JPI_API jpi_status jpi_corr_predict(jpi_corr_handle* h, const float* state, const float* actions,
                                     int batch, int delta, float* out_state, float* out_confidence,
                                     void* stream);

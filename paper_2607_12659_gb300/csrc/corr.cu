@@ -19,6 +19,9 @@
 // 2 H T' T d_vlm * 2 FLOPs per request instead of the 4 T d_vlm d of projecting every token.
 
 #include "jpi_internal.h"
+
+#include <map>
+#include <tuple>
 #include "jpi_corr.h"
 
 #include <cmath>
@@ -106,6 +109,8 @@ __global__ void __launch_bounds__(256) k_corr_linear(const LinArgs a) {
 #pragma unroll
             for (int k = 0; k < LIN_ROWS; ++k) acc[k] = 0.f;
             if (VEC) {
+                // Unrolled so that several 4-wide weight loads of the row are in flight at once.
+#pragma unroll 4
                 for (int i = lane * 4; i < a.in; i += 128) {
                     const float4 w4 = load4(wr + i);
 #pragma unroll
@@ -138,7 +143,10 @@ __global__ void __launch_bounds__(256) k_corr_linear(const LinArgs a) {
     }
 }
 
-// Row-wise LayerNorm with the biased variance; one warp per row (grid-stride over rows).
+// LayerNorm of `rows` rows of width d: one warp per row (grid-stride over rows), three passes
+// (mean, biased variance, output). VEC: every row and vector 16-byte aligned, d a multiple of 4,
+// so the passes move float4s.
+template <bool VEC>
 __global__ void __launch_bounds__(256) k_corr_layernorm(const float* __restrict__ x, int ldx,
                                                         const float* __restrict__ g,
                                                         const float* __restrict__ b,
@@ -147,17 +155,46 @@ __global__ void __launch_bounds__(256) k_corr_layernorm(const float* __restrict_
     const int lane = threadIdx.x & 31, nwarps = (int)((gridDim.x * blockDim.x) >> 5);
     for (int r = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); r < rows; r += nwarps) {
         const float* xr = x + (size_t)r * ldx;
-        float s = 0.f;
-        for (int i = lane; i < d; i += 32) s += xr[i];
-        const float mean = warp_sum(s) / (float)d;
-        float v = 0.f;
-        for (int i = lane; i < d; i += 32) {
-            const float t = xr[i] - mean;
-            v = fmaf(t, t, v);
-        }
-        const float rstd = 1.f / sqrtf(warp_sum(v) / (float)d + eps);
         float* yr = y + (size_t)r * ldy;
-        for (int i = lane; i < d; i += 32) yr[i] = (xr[i] - mean) * rstd * g[i] + b[i];
+        if (VEC) {
+            const int d4 = d >> 2;
+            const float4* x4 = reinterpret_cast<const float4*>(xr);
+            float s = 0.f;
+#pragma unroll 4
+            for (int i = lane; i < d4; i += 32) {
+                const float4 v = x4[i];
+                s += (v.x + v.y) + (v.z + v.w);
+            }
+            const float mean = warp_sum(s) / (float)d;
+            float var = 0.f;
+#pragma unroll 4
+            for (int i = lane; i < d4; i += 32) {
+                const float4 v = x4[i];
+                const float t0 = v.x - mean, t1 = v.y - mean, t2 = v.z - mean, t3 = v.w - mean;
+                var = fmaf(t0, t0, fmaf(t1, t1, fmaf(t2, t2, fmaf(t3, t3, var))));
+            }
+            const float rstd = 1.f / sqrtf(warp_sum(var) / (float)d + eps);
+            float4* y4 = reinterpret_cast<float4*>(yr);
+            const float4* g4 = reinterpret_cast<const float4*>(g);
+            const float4* b4 = reinterpret_cast<const float4*>(b);
+#pragma unroll 4
+            for (int i = lane; i < d4; i += 32) {
+                const float4 v = x4[i], gg = g4[i], bb = b4[i];
+                y4[i] = make_float4((v.x - mean) * rstd * gg.x + bb.x, (v.y - mean) * rstd * gg.y + bb.y,
+                                    (v.z - mean) * rstd * gg.z + bb.z, (v.w - mean) * rstd * gg.w + bb.w);
+            }
+        } else {
+            float s = 0.f;
+            for (int i = lane; i < d; i += 32) s += xr[i];
+            const float mean = warp_sum(s) / (float)d;
+            float var = 0.f;
+            for (int i = lane; i < d; i += 32) {
+                const float t = xr[i] - mean;
+                var = fmaf(t, t, var);
+            }
+            const float rstd = 1.f / sqrtf(warp_sum(var) / (float)d + eps);
+            for (int i = lane; i < d; i += 32) yr[i] = (xr[i] - mean) * rstd * g[i] + b[i];
+        }
     }
 }
 
@@ -258,100 +295,157 @@ __global__ void __launch_bounds__(256) k_corr_qk(const float* __restrict__ qc, c
         if (i < T) qk[((size_t)h * T + i) * dv + c] = acc[i] * scale;
 }
 
-// s[b][m][j] = sum_c qk[m][c] hv[b][j][c] for m < M, j < T. Grid (ceil(T / 32), B): 32 tokens per
-// CTA, warp w holds rows w, w + 8, ..., the c range staged 32 at a time.
+// Partial scores over one chunk of the VLM features: part[b][kc][m][j] = sum over c in chunk kc
+// (CORR_KCHUNK features) of qk[m][c] hv[b][j][c], m < M, j < T. Grid (ceil(T / 32), chunks, B):
+// 32 tokens per CTA; the chunk's query rows and token rows are staged in shared memory with all
+// their loads in flight together, then warp w computes rows w, w + 8, ... for lane = token.
+// Splitting the feature sum over CTAs keeps the whole GPU busy at batch 1 (26 token tiles alone
+// would not); the chunks are added in order by k_corr_softmax_sum.
+constexpr int CORR_KCHUNK = 256;
+constexpr int CORR_KPAD = CORR_KCHUNK + 1;
+constexpr size_t CORR_SCORES_SMEM = (size_t)(CORR_MAX_M + 32) * CORR_KPAD * sizeof(float);
+
 template <typename THV>
 __global__ void __launch_bounds__(256) k_corr_scores(const float* __restrict__ qk, const THV* __restrict__ hv,
-                                                     float* __restrict__ s, int M, int T, int dv) {
-    __shared__ float as[CORR_MAX_M][33];
-    __shared__ float bs[32][33];
-    const int b = blockIdx.y, j0 = blockIdx.x * 32;
+                                                     float* __restrict__ part, int M, int T, int dv) {
+    extern __shared__ float sm_scores[];
+    float* as = sm_scores;                       // [M][CORR_KPAD]
+    float* bs = sm_scores + CORR_MAX_M * CORR_KPAD;   // [32][CORR_KPAD]
+    const int b = blockIdx.z, kc = blockIdx.y, j0 = blockIdx.x * 32;
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int c0 = kc * CORR_KCHUNK, cn = min(CORR_KCHUNK, dv - c0);
+    const THV* hb = hv + (size_t)b * T * dv;
+    for (int idx = threadIdx.x; idx < M * CORR_KCHUNK; idx += 256) {
+        const int m = idx / CORR_KCHUNK, kk = idx % CORR_KCHUNK;
+        as[m * CORR_KPAD + kk] = kk < cn ? qk[(size_t)m * dv + c0 + kk] : 0.f;
+    }
+    for (int idx = threadIdx.x; idx < 32 * CORR_KCHUNK; idx += 256) {
+        const int t = idx / CORR_KCHUNK, kk = idx % CORR_KCHUNK, j = j0 + t;
+        bs[t * CORR_KPAD + kk] = (j < T && kk < cn) ? to_f(hb[(size_t)j * dv + c0 + kk]) : 0.f;
+    }
+    __syncthreads();
     float acc[CORR_MAX_M / 8];
 #pragma unroll
     for (int r = 0; r < CORR_MAX_M / 8; ++r) acc[r] = 0.f;
-    const THV* hb = hv + (size_t)b * T * dv;
-    for (int c0 = 0; c0 < dv; c0 += 32) {
-        for (int idx = threadIdx.x; idx < M * 32; idx += 256) {
-            const int m = idx >> 5, kk = idx & 31;
-            as[m][kk] = c0 + kk < dv ? qk[(size_t)m * dv + c0 + kk] : 0.f;
-        }
-        for (int idx = threadIdx.x; idx < 32 * 32; idx += 256) {
-            const int t = idx >> 5, kk = idx & 31, j = j0 + t;
-            bs[t][kk] = (j < T && c0 + kk < dv) ? to_f(hb[(size_t)j * dv + c0 + kk]) : 0.f;
-        }
-        __syncthreads();
 #pragma unroll 8
-        for (int kk = 0; kk < 32; ++kk) {
-            const float bv = bs[tx][kk];
+    for (int kk = 0; kk < CORR_KCHUNK; ++kk) {
+        const float bv = bs[tx * CORR_KPAD + kk];
 #pragma unroll
-            for (int r = 0; r < CORR_MAX_M / 8; ++r) {
-                const int m = ty + 8 * r;
-                if (m < M) acc[r] = fmaf(as[m][kk], bv, acc[r]);
-            }
+        for (int r = 0; r < CORR_MAX_M / 8; ++r) {
+            const int m = ty + 8 * r;
+            if (m < M) acc[r] = fmaf(as[m * CORR_KPAD + kk], bv, acc[r]);
         }
-        __syncthreads();
     }
     const int j = j0 + tx;
     if (j < T)
 #pragma unroll
         for (int r = 0; r < CORR_MAX_M / 8; ++r) {
             const int m = ty + 8 * r;
-            if (m < M) s[((size_t)b * M + m) * T + j] = acc[r];
+            if (m < M) part[(((size_t)b * gridDim.y + kc) * M + m) * T + j] = acc[r];
         }
 }
 
-// In-place softmax of each row of length n; one warp per row (grid-stride over rows).
-__global__ void __launch_bounds__(256) k_corr_softmax(float* __restrict__ s, int rows, int n) {
-    const int lane = threadIdx.x & 31, nwarps = (int)((gridDim.x * blockDim.x) >> 5);
-    for (int r = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); r < rows; r += nwarps) {
-        float* row = s + (size_t)r * n;
-        float mx = -INFINITY;
-        for (int j = lane; j < n; j += 32) mx = fmaxf(mx, row[j]);
+// Block-wide reductions over 256 threads (8 warps), through `red` [8] in shared memory.
+__device__ __forceinline__ float block_max256(float v, float* red) {
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        float den = 0.f;
-        for (int j = lane; j < n; j += 32) {
-            const float e = expf(row[j] - mx);
-            row[j] = e;
-            den += e;
-        }
-        const float inv = 1.f / warp_sum(den);
-        for (int j = lane; j < n; j += 32) row[j] *= inv;
-    }
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float r = red[0];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) r = fmaxf(r, red[w]);
+    __syncthreads();
+    return r;
+}
+__device__ __forceinline__ float block_sum256(float v, float* red) {
+    v = warp_sum(v);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float r = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) r += red[w];   // fixed order
+    __syncthreads();
+    return r;
 }
 
-// g[b][m][c] = sum_j p[b][m][j] hv[b][j][c]. Grid (ceil(dv / 256), ceil(M / 16), B): one column
-// per thread, 16 rows per CTA, the probabilities staged 64 tokens at a time.
+// Row r = b M + m of the scores (one CTA of 256 threads per row): the nkc feature chunks added in
+// order, then the softmax over its n tokens, written to s[r][.].
+__global__ void __launch_bounds__(256) k_corr_softmax_sum(const float* __restrict__ part, float* __restrict__ s,
+                                                          int M, int n, int nkc) {
+    __shared__ float red[8];
+    const int r = blockIdx.x, b = r / M, m = r - b * M;
+    const float* p0 = part + ((size_t)b * nkc * M + m) * n;
+    float* row = s + (size_t)r * n;
+    float mx = -INFINITY;
+    for (int j = threadIdx.x; j < n; j += 256) {
+        float v = 0.f;
+        for (int kc = 0; kc < nkc; ++kc) v += p0[(size_t)kc * M * n + j];
+        row[j] = v;
+        mx = fmaxf(mx, v);
+    }
+    mx = block_max256(mx, red);
+    float den = 0.f;
+    for (int j = threadIdx.x; j < n; j += 256) {
+        const float e = expf(row[j] - mx);
+        row[j] = e;
+        den += e;
+    }
+    const float inv = 1.f / block_sum256(den, red);
+    for (int j = threadIdx.x; j < n; j += 256) row[j] *= inv;
+}
+
+// Partial weighted sums over one chunk of CORR_TCHUNK tokens: part[b][tc][m][c] = sum over j in
+// chunk tc of p[b][m][j] hv[b][j][c]. Grid (ceil(dv / 256), chunks, B): one column per thread,
+// all M rows, the chunk's probabilities staged in shared memory (read as broadcasts). The token
+// chunks are added in order by k_corr_wsum_reduce.
+constexpr int CORR_TCHUNK = 64;
+
 template <typename THV>
 __global__ void __launch_bounds__(256) k_corr_wsum(const float* __restrict__ p, const THV* __restrict__ hv,
-                                                   float* __restrict__ g, int M, int T, int dv) {
-    __shared__ float ps[16][64];
-    const int b = blockIdx.z, m0 = blockIdx.y * 16, c = blockIdx.x * 256 + threadIdx.x;
-    float acc[16];
-#pragma unroll
-    for (int r = 0; r < 16; ++r) acc[r] = 0.f;
-    const THV* hb = hv + (size_t)b * T * dv;
-    for (int j0 = 0; j0 < T; j0 += 64) {
-        for (int idx = threadIdx.x; idx < 16 * 64; idx += 256) {
-            const int r = idx >> 6, jj = idx & 63;
-            ps[r][jj] = (m0 + r < M && j0 + jj < T) ? p[((size_t)b * M + m0 + r) * T + j0 + jj] : 0.f;
-        }
-        __syncthreads();
-        if (c < dv) {
-            const int jn = T - j0 < 64 ? T - j0 : 64;
-            for (int jj = 0; jj < jn; ++jj) {
-                const float hvv = to_f(hb[(size_t)(j0 + jj) * dv + c]);
-#pragma unroll
-                for (int r = 0; r < 16; ++r) acc[r] = fmaf(ps[r][jj], hvv, acc[r]);
-            }
-        }
-        __syncthreads();
+                                                   float* __restrict__ part, int M, int T, int dv) {
+    __shared__ float ps[CORR_MAX_M][CORR_TCHUNK];
+    const int b = blockIdx.z, tc = blockIdx.y, c = blockIdx.x * 256 + threadIdx.x;
+    const int j0 = tc * CORR_TCHUNK, jn = min(CORR_TCHUNK, T - j0);
+    for (int idx = threadIdx.x; idx < M * CORR_TCHUNK; idx += 256) {
+        const int r = idx / CORR_TCHUNK, jj = idx % CORR_TCHUNK;
+        ps[r][jj] = jj < jn ? p[((size_t)b * M + r) * T + j0 + jj] : 0.f;
     }
-    if (c < dv)
+    __syncthreads();
+    if (c >= dv) return;
+    float acc[CORR_MAX_M];
 #pragma unroll
-        for (int r = 0; r < 16; ++r)
-            if (m0 + r < M) g[((size_t)b * M + m0 + r) * dv + c] = acc[r];
+    for (int r = 0; r < CORR_MAX_M; ++r) acc[r] = 0.f;
+    const THV* hb = hv + ((size_t)b * T + j0) * dv + c;
+    // Eight tokens' values loaded together, then their products (loads of the next eight in
+    // flight behind them).
+    for (int jb = 0; jb < jn; jb += 8) {
+        float hvv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) hvv[u] = jb + u < jn ? to_f(hb[(size_t)(jb + u) * dv]) : 0.f;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+#pragma unroll
+            for (int r = 0; r < CORR_MAX_M; ++r)
+                if (r < M) acc[r] = fmaf(ps[r][jb + u], hvv[u], acc[r]);
+    }
+    float* out = part + ((size_t)b * gridDim.y + tc) * M * dv + c;
+#pragma unroll
+    for (int r = 0; r < CORR_MAX_M; ++r)
+        if (r < M) out[(size_t)r * dv] = acc[r];
+}
+
+// g[b][m][c] = the ntc token-chunk partials added in order.
+__global__ void k_corr_wsum_reduce(const float* __restrict__ part, float* __restrict__ g, int B, int M, int dv,
+                                   int ntc) {
+    const long long total = (long long)B * M * dv;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const long long b = idx / ((long long)M * dv), rest = idx - b * M * dv;
+        const float* p0 = part + (size_t)b * ntc * M * dv + rest;
+        float v = 0.f;
+        for (int tc = 0; tc < ntc; ++tc) v += p0[(size_t)tc * M * dv];
+        g[idx] = v;
+    }
 }
 
 // y[(b n + k)][c] += pos[k][c] for b < B, k < n, c < d.
@@ -378,21 +472,20 @@ __global__ void k_corr_join(const float* __restrict__ state, const float* __rest
     }
 }
 
-// conf[b] = w . mean_i u[b T' + i] + bias; one warp per request (grid-stride over requests).
-__global__ void k_corr_confidence(const float* __restrict__ u, const float* __restrict__ w,
-                                  const float* __restrict__ bias, float* __restrict__ conf, int B,
-                                  int T, int d) {
-    const int lane = threadIdx.x & 31, nwarps = (int)((gridDim.x * blockDim.x) >> 5);
-    for (int b = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); b < B; b += nwarps) {
-        float s = 0.f;
-        for (int c = lane; c < d; c += 32) {
-            float m = 0.f;
-            for (int i = 0; i < T; ++i) m += u[((size_t)b * T + i) * d + c];
-            s = fmaf(w[c], m / (float)T, s);
-        }
-        s = warp_sum(s);
-        if (lane == 0) conf[b] = s + bias[0];
+// conf[b] = w . mean_i u[b T' + i] + bias; one CTA of 256 threads per request.
+__global__ void __launch_bounds__(256) k_corr_confidence(const float* __restrict__ u, const float* __restrict__ w,
+                                                         const float* __restrict__ bias, float* __restrict__ conf,
+                                                         int T, int d) {
+    __shared__ float red[8];
+    const int b = blockIdx.x;
+    float s = 0.f;
+    for (int c = threadIdx.x; c < d; c += 256) {
+        float m = 0.f;
+        for (int i = 0; i < T; ++i) m += u[((size_t)b * T + i) * d + c];
+        s = fmaf(w[c], m / (float)T, s);
     }
+    s = block_sum256(s, red);
+    if (threadIdx.x == 0) conf[b] = s + bias[0];
 }
 
 __global__ void k_corr_cast(const float* __restrict__ src, __nv_bfloat16* __restrict__ dst, long long n) {
@@ -472,7 +565,16 @@ struct jpi_corr_handle {
     float *xj = nullptr, *xf = nullptr, *u = nullptr, *qkv = nullptr, *o = nullptr;   // [B T'] rows
     float* hid = nullptr;                                                 // [B T'][F]
     float *sc = nullptr, *gs = nullptr;                                   // [B][M][Tm], [B][M][dv]
+    float *scp = nullptr, *gsp = nullptr;   // partials: [B][dv / 256][M][Tm], [B][Tm / 64][M][dv]
     float* conf_scratch = nullptr;                                        // [B]
+
+    // Graph replay: the calls copy their inputs into these buffers, replay the kernel sequence
+    // captured once per (call, batch, tokens or delta, input type), and copy the outputs out.
+    void* in_vlm = nullptr;                                               // [B][Tm][dv], fp32 or bf16
+    float *in_state = nullptr, *in_act = nullptr;                         // [B T'][d], [B Dm][A]
+    float *out_st = nullptr, *out_conf = nullptr;                         // [B T'][d], [B]
+    cudaStream_t cap = nullptr;
+    std::map<std::tuple<int, int, int, int>, cudaGraphExec_t> graphs;
 };
 
 namespace {
@@ -617,8 +719,14 @@ jpi_status linear(const jpi_corr_handle* h, cudaStream_t st, const float* x, int
 jpi_status layernorm(const jpi_corr_handle* h, cudaStream_t st, const float* x, int ldx, const float* g,
                      const float* b, float* y, int ldy, int rows) {
     if (rows <= 0) return JPI_OK;
-    k_corr_layernorm<<<grid_for((long long)rows * 32), 256, 0, st>>>(x, ldx, g, b, y, ldy, rows, h->d,
-                                                                     h->cfg.ln_eps);
+    const bool vec = h->d % 4 == 0 && ldx % 4 == 0 && ldy % 4 == 0 &&
+                     (((uintptr_t)x | (uintptr_t)y | (uintptr_t)g | (uintptr_t)b) & 15) == 0;
+    if (vec)
+        k_corr_layernorm<true><<<grid_for((long long)rows * 32), 256, 0, st>>>(x, ldx, g, b, y, ldy, rows, h->d,
+                                                                           h->cfg.ln_eps);
+    else
+        k_corr_layernorm<false><<<grid_for((long long)rows * 32), 256, 0, st>>>(x, ldx, g, b, y, ldy, rows, h->d,
+                                                                            h->cfg.ln_eps);
     JPI_CUDA_TRY(cudaGetLastError());
     return JPI_OK;
 }
@@ -799,6 +907,18 @@ jpi_status setup(jpi_corr_handle* h, const jpi_corr_config* c, const jpi_corr_we
     JPI_TRY(corr_alloc(h, &h->hid, B * T * F));
     JPI_TRY(corr_alloc(h, &h->sc, B * M * (size_t)h->Tm));
     JPI_TRY(corr_alloc(h, &h->gs, B * M * dv));
+    JPI_TRY(corr_alloc(h, &h->scp, B * (size_t)((dv + CORR_KCHUNK - 1) / CORR_KCHUNK) * M * h->Tm));
+    JPI_TRY(corr_alloc(h, &h->gsp, B * (size_t)((h->Tm + CORR_TCHUNK - 1) / CORR_TCHUNK) * M * dv));
+    JPI_TRY(corr_alloc(h, reinterpret_cast<float**>(&h->in_vlm), B * (size_t)h->Tm * dv));
+    JPI_TRY(corr_alloc(h, &h->in_state, B * (size_t)h->Ti * h->d));
+    JPI_TRY(corr_alloc(h, &h->in_act, B * (size_t)h->Dm * h->A));
+    JPI_TRY(corr_alloc(h, &h->out_st, B * (size_t)h->Ti * h->d));
+    JPI_TRY(corr_alloc(h, &h->out_conf, (size_t)B));
+    JPI_CUDA_TRY(cudaStreamCreateWithFlags(&h->cap, cudaStreamNonBlocking));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)CORR_SCORES_SMEM));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)CORR_SCORES_SMEM));
     JPI_TRY(corr_alloc(h, &h->conf_scratch, B));
 
     JPI_TRY(prepare(h, nullptr));
@@ -808,62 +928,28 @@ jpi_status setup(jpi_corr_handle* h, const jpi_corr_config* c, const jpi_corr_we
 
 }  // namespace
 
-extern "C" {
+namespace {
 
-JPI_API jpi_status jpi_corr_create(const jpi_corr_config* cfg, const jpi_corr_weights* w,
-                                   jpi_corr_handle** out) {
-    jpi::clear_error();
-    if (!out) return cfail(JPI_ERR_INVALID_ARG, "out is NULL");
-    *out = nullptr;
-    if (!cfg || !w) return cfail(JPI_ERR_INVALID_ARG, "config or weights is NULL");
-    JPI_TRY(check_corr_config(cfg));
-    if (cfg->n_joint > 0 && !w->jb) return cfail(JPI_ERR_INVALID_ARG, "joint blocks (jb) are NULL");
-    jpi_corr_handle* h = new (std::nothrow) jpi_corr_handle();
-    if (!h) return cfail(JPI_ERR_OOM, "host allocation failed");
-    const jpi_status s = setup(h, cfg, w);
-    if (s != JPI_OK) {
-        cudaStreamSynchronize(nullptr);   // let any conversion in flight finish before its buffers go
-        cudaGetLastError();
-        for (void* p : h->allocs) cudaFree(p);
-        delete h;
-        return s;
-    }
-    *out = h;
-    return JPI_OK;
-}
-
-JPI_API jpi_status jpi_corr_destroy(jpi_corr_handle* h) {
-    jpi::clear_error();
-    if (!h) return JPI_OK;
-    for (void* p : h->allocs) cudaFree(p);
-    delete h;
-    return JPI_OK;
-}
-
-JPI_API jpi_status jpi_corr_compress(jpi_corr_handle* h, const void* h_vlm, int vlm_is_fp32, int batch,
-                                     int n_tokens, float* out_state, void* stream) {
-    jpi::clear_error();
-    if (!h) return cfail(JPI_ERR_INVALID_ARG, "handle is NULL");
-    if (!h_vlm || !out_state) return cfail(JPI_ERR_INVALID_ARG, "NULL input or output");
-    if (batch < 1 || n_tokens < 1) return cfail(JPI_ERR_INVALID_ARG, "batch and n_tokens must be >= 1");
-    if (batch > h->B || n_tokens > h->Tm)
-        return cfail(JPI_ERR_SHAPE, "batch %d / n_tokens %d exceed the maxima %d / %d", batch, n_tokens, h->B,
-                     h->Tm);
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
+// The compressor's kernel sequence on `st`: hvlm [batch][n_tokens][dv] -> out [batch][T'][d].
+jpi_status enqueue_compress(jpi_corr_handle* h, const void* hvlm, int vlm_is_fp32, int batch, int n_tokens,
+                            float* out, cudaStream_t st) {
     const int d = h->d, T = h->Ti, M = h->M, dv = h->dv, rows = batch * T;
-    const dim3 gs((unsigned)((n_tokens + 31) / 32), (unsigned)batch);
-    const dim3 gw((unsigned)((dv + 255) / 256), (unsigned)((M + 15) / 16), (unsigned)batch);
+    const int nkc = (dv + CORR_KCHUNK - 1) / CORR_KCHUNK, ntc = (n_tokens + CORR_TCHUNK - 1) / CORR_TCHUNK;
+    const dim3 gs((unsigned)((n_tokens + 31) / 32), (unsigned)nkc, (unsigned)batch);
+    const dim3 gw((unsigned)((dv + 255) / 256), (unsigned)ntc, (unsigned)batch);
+    const int red_grid = grid_for((long long)batch * M * dv);
     if (vlm_is_fp32) {
-        const float* hv = static_cast<const float*>(h_vlm);
-        k_corr_scores<float><<<gs, 256, 0, st>>>(h->qk, hv, h->sc, M, n_tokens, dv);
-        k_corr_softmax<<<grid_for((long long)batch * M * 32), 256, 0, st>>>(h->sc, batch * M, n_tokens);
-        k_corr_wsum<float><<<gw, 256, 0, st>>>(h->sc, hv, h->gs, M, n_tokens, dv);
+        const float* hv = static_cast<const float*>(hvlm);
+        k_corr_scores<float><<<gs, 256, CORR_SCORES_SMEM, st>>>(h->qk, hv, h->scp, M, n_tokens, dv);
+        k_corr_softmax_sum<<<batch * M, 256, 0, st>>>(h->scp, h->sc, M, n_tokens, nkc);
+        k_corr_wsum<float><<<gw, 256, 0, st>>>(h->sc, hv, h->gsp, M, n_tokens, dv);
     } else {
-        const __nv_bfloat16* hv = static_cast<const __nv_bfloat16*>(h_vlm);
-        k_corr_scores<__nv_bfloat16><<<gs, 256, 0, st>>>(h->qk, hv, h->sc, M, n_tokens, dv);
-        k_corr_softmax<<<grid_for((long long)batch * M * 32), 256, 0, st>>>(h->sc, batch * M, n_tokens);
-        k_corr_wsum<__nv_bfloat16><<<gw, 256, 0, st>>>(h->sc, hv, h->gs, M, n_tokens, dv);
+        const __nv_bfloat16* hv = static_cast<const __nv_bfloat16*>(hvlm);
+        k_corr_scores<__nv_bfloat16><<<gs, 256, CORR_SCORES_SMEM, st>>>(h->qk, hv, h->scp, M, n_tokens, dv);
+        k_corr_softmax_sum<<<batch * M, 256, 0, st>>>(h->scp, h->sc, M, n_tokens, nkc);
+        k_corr_wsum<__nv_bfloat16><<<gw, 256, 0, st>>>(h->sc, hv, h->gsp, M, n_tokens, dv);
     }
+    k_corr_wsum_reduce<<<red_grid, 256, 0, st>>>(h->gsp, h->gs, batch, M, dv, ntc);
     JPI_CUDA_TRY(cudaGetLastError());
     // out_hi = W_v,h g_hi + b_v (head-select rows of gs), then the output projection onto the
     // queries' residual, the MLP, and the output LayerNorm.
@@ -872,19 +958,13 @@ JPI_API jpi_status jpi_corr_compress(jpi_corr_handle* h, const void* h_vlm, int 
     JPI_TRY(layernorm(h, st, h->xf, d, h->qf_ln3_w, h->qf_ln3_b, h->u, d, rows));
     JPI_TRY(linear(h, st, h->u, d, h->qf_w1, h->qf_b1, nullptr, 0, h->hid, h->F, rows, d, h->F, true));
     JPI_TRY(linear(h, st, h->hid, h->F, h->qf_w2, h->qf_b2, h->xf, d, h->xf, d, rows, h->F, d, false));
-    JPI_TRY(layernorm(h, st, h->xf, d, h->qf_lnf_w, h->qf_lnf_b, out_state, d, rows));
+    JPI_TRY(layernorm(h, st, h->xf, d, h->qf_lnf_w, h->qf_lnf_b, out, d, rows));
     return JPI_OK;
 }
 
-JPI_API jpi_status jpi_corr_predict(jpi_corr_handle* h, const float* state, const float* actions, int batch,
-                                    int delta, float* out_state, float* out_confidence, void* stream) {
-    jpi::clear_error();
-    if (!h) return cfail(JPI_ERR_INVALID_ARG, "handle is NULL");
-    if (!state || !actions || !out_state) return cfail(JPI_ERR_INVALID_ARG, "NULL input or output");
-    if (batch < 1 || delta < 1) return cfail(JPI_ERR_INVALID_ARG, "batch and delta must be >= 1");
-    if (batch > h->B || delta > h->Dm)
-        return cfail(JPI_ERR_SHAPE, "batch %d / delta %d exceed the maxima %d / %d", batch, delta, h->B, h->Dm);
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
+// f_corr's kernel sequence on `st`: state, actions -> out [batch][T'][d], conf [batch].
+jpi_status enqueue_predict(jpi_corr_handle* h, const float* state, const float* actions, int batch, int delta,
+                           float* out, float* conf, cudaStream_t st) {
     const int d = h->d, T = h->Ti, F = h->F, ra = batch * delta, rows = batch * T;
     const BlockDev& ab = h->ab;
     // Action tokens: MLP, plus the position row of each action.
@@ -911,11 +991,125 @@ JPI_API jpi_status jpi_corr_predict(jpi_corr_handle* h, const float* state, cons
     for (int i = 0; i < h->J; ++i) JPI_TRY(block(h, st, h->jb[(size_t)i], h->xf, batch, T));
     // Heads.
     JPI_TRY(layernorm(h, st, h->xf, d, h->head_ln_w, h->head_ln_b, h->u, d, rows));
-    JPI_TRY(linear(h, st, h->u, d, h->corr_w, h->corr_b, nullptr, 0, out_state, d, rows, d, d, false));
-    float* conf = out_confidence ? out_confidence : h->conf_scratch;
-    k_corr_confidence<<<grid_for((long long)batch * 32), 256, 0, st>>>(h->u, h->conf_w, h->conf_b, conf, batch,
-                                                                       T, d);
+    JPI_TRY(linear(h, st, h->u, d, h->corr_w, h->corr_b, nullptr, 0, out, d, rows, d, d, false));
+    k_corr_confidence<<<batch, 256, 0, st>>>(h->u, h->conf_w, h->conf_b, conf, T, d);
     JPI_CUDA_TRY(cudaGetLastError());
+    return JPI_OK;
+}
+
+// The graph of one call shape, captured on the handle's own stream the first time it is asked for.
+template <typename F>
+jpi_status corr_graph(jpi_corr_handle* h, std::tuple<int, int, int, int> key, F&& enqueue, cudaGraphExec_t* out) {
+    auto it = h->graphs.find(key);
+    if (it != h->graphs.end()) {
+        *out = it->second;
+        return JPI_OK;
+    }
+    cudaGraph_t g = nullptr;
+    JPI_CUDA_TRY(cudaStreamBeginCapture(h->cap, cudaStreamCaptureModeThreadLocal));
+    const jpi_status s = enqueue(h->cap);
+    const cudaError_t e = cudaStreamEndCapture(h->cap, &g);
+    if (s != JPI_OK) {
+        if (g) cudaGraphDestroy(g);
+        return s;
+    }
+    if (e != cudaSuccess) return cfail(JPI_ERR_CUDA, "graph capture failed: %s", cudaGetErrorString(e));
+    cudaGraphExec_t ex = nullptr;
+    const cudaError_t ei = cudaGraphInstantiate(&ex, g, 0);
+    cudaGraphDestroy(g);
+    if (ei != cudaSuccess) return cfail(JPI_ERR_CUDA, "graph instantiate failed: %s", cudaGetErrorString(ei));
+    h->graphs[key] = ex;
+    *out = ex;
+    return JPI_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+JPI_API jpi_status jpi_corr_create(const jpi_corr_config* cfg, const jpi_corr_weights* w,
+                                   jpi_corr_handle** out) {
+    jpi::clear_error();
+    if (!out) return cfail(JPI_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (!cfg || !w) return cfail(JPI_ERR_INVALID_ARG, "config or weights is NULL");
+    JPI_TRY(check_corr_config(cfg));
+    if (cfg->n_joint > 0 && !w->jb) return cfail(JPI_ERR_INVALID_ARG, "joint blocks (jb) are NULL");
+    jpi_corr_handle* h = new (std::nothrow) jpi_corr_handle();
+    if (!h) return cfail(JPI_ERR_OOM, "host allocation failed");
+    const jpi_status s = setup(h, cfg, w);
+    if (s != JPI_OK) {
+        cudaStreamSynchronize(nullptr);   // let any conversion in flight finish before its buffers go
+        cudaGetLastError();
+        if (h->cap) cudaStreamDestroy(h->cap);
+        for (void* p : h->allocs) cudaFree(p);
+        delete h;
+        return s;
+    }
+    *out = h;
+    return JPI_OK;
+}
+
+JPI_API jpi_status jpi_corr_destroy(jpi_corr_handle* h) {
+    jpi::clear_error();
+    if (!h) return JPI_OK;
+    cudaDeviceSynchronize();
+    for (auto& kv : h->graphs) cudaGraphExecDestroy(kv.second);
+    if (h->cap) cudaStreamDestroy(h->cap);
+    for (void* p : h->allocs) cudaFree(p);
+    cudaGetLastError();
+    delete h;
+    return JPI_OK;
+}
+
+JPI_API jpi_status jpi_corr_compress(jpi_corr_handle* h, const void* h_vlm, int vlm_is_fp32, int batch,
+                                     int n_tokens, float* out_state, void* stream) {
+    jpi::clear_error();
+    if (!h) return cfail(JPI_ERR_INVALID_ARG, "handle is NULL");
+    if (!h_vlm || !out_state) return cfail(JPI_ERR_INVALID_ARG, "NULL input or output");
+    if (batch < 1 || n_tokens < 1) return cfail(JPI_ERR_INVALID_ARG, "batch and n_tokens must be >= 1");
+    if (batch > h->B || n_tokens > h->Tm)
+        return cfail(JPI_ERR_SHAPE, "batch %d / n_tokens %d exceed the maxima %d / %d", batch, n_tokens, h->B,
+                     h->Tm);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t in_bytes = (size_t)batch * n_tokens * h->dv * (vlm_is_fp32 ? 4 : 2);
+    cudaGraphExec_t ex = nullptr;
+    JPI_TRY(corr_graph(h, std::make_tuple(0, batch, n_tokens, vlm_is_fp32 ? 1 : 0),
+                       [&](cudaStream_t cs) {
+                           return enqueue_compress(h, h->in_vlm, vlm_is_fp32, batch, n_tokens, h->out_st, cs);
+                       },
+                       &ex));
+    JPI_CUDA_TRY(cudaMemcpyAsync(h->in_vlm, h_vlm, in_bytes, cudaMemcpyDeviceToDevice, st));
+    JPI_CUDA_TRY(cudaGraphLaunch(ex, st));
+    JPI_CUDA_TRY(cudaMemcpyAsync(out_state, h->out_st, (size_t)batch * h->Ti * h->d * sizeof(float),
+                                 cudaMemcpyDeviceToDevice, st));
+    return JPI_OK;
+}
+
+JPI_API jpi_status jpi_corr_predict(jpi_corr_handle* h, const float* state, const float* actions, int batch,
+                                    int delta, float* out_state, float* out_confidence, void* stream) {
+    jpi::clear_error();
+    if (!h) return cfail(JPI_ERR_INVALID_ARG, "handle is NULL");
+    if (!state || !actions || !out_state) return cfail(JPI_ERR_INVALID_ARG, "NULL input or output");
+    if (batch < 1 || delta < 1) return cfail(JPI_ERR_INVALID_ARG, "batch and delta must be >= 1");
+    if (batch > h->B || delta > h->Dm)
+        return cfail(JPI_ERR_SHAPE, "batch %d / delta %d exceed the maxima %d / %d", batch, delta, h->B, h->Dm);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaGraphExec_t ex = nullptr;
+    JPI_TRY(corr_graph(h, std::make_tuple(1, batch, delta, 0),
+                       [&](cudaStream_t cs) {
+                           return enqueue_predict(h, h->in_state, h->in_act, batch, delta, h->out_st, h->out_conf, cs);
+                       },
+                       &ex));
+    const size_t state_bytes = (size_t)batch * h->Ti * h->d * sizeof(float);
+    JPI_CUDA_TRY(cudaMemcpyAsync(h->in_state, state, state_bytes, cudaMemcpyDeviceToDevice, st));
+    JPI_CUDA_TRY(cudaMemcpyAsync(h->in_act, actions, (size_t)batch * delta * h->A * sizeof(float),
+                                 cudaMemcpyDeviceToDevice, st));
+    JPI_CUDA_TRY(cudaGraphLaunch(ex, st));
+    JPI_CUDA_TRY(cudaMemcpyAsync(out_state, h->out_st, state_bytes, cudaMemcpyDeviceToDevice, st));
+    if (out_confidence)
+        JPI_CUDA_TRY(cudaMemcpyAsync(out_confidence, h->out_conf, (size_t)batch * sizeof(float),
+                                     cudaMemcpyDeviceToDevice, st));
     return JPI_OK;
 }
 
