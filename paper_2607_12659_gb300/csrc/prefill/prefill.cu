@@ -172,8 +172,9 @@ struct LayerW {
 // The products: Y[m][n] = alpha sum_k X[m][k] W[n][k] (+ Y[m][n]), X [M][K] and W [N][K] row-major
 // bf16, Y fp32 or bf16, fp32 accumulation. One output tile = 128 rows of W (the MMA's M) x 128
 // rows of X (its N) over the whole K range, in TMEM as [W row = lane][X row = column]. Persistent:
-// one CTA per SM walks the tiles u = blockIdx.x, + gridDim.x, ... (W tile fastest, so CTAs that run
-// together share X tiles through L2):
+// one CTA per SM walks the tiles u = blockIdx.x, + gridDim.x, ... with the X tile fastest, so the
+// CTAs that run together share one W tile through L2 and every W tile is read from HBM once (W is
+// the large operand: 134 MB for gate/up at Gemma-2B sizes, X 3.3 MB):
 //   warp 0  one thread streams (W block, X block) pairs of 64 K-columns by bulk tensor copies
 //           (128-byte swizzle; rows and columns past the tensors' extents arrive as zeros) into a
 //           ring of PG_STAGES stages;
@@ -248,7 +249,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
             int it = 0, issued = 0;
             bool ok = true;
             for (int u = u0; u < total && ok; u += du) {
-                const int tn = u % ntn, tm = u / ntn;
+                const int tm = u % ntm, tn = u / ntm;
                 for (int kb = 0; kb < nkb; ++kb, ++it) {
                     const int s = it % PG_STAGES, n = it / PG_STAGES;
                     if (it >= PG_STAGES && !ptx::mbar_wait_bounded(&empty[s], (n - 1) & 1, PG_WAIT_NS)) {
@@ -303,7 +304,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         for (int u = u0, j = 0; u < total; u += du, ++j) {
             const int buf = j & 1;
-            const int tn = u % ntn, tm = u / ntn;
+            const int tm = u % ntm, tn = u / ntm;
             const bool ok = ptx::mbar_wait_bounded(&accf[buf], (j >> 1) & 1, PG_WAIT_NS) && *flag == 0;
             ptx::tc_fence_after();
             const int n = tn * PG_TILE + row;
