@@ -119,6 +119,12 @@ typedef struct jpi_weights {
  * Ownership: the weights are copied; the caller may free its buffers when the call returns.
  * Synchronous. Errors: INVALID_ARG (null pointer, bad dims), UNSUPPORTED (dims the kernels
  * do not tile), OOM, CUDA.
+ * The environment read here fixes kernel choices for the handle's lifetime:
+ * JPI_BATCH_INVARIANT=1 makes every launch choose its kernels and splits as for one request, so
+ * a request's actions are identical bit for bit alone and inside any batch (slower from batch 4);
+ * JPI_ATTN_SPLITS=n fixes the key splits of the small-batch attention (results agree across
+ * split counts to rounding only); JPI_ATTN_T5_MIN_BATCH and JPI_BIG_GEMM_MIN_TOKENS move the
+ * batch / token thresholds of the large-batch attention and projection kernels (0 disables them).
  */
 JPI_API jpi_status jpi_expert_create(const jpi_config* cfg, const jpi_weights* w, jpi_handle** out);
 

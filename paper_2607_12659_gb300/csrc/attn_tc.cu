@@ -461,7 +461,8 @@ jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     // themselves (then each CTA runs an online softmax over all keys and nothing is exchanged).
     // The split follows the launch's sizes, so a request's low-order bits depend on the batch
     // size it runs with; they never depend on timing.
-    const int blocks = rblocks * B;
+    // In the batch-invariant mode the split is the one a single request gets, whatever B.
+    const int blocks = rblocks * (h->batch_invariant ? 1 : B);
     int want = (2 * h->num_sms + blocks - 1) / blocks;
     // A split count asked through the environment at create time replaces that choice.
     if (h->attn_force_splits > 0) want = h->attn_force_splits;

@@ -109,6 +109,7 @@ struct jpi_handle {
     int num_sms = 0;
     int attn_max_splits = 8;  // largest key-split cluster of the attention kernel
     int attn_force_splits = 0;  // > 0: key splits asked of the split-KV attention (JPI_ATTN_SPLITS)
+    bool batch_invariant = false;   // kernels and splits of one request at every batch size (JPI_BATCH_INVARIANT)
 
     // Dimensions.
     int L, W, H, D, F, A, Sd, dt, HD, QKV;   // QKV = (H + 2) D

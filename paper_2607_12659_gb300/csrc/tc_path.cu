@@ -472,6 +472,15 @@ jpi_status tc_prepare(jpi_handle* h) {
     JPI_TRY(make_tmap(h->o, h->maxMt, h->HD, NT, &h->xmaps[1]));
     JPI_TRY(make_tmap(h->z, h->maxMt, h->F, NT, &h->xmaps[2]));
     JPI_TRY(mod_tc_prepare(h));
+    // JPI_BATCH_INVARIANT=1: every launch makes the choices it makes for one request (K-split
+    // projections, split-KV attention with a single request's key split), so a request's result
+    // is the same bit for bit alone and inside any batch, at the cost of the batched kernels.
+    const char* inv_env = std::getenv("JPI_BATCH_INVARIANT");
+    if (inv_env && inv_env[0] == '1') {
+        h->batch_invariant = true;
+        h->attn_t5_min_batch = 0;
+        for (int k = 0; k < 4; ++k) h->big_min_tokens[k] = 0;
+    }
     return JPI_OK;
 }
 

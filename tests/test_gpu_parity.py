@@ -300,3 +300,28 @@ def test_split_counts_agree_on_one_pi05_shaped_layer(monkeypatch):
         dv = float(np.abs(got[s][0] - got[16][0]).max())
         print(f"splits {s} vs 14: hidden {dh:.3g} (relative to max |h| {scale:.3g}), velocity {dv:.3g}")
         assert dh <= SPLIT_AGREEMENT, f"{s} key splits: hidden state differs by {dh:.3g} of max |h|"
+
+
+# Batch invariance, bit for bit: with JPI_BATCH_INVARIANT=1 every launch makes the choices it makes
+# for a single request (the K-split projections with their fixed K split, the split-KV attention
+# with one request's key split), so request b of a batch gets exactly the actions it gets alone.
+# Without the switch the attention's split and the projection kernel follow the batch size and the
+# low-order bits may move (test_pi05_batches_sampled_requests bounds that).
+@pytest.mark.parametrize("cfg,P,C,N,B", [(SMALL_BF16, 100, 13, 2, 3), (PI05, 816, 50, 10, 16)],
+                         ids=["small-bf16", "pi05"])
+def test_batch_invariant_mode_is_bitwise(monkeypatch, cfg, P, C, N, B):
+    monkeypatch.setenv("JPI_BATCH_INVARIANT", "1")
+    w = make_weights(cfg, 2800)
+    ex = make_expert(cfg, w, max_batch=B, max_prefix=P, max_chunk=C, max_steps=N)
+    try:
+        r = make_requests(cfg, 2801, B, P, C)
+        got = gpu_denoise(ex, cfg, r, N)
+        for b in sorted({0, B // 2, B - 1}):
+            one = gpu_denoise(ex, cfg, make_requests(cfg, 2801, 1, P, C, first_request=b), N)
+            assert np.array_equal(got[b:b + 1], one), \
+                f"request {b}: max difference {float(np.abs(got[b:b + 1] - one).max()):.3g}"
+        sample = [0, B - 1]
+        assert_close(got[sample], oracle_denoise(cfg, oracle.to_f64(w), r, N, sample), cfg,
+                     f"batch-invariant mode B{B} P{P}")
+    finally:
+        ex.close()
