@@ -170,26 +170,30 @@ struct LayerW {
 
 // ---------------------------------------------------------------------------------------------
 // The products: Y[m][n] = alpha sum_k X[m][k] W[n][k] (+ Y[m][n]), X [M][K] and W [N][K] row-major
-// bf16, Y fp32 or bf16, fp32 accumulation. One output tile = 128 rows of W (the MMA's M) x 128
-// rows of X (its N) over the whole K range, in TMEM as [W row = lane][X row = column]. Persistent:
-// one CTA per SM walks the tiles u = blockIdx.x, + gridDim.x, ... with the X tile fastest, so the
-// CTAs that run together share one W tile through L2 and every W tile is read from HBM once (W is
-// the large operand: 134 MB for gate/up at Gemma-2B sizes, X 3.3 MB):
-//   warp 0  one thread streams (W block, X block) pairs of 64 K-columns by bulk tensor copies
+// bf16, Y fp32 or bf16, fp32 accumulation. One output tile = 128 rows of X (the MMA's M) x 256
+// rows of W (its N) over the whole K range, in TMEM as [X row = lane][W row = column]: each k-block
+// brings 48 KB into the SM for 2 M multiply-adds (a 128 x 128 tile brings 32 KB for 1 M, and one
+// SM takes in only about 85 GB/s from L2), and only the token dimension, 816 rows at Gemma-2B
+// sizes, is padded. Persistent: one CTA per SM walks the tiles u = blockIdx.x, + gridDim.x, ...
+// with the X tile fastest, so the CTAs that run together share one W tile through L2 and every W
+// tile is read from HBM once (W is the large operand: 134 MB for gate/up, X 3.3 MB):
+//   warp 0  one thread streams (X block, W block) pairs of 64 K-columns by bulk tensor copies
 //           (128-byte swizzle; rows and columns past the tensors' extents arrive as zeros) into a
 //           ring of PG_STAGES stages;
-//   warp 1  one thread issues the tcgen05.mma chain (M = 128, N = 128, K = 16 each) into one of two
+//   warp 1  one thread issues the tcgen05.mma chain (M = 128, N = 256, K = 16 each) into one of two
 //           TMEM accumulators and releases each stage through tcgen05.commit;
-//   warps 2-5  one TMEM lane (W row n) per thread: 16 columns (X rows m) at a time, scaled by alpha,
-//           added to Y when accumulating, stored (consecutive lanes write consecutive n), after
+//   warps 2-5  one TMEM lane (X row m) per thread: 16 columns (W rows n) at a time, scaled by
+//           alpha, added to Y when accumulating, stored as 16 consecutive elements of row m, after
 //           which the accumulator goes back to the MMA thread.
 // Every wait is bounded; a timeout records a device error in the handle's word and the CTA returns.
 
-constexpr int PG_TILE = 128;
+constexpr int PG_TM = 128;                                      // X rows per tile (MMA M)
+constexpr int PG_TN = 256;                                      // W rows per tile (MMA N)
 constexpr int PG_KBLK = 64;
-constexpr int PG_STAGES = 6;
-constexpr int PG_BLOCK_BYTES = PG_TILE * PG_KBLK * 2;          // 16 KB
-constexpr int PG_STAGE_BYTES = 2 * PG_BLOCK_BYTES;
+constexpr int PG_STAGES = 4;
+constexpr int PG_XBYTES = PG_TM * PG_KBLK * 2;                  // 16 KB
+constexpr int PG_WBYTES = PG_TN * PG_KBLK * 2;                  // 32 KB
+constexpr int PG_STAGE_BYTES = PG_XBYTES + PG_WBYTES;
 constexpr int PG_THREADS = 192;
 constexpr uint64_t PG_WAIT_NS = 200ull * 1000 * 1000;
 constexpr size_t PG_SMEM = 1024 + (size_t)PG_STAGES * PG_STAGE_BYTES + 128;
@@ -201,6 +205,7 @@ struct PfGemmArgs {
     float alpha;
     int accumulate;       // Y += ... (fp32 Y only)
     int out_bf16;
+    int vec;              // Y and ldy allow 16-byte stores of 16 consecutive elements
     void* Y;
     long long ldy;        // elements
     int* err;
@@ -212,7 +217,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
     namespace ptx = jpi::ptx;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (ptx::smem_u32(smem_raw) & 1023u)) & 1023u);
-    uint8_t* stages = smem;
+    uint8_t* stages = smem;                                  // [stage][X 16 KB | W 32 KB]
     uint64_t* full = (uint64_t*)(smem + (size_t)PG_STAGES * PG_STAGE_BYTES);
     uint64_t* empty = full + PG_STAGES;
     uint64_t* accf = empty + PG_STAGES;
@@ -222,12 +227,12 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nkb = (a.K + PG_KBLK - 1) / PG_KBLK;
-    const int ntn = (a.N + PG_TILE - 1) / PG_TILE, ntm = (a.M + PG_TILE - 1) / PG_TILE;
+    const int ntn = (a.N + PG_TN - 1) / PG_TN, ntm = (a.M + PG_TM - 1) / PG_TM;
     const int total = ntn * ntm;
     const int u0 = blockIdx.x, du = gridDim.x;
 
     if (warp == 1) {
-        ptx::tmem_alloc(tmem_slot, 2 * PG_TILE);
+        ptx::tmem_alloc(tmem_slot, 2 * PG_TN);
         ptx::tmem_relinquish();
     }
     if (tid == 0) {
@@ -259,8 +264,8 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
                     }
                     uint8_t* st = stages + (size_t)s * PG_STAGE_BYTES;
                     ptx::mbar_expect_tx(&full[s], (uint32_t)PG_STAGE_BYTES);
-                    ptx::tma_load_2d_plain(st, &wmap, &full[s], kb * PG_KBLK, tn * PG_TILE);
-                    ptx::tma_load_2d_plain(st + PG_BLOCK_BYTES, &xmap, &full[s], kb * PG_KBLK, tm * PG_TILE);
+                    ptx::tma_load_2d_plain(st, &xmap, &full[s], kb * PG_KBLK, tm * PG_TM);
+                    ptx::tma_load_2d_plain(st + PG_XBYTES, &wmap, &full[s], kb * PG_KBLK, tn * PG_TN);
                     issued = it + 1;
                 }
             }
@@ -272,7 +277,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            constexpr uint32_t IDESC = ptx::idesc_bf16_f32(PG_TILE, PG_TILE);
+            constexpr uint32_t IDESC = ptx::idesc_bf16_f32(PG_TM, PG_TN);
             const uint32_t base = ptx::smem_u32(stages);
             bool good = true;
             int it = 0;
@@ -280,16 +285,16 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
                 const int buf = j & 1;
                 if (j >= 2 && !ptx::mbar_wait_bounded(&acce[buf], ((j - 2) >> 1) & 1, PG_WAIT_NS)) good = false;
                 ptx::tc_fence_after();
-                const uint32_t acc = tmem + (uint32_t)(buf * PG_TILE);
+                const uint32_t acc = tmem + (uint32_t)(buf * PG_TN);
                 for (int kb = 0; kb < nkb; ++kb, ++it) {
                     const int s = it % PG_STAGES, n = it / PG_STAGES;
                     if (good && !ptx::mbar_wait_bounded(&full[s], n & 1, PG_WAIT_NS)) good = false;
                     ptx::tc_fence_after();
                     if (good) {
-                        const uint32_t w = base + (uint32_t)(s * PG_STAGE_BYTES), x = w + PG_BLOCK_BYTES;
+                        const uint32_t x = base + (uint32_t)(s * PG_STAGE_BYTES), w = x + PG_XBYTES;
 #pragma unroll
                         for (int kk = 0; kk < PG_KBLK / 16; ++kk)
-                            ptx::mma_bf16(acc, ptx::desc_sw128(w + kk * 32), ptx::desc_sw128(x + kk * 32), IDESC,
+                            ptx::mma_bf16(acc, ptx::desc_sw128(x + kk * 32), ptx::desc_sw128(w + kk * 32), IDESC,
                                           (kb | kk) != 0);
                     }
                     ptx::mma_commit(&empty[s]);
@@ -300,30 +305,61 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
             if (!good) *flag = PF_DEV_TIMEOUT_MMA;
         }
     } else {
-        const int row = (warp & 3) * 32 + lane;   // TMEM lane: W row of the tile
+        const int row = (warp & 3) * 32 + lane;   // TMEM lane: X row of the tile
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         for (int u = u0, j = 0; u < total; u += du, ++j) {
             const int buf = j & 1;
             const int tm = u % ntm, tn = u / ntm;
             const bool ok = ptx::mbar_wait_bounded(&accf[buf], (j >> 1) & 1, PG_WAIT_NS) && *flag == 0;
             ptx::tc_fence_after();
-            const int n = tn * PG_TILE + row;
-            for (int c0 = 0; c0 < PG_TILE; c0 += 16) {
+            const int m = tm * PG_TM + row;
+            const bool live = ok && m < a.M;
+            for (int c0 = 0; c0 < PG_TN; c0 += 16) {
                 uint32_t r[16];
-                ptx::tmem_ld_x16(lane_base + (uint32_t)(buf * PG_TILE + c0), r);
+                ptx::tmem_ld_x16(lane_base + (uint32_t)(buf * PG_TN + c0), r);
                 ptx::tmem_ld_wait();
-                if (!ok || n >= a.N) continue;
+                const int n0 = tn * PG_TN + c0;
+                if (!live || n0 >= a.N) continue;
+                float v[16];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int m = tm * PG_TILE + c0 + i;
-                    if (m >= a.M) break;
-                    const float v = a.alpha * __uint_as_float(r[i]);
-                    const size_t o = (size_t)m * a.ldy + n;
+                for (int i = 0; i < 16; ++i) v[i] = a.alpha * __uint_as_float(r[i]);
+                const size_t o = (size_t)m * a.ldy + n0;
+                if (a.vec && n0 + 16 <= a.N) {
                     if (a.out_bf16) {
-                        static_cast<__nv_bfloat16*>(a.Y)[o] = __float2bfloat16_rn(v);
+                        uint4* y = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.Y) + o);
+                        uint32_t p[8];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            __nv_bfloat162 t = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+                            p[i] = *reinterpret_cast<uint32_t*>(&t);
+                        }
+                        y[0] = make_uint4(p[0], p[1], p[2], p[3]);
+                        y[1] = make_uint4(p[4], p[5], p[6], p[7]);
                     } else {
-                        float* y = static_cast<float*>(a.Y) + o;
-                        *y = a.accumulate ? *y + v : v;
+                        float4* y = reinterpret_cast<float4*>(static_cast<float*>(a.Y) + o);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            float4 t = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                            if (a.accumulate) {
+                                const float4 old = y[q];
+                                t.x += old.x;
+                                t.y += old.y;
+                                t.z += old.z;
+                                t.w += old.w;
+                            }
+                            y[q] = t;
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        if (n0 + i >= a.N) continue;
+                        if (a.out_bf16) {
+                            static_cast<__nv_bfloat16*>(a.Y)[o + i] = __float2bfloat16_rn(v[i]);
+                        } else {
+                            float* y = static_cast<float*>(a.Y) + o + i;
+                            *y = a.accumulate ? *y + v[i] : v[i];
+                        }
                     }
                 }
             }
@@ -337,7 +373,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
-    if (warp == 1) ptx::tmem_dealloc(tmem, 2 * PG_TILE);
+    if (warp == 1) ptx::tmem_dealloc(tmem, 2 * PG_TN);
 }
 
 // vt[d][p] = v[p][d] for one request (p < P), so that P V runs as a product of K-major operands.
@@ -415,15 +451,15 @@ void release(jpi_prefill_handle* h) {
 }
 
 // 2D bf16 tensor map over a row-major [rows][cols] matrix of leading dimension ld (elements),
-// 128-byte swizzle, boxes of 64 columns x 128 rows; reads past the extents return zeros.
-jpi_status make_map(const void* base, long long rows, long long cols, long long ld, CUtensorMap* map) {
+// 128-byte swizzle, boxes of 64 columns x box_rows rows; reads past the extents return zeros.
+jpi_status make_map(const void* base, long long rows, long long cols, long long ld, int box_rows, CUtensorMap* map) {
     auto enc = get_encode();
     if (!enc) return pfail(JPI_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
     if ((reinterpret_cast<uintptr_t>(base) & 15) || (ld * 2) % 16)
         return pfail(JPI_ERR_INVALID_ARG, "a GEMM operand is not 16-byte aligned (address or row stride)");
     const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     const cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
-    const cuuint32_t box[2] = {(cuuint32_t)PG_KBLK, (cuuint32_t)PG_TILE};
+    const cuuint32_t box[2] = {(cuuint32_t)PG_KBLK, (cuuint32_t)box_rows};
     const cuuint32_t estr[2] = {1, 1};
     const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
                            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -438,8 +474,8 @@ jpi_status row_gemm(jpi_prefill_handle* h, cudaStream_t st, const __nv_bfloat16*
                     const __nv_bfloat16* Wm, long long ldw, void* Y, bool y_bf16, long long ldy, int M, int N,
                     int K, float alpha, bool accumulate) {
     CUtensorMap wmap, xmap;
-    PF_TRY(make_map(Wm, N, K, ldw, &wmap));
-    PF_TRY(make_map(X, M, K, ldx, &xmap));
+    PF_TRY(make_map(Wm, N, K, ldw, PG_TN, &wmap));
+    PF_TRY(make_map(X, M, K, ldx, PG_TM, &xmap));
     PfGemmArgs a;
     a.M = M;
     a.N = N;
@@ -449,8 +485,9 @@ jpi_status row_gemm(jpi_prefill_handle* h, cudaStream_t st, const __nv_bfloat16*
     a.out_bf16 = y_bf16 ? 1 : 0;
     a.Y = Y;
     a.ldy = ldy;
+    a.vec = (reinterpret_cast<uintptr_t>(Y) % 16 == 0 && ldy % (y_bf16 ? 8 : 4) == 0) ? 1 : 0;
     a.err = h->dev_err;
-    const long long tiles = (long long)((N + PG_TILE - 1) / PG_TILE) * ((M + PG_TILE - 1) / PG_TILE);
+    const long long tiles = (long long)((N + PG_TN - 1) / PG_TN) * ((M + PG_TM - 1) / PG_TM);
     const int grid = (int)(tiles < h->num_sms ? tiles : h->num_sms);
     k_pf_gemm<<<grid, PG_THREADS, PG_SMEM, st>>>(wmap, xmap, a);
     PF_CUDA(cudaGetLastError());
