@@ -587,8 +587,25 @@ def profile_forward(args):
     print(json.dumps({"profile_forward": "ok", "passes": args.forward_passes}))
 
 
+def primitives_arm():
+    """The hardware-primitive costs that bound the batch-1 chain (csrc/probe/primitives.cu): one
+    JSON line (a diagnostic, not a bench line)."""
+    from paper_2607_12659_gb300 import build
+    binary = build.build_probe()
+    r = subprocess.run([binary], capture_output=True, text=True, timeout=300)
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    if r.returncode != 0 or not lines:
+        raise SystemExit(f"primitives probe failed ({r.returncode}): {r.stdout[-400:]} {r.stderr[-400:]}")
+    out = json.loads(lines[-1])
+    print(json.dumps({"metric": "GB300 primitive costs behind the batch-1 chain (diagnostic)",
+                      "primitives": out, "clocks_note": "not sampled; durations are medians of short loops"}),
+          flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--primitives", action="store_true",
+                    help="measure the hand-off, barrier, reduction, copy and MMA-issue costs (diagnostic)")
     ap.add_argument("--profile-forward", action="store_true",
                     help="run eager expert passes of the workload (small case for ncu captures)")
     ap.add_argument("--forward-passes", type=int, default=2)
@@ -612,6 +629,9 @@ def main():
         return
     if args.profile_forward:
         profile_forward(args)
+        return
+    if args.primitives:
+        primitives_arm()
         return
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -86,6 +86,23 @@ def build_prefill(verbose: bool = False, force: bool = False) -> str:
     return PREFILL_LIB
 
 
+PROBE_SRC = os.path.join(CSRC, "probe", "primitives.cu")
+PROBE_BIN = os.path.join(BUILD, "primitives")
+
+
+def build_probe(force: bool = False) -> str:
+    """Compile the hardware-primitive diagnostic (csrc/probe/primitives.cu, a standalone
+    executable, not part of either library) and return its path."""
+    os.makedirs(BUILD, exist_ok=True)
+    deps = [PROBE_SRC, os.path.join(CSRC, "ptx.h")]
+    if force or not os.path.exists(PROBE_BIN) or any(os.path.getmtime(d) > os.path.getmtime(PROBE_BIN) for d in deps):
+        r = subprocess.run([nvcc()] + ARCH + ["-O2", "-std=c++17", "-o", PROBE_BIN, PROBE_SRC],
+                           capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed for primitives.cu:\n{r.stderr}")
+    return PROBE_BIN
+
+
 def build(verbose: bool = False, force: bool = False) -> str:
     """Compile every .cu directly under csrc/ and link libjpi.so, then the prefill library;
     returns libjpi.so's path."""
