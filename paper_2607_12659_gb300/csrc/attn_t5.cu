@@ -8,14 +8,17 @@
 //
 // One CTA = 128 query rows of one request over all of its keys, in blocks of 64 keys (two TMEM
 // score buffers and two shared-memory P buffers, so block i+1's softmax overlaps block i's P V):
-//   warp 0  one thread: bulk tensor copies of the query tile once, then K and V blocks through
-//           two-slot rings of their own (K of block i+2 as soon as S_i is done, V of block i+2
-//           once P_i V_i is done; prefix blocks may be fetched before the grid-dependency wait);
-//   warp 1  one thread: S_i = Q K_i^T (M = 128, N = 64, K = D) into one of two TMEM score
-//           buffers, and O += P_i V_i (M = 128, N = D, K = 64) into the TMEM output with V read
-//           as an MN-major operand straight from its bulk copy; order S_0, S_1, then P_i V_i as
-//           soon as P_i is written followed by S_{i+2}, so P V never waits for a copy;
-//   warps 2-5  one query row per thread (its TMEM lane): scale, mask, block maximum, softmax
+//   warp 0  one thread: bulk tensor copies of the query tile once, then K blocks through a
+//           two-slot ring (K of block i+2 as soon as S_i is done);
+//   warp 1  one thread: V blocks through a two-slot ring of their own (V of block i+2 once
+//           P_i V_i is done); prefix blocks of either may be fetched before the dependency wait;
+//   warp 2  one thread: S_i = Q K_i^T (M = 128, N = 64, K = D) into one of two TMEM score
+//           buffers: S_0, S_1, then S_{i+2} as soon as P_i is written (its score buffer is free);
+//   warp 3  one thread: O += P_i V_i (M = 128, N = D, K = 64) into the TMEM output with V read
+//           as an MN-major operand straight from its bulk copy, as soon as P_i and V_i are in.
+//           The two MMA chains are issued by two threads, so neither waits on the other's issue
+//           (one thread issues an N = 64 MMA every ~50-75 cycles, longer than it runs);
+//   warps 4-7  one query row per thread (its TMEM lane): scale, mask, block maximum, softmax
 //           probabilities P_i written to shared memory (bf16, 128-byte swizzled K-major rows).
 //           The running maximum is only moved, and O rescaled in TMEM, when a block's maximum
 //           exceeds it by more than 8 (log2 units), so probabilities stay below 2^8.
@@ -34,7 +37,7 @@ namespace {
 constexpr int T5_ROWS = 128;
 constexpr int T5_KEYS = 64;
 constexpr int T5_STAGES = 2;
-constexpr int T5_THREADS = 192;
+constexpr int T5_THREADS = 256;
 constexpr uint64_t T5_WAIT_NS = 200ull * 1000 * 1000;
 constexpr float T5_RESCALE = 8.f;   // log2 units
 
@@ -130,60 +133,47 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
+    if (warp <= 1) {
+        // Warp 0 streams Q and K, warp 1 streams V.
         if (lane == 0) {
+            const bool is_v = warp == 1;
             const uint64_t pol = ptx::l2_policy_evict_first();
             const int kv0 = (a.layer * a.maxB + b) * a.kv_rows;
-            // One half-stage (K or V of block i, ring slot i mod 2): NDB column boxes.
-            auto load_half = [&](bool is_v, int i) {
+            uint64_t* fullb = is_v ? vfull : kfull;
+            uint64_t* emptyb = is_v ? vempty : kempty;
+            const CUtensorMap* map = is_v ? &vmap : &kmap;
+            // Block i into ring slot i mod 2: NDB column boxes.
+            auto load = [&](int i) {
                 const int sl = i % T5_STAGES;
-                uint64_t* bar = is_v ? &vfull[sl] : &kfull[sl];
                 uint8_t* base = stages + sl * L::STAGE + (is_v ? L::KVBYTES : 0);
-                const CUtensorMap* map = is_v ? &vmap : &kmap;
-                ptx::mbar_expect_tx(bar, (uint32_t)L::KVBYTES);
+                ptx::mbar_expect_tx(&fullb[sl], (uint32_t)L::KVBYTES);
                 for (int db = 0; db < NDB; ++db)
-                    ptx::tma_load_2d(base + db * (T5_KEYS * 128), map, bar, db * 64, kv0 + i * T5_KEYS, pol);
+                    ptx::tma_load_2d(base + db * (T5_KEYS * 128), map, &fullb[sl], db * 64, kv0 + i * T5_KEYS, pol);
             };
             // First use of both slots: blocks made only of prefix keys were written before this
             // graph ran and are fetched before the dependency wait.
             int first = 0;
-            while (first < T5_STAGES && first < nb && (first + 1) * T5_KEYS <= a.P) {
-                load_half(false, first);
-                load_half(true, first);
-                ++first;
-            }
-            ptx::prefetch_tmap(&qmap);
+            while (first < T5_STAGES && first < nb && (first + 1) * T5_KEYS <= a.P) load(first++);
+            if (!is_v) ptx::prefetch_tmap(&qmap);
             ptx::grid_dep_wait();
-            ptx::mbar_expect_tx(qfull, (uint32_t)L::QBYTES);
-            for (int db = 0; db < NDB; ++db)
-                ptx::tma_load_2d(qs + db * (T5_ROWS * 128), &qmap, qfull, db * 64, b * nrows + row0, pol);
-            for (; first < T5_STAGES && first < nb; ++first) {
-                load_half(false, first);
-                load_half(true, first);
+            if (!is_v) {
+                ptx::mbar_expect_tx(qfull, (uint32_t)L::QBYTES);
+                for (int db = 0; db < NDB; ++db)
+                    ptx::tma_load_2d(qs + db * (T5_ROWS * 128), &qmap, qfull, db * 64, b * nrows + row0, pol);
             }
-            // Refills in the order the MMA thread frees them (S_0, S_1, P_0 V_0, S_2, P_1 V_1, ...):
-            // K of block j once S_{j-2} is done, then V of block j-1 once P_{j-3} V_{j-3} is done.
-            for (int j = T5_STAGES; j <= nb; ++j) {
-                if (j < nb) {
-                    if (!ptx::mbar_wait_bounded(&kempty[j % T5_STAGES], ((j - 2) >> 1) & 1, T5_WAIT_NS)) {
-                        *flag = DEV_TIMEOUT_WEIGHTS;
-                        break;
-                    }
-                    load_half(false, j);
+            for (; first < T5_STAGES && first < nb; ++first) load(first);
+            // Block j once the MMAs that read block j - 2 (S_{j-2}, or P_{j-2} V_{j-2}) are done.
+            for (int j = T5_STAGES; j < nb; ++j) {
+                if (!ptx::mbar_wait_bounded(&emptyb[j % T5_STAGES], ((j - 2) >> 1) & 1, T5_WAIT_NS)) {
+                    *flag = DEV_TIMEOUT_WEIGHTS;
+                    break;
                 }
-                const int jv = j - 1;
-                if (jv >= T5_STAGES && jv < nb) {
-                    if (!ptx::mbar_wait_bounded(&vempty[jv % T5_STAGES], ((jv - 2) >> 1) & 1, T5_WAIT_NS)) {
-                        *flag = DEV_TIMEOUT_WEIGHTS;
-                        break;
-                    }
-                    load_half(true, jv);
-                }
+                load(j);
             }
         }
-    } else if (warp == 1) {
+    } else if (warp == 2) {
         if (lane == 0) {
-            const uint32_t qb = ptx::smem_u32(qs), sb = ptx::smem_u32(stages), pb = ptx::smem_u32(ps);
+            const uint32_t qb = ptx::smem_u32(qs), sb = ptx::smem_u32(stages);
             bool good = ptx::mbar_wait_bounded(qfull, 0, T5_WAIT_NS);
             // S_i = Q K_i^T into score buffer i mod 2; K slot i mod 2 is released when it is done.
             auto issue_s = [&](int i) {
@@ -203,10 +193,20 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                 ptx::mma_commit(&sfull[i & 1]);
                 if (i + T5_STAGES < nb) ptx::mma_commit(&kempty[sl]);
             };
-            // Issue order S_0, S_1, then P_i V_i as soon as P_i is written, followed by S_{i+2}
-            // (its score buffer was read by the softmax of block i): P V never waits for a copy.
             issue_s(0);
             if (nb > 1) issue_s(1);
+            // S_{i+2} once P_i is written: the softmax of block i has read score buffer i mod 2.
+            for (int i = 0; i + 2 < nb; ++i) {
+                if (!ptx::mbar_wait_bounded(&pfull[i & 1], (i >> 1) & 1, T5_WAIT_NS)) good = false;
+                ptx::tc_fence_after();
+                issue_s(i + 2);
+            }
+            if (!good) *flag = DEV_TIMEOUT_MMA;
+        }
+    } else if (warp == 3) {
+        if (lane == 0) {
+            const uint32_t sb = ptx::smem_u32(stages), pb = ptx::smem_u32(ps);
+            bool good = true;
             for (int i = 0; i < nb; ++i) {
                 const int sl = i % T5_STAGES;
                 if (!ptx::mbar_wait_bounded(&pfull[i & 1], (i >> 1) & 1, T5_WAIT_NS)) good = false;
@@ -223,7 +223,6 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                 }
                 if (i + T5_STAGES < nb) ptx::mma_commit(&vempty[sl]);
                 ptx::mma_commit(&odone[i & 1]);
-                if (i + 2 < nb) issue_s(i + 2);
             }
             if (!good) *flag = DEV_TIMEOUT_MMA;
         }
