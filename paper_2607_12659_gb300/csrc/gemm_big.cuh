@@ -2,7 +2,9 @@
 // namespace), used when a launch has enough tokens to fill the GPU without splitting K.
 //
 // Output tile = one 128-row weight tile x one 128-row operand tile (128 tokens, or for the
-// RMSNorm-fed kinds two 64-row tiles of 63 tokens + one beta row) over the whole K range.
+// RMSNorm-fed kinds two 64-row tiles of 63 tokens + one beta row) over the whole K range. At
+// large batch these projections are bound by the rate at which one SM takes operands in from
+// L2 (87-100 GB/s measured per SM), not by the MMAs.
 // Persistent: one CTA per SM walks the tiles u = blockIdx.x, + gridDim.x, ... (weight tile
 // fastest), and its roles overlap consecutive tiles:
 //   warp 0  one thread streams (weight block, operand block) pairs by bulk tensor copies into a
@@ -11,12 +13,18 @@
 //           into one of two TMEM accumulators (tile j into buffer j mod 2, once the epilogue has
 //           read tile j - 2 out of it) and releases each stage through tcgen05.commit;
 //   warps 2-9  the epilogue, two groups of four warps (group g takes accumulator columns
-//           64g..64g+63): one TMEM lane (weight row) per thread copies its half row to a
-//           shared fp32 staging tile, hands the TMEM buffer back, then runs the per-kind
-//           epilogue (rotary + scatter, GeGLU, gated residual with the next norm's operand and
-//           sums of squares) while the MMAs of the next tile run. Row pairs (p, p + 64) meet
-//           through the staging tile; residual rows and rotary factors are loaded in chunks of
-//           16 columns (each chunk's loads issued together, the next chunk's in flight).
+//           64g..64g+63, one TMEM lane = weight row per thread). Every global input of a tile
+//           (residual rows, rotary factors, the norm's sums of squares) is fetched before the
+//           accumulator is waited for, all loads in flight together, so their latency hides
+//           behind the MMAs (fetched in dependent chunks after it, it made the epilogue as long
+//           as the tile's operand stream); one thread waits for the accumulator and the others
+//           at a named barrier. Residual kinds copy the residual rows of the tile into a shared fp32
+//           tile [token][feature] with 16-byte async copies, add their accumulator rows into it,
+//           then write the new residual, the next norm's operand and each token's sum of squares
+//           a token row per warp instruction (16 / 8 bytes per lane). The RMSNorm-fed kinds copy
+//           their accumulator to a shared staging tile [row][token] where the row pairs
+//           (p, p + 64) of rotary / GeGLU meet. After the read-out the TMEM buffer goes back to
+//           the MMA thread.
 // The next kernel is released once this CTA's last accumulator is complete. All waits are
 // bounded.
 
@@ -26,8 +34,9 @@ constexpr int BIG_EPI = 256;                     // epilogue threads: two groups
 constexpr int BIG_THREADS = 64 + BIG_EPI;
 constexpr int BIG_XBYTES = BIG_NT * KBLK * 2;     // 16 KB operand block
 constexpr int BIG_STAGE_BYTES = TILE_BYTES + BIG_XBYTES;
-constexpr int BIG_YS = BIG_NT + 1;                // fp32 staging row stride: conflict-free rows and columns
-constexpr int BIG_YBYTES = TILE_ROWS * BIG_YS * 4;
+constexpr int BIG_YS = BIG_NT + 1;                // [row][token] staging stride: conflict-free rows and columns
+constexpr int BIG_HS = BIG_NT + 4;                // [token][feature] residual stride: 16-byte rows
+constexpr int BIG_YBYTES = BIG_NT * BIG_HS * 4;   // room for either layout
 
 __host__ __device__ constexpr int big_smem_bytes() {
     // stages | staging tile | rinv[128] | bars (full, empty, acc full[2], acc empty[2]) + TMEM slot + flag
@@ -45,8 +54,8 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (ptx::smem_u32(smem_raw) & 1023u)) & 1023u);
     uint8_t* stages = smem;                                             // [stage][W 16 KB | X 16 KB]
-    float* ystage = (float*)(smem + BIG_STAGES * BIG_STAGE_BYTES);      // [128][BIG_YS]
-    float* rinv_s = (float*)((uint8_t*)ystage + BIG_YBYTES);            // [128]
+    float* ystage = (float*)(smem + BIG_STAGES * BIG_STAGE_BYTES);      // staging tile
+    float* rinv_s = (float*)((uint8_t*)ystage + BIG_YBYTES);            // [128] column scales (norm-fed kinds)
     uint64_t* full = (uint64_t*)(rinv_s + BIG_NT);
     uint64_t* empty = full + BIG_STAGES;
     uint64_t* accf = empty + BIG_STAGES;   // [2] accumulator buffer holds a finished tile
@@ -66,7 +75,10 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
         ptx::tmem_relinquish();
     }
     if (tid == 0) {
-        for (int i = 0; i < 2 * BIG_STAGES; ++i) ptx::mbar_init(&full[i], 1);
+        for (int i = 0; i < BIG_STAGES; ++i) {
+            ptx::mbar_init(&full[i], 1);
+            ptx::mbar_init(&empty[i], 1);
+        }
         ptx::mbar_init(&accf[0], 1);
         ptx::mbar_init(&accf[1], 1);
         ptx::mbar_init(&acce[0], BIG_EPI);
@@ -96,7 +108,7 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
             const int npre = u0 < total ? (nkb < BIG_STAGES ? nkb : BIG_STAGES) : 0;
             for (int kb = 0; kb < npre; ++kb) load_w(u0 % ntiles, kb, kb);
             ptx::grid_dep_wait();
-            int it = 0;   // k-block counter over this CTA's tiles: stage it mod STAGES
+            int it = 0;   // k-block counter over this CTA's tiles: stage it mod BIG_STAGES
             bool ok = true;
             for (int u = u0; u < total && ok; u += du) {
                 const int tile = u % ntiles, xt = u / ntiles;
@@ -146,27 +158,55 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
             if (!good) *flag = DEV_TIMEOUT_MMA;
         }
     } else {
-        // ---- epilogue: thread et = TMEM lane (weight row) of the accumulator ----
+        // ---- epilogue: TMEM lane `row` (weight row) of the accumulator per thread ----
         const int et = (tid - 64) & 127, eg = (tid - 64) >> 7;   // thread within its group, group
         const int row = (warp & 3) * 32 + lane;
         ptx::grid_dep_wait();
-        // Pair / token-half of this thread in the norm-fed epilogues.
+        // Norm-fed kinds: thread (pair p, token half h) of the staging tile, tokens j_lo.. of the half.
         const int p = et & 63, h = et >> 6;
+        const int j_lo = 32 * eg, nj = eg ? XS_TOKENS - 32 : 32;
         bool ok = true;
+        // A tile's global inputs, all loads in flight together: the residual rows of the tile's
+        // tokens (residual kinds: epilogue warp ew copies tokens 16 ew.. into the shared tile
+        // [token][feature], 16 bytes per lane), or the rotary factors of this thread's tokens (QKV).
+        const int ew = (tid - 64) >> 5;
+        float2 cs[32];
+        float gam = 0.f;
+        float4 sg4 = make_float4(0.f, 0.f, 0.f, 0.f);   // next norm's scale of features 4 lane..
+        auto fetch = [&](int tile, int tok0) {
+            if constexpr (!NORM_IN) {
+                const int f0 = tile * TILE_ROWS;
+                gam = a.gamma[f0 + row];
+                if (a.xs) sg4 = *(const float4*)(a.sigma_next + f0 + 4 * lane);
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    const int c = 16 * ew + k, t = tok0 + c;
+                    const bool in = t < a.Mt;
+                    ptx::cp_async_16(ptx::smem_u32(ystage + c * BIG_HS + 4 * lane),
+                                     a.hres + (in ? (size_t)t * a.W + f0 + 4 * lane : 0), in);
+                }
+            } else if constexpr (KIND == G_QKV) {
+                const int hd = a.D >> 1;
+                const int pair = tile * 64 + p;
+                const int sec = pair / hd, d = pair - sec * hd;
+                const bool rot = a.rope && sec <= a.H;
+                const int tfirst = tok0 + h * XS_TOKENS + j_lo;
+                int ql = tfirst % a.S;   // position of the token in its request
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const bool in = rot && i < nj && tfirst + i < a.Mt;
+                    cs[i] = in ? __ldg(a.rope + (size_t)(a.P + ql) * hd + d) : make_float2(1.f, 0.f);
+                    if (++ql == a.S) ql = 0;
+                }
+            }
+        };
         for (int u = u0, j = 0; u < total; u += du, ++j) {
             const int buf = j & 1;
             const int tile = u % ntiles, xt = u / ntiles;
             const int tok0 = xt * TT;
-            const int pair = tile * 64 + p;
-            int sec = 0, d = 0;
-            if (KIND == G_QKV) {
-                const int hd = a.D >> 1;
-                sec = pair / hd;
-                d = pair - sec * hd;
-            }
             if (NORM_IN && eg == 0) {
-                // Column scale: rinv of the column's token (sums of squares in slot order), 1 for
-                // the beta columns 63 and 127.
+                // Column scale: rinv of the column's token from the sums of squares (added in slot
+                // order, loaded 8 at a time), 1 for the beta columns 63 and 127.
                 const int c = et;
                 const int t = tok0 + (c >> 6) * XS_TOKENS + (c & 63);
                 float r = 1.f;
@@ -174,76 +214,72 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
                     r = 0.f;
                     if (t < a.Mt) {
                         float s = 0.f;
-                        for (int sl = 0; sl < a.nslot; ++sl) s += a.ss[(size_t)sl * a.ss_ld + t];
+                        for (int s0 = 0; s0 < a.nslot; s0 += 8) {
+                            float v[8];
+#pragma unroll
+                            for (int k = 0; k < 8; ++k)
+                                v[k] = s0 + k < a.nslot ? a.ss[(size_t)(s0 + k) * a.ss_ld + t] : 0.f;
+#pragma unroll
+                            for (int k = 0; k < 8; ++k) s += v[k];
+                        }
                         r = rsqrtf(s * a.inv_w + a.eps);
                     }
                 }
                 rinv_s[c] = r;
             }
-            if (!ptx::mbar_wait_bounded(&accf[buf], (j >> 1) & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
-            ptx::named_bar_sync(1, BIG_EPI);   // rinv_s published; every epilogue thread saw the MMAs done
+            fetch(tile, tok0);
+            if (!NORM_IN) ptx::cp_async_wait_all();
+            if (tid == 64 && !ptx::mbar_wait_bounded(&accf[buf], (j >> 1) & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
+            // rinv or the residual rows published; the MMAs of the tile are done.
+            ptx::named_bar_sync(1, BIG_EPI);
             ptx::tc_fence_after();
             // This CTA's last accumulator is complete: the next kernel may start streaming its weights.
             if (u + du >= total) ptx::grid_dep_launch();
             ok = ok && *flag == 0;
-
-            const uint32_t lane_base = tmem + (uint32_t)(buf * BIG_NT) + ((uint32_t)((warp & 3) * 32) << 16);
-            // Accumulator row -> staging row (NORM_IN: y = rinv * acc + W beta of the column's
-            // 64-group), then the TMEM buffer goes back to the MMA thread.
-            float beta = 0.f;   // W beta of this group's 64 columns (column 64 eg + 63)
-            if (NORM_IN) {
-                uint32_t r0[16];
-                ptx::tmem_ld_x16(lane_base + (uint32_t)(64 * eg + 48), r0);
-                ptx::tmem_ld_wait();
-                beta = __uint_as_float(r0[15]);
-            }
-#pragma unroll
-            for (int c0 = 64 * eg; c0 < 64 * eg + 64; c0 += 32) {
-                uint32_t r[2][16];
-                ptx::tmem_ld_x16(lane_base + (uint32_t)c0, r[0]);
-                ptx::tmem_ld_x16(lane_base + (uint32_t)(c0 + 16), r[1]);
-                ptx::tmem_ld_wait();
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh)
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int c = c0 + 16 * hh + i;
-                        const float v = __uint_as_float(r[hh][i]);
-                        ystage[row * BIG_YS + c] =
-                            !NORM_IN ? v : (c & 63) == 63 ? 0.f : rinv_s[c] * v + beta;
+            {
+                const uint32_t lane_base = tmem + (uint32_t)(buf * BIG_NT) + ((uint32_t)((warp & 3) * 32) << 16);
+                if constexpr (NORM_IN) {
+                    // Accumulator row -> staging row: y = rinv * acc + W beta of the column's
+                    // 64-group (column 64 eg + 63 holds W beta).
+                    float beta;
+                    {
+                        uint32_t r0[16];
+                        ptx::tmem_ld_x16(lane_base + (uint32_t)(64 * eg + 48), r0);
+                        ptx::tmem_ld_wait();
+                        beta = __uint_as_float(r0[15]);
                     }
-            }
-            ptx::tc_fence_before();
-            ptx::mbar_arrive(&acce[buf]);
-
-            if (NORM_IN) {
-                ptx::named_bar_sync(1, BIG_EPI);   // staging rows of the pair partners written
-                // Thread (pair p, column half h): rows p and p + 64 of this tile for 63 tokens, in
-                // chunks of 16 tokens whose rotary factors are loaded together.
-                const int j_lo = 32 * eg, j_hi = eg ? XS_TOKENS : 32;   // this group's tokens
-                const int tfirst = tok0 + h * XS_TOKENS + j_lo;
-                int qb = tfirst / a.S, qi = tfirst - qb * a.S;   // request and position of the token
-                const bool rot = KIND == G_QKV && a.rope && sec <= a.H;
-                // Rotary factors of tokens j0..j0+15, loaded together; position ql advances with j.
-                int ql = qi;
-                auto load_cs = [&](int j0, float2 (&dst)[16]) {
-                    const int hd = a.D >> 1;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const bool in = rot && j0 + i < j_hi - j_lo && tfirst + j0 + i < a.Mt;
-                        dst[i] = in ? __ldg(a.rope + (size_t)(a.P + ql) * hd + d) : make_float2(1.f, 0.f);
-                        if (++ql == a.S) ql = 0;
+                    for (int c0 = 64 * eg; c0 < 64 * eg + 64; c0 += 32) {
+                        uint32_t r[2][16];
+                        ptx::tmem_ld_x16(lane_base + (uint32_t)c0, r[0]);
+                        ptx::tmem_ld_x16(lane_base + (uint32_t)(c0 + 16), r[1]);
+                        ptx::tmem_ld_wait();
+#pragma unroll
+                        for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                const int c = c0 + 16 * hh + i;
+                                const float v = __uint_as_float(r[hh][i]);
+                                ystage[row * BIG_YS + c] = (c & 63) == 63 ? 0.f : rinv_s[c] * v + beta;
+                            }
                     }
-                };
-                float2 cs[16];
-                load_cs(0, cs);
-                for (int j0 = 0; j0 < j_hi - j_lo; j0 += 16) {
-                    float2 cn[16];
-                    if (j0 + 16 < j_hi - j_lo) load_cs(j0 + 16, cn);   // the next chunk's factors in flight
+                    ptx::tc_fence_before();
+                    ptx::mbar_arrive(&acce[buf]);
+                    ptx::named_bar_sync(1, BIG_EPI);   // staging rows of the pair partners written
+                    // Rows p and p + 64 of this tile for this thread's tokens of half h.
+                    const int pair = tile * 64 + p;
+                    int sec = 0, d = 0;
+                    if (KIND == G_QKV) {
+                        const int hd = a.D >> 1;
+                        sec = pair / hd;
+                        d = pair - sec * hd;
+                    }
+                    const bool rot = KIND == G_QKV && a.rope && sec <= a.H;
+                    const int tfirst = tok0 + h * XS_TOKENS + j_lo;
+                    int qb = tfirst / a.S, qi = tfirst - qb * a.S;   // request and position of the token
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int jj = j0 + i;
-                        if (jj >= j_hi - j_lo) break;
+                    for (int jj = 0; jj < 32; ++jj) {
+                        if (jj >= nj) break;
                         const int t = tfirst + jj;
                         const int b = qb, ii = qi;
                         if (++qi == a.S) {
@@ -257,8 +293,8 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
                             const int hd = a.D >> 1;
                             float r1 = u1, r2 = u2;
                             if (rot) {
-                                r1 = u1 * cs[i].x - u2 * cs[i].y;
-                                r2 = u2 * cs[i].x + u1 * cs[i].y;
+                                r1 = u1 * cs[jj].x - u2 * cs[jj].y;
+                                r2 = u2 * cs[jj].x + u1 * cs[jj].y;
                             }
                             __nv_bfloat16* dst = (sec < a.H) ? a.q + ((size_t)t * a.H + sec) * a.D
                                                              : (sec == a.H ? a.kst : a.vst) + ((size_t)b * a.kv_rows + a.P + ii) * a.D;
@@ -268,61 +304,56 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
                             a.z[(size_t)t * a.F + pair] = __float2bfloat16_rn(gelu_tanh(u1) * u2);
                         }
                     }
+                } else {
+                    const int f0 = tile * TILE_ROWS, f = f0 + row;
+                    // n = h + gamma * y in place of h: accumulator row `row` (feature f), 32 token
+                    // columns at a time, into column f of the [token][feature] tile.
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) cs[i] = cn[i];
-                }
-            } else {
-                const int f = tile * TILE_ROWS + row;
-                const float g = a.gamma[f];
-                const float sn = a.xs ? a.sigma_next[f] : 0.f;
-                // 16 columns at a time; the next chunk's residual values are loaded (together)
-                // before this chunk is updated, so their latency overlaps the updates.
-                float hv[16];
-                auto load_h = [&](int c0, float (&dst)[16]) {
+                    for (int c0 = 0; c0 < 64; c0 += 32) {
+                        uint32_t r[2][16];
+                        ptx::tmem_ld_x16(lane_base + (uint32_t)(64 * eg + c0), r[0]);
+                        ptx::tmem_ld_x16(lane_base + (uint32_t)(64 * eg + c0 + 16), r[1]);
+                        ptx::tmem_ld_wait();
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int t = tok0 + c0 + i;
-                        dst[i] = t < a.Mt ? a.hres[(size_t)t * a.W + f] : 0.f;
-                    }
-                };
-                const int cb = 64 * eg, ce = cb + 64;   // this group's columns
-                load_h(cb, hv);
-#pragma unroll 1
-                for (int c0 = cb; c0 < ce; c0 += 16) {
-                    float hn[16];
-                    if (c0 + 16 < ce) load_h(c0 + 16, hn);
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int c = c0 + i, t = tok0 + c;
-                        float sq = 0.f;
-                        if (t < a.Mt && ok) {
-                            const float n = hv[i] + g * ystage[row * BIG_YS + c];
-                            a.hres[(size_t)t * a.W + f] = n;
-                            if (a.xs) a.xs[(size_t)xs_row(t) * a.W + f] = __float2bfloat16_rn((1.f + sn) * n);
-                            sq = n * n;
+                        for (int i = 0; i < 32; ++i) {
+                            float* hp = ystage + (64 * eg + c0 + i) * BIG_HS + row;
+                            *hp = *hp + gam * __uint_as_float(r[i >> 4][i & 15]);
                         }
-                        ystage[row * BIG_YS + c] = sq;
                     }
+                    ptx::tc_fence_before();
+                    ptx::mbar_arrive(&acce[buf]);
+                    // The next norm's shift in the last row of each of its token tiles (this tile's rows).
+                    if (a.xs && xt == 0 && ok && eg == 0) {
+                        const float bn = a.beta_next[f];
+                        for (int x = 0; x < xs_tiles(a.Mt); ++x)
+                            a.xs[((size_t)x * 64 + 63) * a.W + f] = __float2bfloat16_rn(bn);
+                    }
+                    ptx::named_bar_sync(1, BIG_EPI);   // the tile's new residual rows are complete
+                    // Warp ew writes tokens 16 ew..: lane l the features 4 l..4 l + 3 of the new
+                    // residual (16 bytes) and of the next norm's operand (8 bytes); the token's sum of
+                    // squares over the tile's 128 features is lane 0's butterfly total (slot `tile`).
+                    // (A timeout flag may be seen by some lanes only: the warp decides together.)
+                    const bool okw = __all_sync(0xffffffffu, ok);
+#pragma unroll 4
+                    for (int k = 0; k < 16; ++k) {
+                        const int c = 16 * ew + k, t = tok0 + c;
+                        if (t >= a.Mt || !okw) break;
+                        const float4 n = *(const float4*)(ystage + c * BIG_HS + 4 * lane);
+                        *(float4*)(a.hres + (size_t)t * a.W + f0 + 4 * lane) = n;
+                        if (a.xs) {
+                            const uint2 v = make_uint2(pack_bf16x2((1.f + sg4.x) * n.x, (1.f + sg4.y) * n.y),
+                                                       pack_bf16x2((1.f + sg4.z) * n.z, (1.f + sg4.w) * n.w));
+                            *(uint2*)(a.xs + (size_t)xs_row(t) * a.W + f0 + 4 * lane) = v;
+                        }
+                        float sq = ((n.x * n.x + n.y * n.y) + n.z * n.z) + n.w * n.w;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) hv[i] = hn[i];
+                        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+                        if (lane == 0) a.ss_out[(size_t)tile * a.ss_ld + t] = sq;
+                    }
                 }
-                // The next norm's shift in the last row of each of its token tiles (this tile's rows).
-                if (a.xs && xt == 0 && ok && eg == 0) {
-                    const float bn = a.beta_next[f];
-                    for (int x = 0; x < xs_tiles(a.Mt); ++x)
-                        a.xs[((size_t)x * 64 + 63) * a.W + f] = __float2bfloat16_rn(bn);
-                }
+                // Every epilogue thread is done with the staging tile (and rinv) of this tile.
                 ptx::named_bar_sync(1, BIG_EPI);
-                // Sum of squares of token c over this tile's 128 features, in row order: slot `tile`.
-                const int c = et, t = tok0 + c;
-                if (eg == 0 && t < a.Mt && ok) {
-                    float s = 0.f;
-                    for (int r = 0; r < TILE_ROWS; ++r) s += ystage[r * BIG_YS + c];
-                    a.ss_out[(size_t)tile * a.ss_ld + t] = s;
-                }
             }
-            // Every epilogue thread is done with the staging tile and rinv_s of this tile.
-            ptx::named_bar_sync(1, BIG_EPI);
         }
     }
 

@@ -80,6 +80,17 @@ __device__ __forceinline__ void tma_load_2d_plain(void* dst, const void* tmap, u
 __device__ __forceinline__ void prefetch_tmap(const void* tmap) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
 }
+// Per-thread asynchronous copy of 16 bytes global -> shared (both 16-byte aligned), not cached in
+// L1, zero-filled (nothing read) when !valid; cp_async_wait_all() waits for every such copy of
+// the calling thread.
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
 // Generic-proxy writes to shared memory become visible to the async proxy (tensor cores).
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

@@ -10,7 +10,7 @@ import numpy as np
 import pytest
 
 import oracle
-from synth import PI05, TINY, make_requests, make_weights
+from synth import PI05, TINY, ExpertConfig, make_requests, make_weights
 from tests.gpu_util import (SMALL_BF16, assert_close, errors, gpu_denoise, lib, make_expert,
                             oracle_denoise, to_dev_kv)
 
@@ -188,6 +188,25 @@ def test_small_bf16_large_m_projection_path(large_m_everywhere, B, P, C, N):
         got = gpu_denoise(ex, SMALL_BF16, r, N)
         assert_close(got, oracle_denoise(SMALL_BF16, oracle.to_f64(w), r, N), SMALL_BF16,
                      f"small bf16 large-M B{B} P{P} C{C} N{N}")
+    finally:
+        ex.close()
+
+
+# One head of 128: the QKV projection has an odd number of weight tiles (3), and a single
+# 128-row weight tile carries both halves of the head's rotary pairs.
+SMALL_ONE_HEAD = ExpertConfig(n_layers=2, width=256, n_heads=1, head_dim=128, mlp_dim=512,
+                              action_dim=7, state_dim=7, time_dim=64, precision="bf16")
+
+
+@pytest.mark.parametrize("B,P,C", [(2, 100, 50), (5, 64, 31)])
+def test_odd_weight_tile_count_large_m_path(large_m_everywhere, B, P, C):
+    w = make_weights(SMALL_ONE_HEAD, 2250)
+    ex = make_expert(SMALL_ONE_HEAD, w, max_batch=B, max_prefix=P, max_chunk=C, max_steps=2)
+    try:
+        r = make_requests(SMALL_ONE_HEAD, 2251 + B, B, P, C)
+        got = gpu_denoise(ex, SMALL_ONE_HEAD, r, 2)
+        assert_close(got, oracle_denoise(SMALL_ONE_HEAD, oracle.to_f64(w), r, 2), SMALL_ONE_HEAD,
+                     f"one-head large-M B{B} P{P} C{C}")
     finally:
         ex.close()
 
