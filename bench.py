@@ -588,8 +588,9 @@ def profile_forward(args):
 
 
 def primitives_arm():
-    """The hardware-primitive costs that bound the batch-1 chain (csrc/probe/primitives.cu): one
-    JSON line (a diagnostic, not a bench line)."""
+    """The hardware-primitive costs that bound the denoise (csrc/probe/primitives.cu): hand-offs
+    behind the batch-1 chain, per-SM operand intake behind large batches. One JSON line (a
+    diagnostic, not a bench line)."""
     from paper_2607_12659_gb300 import build
     binary = build.build_probe()
     r = subprocess.run([binary], capture_output=True, text=True, timeout=300)
@@ -597,7 +598,7 @@ def primitives_arm():
     if r.returncode != 0 or not lines:
         raise SystemExit(f"primitives probe failed ({r.returncode}): {r.stdout[-400:]} {r.stderr[-400:]}")
     out = json.loads(lines[-1])
-    print(json.dumps({"metric": "GB300 primitive costs behind the batch-1 chain (diagnostic)",
+    print(json.dumps({"metric": "GB300 primitive costs behind the denoise (diagnostic)",
                       "primitives": out, "clocks_note": "not sampled; durations are medians of short loops"}),
           flush=True)
 

@@ -1,16 +1,27 @@
-// Costs of the hardware primitives that bound the batch-1 denoise on this GPU, measured directly
-// (a diagnostic executable, not part of the library; `python bench.py --primitives` builds and
-// runs it and prints its JSON line).
+// Costs of the hardware primitives that bound the denoise on this GPU, measured directly (a
+// diagnostic executable, not part of the library; `python bench.py --primitives` builds and runs
+// it and prints its JSON line).
 //
 // At batch 1 every expert layer is a chain of five stages that each need all of the previous
 // stage's output, so the denoise time is set by what it costs to hand data from one set of SMs to
-// another and to run a short chain of tensor-core work, not by HBM. Measured here:
+// another and to run a short chain of tensor-core work, not by HBM. At large batch the
+// projections and attention are bound by the rate at which an SM takes operands in. Measured here:
 //   handoff_flag_us     one SM releases a flag in global memory, another SM polls it with acquire
 //                       loads and answers; half the round trip (several SM pairs, median)
 //   handoff_8kb_us      the same with 8 KB written before the flag and read after it
 //   grid_barrier_us     all co-resident CTAs arrive on one counter and poll it (one CTA per SM)
 //   l2_reduce_us        every CTA adds a 32 KB fp32 partial into L2 with red.add (20 targets)
 //   l2_bulk_load_us     one CTA's 8 KB bulk copy of L2-resident data into its shared memory
+//   stream_gbs          rate at which one CTA per SM takes data in by bulk copies (4 x 16 KB in
+//                       flight), from a 32 MB L2-resident buffer with 1, 8, 38, 76 and 152 CTAs
+//                       streaming at once (median per CTA), and from a 1 GB buffer (HBM) with 152;
+//                       then with 8 and 12 copies in flight (1 and 152 CTAs, L2); then per-thread
+//                       16-byte async copies (cp.async, 256 threads, 4 x 16 KB rounds in flight),
+//                       and both at once in one CTA (a bulk-copy thread and 256 cp.async threads);
+//                       then clusters of 2 and 4 where every CTA fetches 1/2 or 1/4 of each chunk
+//                       with a multicast bulk copy into all CTAs of its cluster (bytes received per
+//                       CTA: whole chunks; 12 chunks per epoch, a cluster barrier between epochs,
+//                       and the same epochs without multicast as the control)
 //   mma_cycles          tcgen05.mma issued back to back by one thread (64 in a row, and 4)
 //   dsmem_ring_us       4 KB pushed around a ring of 8 CTAs of a cluster, with a cluster barrier
 //   coresident_ctas     CTAs of 200 KB shared memory co-resident per cluster size, and whether a
@@ -139,6 +150,161 @@ __global__ void k_bulk_load(const uint8_t* src, int reps, unsigned long long* ou
     }
 }
 
+// One thread per CTA streams `reps` 16 KB bulk copies, NS in flight, from chunks of `src`
+// (`nchunks` of them; CTA b starts at chunk b * stride) into an NS-slot ring; out[blockIdx.x] =
+// elapsed ns.
+template <int NS>
+__global__ void k_stream(const uint8_t* src, int nchunks, int stride, int reps, unsigned long long* out,
+                         int* err) {
+    extern __shared__ __align__(128) uint8_t sm[];
+    __shared__ __align__(8) uint64_t bar[NS];
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < NS; ++i) ptx::mbar_init(&bar[i], 1);
+        ptx::fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    const uint64_t t0 = ptx::globaltimer_ns();
+    bool ok = true;
+    for (int r = 0; r < reps && ok; ++r) {
+        const int s = r % NS;
+        if (r >= NS && !ptx::mbar_wait_bounded(&bar[s], ((r - NS) / NS) & 1, LIMIT_NS)) {
+            atomicExch(err, 7);
+            ok = false;
+            break;
+        }
+        ptx::mbar_expect_tx(&bar[s], 16384);
+        const size_t chunk = ((size_t)blockIdx.x * stride + r) % nchunks;
+        asm volatile(
+            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                ptx::smem_u32(sm + s * 16384)),
+            "l"(src + chunk * 16384), "r"(16384), "r"(ptx::smem_u32(&bar[s]))
+            : "memory");
+    }
+    // The last copies have landed before the CTA exits.
+    for (int r = reps - NS < 0 ? 0 : reps - NS; r < reps; ++r)
+        if (!ptx::mbar_wait_bounded(&bar[r % NS], (r / NS) & 1, LIMIT_NS)) atomicExch(err, 8);
+    out[blockIdx.x] = ptx::globaltimer_ns() - t0;
+}
+
+// Warps 1..8 of the CTA stream `reps` rounds of 16 KB with per-thread 16-byte async copies
+// (thread k copies bytes 64 k..64 k + 63 of a round), 4 rounds in flight, into a 64 KB ring at
+// sm + ring_off; with `bulk` set, thread 0 meanwhile streams `reps` 16 KB bulk copies into
+// sm[0, 64 KB) as k_stream<4> does. out[blockIdx.x] = elapsed ns of the slower of the two.
+__global__ void k_stream_lsu(const uint8_t* src, int nchunks, int stride, int reps, int bulk,
+                             unsigned long long* out, int* err) {
+    extern __shared__ __align__(128) uint8_t sm[];
+    __shared__ __align__(8) uint64_t bar[4];
+    __shared__ unsigned long long t_end[2];
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 4; ++i) ptx::mbar_init(&bar[i], 1);
+        ptx::fence_mbar_init();
+        t_end[0] = t_end[1] = 0;
+    }
+    __syncthreads();
+    const uint64_t t0 = ptx::globaltimer_ns();
+    if (threadIdx.x < 32) {
+        if (threadIdx.x == 0 && bulk) {
+            bool ok = true;
+            for (int r = 0; r < reps && ok; ++r) {
+                const int s = r & 3;
+                if (r >= 4 && !ptx::mbar_wait_bounded(&bar[s], ((r - 4) >> 2) & 1, LIMIT_NS)) {
+                    atomicExch(err, 9);
+                    ok = false;
+                    break;
+                }
+                ptx::mbar_expect_tx(&bar[s], 16384);
+                const size_t chunk = ((size_t)blockIdx.x * stride + r) % nchunks;
+                asm volatile(
+                    "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                        ptx::smem_u32(sm + s * 16384)),
+                    "l"(src + chunk * 16384), "r"(16384), "r"(ptx::smem_u32(&bar[s]))
+                    : "memory");
+            }
+            for (int r = reps - 4 < 0 ? 0 : reps - 4; r < reps; ++r)
+                if (!ptx::mbar_wait_bounded(&bar[r & 3], (r >> 2) & 1, LIMIT_NS)) atomicExch(err, 10);
+            t_end[0] = ptx::globaltimer_ns() - t0;
+        }
+    } else {
+        const int k = threadIdx.x - 32;   // 0..255
+        uint8_t* ring = sm + 65536;
+        for (int r = 0; r < reps; ++r) {
+            // Chunks offset from the bulk stream's, so the two do not read the same lines.
+            const size_t chunk = ((size_t)blockIdx.x * stride + r + nchunks / 2) % nchunks;
+            const uint8_t* g = src + chunk * 16384 + 64 * k;
+            const uint32_t d = ptx::smem_u32(ring + (r & 3) * 16384 + 64 * k);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) ptx::cp_async_16(d + 16 * q, g + 16 * q, true);
+            asm volatile("cp.async.commit_group;" ::: "memory");
+            asm volatile("cp.async.wait_group 3;" ::: "memory");
+        }
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        if (k == 0) t_end[1] = ptx::globaltimer_ns() - t0;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) out[blockIdx.x] = t_end[0] > t_end[1] ? t_end[0] : t_end[1];
+}
+
+// Clusters of CL CTAs (CL = 1: the same protocol without multicast), thread 0 of each, in epochs:
+// arm 12 slots of 16 KB (one arrival + 16 KB each), cluster barrier (every CTA of the cluster has
+// armed its slots and read the previous epoch's), then piece `rank` (16 KB / CL) of each of the
+// epoch's 12 chunks is fetched by a multicast bulk copy into that slot of every CTA of the
+// cluster, and each CTA waits for its 12 slots: each CTA receives 192 KB an epoch while fetching
+// 1/CL of it. Every wait is bounded; the final cluster barrier keeps each CTA alive until nothing
+// can still land in it. out[blockIdx.x] = elapsed ns.
+template <int CL>
+__global__ void k_stream_mc(const uint8_t* src, int nchunks, int stride, int epochs, unsigned long long* out,
+                            int* err) {
+    constexpr int NSLOT = 12;
+    extern __shared__ __align__(128) uint8_t sm[];
+    __shared__ __align__(8) uint64_t full[NSLOT];
+    const uint32_t rank = ptx::cluster_rank();
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < NSLOT; ++i) ptx::mbar_init(&full[i], 1);
+        ptx::fence_mbar_init();
+    }
+    __syncthreads();
+    const uint64_t t0 = ptx::globaltimer_ns();
+    constexpr uint32_t piece = 16384 / CL;
+    const uint16_t mask = (uint16_t)((1u << CL) - 1);
+    const size_t cluster_id = blockIdx.x / CL;
+    bool ok = true;
+    for (int e = 0; e < epochs; ++e) {
+        if (threadIdx.x == 0)
+            for (int i = 0; i < NSLOT; ++i) ptx::mbar_expect_tx(&full[i], 16384);
+        __syncwarp();
+        ptx::cluster_arrive();
+        ptx::cluster_wait();
+        if (threadIdx.x == 0) {
+            for (int i = 0; i < NSLOT; ++i) {
+                const size_t chunk = (cluster_id * stride + (size_t)e * NSLOT + i) % nchunks;
+                if (CL == 1)
+                    asm volatile(
+                        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                            ptx::smem_u32(sm + i * 16384)),
+                        "l"(src + chunk * 16384), "r"(16384), "r"(ptx::smem_u32(&full[i]))
+                        : "memory");
+                else
+                    asm volatile(
+                        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], "
+                        "[%1], %2, [%3], %4;" ::"r"(ptx::smem_u32(sm + i * 16384 + rank * piece)),
+                        "l"(src + chunk * 16384 + rank * piece), "r"(piece), "r"(ptx::smem_u32(&full[i])), "h"(mask)
+                        : "memory");
+            }
+            for (int i = 0; i < NSLOT; ++i)
+                if (ok && !ptx::mbar_wait_bounded(&full[i], e & 1, LIMIT_NS)) {
+                    atomicExch(err, 11);
+                    ok = false;
+                }
+        }
+        __syncwarp();
+    }
+    if (threadIdx.x == 0) out[blockIdx.x] = ptx::globaltimer_ns() - t0;
+    __syncwarp();
+    ptx::cluster_arrive();
+    ptx::cluster_wait();
+}
+
 // One thread issues `nmma` tcgen05.mma of 128 x N x 16 (bf16, fp32 accumulate) back to back.
 // out[0] = cycles to issue them, out[1] = cycles until their commit has arrived.
 template <int N>
@@ -248,7 +414,7 @@ int main() {
     float* d_data = nullptr;
     CK(cudaMalloc(&d_int, 4096));
     CK(cudaMalloc(&d_err, 64));
-    CK(cudaMalloc(&d_out, 64));
+    CK(cudaMalloc(&d_out, 64 * 8 * 4));
     CK(cudaMalloc(&d_data, 4 << 20));
     CK(cudaMemset(d_err, 0, 64));
     CK(cudaMemset(d_data, 0, 4 << 20));
@@ -307,6 +473,94 @@ int main() {
     CK(cudaDeviceSynchronize());
     CK(cudaMemcpy(h, d_out, 8, cudaMemcpyDeviceToHost));
     const double load_us = h[0] / 1e3 / 256;
+
+    // Streaming intake per SM: one CTA per SM (120 KB of shared memory requested, 64 KB used).
+    double stream_gbs[5], hbm_gbs = 0.0, deep_gbs[4] = {0.0, 0.0, 0.0, 0.0}, lsu_gbs[4] = {0.0, 0.0, 0.0, 0.0};
+    double mc_gbs[4] = {0.0, 0.0, 0.0, 0.0};
+    const int nstream[5] = {1, 8, 38, 76, 152};
+    {
+        uint8_t* d_l2 = nullptr;
+        uint8_t* d_hbm = nullptr;
+        const size_t l2_bytes = 32u << 20, hbm_bytes = 1ull << 30;
+        CK(cudaMalloc(&d_l2, l2_bytes));
+        CK(cudaMalloc(&d_hbm, hbm_bytes));
+        CK(cudaMemset(d_l2, 1, l2_bytes));
+        CK(cudaMemset(d_hbm, 1, hbm_bytes));
+        const int smem = 200 * 1024;   // one CTA per SM; 12 slots of 16 KB at most
+        CK(cudaFuncSetAttribute(k_stream<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+        CK(cudaFuncSetAttribute(k_stream<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+        CK(cudaFuncSetAttribute(k_stream<12>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+        std::vector<unsigned long long> t(sms);
+        auto run = [&](auto kern, const uint8_t* src, size_t bytes, int ctas, int stride, int reps) -> double {
+            for (int rep = 0; rep < 2; ++rep) {
+                kern<<<ctas, 32, smem>>>(src, (int)(bytes / 16384), stride, reps, d_out, d_err);
+                if (cudaDeviceSynchronize() != cudaSuccess) return -1.0;
+            }
+            if (cudaMemcpy(t.data(), d_out, 8 * ctas, cudaMemcpyDeviceToHost) != cudaSuccess) return -1.0;
+            std::vector<double> gbs;
+            for (int c = 0; c < ctas; ++c) gbs.push_back((double)reps * 16384 / (double)t[c]);
+            return median(gbs);
+        };
+        // L2: every CTA walks the whole 32 MB buffer from its own offset (resident after the
+        // first run); HBM: disjoint windows of 400 chunks (6.5 MB) of the 1 GB buffer per CTA.
+        for (int i = 0; i < 5; ++i)
+            stream_gbs[i] = nstream[i] <= sms ? run(k_stream<4>, d_l2, l2_bytes, nstream[i], 131, 2048) : 0.0;
+        hbm_gbs = run(k_stream<4>, d_hbm, hbm_bytes, sms, (int)(hbm_bytes / 16384 / sms), 400);
+        deep_gbs[0] = run(k_stream<8>, d_l2, l2_bytes, 1, 131, 2048);
+        deep_gbs[1] = run(k_stream<8>, d_l2, l2_bytes, sms, 131, 2048);
+        deep_gbs[2] = run(k_stream<12>, d_l2, l2_bytes, 1, 131, 2048);
+        deep_gbs[3] = run(k_stream<12>, d_l2, l2_bytes, sms, 131, 2048);
+        CK(cudaFuncSetAttribute(k_stream_lsu, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+        // Bytes per CTA: 16 KB per round for cp.async, plus 16 KB per copy for the bulk stream.
+        auto run_lsu = [&](int ctas, int bulk) -> double {
+            const int reps = 2048;
+            for (int rep = 0; rep < 2; ++rep) {
+                k_stream_lsu<<<ctas, 288, smem>>>(d_l2, (int)(l2_bytes / 16384), 131, reps, bulk, d_out, d_err);
+                if (cudaDeviceSynchronize() != cudaSuccess) return -1.0;
+            }
+            if (cudaMemcpy(t.data(), d_out, 8 * ctas, cudaMemcpyDeviceToHost) != cudaSuccess) return -1.0;
+            std::vector<double> gbs;
+            for (int c = 0; c < ctas; ++c) gbs.push_back((double)reps * 16384 * (bulk ? 2 : 1) / (double)t[c]);
+            return median(gbs);
+        };
+        lsu_gbs[0] = run_lsu(1, 0);
+        lsu_gbs[1] = run_lsu(sms, 0);
+        lsu_gbs[2] = run_lsu(1, 1);
+        lsu_gbs[3] = run_lsu(sms, 1);
+        // Multicast within clusters of 2 and 4 (and the same protocol in clusters of 1): bytes
+        // received per CTA, 192 KB an epoch.
+        auto run_mc = [&](auto kern, int cl, int ctas) -> double {
+            CK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(ctas);
+            cfg.blockDim = dim3(32);
+            cfg.dynamicSmemBytes = smem;
+            cudaLaunchAttribute at;
+            at.id = cudaLaunchAttributeClusterDimension;
+            at.val.clusterDim.x = cl;
+            at.val.clusterDim.y = 1;
+            at.val.clusterDim.z = 1;
+            cfg.attrs = &at;
+            cfg.numAttrs = 1;
+            const int epochs = 170;   // 2040 chunks of 16 KB per CTA
+            for (int rep = 0; rep < 2; ++rep) {
+                if (cudaLaunchKernelEx(&cfg, kern, (const uint8_t*)d_l2, (int)(l2_bytes / 16384), 131, epochs, d_out,
+                                       d_err) != cudaSuccess)
+                    return -1.0;
+                if (cudaDeviceSynchronize() != cudaSuccess) return -1.0;
+            }
+            if (cudaMemcpy(t.data(), d_out, 8 * ctas, cudaMemcpyDeviceToHost) != cudaSuccess) return -1.0;
+            std::vector<double> gbs;
+            for (int c = 0; c < ctas; ++c) gbs.push_back((double)epochs * 12 * 16384 / (double)t[c]);
+            return median(gbs);
+        };
+        mc_gbs[0] = run_mc(k_stream_mc<1>, 1, 152);
+        mc_gbs[1] = run_mc(k_stream_mc<2>, 2, 152);
+        mc_gbs[2] = run_mc(k_stream_mc<4>, 4, 144);
+        mc_gbs[3] = run_mc(k_stream_mc<2>, 2, 2);
+        CK(cudaFree(d_l2));
+        CK(cudaFree(d_hbm));
+    }
 
     // tcgen05.mma issue (the second of two runs, so the code is warm).
     double mma[4];
@@ -393,11 +647,19 @@ int main() {
            "\"mma_cycles\": {\"128x64x16\": %.1f, \"128x64x16_run_of_4\": %.1f, \"128x128x16\": %.1f, "
            "\"128x256x16\": %.1f}, \"dsmem_ring_us\": %.3f, "
            "\"coresident_ctas_200kb\": {\"1\": %d, \"2\": %d, \"4\": %d, \"8\": %d, \"16\": %d}, "
-           "\"cooperative_clusters_of_8\": %s, \"errors\": %d}\n",
+           "\"cooperative_clusters_of_8\": %s, \"stream_gbs_per_cta\": {\"l2_1\": %.1f, \"l2_8\": %.1f, "
+           "\"l2_38\": %.1f, \"l2_76\": %.1f, \"l2_152\": %.1f, \"hbm_152\": %.1f, \"l2_1_depth8\": %.1f, "
+           "\"l2_152_depth8\": %.1f, \"l2_1_depth12\": %.1f, \"l2_152_depth12\": %.1f, \"l2_1_cp_async\": %.1f, "
+           "\"l2_152_cp_async\": %.1f, \"l2_1_bulk_plus_cp_async\": %.1f, \"l2_152_bulk_plus_cp_async\": %.1f, "
+           "\"l2_epochs_cluster1_x152\": %.1f, \"l2_multicast_cluster2_x76\": %.1f, "
+           "\"l2_multicast_cluster4_x36\": %.1f, \"l2_multicast_cluster2_x1\": %.1f}, \"errors\": %d}\n",
            sms, median(flag_us), *std::min_element(flag_us.begin(), flag_us.end()),
            *std::max_element(flag_us.begin(), flag_us.end()), median(data_us),
            *std::min_element(data_us.begin(), data_us.end()), *std::max_element(data_us.begin(), data_us.end()),
            barrier_us, reduce_us, sms * 32768, load_us, mma[0], mma[1], mma[2], mma[3], ring_us, coresident[0],
-           coresident[1], coresident[2], coresident[3], coresident[4], coop8 ? "true" : "false", errs);
+           coresident[1], coresident[2], coresident[3], coresident[4], coop8 ? "true" : "false", stream_gbs[0],
+           stream_gbs[1], stream_gbs[2], stream_gbs[3], stream_gbs[4], hbm_gbs, deep_gbs[0], deep_gbs[1], deep_gbs[2],
+           deep_gbs[3], lsu_gbs[0], lsu_gbs[1], lsu_gbs[2], lsu_gbs[3], mc_gbs[0], mc_gbs[1], mc_gbs[2], mc_gbs[3],
+           errs);
     return 0;
 }
