@@ -16,6 +16,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdint>
@@ -74,22 +75,59 @@ __global__ void k_pf_load_x(const void* __restrict__ x, int x_fp32, float* __res
         h[i] = x_fp32 ? static_cast<const float*>(x)[i] : __bfloat162float(static_cast<const __nv_bfloat16*>(x)[i]);
 }
 
-// y = h / sqrt(mean(h^2) + eps) * (1 + w), row by row; one warp per row (grid-stride).
+// y = h / sqrt(mean(h^2) + eps) * (1 + w), row by row; one warp per row (grid-stride). A row of
+// up to RN_CAP float4 per lane is loaded into registers at once (every load in flight together,
+// one pass over memory); longer rows take a strided loop. W is a multiple of 4.
+constexpr int RN_CAP = 16;   // 2048 floats per row
 template <typename TO>
 __global__ void __launch_bounds__(256) k_pf_rmsnorm(const float* __restrict__ h, const float* __restrict__ w,
                                                     TO* __restrict__ y, long long rows, int W, float eps) {
     const int lane = threadIdx.x & 31;
     const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    const int n4 = W >> 2;
+    const float4* w4 = reinterpret_cast<const float4*>(w);
     for (long long r = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += nwarps) {
-        const float* hr = h + r * W;
-        float s = 0.f;
-        for (int i = lane; i < W; i += 32) s = fmaf(hr[i], hr[i], s);
-        const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
-        TO* yr = y + r * W;
-        for (int i = lane; i < W; i += 32) {
-            const float v = hr[i] * rinv * (1.f + w[i]);
-            if constexpr (sizeof(TO) == 2) yr[i] = __float2bfloat16_rn(v);
-            else yr[i] = v;
+        const float4* hr = reinterpret_cast<const float4*>(h + r * W);
+        auto store4 = [&](int i, float4 v, float rinv) {
+            const float4 g = w4[i];
+            const float a0 = v.x * rinv * (1.f + g.x), a1 = v.y * rinv * (1.f + g.y);
+            const float a2 = v.z * rinv * (1.f + g.z), a3 = v.w * rinv * (1.f + g.w);
+            if constexpr (sizeof(TO) == 2) {
+                const __nv_bfloat162 lo = __floats2bfloat162_rn(a0, a1), hi = __floats2bfloat162_rn(a2, a3);
+                uint2 u;
+                u.x = *reinterpret_cast<const uint32_t*>(&lo);
+                u.y = *reinterpret_cast<const uint32_t*>(&hi);
+                *reinterpret_cast<uint2*>(y + r * W + 4 * i) = u;
+            } else {
+                *reinterpret_cast<float4*>(y + r * W + 4 * i) = make_float4(a0, a1, a2, a3);
+            }
+        };
+        if (n4 <= 32 * RN_CAP) {
+            float4 v[RN_CAP];
+            float s = 0.f;
+#pragma unroll
+            for (int k = 0; k < RN_CAP; ++k) {
+                const int i = lane + 32 * k;
+                v[k] = i < n4 ? hr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int k = 0; k < RN_CAP; ++k) s += (v[k].x * v[k].x + v[k].y * v[k].y) + (v[k].z * v[k].z + v[k].w * v[k].w);
+            const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
+#pragma unroll
+            for (int k = 0; k < RN_CAP; ++k) {
+                const int i = lane + 32 * k;
+                if (i < n4) store4(i, v[k], rinv);
+            }
+        } else {
+            float s = 0.f;
+#pragma unroll 4
+            for (int i = lane; i < n4; i += 32) {
+                const float4 v = hr[i];
+                s += (v.x * v.x + v.y * v.y) + (v.z * v.z + v.w * v.w);
+            }
+            const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
+#pragma unroll 4
+            for (int i = lane; i < n4; i += 32) store4(i, hr[i], rinv);
         }
     }
 }
@@ -125,34 +163,162 @@ __global__ void k_pf_rope_scatter(const float* __restrict__ qkv, const float2* _
     }
 }
 
-// probs[r][0 .. n) = softmax(s[r][0 .. n)) as bf16 (rows of stride ld); one warp per row.
+// probs[r][0 .. n) = softmax(s[r][0 .. n)) as bf16 (rows of stride ld); one warp per row. Rows of
+// up to SM_CAP values per lane are read once into registers (all loads in flight together);
+// longer rows take three strided passes.
+constexpr int SM_CAP = 32;   // 1024 keys
 __global__ void __launch_bounds__(256) k_pf_softmax(const float* __restrict__ s, __nv_bfloat16* __restrict__ p,
                                                     long long rows, int n, int ld) {
     const int lane = threadIdx.x & 31;
     const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
     for (long long r = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += nwarps) {
         const float* sr = s + r * ld;
-        float mx = -INFINITY;
-        for (int j = lane; j < n; j += 32) mx = fmaxf(mx, sr[j]);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        float den = 0.f;
-        for (int j = lane; j < n; j += 32) den += expf(sr[j] - mx);
-        const float inv = 1.f / warp_sum(den);
         __nv_bfloat16* pr = p + r * ld;
-        for (int j = lane; j < n; j += 32) pr[j] = __float2bfloat16_rn(expf(sr[j] - mx) * inv);
+        if (n <= 32 * SM_CAP) {
+            float v[SM_CAP];
+            float mx = -INFINITY;
+#pragma unroll
+            for (int k = 0; k < SM_CAP; ++k) {
+                const int j = lane + 32 * k;
+                v[k] = j < n ? sr[j] : -INFINITY;
+            }
+#pragma unroll
+            for (int k = 0; k < SM_CAP; ++k) mx = fmaxf(mx, v[k]);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            float den = 0.f;
+#pragma unroll
+            for (int k = 0; k < SM_CAP; ++k) {
+                v[k] = lane + 32 * k < n ? expf(v[k] - mx) : 0.f;
+                den += v[k];
+            }
+            const float inv = 1.f / warp_sum(den);
+#pragma unroll
+            for (int k = 0; k < SM_CAP; ++k) {
+                const int j = lane + 32 * k;
+                if (j < n) pr[j] = __float2bfloat16_rn(v[k] * inv);
+            }
+        } else {
+            float mx = -INFINITY;
+            for (int j = lane; j < n; j += 32) mx = fmaxf(mx, sr[j]);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            float den = 0.f;
+            for (int j = lane; j < n; j += 32) den += expf(sr[j] - mx);
+            const float inv = 1.f / warp_sum(den);
+            for (int j = lane; j < n; j += 32) pr[j] = __float2bfloat16_rn(expf(sr[j] - mx) * inv);
+        }
     }
 }
 
-// z[r][j] = gelu_tanh(gu[r][j]) * gu[r][F + j] (gate rows first, then up rows, in the packed matrix).
-__global__ void k_pf_geglu(const float* __restrict__ gu, __nv_bfloat16* __restrict__ z, long long rows, int F) {
-    const long long total = rows * F;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const long long r = idx / F;
-        const int j = (int)(idx % F);
-        const float* row = gu + r * 2 * (long long)F;
-        z[idx] = __float2bfloat16_rn(gelu_tanh_f(row[j]) * row[F + j]);
+// After a product split over K ranges: h += (part_0 + part_1 + ...) in range order (parts [rows][W]
+// fp32, `pstride` elements apart), then, when w is set, the next RMSNorm y = h / sqrt(mean(h^2) +
+// eps) * (1 + w) as k_pf_rmsnorm computes it. One warp per row; a row of up to RN_CAP float4 per
+// lane stays in registers (W a multiple of 4).
+template <typename TO>
+__global__ void __launch_bounds__(256) k_pf_residual_norm(float* __restrict__ h, const float* __restrict__ parts,
+                                                          int nparts, long long pstride, const float* __restrict__ w,
+                                                          TO* __restrict__ y, long long rows, int W, float eps) {
+    const int lane = threadIdx.x & 31;
+    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    const int n4 = W >> 2;
+    const float4* w4 = reinterpret_cast<const float4*>(w);
+    for (long long r = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += nwarps) {
+        float4* hr = reinterpret_cast<float4*>(h + r * W);
+        auto update = [&](int i) {
+            float4 d = reinterpret_cast<const float4*>(parts + r * W)[i];
+            for (int q = 1; q < nparts; ++q) {
+                const float4 e = reinterpret_cast<const float4*>(parts + (size_t)q * pstride + r * W)[i];
+                d.x += e.x;
+                d.y += e.y;
+                d.z += e.z;
+                d.w += e.w;
+            }
+            float4 v = hr[i];
+            v.x += d.x;
+            v.y += d.y;
+            v.z += d.z;
+            v.w += d.w;
+            hr[i] = v;
+            return v;
+        };
+        auto store4 = [&](int i, float4 v, float rinv) {
+            const float4 g = w4[i];
+            const float a0 = v.x * rinv * (1.f + g.x), a1 = v.y * rinv * (1.f + g.y);
+            const float a2 = v.z * rinv * (1.f + g.z), a3 = v.w * rinv * (1.f + g.w);
+            if constexpr (sizeof(TO) == 2) {
+                const __nv_bfloat162 lo = __floats2bfloat162_rn(a0, a1), hi = __floats2bfloat162_rn(a2, a3);
+                uint2 u;
+                u.x = *reinterpret_cast<const uint32_t*>(&lo);
+                u.y = *reinterpret_cast<const uint32_t*>(&hi);
+                *reinterpret_cast<uint2*>(y + r * W + 4 * i) = u;
+            } else {
+                *reinterpret_cast<float4*>(y + r * W + 4 * i) = make_float4(a0, a1, a2, a3);
+            }
+        };
+        if (n4 <= 32 * RN_CAP) {
+            // Passes over the row held in registers: part 0, each further part, then h.
+            float4 v[RN_CAP];
+            float s = 0.f;
+            const float4* p0 = reinterpret_cast<const float4*>(parts + r * W);
+#pragma unroll
+            for (int k = 0; k < RN_CAP; ++k) {
+                const int i = lane + 32 * k;
+                v[k] = i < n4 ? p0[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            for (int q = 1; q < nparts; ++q) {
+                const float4* pq = reinterpret_cast<const float4*>(parts + (size_t)q * pstride + r * W);
+#pragma unroll
+                for (int k = 0; k < RN_CAP; ++k) {
+                    const int i = lane + 32 * k;
+                    if (i < n4) {
+                        const float4 e = pq[i];
+                        v[k].x += e.x;
+                        v[k].y += e.y;
+                        v[k].z += e.z;
+                        v[k].w += e.w;
+                    }
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < RN_CAP; ++k) {
+                const int i = lane + 32 * k;
+                if (i < n4) {
+                    const float4 o = hr[i];
+                    v[k] = make_float4(o.x + v[k].x, o.y + v[k].y, o.z + v[k].z, o.w + v[k].w);
+                    hr[i] = v[k];
+                }
+            }
+            if (!w) continue;
+#pragma unroll
+            for (int k = 0; k < RN_CAP; ++k) s += (v[k].x * v[k].x + v[k].y * v[k].y) + (v[k].z * v[k].z + v[k].w * v[k].w);
+            const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
+#pragma unroll
+            for (int k = 0; k < RN_CAP; ++k) {
+                const int i = lane + 32 * k;
+                if (i < n4) store4(i, v[k], rinv);
+            }
+        } else {
+            float s = 0.f;
+            for (int i = lane; i < n4; i += 32) {
+                const float4 v = update(i);
+                s += (v.x * v.x + v.y * v.y) + (v.z * v.z + v.w * v.w);
+            }
+            if (!w) continue;
+            const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
+            for (int i = lane; i < n4; i += 32) store4(i, hr[i], rinv);
+        }
+    }
+}
+
+// Gate (off = 0) or up (off = 128) rows [F][W] fp32 -> bf16 rows of the packed gate/up matrix,
+// where 256-row tile t holds gate rows 128 t..128 t + 127, then the up rows of the same features.
+__global__ void k_pf_cast_gu(const float* __restrict__ src, __nv_bfloat16* __restrict__ dst, int F, int W, int off) {
+    const long long n = (long long)F * W;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const int f = (int)(i / W), c = (int)(i - (long long)f * W);
+        const long long row = (long long)(f >> 7) * 256 + off + (f & 127);
+        dst[row * W + c] = __float2bfloat16_rn(src[i]);
     }
 }
 
@@ -208,6 +374,13 @@ struct PfGemmArgs {
     int vec;              // Y and ldy allow 16-byte stores of 16 consecutive elements
     void* Y;
     long long ldy;        // elements
+    // K split: k-blocks in ksplit consecutive ranges; range s writes its partial products to
+    // Y + s * ysplit (fp32, never accumulating), summed in range order by the consumer.
+    int ksplit;
+    long long ysplit;
+    // GeGLU: W tile t holds gate rows 128 t.. then the up rows of the same features; Y is bf16
+    // z [M][ldy] = gelu_tanh(alpha gate) * (alpha up) for the nz features.
+    int geglu, nz;
     int* err;
 };
 
@@ -228,8 +401,17 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nkb = (a.K + PG_KBLK - 1) / PG_KBLK;
     const int ntn = (a.N + PG_TN - 1) / PG_TN, ntm = (a.M + PG_TM - 1) / PG_TM;
-    const int total = ntn * ntm;
+    const int total = ntn * ntm * a.ksplit;
     const int u0 = blockIdx.x, du = gridDim.x;
+    // Unit u: X tile fastest, then W tile, then K range; k-blocks [kb_lo, kb_hi) of the range.
+    const int nkr = (nkb + a.ksplit - 1) / a.ksplit;
+    auto unit = [&](int u, int& tm, int& tn, int& sk, int& kb_lo, int& kb_hi) {
+        tm = u % ntm;
+        tn = (u / ntm) % ntn;
+        sk = u / (ntm * ntn);
+        kb_lo = sk * nkr;
+        kb_hi = min(nkb, kb_lo + nkr);
+    };
 
     if (warp == 1) {
         ptx::tmem_alloc(tmem_slot, 2 * PG_TN);
@@ -254,8 +436,9 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
             int it = 0, issued = 0;
             bool ok = true;
             for (int u = u0; u < total && ok; u += du) {
-                const int tm = u % ntm, tn = u / ntm;
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                int tm, tn, sk, kb_lo, kb_hi;
+                unit(u, tm, tn, sk, kb_lo, kb_hi);
+                for (int kb = kb_lo; kb < kb_hi; ++kb, ++it) {
                     const int s = it % PG_STAGES, n = it / PG_STAGES;
                     if (it >= PG_STAGES && !ptx::mbar_wait_bounded(&empty[s], (n - 1) & 1, PG_WAIT_NS)) {
                         *flag = PF_DEV_TIMEOUT_LOAD;
@@ -286,7 +469,9 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
                 if (j >= 2 && !ptx::mbar_wait_bounded(&acce[buf], ((j - 2) >> 1) & 1, PG_WAIT_NS)) good = false;
                 ptx::tc_fence_after();
                 const uint32_t acc = tmem + (uint32_t)(buf * PG_TN);
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                int tm, tn, sk, kb_lo, kb_hi;
+                unit(u, tm, tn, sk, kb_lo, kb_hi);
+                for (int kb = kb_lo; kb < kb_hi; ++kb, ++it) {
                     const int s = it % PG_STAGES, n = it / PG_STAGES;
                     if (good && !ptx::mbar_wait_bounded(&full[s], n & 1, PG_WAIT_NS)) good = false;
                     ptx::tc_fence_after();
@@ -295,7 +480,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
 #pragma unroll
                         for (int kk = 0; kk < PG_KBLK / 16; ++kk)
                             ptx::mma_bf16(acc, ptx::desc_sw128(x + kk * 32), ptx::desc_sw128(w + kk * 32), IDESC,
-                                          (kb | kk) != 0);
+                                          (kb != kb_lo) || (kk != 0));
                     }
                     ptx::mma_commit(&empty[s]);
                 }
@@ -309,11 +494,49 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         for (int u = u0, j = 0; u < total; u += du, ++j) {
             const int buf = j & 1;
-            const int tm = u % ntm, tn = u / ntm;
+            int tm, tn, sk, kb_lo, kb_hi;
+            unit(u, tm, tn, sk, kb_lo, kb_hi);
             const bool ok = ptx::mbar_wait_bounded(&accf[buf], (j >> 1) & 1, PG_WAIT_NS) && *flag == 0;
             ptx::tc_fence_after();
             const int m = tm * PG_TM + row;
             const bool live = ok && m < a.M;
+            if (a.geglu) {
+                // Gate columns c0.. and up columns 128 + c0.. of this tile: 16 features of z.
+                for (int c0 = 0; c0 < PG_TN / 2; c0 += 16) {
+                    uint32_t rg[16], ru[16];
+                    ptx::tmem_ld_x16(lane_base + (uint32_t)(buf * PG_TN + c0), rg);
+                    ptx::tmem_ld_x16(lane_base + (uint32_t)(buf * PG_TN + PG_TN / 2 + c0), ru);
+                    ptx::tmem_ld_wait();
+                    const int f0 = tn * (PG_TN / 2) + c0;
+                    if (!live || f0 >= a.nz) continue;
+                    float v[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i)
+                        v[i] = gelu_tanh_f(a.alpha * __uint_as_float(rg[i])) * (a.alpha * __uint_as_float(ru[i]));
+                    __nv_bfloat16* z = static_cast<__nv_bfloat16*>(a.Y) + (size_t)m * a.ldy + f0;
+                    if (a.vec && f0 + 16 <= a.nz) {
+                        uint32_t p[8];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            __nv_bfloat162 t = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+                            p[i] = *reinterpret_cast<uint32_t*>(&t);
+                        }
+                        reinterpret_cast<uint4*>(z)[0] = make_uint4(p[0], p[1], p[2], p[3]);
+                        reinterpret_cast<uint4*>(z)[1] = make_uint4(p[4], p[5], p[6], p[7]);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i)
+                            if (f0 + i < a.nz) z[i] = __float2bfloat16_rn(v[i]);
+                    }
+                }
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(&acce[buf]);
+                if (!ok && lane == 0) *flag = PF_DEV_TIMEOUT_MMA;
+                continue;
+            }
+            // K range sk writes its own partial (never accumulating).
+            void* Yu = a.ksplit > 1 ? (void*)(static_cast<float*>(a.Y) + (size_t)sk * a.ysplit) : a.Y;
+            const bool accum = a.accumulate && a.ksplit == 1;
             for (int c0 = 0; c0 < PG_TN; c0 += 16) {
                 uint32_t r[16];
                 ptx::tmem_ld_x16(lane_base + (uint32_t)(buf * PG_TN + c0), r);
@@ -326,7 +549,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
                 const size_t o = (size_t)m * a.ldy + n0;
                 if (a.vec && n0 + 16 <= a.N) {
                     if (a.out_bf16) {
-                        uint4* y = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.Y) + o);
+                        uint4* y = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(Yu) + o);
                         uint32_t p[8];
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
@@ -336,11 +559,11 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
                         y[0] = make_uint4(p[0], p[1], p[2], p[3]);
                         y[1] = make_uint4(p[4], p[5], p[6], p[7]);
                     } else {
-                        float4* y = reinterpret_cast<float4*>(static_cast<float*>(a.Y) + o);
+                        float4* y = reinterpret_cast<float4*>(static_cast<float*>(Yu) + o);
 #pragma unroll
                         for (int q = 0; q < 4; ++q) {
                             float4 t = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                            if (a.accumulate) {
+                            if (accum) {
                                 const float4 old = y[q];
                                 t.x += old.x;
                                 t.y += old.y;
@@ -355,10 +578,10 @@ __global__ void __launch_bounds__(PG_THREADS, 1) k_pf_gemm(const __grid_constant
                     for (int i = 0; i < 16; ++i) {
                         if (n0 + i >= a.N) continue;
                         if (a.out_bf16) {
-                            static_cast<__nv_bfloat16*>(a.Y)[o + i] = __float2bfloat16_rn(v[i]);
+                            static_cast<__nv_bfloat16*>(Yu)[o + i] = __float2bfloat16_rn(v[i]);
                         } else {
-                            float* y = static_cast<float*>(a.Y) + o + i;
-                            *y = a.accumulate ? *y + v[i] : v[i];
+                            float* y = static_cast<float*>(Yu) + o + i;
+                            *y = accum ? *y + v[i] : v[i];
                         }
                     }
                 }
@@ -416,11 +639,14 @@ struct jpi_prefill_handle {
     float* final_norm = nullptr;
     float2* rope = nullptr;          // [Pm][D / 2]
     float* h = nullptr;              // [Bm Pm][W] residual stream
-    __nv_bfloat16* xn = nullptr;     // [Bm Pm][max(W, F)] GEMM operand (normed h, or z)
+    __nv_bfloat16* xn = nullptr;     // [Bm Pm][W] GEMM operand: normed h
     float* qkv = nullptr;            // [Bm Pm][(H + 2) D]
     __nv_bfloat16* q = nullptr;      // [Bm Pm][H][D]
     __nv_bfloat16* o = nullptr;      // [Bm Pm][H D]
-    float* gu = nullptr;             // [Bm Pm][2 F]
+    __nv_bfloat16* z = nullptr;      // [Bm Pm][F] GeGLU output (the gate/up product's epilogue)
+    float* part = nullptr;           // [part_rows][W] partial products of a K-split projection
+    long long part_rows = 0;         // rows the partials hold (parts x rows of one part)
+    int Fp = 0;                      // F rounded up to 128: gate/up tiles of 128 features
     float* sc = nullptr;             // [H Pm][Pp] scores of one request
     __nv_bfloat16* pr = nullptr;     // [H Pm][Pp] probabilities of one request
     __nv_bfloat16* vt = nullptr;     // [D][Pp] one request's values, transposed
@@ -469,10 +695,12 @@ jpi_status make_map(const void* base, long long rows, long long cols, long long 
 }
 
 // Y [M][N] (leading dimension ldy; fp32, or bf16 when y_bf16) = alpha X [M][K] W[N][K]^T, plus Y
-// when accumulating. X and W are bf16 with leading dimensions ldx and ldw.
+// when accumulating. X and W are bf16 with leading dimensions ldx and ldw. With ksplit > 1 the
+// k-blocks are cut into ksplit ranges and range s writes fp32 Y + s * ysplit (not accumulating);
+// with nz > 0, Y is the bf16 GeGLU output z [M][ldy] of nz features (gate/up tiles packed).
 jpi_status row_gemm(jpi_prefill_handle* h, cudaStream_t st, const __nv_bfloat16* X, long long ldx,
                     const __nv_bfloat16* Wm, long long ldw, void* Y, bool y_bf16, long long ldy, int M, int N,
-                    int K, float alpha, bool accumulate) {
+                    int K, float alpha, bool accumulate, int ksplit = 1, long long ysplit = 0, int nz = 0) {
     CUtensorMap wmap, xmap;
     PF_TRY(make_map(Wm, N, K, ldw, PG_TN, &wmap));
     PF_TRY(make_map(X, M, K, ldx, PG_TM, &xmap));
@@ -486,12 +714,28 @@ jpi_status row_gemm(jpi_prefill_handle* h, cudaStream_t st, const __nv_bfloat16*
     a.Y = Y;
     a.ldy = ldy;
     a.vec = (reinterpret_cast<uintptr_t>(Y) % 16 == 0 && ldy % (y_bf16 ? 8 : 4) == 0) ? 1 : 0;
+    a.ksplit = ksplit;
+    a.ysplit = ysplit;
+    a.geglu = nz > 0 ? 1 : 0;
+    a.nz = nz;
     a.err = h->dev_err;
-    const long long tiles = (long long)((N + PG_TN - 1) / PG_TN) * ((M + PG_TM - 1) / PG_TM);
+    const long long tiles = (long long)((N + PG_TN - 1) / PG_TN) * ((M + PG_TM - 1) / PG_TM) * ksplit;
     const int grid = (int)(tiles < h->num_sms ? tiles : h->num_sms);
     k_pf_gemm<<<grid, PG_THREADS, PG_SMEM, st>>>(wmap, xmap, a);
     PF_CUDA(cudaGetLastError());
     return JPI_OK;
+}
+
+// K ranges for a product with few output tiles (the O and down projections at small B x P have
+// W / 256 x (B P) / 128 tiles, 56 at Gemma-2B sizes): as many as keep one wave on the GPU, at
+// most 4, each of at least 8 k-blocks, and only while the partials fit.
+int split_for(const jpi_prefill_handle* h, int M, int N, int K) {
+    const long long tiles = (long long)((N + PG_TN - 1) / PG_TN) * ((M + PG_TM - 1) / PG_TM);
+    const int nkb = (K + PG_KBLK - 1) / PG_KBLK;
+    int s = 1;
+    while (s < 4 && tiles * (s + 1) <= h->num_sms && nkb / (s + 1) >= 8 && (long long)(s + 1) * M <= h->part_rows)
+        ++s;
+    return s;
 }
 
 jpi_status check_config(const jpi_prefill_config* c) {
@@ -524,6 +768,22 @@ jpi_status put_bf16(jpi_prefill_handle* h, bool dev, float* staging, __nv_bfloat
     return JPI_OK;
 }
 
+// Gate (off 0) or up (off 128) rows [F][W] (host or device fp32) into the packed gate/up matrix.
+jpi_status put_gu(jpi_prefill_handle* h, bool dev, float* staging, __nv_bfloat16* dst, const float* src, int off,
+                  const char* name, int layer) {
+    if (!src) return pfail(JPI_ERR_INVALID_ARG, "weight %s of layer %d is NULL", name, layer);
+    const size_t n = (size_t)h->F * h->W;
+    const float* s = src;
+    if (!dev) {
+        PF_CUDA(cudaMemcpy(staging, src, n * sizeof(float), cudaMemcpyHostToDevice));
+        s = staging;
+    }
+    k_pf_cast_gu<<<grid_for((long long)n), 256>>>(s, dst, h->F, h->W, off);
+    PF_CUDA(cudaGetLastError());
+    PF_CUDA(cudaStreamSynchronize(nullptr));
+    return JPI_OK;
+}
+
 jpi_status put_f32(jpi_prefill_handle* h, bool dev, float** dst, const float* src, size_t n, const char* name,
                    int layer) {
     if (!src) return pfail(JPI_ERR_INVALID_ARG, "weight %s of layer %d is NULL", name, layer);
@@ -545,6 +805,8 @@ jpi_status setup(jpi_prefill_handle* h, const jpi_prefill_config* c, const jpi_p
     h->Pp = (h->Pm + 7) / 8 * 8;
     const size_t W = (size_t)h->W, D = (size_t)h->D, F = (size_t)h->F, HD = (size_t)h->H * D;
     const size_t Mm = (size_t)h->Bm * h->Pm;
+    h->Fp = (h->F + 127) / 128 * 128;
+    const size_t Fp = (size_t)h->Fp;
     const bool dev = w->on_device != 0;
     if (!w->attn_norm || !w->wq || !w->wk || !w->wv || !w->wo || !w->mlp_norm || !w->w_gate || !w->w_up ||
         !w->w_down || !w->final_norm)
@@ -567,9 +829,10 @@ jpi_status setup(jpi_prefill_handle* h, const jpi_prefill_config* c, const jpi_p
         PF_TRY(put_bf16(h, dev, staging, lw.wqkv + (HD + D) * W, w->wv[l], D * W, "wv", l));
         PF_TRY(pf_alloc(h, &lw.wo, W * HD));
         PF_TRY(put_bf16(h, dev, staging, lw.wo, w->wo[l], W * HD, "wo", l));
-        PF_TRY(pf_alloc(h, &lw.wgu, 2 * F * W));
-        PF_TRY(put_bf16(h, dev, staging, lw.wgu, w->w_gate[l], F * W, "w_gate", l));
-        PF_TRY(put_bf16(h, dev, staging, lw.wgu + F * W, w->w_up[l], F * W, "w_up", l));
+        PF_TRY(pf_alloc(h, &lw.wgu, 2 * Fp * W));
+        PF_CUDA(cudaMemset(lw.wgu, 0, 2 * Fp * W * sizeof(__nv_bfloat16)));   // rows of features past F
+        PF_TRY(put_gu(h, dev, staging, lw.wgu, w->w_gate[l], 0, "w_gate", l));
+        PF_TRY(put_gu(h, dev, staging, lw.wgu, w->w_up[l], 128, "w_up", l));
         PF_TRY(pf_alloc(h, &lw.wd, W * F));
         PF_TRY(put_bf16(h, dev, staging, lw.wd, w->w_down[l], W * F, "w_down", l));
         PF_TRY(put_f32(h, dev, &lw.attn_norm, w->attn_norm[l], W, "attn_norm", l));
@@ -592,11 +855,19 @@ jpi_status setup(jpi_prefill_handle* h, const jpi_prefill_config* c, const jpi_p
     PF_CUDA(cudaMemcpy(h->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice));
 
     PF_TRY(pf_alloc(h, &h->h, Mm * W));
-    PF_TRY(pf_alloc(h, &h->xn, Mm * (W > F ? W : F)));
+    PF_TRY(pf_alloc(h, &h->xn, Mm * W));
+    PF_TRY(pf_alloc(h, &h->z, Mm * F));
+    // Partials of K-split projections (N = W): a split needs at most num_sms / 2 output tiles,
+    // so a part has at most that many 128-row tiles of rows, and there are at most 4 parts.
+    {
+        const long long ntn = (h->W + PG_TN - 1) / PG_TN;
+        const long long rows2 = std::min<long long>((long long)Mm, (h->num_sms / 2 / ntn) * PG_TM);
+        h->part_rows = 4 * rows2;
+        if (h->part_rows > 0) PF_TRY(pf_alloc(h, &h->part, (size_t)h->part_rows * W));
+    }
     PF_TRY(pf_alloc(h, &h->qkv, Mm * (size_t)h->QKV));
     PF_TRY(pf_alloc(h, &h->q, Mm * HD));
     PF_TRY(pf_alloc(h, &h->o, Mm * HD));
-    PF_TRY(pf_alloc(h, &h->gu, Mm * 2 * F));
     PF_TRY(pf_alloc(h, &h->sc, (size_t)h->H * h->Pm * h->Pp));
     PF_TRY(pf_alloc(h, &h->pr, (size_t)h->H * h->Pm * h->Pp));
     PF_TRY(pf_alloc(h, &h->vt, D * (size_t)h->Pp));
@@ -659,13 +930,19 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
 
     k_pf_load_x<<<grid_for(M * W), 256, 0, st>>>(x, x_is_fp32, h->h, M * W);
     PF_CUDA(cudaGetLastError());
+    // After a K-split down projection, the step that adds its partials to h also writes the next
+    // layer's attention norm into xn.
+    bool xn_ready = false;
+    const long long pstride = M * W;   // elements between the parts of a split product
     for (int l = 0; l < h->L; ++l) {
         const LayerW& lw = h->layers[(size_t)l];
         __nv_bfloat16* kd = static_cast<__nv_bfloat16*>(k_layers[l]);
         __nv_bfloat16* vd = static_cast<__nv_bfloat16*>(v_layers[l]);
         // Attention sublayer.
-        k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, lw.attn_norm, h->xn, M, W, eps);
-        PF_CUDA(cudaGetLastError());
+        if (!xn_ready) {
+            k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, lw.attn_norm, h->xn, M, W, eps);
+            PF_CUDA(cudaGetLastError());
+        }
         PF_TRY(row_gemm(h, st, h->xn, W, lw.wqkv, W, h->qkv, false, h->QKV, (int)M, h->QKV, W, 1.f, false));
         k_pf_rope_scatter<<<grid_for(M * (H + 2) * (D / 2)), 256, 0, st>>>(h->qkv, h->rope, h->q, kd, vd,
                                                                              request_stride, batch, P, H, D);
@@ -682,17 +959,41 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
             PF_CUDA(cudaGetLastError());
             PF_TRY(row_gemm(h, st, h->pr, Pp, h->vt, Pp, ob, true, D, P * H, D, P, 1.f, false));
         }
-        PF_TRY(row_gemm(h, st, h->o, H * D, lw.wo, H * D, h->h, false, W, (int)M, W, H * D, 1.f, true));
-        // MLP sublayer.
-        k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, lw.mlp_norm, h->xn, M, W, eps);
+        // Output projection into the residual stream, then the MLP norm: split over K when the
+        // product has too few tiles to fill the GPU (partials added in order with the norm).
+        const int so = split_for(h, (int)M, W, H * D);
+        if (so > 1) {
+            PF_TRY(row_gemm(h, st, h->o, H * D, lw.wo, H * D, h->part, false, W, (int)M, W, H * D, 1.f, false, so,
+                            pstride));
+            k_pf_residual_norm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->part, so, pstride,
+                                                                                  lw.mlp_norm, h->xn, M, W, eps);
+        } else {
+            PF_TRY(row_gemm(h, st, h->o, H * D, lw.wo, H * D, h->h, false, W, (int)M, W, H * D, 1.f, true));
+            k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, lw.mlp_norm, h->xn, M, W, eps);
+        }
         PF_CUDA(cudaGetLastError());
-        PF_TRY(row_gemm(h, st, h->xn, W, lw.wgu, W, h->gu, false, 2 * F, (int)M, 2 * F, W, 1.f, false));
-        k_pf_geglu<<<grid_for(M * F), 256, 0, st>>>(h->gu, h->xn, M, F);
-        PF_CUDA(cudaGetLastError());
-        PF_TRY(row_gemm(h, st, h->xn, F, lw.wd, F, h->h, false, W, (int)M, W, F, 1.f, true));
-    }
-    if (out_final) {
-        k_pf_rmsnorm<float><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->final_norm, out_final, M, W, eps);
+        // MLP sublayer: gate/up with GeGLU in its epilogue (z bf16), then down into the residual.
+        PF_TRY(row_gemm(h, st, h->xn, W, lw.wgu, W, h->z, true, F, (int)M, 2 * h->Fp, W, 1.f, false, 1, 0, F));
+        const int sd = split_for(h, (int)M, W, F);
+        if (sd > 1) {
+            PF_TRY(row_gemm(h, st, h->z, F, lw.wd, F, h->part, false, W, (int)M, W, F, 1.f, false, sd, pstride));
+            if (l + 1 < h->L) {
+                k_pf_residual_norm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(
+                    h->h, h->part, sd, pstride, h->layers[(size_t)l + 1].attn_norm, h->xn, M, W, eps);
+                xn_ready = true;
+            } else if (out_final) {
+                k_pf_residual_norm<float><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->part, sd, pstride,
+                                                                            h->final_norm, out_final, M, W, eps);
+            } else {
+                k_pf_residual_norm<float><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->part, sd, pstride, nullptr,
+                                                                            nullptr, M, W, eps);
+            }
+        } else {
+            PF_TRY(row_gemm(h, st, h->z, F, lw.wd, F, h->h, false, W, (int)M, W, F, 1.f, true));
+            xn_ready = false;
+            if (l + 1 == h->L && out_final)
+                k_pf_rmsnorm<float><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->final_norm, out_final, M, W, eps);
+        }
         PF_CUDA(cudaGetLastError());
     }
     return JPI_OK;

@@ -57,6 +57,31 @@ def test_prefill_matches_the_oracle(B, P, x_dtype):
     pre.close()
 
 
+def test_split_products_and_padded_gate_up():
+    # H D = 1024 and F = 1096 give the output and down products 16 and 18 k-blocks over few
+    # tiles, so both run split over K (partials added to the residual with the next norm), and
+    # F is not a multiple of 128, so the last gate/up tile is zero-padded. Without the final
+    # output the last split only updates the residual; K and V must not change.
+    import torch
+    prefill = _mods()
+    cfg = GEMMA2B.with_(n_layers=2, width=256, n_heads=4, head_dim=256, mlp_dim=1096)
+    w = make_llm_weights(cfg, 91, std=0.05, norm_std=0.1)
+    x = make_prefix_embeddings(cfg, 92, 2, 50)
+    pre = prefill.Prefill(cfg, w, max_batch=2, max_prefix=50)
+    xt = torch.from_numpy(x).cuda()
+    K, V, out = pre.into_tensors(xt)
+    K2, V2, _ = pre.into_tensors(xt, final=False)
+    torch.cuda.synchronize()
+    pre.device_status()
+    Kw, Vw, want = pf.prefill_batch(x, w, cfg)
+    for l in range(cfg.n_layers):
+        _close(K[l].float().cpu().numpy(), Kw[l], f"split K layer {l}")
+        _close(V[l].float().cpu().numpy(), Vw[l], f"split V layer {l}")
+        assert torch.equal(K[l], K2[l]) and torch.equal(V[l], V2[l])
+    _close(out.cpu().numpy(), want, "split final output")
+    pre.close()
+
+
 def test_gemma2b_sized_layers():
     # Width 2048, 8 heads x 256, GeGLU 16384, 816 prefix tokens; two layers keep the fp64 oracle
     # to seconds.
