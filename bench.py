@@ -47,7 +47,7 @@ NCU_TRAFFIC = {
 
 # The sources the expert's kernels and their launches are built from. The correction module
 # (CORRECTION_SOURCES) is compiled into the same library but none of the measured kernels uses it.
-EXPERT_SOURCES = ("api.cu", "attn_t5.cu", "attn_tc.cu", "gemm_big.cuh", "gemm_kernel.cuh",
+EXPERT_SOURCES = ("api.cu", "attn_t5.cu", "attn_t5_kernel.cuh", "attn_tc.cu", "gemm_big.cuh", "gemm_kernel.cuh",
                   "jpi_internal.h", "kernels_simt.cu", "mod_tc.cu", "noalloc.cu", "ptx.h", "tc_path.cu",
                   "tc_path.h")
 CORRECTION_SOURCES = ("corr.cu",)

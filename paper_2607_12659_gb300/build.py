@@ -62,7 +62,8 @@ def build_prefill(verbose: bool = False, force: bool = False) -> str:
     out = os.path.join(BUILD, "prefill")
     os.makedirs(out, exist_ok=True)
     srcs = sorted(os.path.join(PREFILL_SRC, f) for f in os.listdir(PREFILL_SRC) if f.endswith(".cu"))
-    headers = [os.path.join(ROOT, "include", f) for f in ("jpi.h", "jpi_prefill.h")] + [os.path.join(CSRC, "ptx.h")]
+    headers = [os.path.join(ROOT, "include", f) for f in ("jpi.h", "jpi_prefill.h")] + [
+        os.path.join(CSRC, f) for f in ("ptx.h", "attn_t5_kernel.cuh")]
     objs = []
     for src in srcs:
         obj = os.path.join(out, os.path.basename(src)[:-3] + ".o")

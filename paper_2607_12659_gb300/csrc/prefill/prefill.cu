@@ -26,6 +26,7 @@
 
 #include "jpi_prefill.h"
 #include "../ptx.h"
+#include "../attn_t5_kernel.cuh"
 
 namespace {
 
@@ -644,8 +645,8 @@ struct jpi_prefill_handle {
     __nv_bfloat16* q = nullptr;      // [Bm Pm][H][D]
     __nv_bfloat16* o = nullptr;      // [Bm Pm][H D]
     __nv_bfloat16* z = nullptr;      // [Bm Pm][F] GeGLU output (the gate/up product's epilogue)
-    float* part = nullptr;           // [part_rows][W] partial products of a K-split projection
-    long long part_rows = 0;         // rows the partials hold (parts x rows of one part)
+    float* part = nullptr;           // partial products of a K-split projection
+    long long part_elems = 0;        // floats `part` holds
     int Fp = 0;                      // F rounded up to 128: gate/up tiles of 128 features
     float* sc = nullptr;             // [H Pm][Pp] scores of one request
     __nv_bfloat16* pr = nullptr;     // [H Pm][Pp] probabilities of one request
@@ -726,16 +727,48 @@ jpi_status row_gemm(jpi_prefill_handle* h, cudaStream_t st, const __nv_bfloat16*
     return JPI_OK;
 }
 
-// K ranges for a product with few output tiles (the O and down projections at small B x P have
-// W / 256 x (B P) / 128 tiles, 56 at Gemma-2B sizes): as many as keep one wave on the GPU, at
-// most 4, each of at least 8 k-blocks, and only while the partials fit.
+// K ranges for a product with few output tiles (at small B x P the O and down projections have
+// 56 tiles at Gemma-2B sizes): as many as keep one wave on the GPU, at most 4, each of at least
+// 8 k-blocks, and only while the partials [M][N] fit.
 int split_for(const jpi_prefill_handle* h, int M, int N, int K) {
     const long long tiles = (long long)((N + PG_TN - 1) / PG_TN) * ((M + PG_TM - 1) / PG_TM);
     const int nkb = (K + PG_KBLK - 1) / PG_KBLK;
     int s = 1;
-    while (s < 4 && tiles * (s + 1) <= h->num_sms && nkb / (s + 1) >= 8 && (long long)(s + 1) * M <= h->part_rows)
+    while (s < 4 && tiles * (s + 1) <= h->num_sms && nkb / (s + 1) >= 8 &&
+           (long long)(s + 1) * M * N <= h->part_elems)
         ++s;
     return s;
+}
+
+// Attention of the requests of one layer on the tcgen05 attention kernel: the queries h->q
+// [B P H][D] against this layer's keys and values kd / vd (request b at row b * kv_rows, P rows
+// each), every key visible, into h->o. Used for head dims 128 and 256 when the request stride is
+// a whole number of rows; the maps' row extents end at the last request's last key, so no copy
+// reads past what the caller owns (the kernel masks the zero-filled rows past P).
+template <int D>
+jpi_status attention_t5(jpi_prefill_handle* h, cudaStream_t st, const __nv_bfloat16* kd, const __nv_bfloat16* vd,
+                        int batch, int P, long long kv_rows) {
+    CUtensorMap qmap, kmap, vmap;
+    const long long nrows = (long long)P * h->H;
+    const long long krows = (long long)(batch - 1) * kv_rows + P;
+    PF_TRY(make_map(h->q, (long long)batch * nrows, D, D, jpi::T5_ROWS, &qmap));
+    PF_TRY(make_map(kd, krows, D, D, jpi::T5_KEYS, &kmap));
+    PF_TRY(make_map(vd, krows, D, D, jpi::T5_KEYS, &vmap));
+    jpi::T5Args a;
+    a.S = P;
+    a.nctx = 0;
+    a.H = h->H;
+    a.P = 0;
+    a.kv_rows = (int)kv_rows;
+    a.maxB = batch;
+    a.layer = 0;
+    a.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
+    a.o = h->o;
+    a.err = h->dev_err;
+    const dim3 grid((unsigned)((nrows + jpi::T5_ROWS - 1) / jpi::T5_ROWS), (unsigned)batch);
+    jpi::k_attn_t5<D><<<grid, jpi::T5_THREADS, 1024 + jpi::T5Smem<D>::TOTAL, st>>>(qmap, kmap, vmap, a);
+    PF_CUDA(cudaGetLastError());
+    return JPI_OK;
 }
 
 jpi_status check_config(const jpi_prefill_config* c) {
@@ -816,6 +849,10 @@ jpi_status setup(jpi_prefill_handle* h, const jpi_prefill_config* c, const jpi_p
     PF_CUDA(cudaGetDevice(&device));
     PF_CUDA(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, device));
     PF_CUDA(cudaFuncSetAttribute(k_pf_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PG_SMEM));
+    PF_CUDA(cudaFuncSetAttribute(jpi::k_attn_t5<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 1024 + jpi::T5Smem<128>::TOTAL));
+    PF_CUDA(cudaFuncSetAttribute(jpi::k_attn_t5<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 1024 + jpi::T5Smem<256>::TOTAL));
     PF_TRY(pf_alloc(h, &h->dev_err, 1));
     PF_CUDA(cudaMemset(h->dev_err, 0, sizeof(int)));
     float* staging = nullptr;
@@ -862,8 +899,8 @@ jpi_status setup(jpi_prefill_handle* h, const jpi_prefill_config* c, const jpi_p
     {
         const long long ntn = (h->W + PG_TN - 1) / PG_TN;
         const long long rows2 = std::min<long long>((long long)Mm, (h->num_sms / 2 / ntn) * PG_TM);
-        h->part_rows = 4 * rows2;
-        if (h->part_rows > 0) PF_TRY(pf_alloc(h, &h->part, (size_t)h->part_rows * W));
+        h->part_elems = 4 * rows2 * h->W;
+        if (h->part_elems > 0) PF_TRY(pf_alloc(h, &h->part, (size_t)h->part_elems));
     }
     PF_TRY(pf_alloc(h, &h->qkv, Mm * (size_t)h->QKV));
     PF_TRY(pf_alloc(h, &h->q, Mm * HD));
@@ -947,7 +984,14 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
         k_pf_rope_scatter<<<grid_for(M * (H + 2) * (D / 2)), 256, 0, st>>>(h->qkv, h->rope, h->q, kd, vd,
                                                                              request_stride, batch, P, H, D);
         PF_CUDA(cudaGetLastError());
-        for (int b = 0; b < batch; ++b) {
+        // Attention: on the tcgen05 attention kernel (scores and probabilities never leave the
+        // SM), else per request through the GEMM: scores, softmax, V^T, probabilities times V.
+        const bool t5 = (D == 128 || D == 256) && request_stride % D == 0 && request_stride / D <= INT32_MAX;
+        if (t5) {
+            PF_TRY(D == 256 ? attention_t5<256>(h, st, kd, vd, batch, P, request_stride / D)
+                            : attention_t5<128>(h, st, kd, vd, batch, P, request_stride / D));
+        }
+        for (int b = 0; b < batch && !t5; ++b) {
             const __nv_bfloat16* qb = h->q + (size_t)b * P * H * D;     // [(P H)][D]
             const __nv_bfloat16* kb = kd + (size_t)b * request_stride;  // [P][D]
             const __nv_bfloat16* vb = vd + (size_t)b * request_stride;  // [P][D]
