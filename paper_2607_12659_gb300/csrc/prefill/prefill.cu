@@ -76,91 +76,102 @@ __global__ void k_pf_load_x(const void* __restrict__ x, int x_fp32, float* __res
         h[i] = x_fp32 ? static_cast<const float*>(x)[i] : __bfloat162float(static_cast<const __nv_bfloat16*>(x)[i]);
 }
 
-// y = h / sqrt(mean(h^2) + eps) * (1 + w), row by row; one warp per row (grid-stride). A row of
-// up to RN_CAP float4 per lane is loaded into registers at once (every load in flight together,
-// one pass over memory); longer rows take a strided loop. W is a multiple of 4.
-constexpr int RN_CAP = 16;   // 2048 floats per row
+// Row kernels of W floats (W a multiple of 4): one block of RB threads per row (grid-stride over
+// rows), a row of up to RB x RB_CAP float4 held in registers with every load in flight, the sum
+// of squares reduced over the block.
+constexpr int RB = 128;
+constexpr int RB_CAP = 8;   // 4096 floats per row
+__device__ __forceinline__ float block_sum_rb(float v, float* red) {
+    v = warp_sum(v);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float t = 0.f;
+#pragma unroll
+    for (int i = 0; i < RB / 32; ++i) t += red[i];
+    __syncthreads();   // red is reused by the next row
+    return t;
+}
+// y[4 i .. 4 i + 3] of row r = v * rinv * (1 + w).
 template <typename TO>
-__global__ void __launch_bounds__(256) k_pf_rmsnorm(const float* __restrict__ h, const float* __restrict__ w,
-                                                    TO* __restrict__ y, long long rows, int W, float eps) {
-    const int lane = threadIdx.x & 31;
-    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
-    const int n4 = W >> 2;
-    const float4* w4 = reinterpret_cast<const float4*>(w);
-    for (long long r = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += nwarps) {
+__device__ __forceinline__ void store_normed4(TO* y, const float* w, long long r, int W, int i, float4 v, float rinv) {
+    const float4 g = reinterpret_cast<const float4*>(w)[i];
+    const float a0 = v.x * rinv * (1.f + g.x), a1 = v.y * rinv * (1.f + g.y);
+    const float a2 = v.z * rinv * (1.f + g.z), a3 = v.w * rinv * (1.f + g.w);
+    if constexpr (sizeof(TO) == 2) {
+        const __nv_bfloat162 lo = __floats2bfloat162_rn(a0, a1), hi = __floats2bfloat162_rn(a2, a3);
+        uint2 u;
+        u.x = *reinterpret_cast<const uint32_t*>(&lo);
+        u.y = *reinterpret_cast<const uint32_t*>(&hi);
+        *reinterpret_cast<uint2*>(y + r * W + 4 * i) = u;
+    } else {
+        *reinterpret_cast<float4*>(y + r * W + 4 * i) = make_float4(a0, a1, a2, a3);
+    }
+}
+__device__ __forceinline__ float sq4(float4 v) {
+    return (v.x * v.x + v.y * v.y) + (v.z * v.z + v.w * v.w);
+}
+
+// y = h / sqrt(mean(h^2) + eps) * (1 + w), row by row.
+template <typename TO>
+__global__ void __launch_bounds__(RB) k_pf_rmsnorm(const float* __restrict__ h, const float* __restrict__ w,
+                                                   TO* __restrict__ y, long long rows, int W, float eps) {
+    __shared__ float red[RB / 32];
+    const int t = threadIdx.x, n4 = W >> 2;
+    for (long long r = blockIdx.x; r < rows; r += gridDim.x) {
         const float4* hr = reinterpret_cast<const float4*>(h + r * W);
-        auto store4 = [&](int i, float4 v, float rinv) {
-            const float4 g = w4[i];
-            const float a0 = v.x * rinv * (1.f + g.x), a1 = v.y * rinv * (1.f + g.y);
-            const float a2 = v.z * rinv * (1.f + g.z), a3 = v.w * rinv * (1.f + g.w);
-            if constexpr (sizeof(TO) == 2) {
-                const __nv_bfloat162 lo = __floats2bfloat162_rn(a0, a1), hi = __floats2bfloat162_rn(a2, a3);
-                uint2 u;
-                u.x = *reinterpret_cast<const uint32_t*>(&lo);
-                u.y = *reinterpret_cast<const uint32_t*>(&hi);
-                *reinterpret_cast<uint2*>(y + r * W + 4 * i) = u;
-            } else {
-                *reinterpret_cast<float4*>(y + r * W + 4 * i) = make_float4(a0, a1, a2, a3);
-            }
-        };
-        if (n4 <= 32 * RN_CAP) {
-            float4 v[RN_CAP];
+        if (n4 <= RB * RB_CAP) {
+            float4 v[RB_CAP];
             float s = 0.f;
 #pragma unroll
-            for (int k = 0; k < RN_CAP; ++k) {
-                const int i = lane + 32 * k;
+            for (int k = 0; k < RB_CAP; ++k) {
+                const int i = t + RB * k;
                 v[k] = i < n4 ? hr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
             }
 #pragma unroll
-            for (int k = 0; k < RN_CAP; ++k) s += (v[k].x * v[k].x + v[k].y * v[k].y) + (v[k].z * v[k].z + v[k].w * v[k].w);
-            const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
+            for (int k = 0; k < RB_CAP; ++k) s += sq4(v[k]);
+            const float rinv = 1.f / sqrtf(block_sum_rb(s, red) / (float)W + eps);
 #pragma unroll
-            for (int k = 0; k < RN_CAP; ++k) {
-                const int i = lane + 32 * k;
-                if (i < n4) store4(i, v[k], rinv);
+            for (int k = 0; k < RB_CAP; ++k) {
+                const int i = t + RB * k;
+                if (i < n4) store_normed4(y, w, r, W, i, v[k], rinv);
             }
         } else {
             float s = 0.f;
-#pragma unroll 4
-            for (int i = lane; i < n4; i += 32) {
-                const float4 v = hr[i];
-                s += (v.x * v.x + v.y * v.y) + (v.z * v.z + v.w * v.w);
-            }
-            const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
-#pragma unroll 4
-            for (int i = lane; i < n4; i += 32) store4(i, hr[i], rinv);
+            for (int i = t; i < n4; i += RB) s += sq4(hr[i]);
+            const float rinv = 1.f / sqrtf(block_sum_rb(s, red) / (float)W + eps);
+            for (int i = t; i < n4; i += RB) store_normed4(y, w, r, W, i, hr[i], rinv);
         }
     }
 }
 
 // From the projections qkv [B P][(H + 2) D] (fp32): rotated queries q [B P][H][D] (bf16), and the
-// rotated keys and the values of request b, row p into kd / vd + b stride + p D (bf16). One thread
-// per (row, section, rotary pair); rope[p][j] = (cos, sin) of p base^(-2j/D).
+// rotated keys and the values of request b, row p into kd / vd + b stride + p D (bf16). One block
+// per token row (grid-stride), its threads over the (section, rotary pair) slots of the row;
+// rope[p][j] = (cos, sin) of p base^(-2j/D).
 __global__ void k_pf_rope_scatter(const float* __restrict__ qkv, const float2* __restrict__ rope,
                                   __nv_bfloat16* __restrict__ q, __nv_bfloat16* __restrict__ kd,
                                   __nv_bfloat16* __restrict__ vd, long long stride, int B, int P, int H,
                                   int D) {
-    const int half = D / 2, secs = H + 2;
-    const long long total = (long long)B * P * secs * half;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const int j = (int)(idx % half);
-        const int s = (int)((idx / half) % secs);
-        const long long r = idx / ((long long)half * secs);   // b P + p
+    const int half = D / 2, secs = H + 2, slots = secs * half;
+    for (long long r = blockIdx.x; r < (long long)B * P; r += gridDim.x) {   // r = b P + p
         const int p = (int)(r % P), b = (int)(r / P);
-        const float* src = qkv + r * (long long)secs * D + (long long)s * D;
-        float x1 = src[j], x2 = src[j + half];
-        if (s <= H) {
-            const float2 cs = rope[(size_t)p * half + j];
-            const float r1 = x1 * cs.x - x2 * cs.y, r2 = x2 * cs.x + x1 * cs.y;
-            x1 = r1;
-            x2 = r2;
+        const float* row = qkv + r * (long long)secs * D;
+        for (int t = threadIdx.x; t < slots; t += blockDim.x) {
+            const int s = t / half, j = t - s * half;
+            const float* src = row + s * D;
+            float x1 = src[j], x2 = src[j + half];
+            if (s <= H) {
+                const float2 cs = rope[(size_t)p * half + j];
+                const float r1 = x1 * cs.x - x2 * cs.y, r2 = x2 * cs.x + x1 * cs.y;
+                x1 = r1;
+                x2 = r2;
+            }
+            __nv_bfloat16* dst;
+            if (s < H) dst = q + (r * H + s) * (long long)D;
+            else dst = (s == H ? kd : vd) + b * stride + (long long)p * D;
+            dst[j] = __float2bfloat16_rn(x1);
+            dst[j + half] = __float2bfloat16_rn(x2);
         }
-        __nv_bfloat16* dst;
-        if (s < H) dst = q + (r * H + s) * (long long)D;
-        else dst = (s == H ? kd : vd) + b * stride + (long long)p * D;
-        dst[j] = __float2bfloat16_rn(x1);
-        dst[j + half] = __float2bfloat16_rn(x2);
     }
 }
 
@@ -214,76 +225,50 @@ __global__ void __launch_bounds__(256) k_pf_softmax(const float* __restrict__ s,
 
 // After a product split over K ranges: h += (part_0 + part_1 + ...) in range order (parts [rows][W]
 // fp32, `pstride` elements apart), then, when w is set, the next RMSNorm y = h / sqrt(mean(h^2) +
-// eps) * (1 + w) as k_pf_rmsnorm computes it. One warp per row; a row of up to RN_CAP float4 per
-// lane stays in registers (W a multiple of 4).
+// eps) * (1 + w) as k_pf_rmsnorm computes it.
 template <typename TO>
-__global__ void __launch_bounds__(256) k_pf_residual_norm(float* __restrict__ h, const float* __restrict__ parts,
-                                                          int nparts, long long pstride, const float* __restrict__ w,
-                                                          TO* __restrict__ y, long long rows, int W, float eps) {
-    const int lane = threadIdx.x & 31;
-    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
-    const int n4 = W >> 2;
-    const float4* w4 = reinterpret_cast<const float4*>(w);
-    for (long long r = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += nwarps) {
+__global__ void __launch_bounds__(RB) k_pf_residual_norm(float* __restrict__ h, const float* __restrict__ parts,
+                                                         int nparts, long long pstride, const float* __restrict__ w,
+                                                         TO* __restrict__ y, long long rows, int W, float eps) {
+    __shared__ float red[RB / 32];
+    const int t = threadIdx.x, n4 = W >> 2;
+    for (long long r = blockIdx.x; r < rows; r += gridDim.x) {
         float4* hr = reinterpret_cast<float4*>(h + r * W);
+        // h + (part_0 + part_1 + ...) for float4 i.
         auto update = [&](int i) {
             float4 d = reinterpret_cast<const float4*>(parts + r * W)[i];
             for (int q = 1; q < nparts; ++q) {
                 const float4 e = reinterpret_cast<const float4*>(parts + (size_t)q * pstride + r * W)[i];
-                d.x += e.x;
-                d.y += e.y;
-                d.z += e.z;
-                d.w += e.w;
+                d = make_float4(d.x + e.x, d.y + e.y, d.z + e.z, d.w + e.w);
             }
-            float4 v = hr[i];
-            v.x += d.x;
-            v.y += d.y;
-            v.z += d.z;
-            v.w += d.w;
+            const float4 o = hr[i];
+            const float4 v = make_float4(o.x + d.x, o.y + d.y, o.z + d.z, o.w + d.w);
             hr[i] = v;
             return v;
         };
-        auto store4 = [&](int i, float4 v, float rinv) {
-            const float4 g = w4[i];
-            const float a0 = v.x * rinv * (1.f + g.x), a1 = v.y * rinv * (1.f + g.y);
-            const float a2 = v.z * rinv * (1.f + g.z), a3 = v.w * rinv * (1.f + g.w);
-            if constexpr (sizeof(TO) == 2) {
-                const __nv_bfloat162 lo = __floats2bfloat162_rn(a0, a1), hi = __floats2bfloat162_rn(a2, a3);
-                uint2 u;
-                u.x = *reinterpret_cast<const uint32_t*>(&lo);
-                u.y = *reinterpret_cast<const uint32_t*>(&hi);
-                *reinterpret_cast<uint2*>(y + r * W + 4 * i) = u;
-            } else {
-                *reinterpret_cast<float4*>(y + r * W + 4 * i) = make_float4(a0, a1, a2, a3);
-            }
-        };
-        if (n4 <= 32 * RN_CAP) {
+        if (n4 <= RB * RB_CAP) {
             // Passes over the row held in registers: part 0, each further part, then h.
-            float4 v[RN_CAP];
-            float s = 0.f;
+            float4 v[RB_CAP];
             const float4* p0 = reinterpret_cast<const float4*>(parts + r * W);
 #pragma unroll
-            for (int k = 0; k < RN_CAP; ++k) {
-                const int i = lane + 32 * k;
+            for (int k = 0; k < RB_CAP; ++k) {
+                const int i = t + RB * k;
                 v[k] = i < n4 ? p0[i] : make_float4(0.f, 0.f, 0.f, 0.f);
             }
             for (int q = 1; q < nparts; ++q) {
                 const float4* pq = reinterpret_cast<const float4*>(parts + (size_t)q * pstride + r * W);
 #pragma unroll
-                for (int k = 0; k < RN_CAP; ++k) {
-                    const int i = lane + 32 * k;
+                for (int k = 0; k < RB_CAP; ++k) {
+                    const int i = t + RB * k;
                     if (i < n4) {
                         const float4 e = pq[i];
-                        v[k].x += e.x;
-                        v[k].y += e.y;
-                        v[k].z += e.z;
-                        v[k].w += e.w;
+                        v[k] = make_float4(v[k].x + e.x, v[k].y + e.y, v[k].z + e.z, v[k].w + e.w);
                     }
                 }
             }
 #pragma unroll
-            for (int k = 0; k < RN_CAP; ++k) {
-                const int i = lane + 32 * k;
+            for (int k = 0; k < RB_CAP; ++k) {
+                const int i = t + RB * k;
                 if (i < n4) {
                     const float4 o = hr[i];
                     v[k] = make_float4(o.x + v[k].x, o.y + v[k].y, o.z + v[k].z, o.w + v[k].w);
@@ -291,23 +276,21 @@ __global__ void __launch_bounds__(256) k_pf_residual_norm(float* __restrict__ h,
                 }
             }
             if (!w) continue;
+            float s = 0.f;
 #pragma unroll
-            for (int k = 0; k < RN_CAP; ++k) s += (v[k].x * v[k].x + v[k].y * v[k].y) + (v[k].z * v[k].z + v[k].w * v[k].w);
-            const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
+            for (int k = 0; k < RB_CAP; ++k) s += sq4(v[k]);
+            const float rinv = 1.f / sqrtf(block_sum_rb(s, red) / (float)W + eps);
 #pragma unroll
-            for (int k = 0; k < RN_CAP; ++k) {
-                const int i = lane + 32 * k;
-                if (i < n4) store4(i, v[k], rinv);
+            for (int k = 0; k < RB_CAP; ++k) {
+                const int i = t + RB * k;
+                if (i < n4) store_normed4(y, w, r, W, i, v[k], rinv);
             }
         } else {
             float s = 0.f;
-            for (int i = lane; i < n4; i += 32) {
-                const float4 v = update(i);
-                s += (v.x * v.x + v.y * v.y) + (v.z * v.z + v.w * v.w);
-            }
+            for (int i = t; i < n4; i += RB) s += sq4(update(i));
             if (!w) continue;
-            const float rinv = 1.f / sqrtf(warp_sum(s) / (float)W + eps);
-            for (int i = lane; i < n4; i += 32) store4(i, hr[i], rinv);
+            const float rinv = 1.f / sqrtf(block_sum_rb(s, red) / (float)W + eps);
+            for (int i = t; i < n4; i += RB) store_normed4(y, w, r, W, i, hr[i], rinv);
         }
     }
 }
@@ -977,11 +960,11 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
         __nv_bfloat16* vd = static_cast<__nv_bfloat16*>(v_layers[l]);
         // Attention sublayer.
         if (!xn_ready) {
-            k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, lw.attn_norm, h->xn, M, W, eps);
+            k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M, 1, 16384), RB, 0, st>>>(h->h, lw.attn_norm, h->xn, M, W, eps);
             PF_CUDA(cudaGetLastError());
         }
         PF_TRY(row_gemm(h, st, h->xn, W, lw.wqkv, W, h->qkv, false, h->QKV, (int)M, h->QKV, W, 1.f, false));
-        k_pf_rope_scatter<<<grid_for(M * (H + 2) * (D / 2)), 256, 0, st>>>(h->qkv, h->rope, h->q, kd, vd,
+        k_pf_rope_scatter<<<grid_for(M, 1, 16384), 256, 0, st>>>(h->qkv, h->rope, h->q, kd, vd,
                                                                              request_stride, batch, P, H, D);
         PF_CUDA(cudaGetLastError());
         // Attention: on the tcgen05 attention kernel (scores and probabilities never leave the
@@ -1009,11 +992,11 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
         if (so > 1) {
             PF_TRY(row_gemm(h, st, h->o, H * D, lw.wo, H * D, h->part, false, W, (int)M, W, H * D, 1.f, false, so,
                             pstride));
-            k_pf_residual_norm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->part, so, pstride,
+            k_pf_residual_norm<__nv_bfloat16><<<grid_for(M, 1, 16384), RB, 0, st>>>(h->h, h->part, so, pstride,
                                                                                   lw.mlp_norm, h->xn, M, W, eps);
         } else {
             PF_TRY(row_gemm(h, st, h->o, H * D, lw.wo, H * D, h->h, false, W, (int)M, W, H * D, 1.f, true));
-            k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(h->h, lw.mlp_norm, h->xn, M, W, eps);
+            k_pf_rmsnorm<__nv_bfloat16><<<grid_for(M, 1, 16384), RB, 0, st>>>(h->h, lw.mlp_norm, h->xn, M, W, eps);
         }
         PF_CUDA(cudaGetLastError());
         // MLP sublayer: gate/up with GeGLU in its epilogue (z bf16), then down into the residual.
@@ -1022,21 +1005,21 @@ JPI_API jpi_status jpi_prefill_run(jpi_prefill_handle* h, const void* x, int x_i
         if (sd > 1) {
             PF_TRY(row_gemm(h, st, h->z, F, lw.wd, F, h->part, false, W, (int)M, W, F, 1.f, false, sd, pstride));
             if (l + 1 < h->L) {
-                k_pf_residual_norm<__nv_bfloat16><<<grid_for(M * 32), 256, 0, st>>>(
+                k_pf_residual_norm<__nv_bfloat16><<<grid_for(M, 1, 16384), RB, 0, st>>>(
                     h->h, h->part, sd, pstride, h->layers[(size_t)l + 1].attn_norm, h->xn, M, W, eps);
                 xn_ready = true;
             } else if (out_final) {
-                k_pf_residual_norm<float><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->part, sd, pstride,
+                k_pf_residual_norm<float><<<grid_for(M, 1, 16384), RB, 0, st>>>(h->h, h->part, sd, pstride,
                                                                             h->final_norm, out_final, M, W, eps);
             } else {
-                k_pf_residual_norm<float><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->part, sd, pstride, nullptr,
+                k_pf_residual_norm<float><<<grid_for(M, 1, 16384), RB, 0, st>>>(h->h, h->part, sd, pstride, nullptr,
                                                                             nullptr, M, W, eps);
             }
         } else {
             PF_TRY(row_gemm(h, st, h->z, F, lw.wd, F, h->h, false, W, (int)M, W, F, 1.f, true));
             xn_ready = false;
             if (l + 1 == h->L && out_final)
-                k_pf_rmsnorm<float><<<grid_for(M * 32), 256, 0, st>>>(h->h, h->final_norm, out_final, M, W, eps);
+                k_pf_rmsnorm<float><<<grid_for(M, 1, 16384), RB, 0, st>>>(h->h, h->final_norm, out_final, M, W, eps);
         }
         PF_CUDA(cudaGetLastError());
     }
