@@ -19,6 +19,7 @@
 // 2 H T' T d_vlm * 2 FLOPs per request instead of the 4 T d_vlm d of projecting every token.
 
 #include "jpi_internal.h"
+#include "ptx.h"
 
 #include <map>
 #include <tuple>
@@ -28,6 +29,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <new>
+#include <utility>
 
 namespace {
 
@@ -89,6 +91,10 @@ struct LinArgs {
 
 template <typename TW, bool VEC>
 __global__ void __launch_bounds__(256) k_corr_linear(const LinArgs a) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     const int lane = threadIdx.x & 31;
     const int nwarps = (gridDim.x * blockDim.x) >> 5;
     const TW* W = static_cast<const TW*>(a.w);
@@ -143,6 +149,230 @@ __global__ void __launch_bounds__(256) k_corr_linear(const LinArgs a) {
     }
 }
 
+// The same product for bf16 weights with 16-byte aligned rows and 16-byte aligned activation rows
+// (in a multiple of 8 KS, ldx of 4): a lane streams 16-byte weight chunks, LIN_CH of them in
+// flight, and the KS consecutive warps of a block share an output feature, each over in / KS
+// inputs, their sums added in warp order through shared memory (deterministic). Blocks of
+// 8 / KS output features walk the outputs grid-stride.
+constexpr int LIN_CH = 8;
+template <int KS>
+__global__ void __launch_bounds__(256) k_corr_linear16(const LinArgs a) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
+    __shared__ float part[8][LIN_ROWS];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int slice = warp % KS, og = warp / KS;
+    constexpr int OPB = 8 / KS;
+    const int kper = a.in / KS, k0 = slice * kper;
+    const __nv_bfloat16* W = static_cast<const __nv_bfloat16*>(a.w);
+    const int ngroups = (a.out + OPB - 1) / OPB;
+    for (int gi = blockIdx.x; gi < ngroups; gi += gridDim.x) {
+        const int o = gi * OPB + og;
+        const bool live = o < a.out;
+        const int oc = live ? o : a.out - 1;   // clamped; result unused
+        const __nv_bfloat16* wr = W + (size_t)oc * a.in + k0;
+        const float bo = (a.bias && live) ? a.bias[oc] : 0.f;
+        for (int r0 = 0; r0 < a.rows; r0 += LIN_ROWS) {
+            const float* xr[LIN_ROWS];
+#pragma unroll
+            for (int k = 0; k < LIN_ROWS; ++k) {
+                const int r = r0 + k < a.rows ? r0 + k : a.rows - 1;   // clamped; result unused
+                long long row = r;
+                if (a.hs_items > 0)
+                    row = ((long long)(r / a.hs_items) * a.hs_heads + oc / a.hs_dh) * a.hs_items + r % a.hs_items;
+                xr[k] = a.x + row * a.ldx + k0;
+            }
+            float acc[LIN_ROWS];
+#pragma unroll
+            for (int k = 0; k < LIN_ROWS; ++k) acc[k] = 0.f;
+            for (int base = 0; base < kper; base += 256 * LIN_CH) {
+                uint4 wv[LIN_CH];
+#pragma unroll
+                for (int j = 0; j < LIN_CH; ++j) {
+                    const int i = base + 256 * j + 8 * lane;
+                    wv[j] = i < kper ? __ldg(reinterpret_cast<const uint4*>(wr + i)) : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int j = 0; j < LIN_CH; ++j) {
+                    const int i = base + 256 * j + 8 * lane;
+                    if (i < kper) {
+                        const uint32_t u[4] = {wv[j].x, wv[j].y, wv[j].z, wv[j].w};
+                        float w[8];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u[q]));
+                            w[2 * q] = f.x;
+                            w[2 * q + 1] = f.y;
+                        }
+#pragma unroll
+                        for (int k = 0; k < LIN_ROWS; ++k) {
+                            const float4 x0 = *reinterpret_cast<const float4*>(xr[k] + i);
+                            const float4 x1 = *reinterpret_cast<const float4*>(xr[k] + i + 4);
+                            float t = acc[k];
+                            t = fmaf(w[0], x0.x, t);
+                            t = fmaf(w[1], x0.y, t);
+                            t = fmaf(w[2], x0.z, t);
+                            t = fmaf(w[3], x0.w, t);
+                            t = fmaf(w[4], x1.x, t);
+                            t = fmaf(w[5], x1.y, t);
+                            t = fmaf(w[6], x1.z, t);
+                            t = fmaf(w[7], x1.w, t);
+                            acc[k] = t;
+                        }
+                    }
+                }
+            }
+            float mine = 0.f;   // lane k keeps row r0 + k
+#pragma unroll
+            for (int k = 0; k < LIN_ROWS; ++k) {
+                const float v = warp_sum(acc[k]);
+                if (lane == k) mine = v;
+            }
+            if (KS > 1) {
+                if (lane < LIN_ROWS) part[warp][lane] = mine;
+                __syncthreads();
+                if (slice == 0 && lane < LIN_ROWS) {
+                    float t = part[warp][lane];
+#pragma unroll
+                    for (int sl = 1; sl < KS; ++sl) t += part[warp + sl][lane];
+                    mine = t;
+                }
+                __syncthreads();   // part is reused by the next row group
+            }
+            const int r = r0 + lane;
+            if (slice == 0 && live && lane < LIN_ROWS && r < a.rows) {
+                float v = mine + bo;
+                if (a.gelu) v = gelu_tanh_f(v);
+                if (a.res) v += a.res[(size_t)r * a.ldr + o];
+                a.y[(size_t)r * a.ldy + o] = v;
+            }
+        }
+    }
+}
+
+// The same product streamed through shared memory, for bf16 weights (16-byte aligned, in a
+// multiple of 8 and at most LP_MAX_IN), 16-byte aligned activation rows (ldx a multiple of 4) and
+// no head-select: a persistent CTA walks groups of LP_ROWS consecutive output features; their
+// weight rows (contiguous) arrive by per-thread 16-byte cp.async copies into a ring of NST
+// stages, the first ones issued before the dependency wait (weights do not depend on the previous
+// kernel). Thread t takes the 8-column chunks t, t + 256, ... of the inputs for all LP_ROWS
+// features of a group, so each chunk of LP_XR activation rows it loads serves all of them (as
+// many activation bytes as weight bytes, where one warp per feature read LIN_ROWS activation
+// chunks per weight chunk and was bound by those L1 reads); the per-feature sums are reduced over
+// the block in a fixed order. No waits that can spin: the copies are waited with
+// cp.async.wait_group.
+constexpr int LP_ROWS = 8;
+constexpr int LP_XR = 4;          // activation rows per pass
+constexpr int LP_MAX_IN = 4096;
+__host__ __device__ constexpr int lp_stages(int in) {
+    return in <= 2048 ? 4 : 3;
+}
+template <int NST>
+__global__ void __launch_bounds__(256) k_corr_linear_pipe(const LinArgs a) {
+    extern __shared__ __align__(128) uint8_t lp_smem[];
+    __shared__ float red[8][LP_ROWS * LP_XR];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int in = a.in, nch = in / 8;
+    const int sbytes = LP_ROWS * in * 2;
+    const int ngroups = (a.out + LP_ROWS - 1) / LP_ROWS;
+    const uint8_t* W = static_cast<const uint8_t*>(a.w);
+    // Group k of this CTA: blockIdx.x + k gridDim.x; its rows into stage k mod NST (one commit
+    // group per k, empty past the last group, so the group count stays uniform).
+    auto issue = [&](int k) {
+        const int g = blockIdx.x + k * gridDim.x;
+        if (g < ngroups) {
+            const int rows = min(LP_ROWS, a.out - g * LP_ROWS);
+            const int chunks = rows * nch;
+            const uint8_t* src = W + (size_t)g * LP_ROWS * in * 2;
+            const uint32_t dst = jpi::ptx::smem_u32(lp_smem + (size_t)(k % NST) * sbytes);
+            for (int c = tid; c < chunks; c += 256) jpi::ptx::cp_async_16(dst + 16 * c, src + 16 * (size_t)c, true);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+#pragma unroll
+    for (int k = 0; k < NST - 1; ++k) issue(k);
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
+    for (int k = 0; blockIdx.x + k * gridDim.x < ngroups; ++k) {
+        issue(k + NST - 1);
+        asm volatile("cp.async.wait_group %0;" ::"n"(NST - 1) : "memory");
+        __syncthreads();   // stage k mod NST holds group k for every thread
+        const int o0 = (blockIdx.x + k * gridDim.x) * LP_ROWS;
+        const int nout = min(LP_ROWS, a.out - o0);
+        const uint4* wst = reinterpret_cast<const uint4*>(lp_smem + (size_t)(k % NST) * sbytes);
+        for (int r0 = 0; r0 < a.rows; r0 += LP_XR) {
+            const int nr = min(LP_XR, a.rows - r0);
+            float acc[LP_ROWS][LP_XR];
+#pragma unroll
+            for (int o = 0; o < LP_ROWS; ++o)
+#pragma unroll
+                for (int q = 0; q < LP_XR; ++q) acc[o][q] = 0.f;
+            for (int c = tid; c < nch; c += 256) {
+                float x[LP_XR][8];
+#pragma unroll
+                for (int q = 0; q < LP_XR; ++q) {
+                    float4 x0 = make_float4(0.f, 0.f, 0.f, 0.f), x1 = x0;
+                    if (q < nr) {
+                        const float* xr = a.x + (size_t)(r0 + q) * a.ldx + 8 * c;
+                        x0 = *reinterpret_cast<const float4*>(xr);
+                        x1 = *reinterpret_cast<const float4*>(xr + 4);
+                    }
+                    x[q][0] = x0.x; x[q][1] = x0.y; x[q][2] = x0.z; x[q][3] = x0.w;
+                    x[q][4] = x1.x; x[q][5] = x1.y; x[q][6] = x1.z; x[q][7] = x1.w;
+                }
+#pragma unroll
+                for (int o = 0; o < LP_ROWS; ++o) {
+                    if (o >= nout) break;
+                    const uint4 wv = wst[(size_t)o * nch + c];
+                    const uint32_t u[4] = {wv.x, wv.y, wv.z, wv.w};
+                    float w[8];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u[e]));
+                        w[2 * e] = f.x;
+                        w[2 * e + 1] = f.y;
+                    }
+#pragma unroll
+                    for (int q = 0; q < LP_XR; ++q) {
+                        float t = acc[o][q];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) t = fmaf(w[e], x[q][e], t);
+                        acc[o][q] = t;
+                    }
+                }
+            }
+            // (feature o, row q) sums: over the warp's lanes, then over the 8 warps in order.
+            float mine = 0.f;   // lane o * LP_XR + q keeps pair (o, q)
+#pragma unroll
+            for (int o = 0; o < LP_ROWS; ++o)
+#pragma unroll
+                for (int q = 0; q < LP_XR; ++q) {
+                    const float v = warp_sum(acc[o][q]);
+                    if (lane == o * LP_XR + q) mine = v;
+                }
+            red[warp][lane] = mine;
+            __syncthreads();
+            if (tid < LP_ROWS * LP_XR) {
+                const int o = tid / LP_XR, q = tid % LP_XR;
+                float v = 0.f;
+#pragma unroll
+                for (int w8 = 0; w8 < 8; ++w8) v += red[w8][tid];
+                const int of = o0 + o, r = r0 + q;
+                if (o < nout && q < nr) {
+                    v += a.bias ? a.bias[of] : 0.f;
+                    if (a.gelu) v = gelu_tanh_f(v);
+                    if (a.res) v += a.res[(size_t)r * a.ldr + of];
+                    a.y[(size_t)r * a.ldy + of] = v;
+                }
+            }
+            __syncthreads();   // red is reused by the next pass
+        }
+    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");   // nothing lands after exit
+}
+
 // LayerNorm of `rows` rows of width d: one warp per row (grid-stride over rows), three passes
 // (mean, biased variance, output). VEC: every row and vector 16-byte aligned, d a multiple of 4,
 // so the passes move float4s.
@@ -152,6 +382,10 @@ __global__ void __launch_bounds__(256) k_corr_layernorm(const float* __restrict_
                                                         const float* __restrict__ b,
                                                         float* __restrict__ y, int ldy, int rows,
                                                         int d, float eps) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     const int lane = threadIdx.x & 31, nwarps = (int)((gridDim.x * blockDim.x) >> 5);
     for (int r = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); r < rows; r += nwarps) {
         const float* xr = x + (size_t)r * ldx;
@@ -214,6 +448,10 @@ struct AttnSmallArgs {
 };
 
 __global__ void __launch_bounds__(256) k_corr_attn(const AttnSmallArgs a) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     __shared__ float sp[8][JPI_CORR_MAX_DELTA];
     const int wib = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int gw = blockIdx.x * 8 + wib;
@@ -275,6 +513,10 @@ template <typename TW>
 __global__ void __launch_bounds__(256) k_corr_qk(const float* __restrict__ qc, const TW* __restrict__ wk,
                                                  float* __restrict__ qk, int T, int Dh, int d, int dv,
                                                  float scale) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     __shared__ float qs[JPI_MAX_CORRECTION][256];
     const int h = blockIdx.y, c = blockIdx.x * 256 + threadIdx.x;
     for (int idx = threadIdx.x; idx < T * Dh; idx += 256)
@@ -308,6 +550,10 @@ constexpr size_t CORR_SCORES_SMEM = (size_t)(CORR_MAX_M + 32) * CORR_KPAD * size
 template <typename THV>
 __global__ void __launch_bounds__(256) k_corr_scores(const float* __restrict__ qk, const THV* __restrict__ hv,
                                                      float* __restrict__ part, int M, int T, int dv) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     extern __shared__ float sm_scores[];
     float* as = sm_scores;                       // [M][CORR_KPAD]
     float* bs = sm_scores + CORR_MAX_M * CORR_KPAD;   // [32][CORR_KPAD]
@@ -372,6 +618,10 @@ __device__ __forceinline__ float block_sum256(float v, float* red) {
 // order, then the softmax over its n tokens, written to s[r][.].
 __global__ void __launch_bounds__(256) k_corr_softmax_sum(const float* __restrict__ part, float* __restrict__ s,
                                                           int M, int n, int nkc) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     __shared__ float red[8];
     const int r = blockIdx.x, b = r / M, m = r - b * M;
     const float* p0 = part + ((size_t)b * nkc * M + m) * n;
@@ -403,6 +653,10 @@ constexpr int CORR_TCHUNK = 64;
 template <typename THV>
 __global__ void __launch_bounds__(256) k_corr_wsum(const float* __restrict__ p, const THV* __restrict__ hv,
                                                    float* __restrict__ part, int M, int T, int dv) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     __shared__ float ps[CORR_MAX_M][CORR_TCHUNK];
     const int b = blockIdx.z, tc = blockIdx.y, c = blockIdx.x * 256 + threadIdx.x;
     const int j0 = tc * CORR_TCHUNK, jn = min(CORR_TCHUNK, T - j0);
@@ -437,6 +691,10 @@ __global__ void __launch_bounds__(256) k_corr_wsum(const float* __restrict__ p, 
 // g[b][m][c] = the ntc token-chunk partials added in order.
 __global__ void k_corr_wsum_reduce(const float* __restrict__ part, float* __restrict__ g, int B, int M, int dv,
                                    int ntc) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     const long long total = (long long)B * M * dv;
     for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
          idx += (long long)gridDim.x * blockDim.x) {
@@ -450,6 +708,10 @@ __global__ void k_corr_wsum_reduce(const float* __restrict__ part, float* __rest
 
 // y[(b n + k)][c] += pos[k][c] for b < B, k < n, c < d.
 __global__ void k_corr_add_pos(float* __restrict__ y, const float* __restrict__ pos, int B, int n, int d) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     const long long total = (long long)B * n * d;
     for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
          idx += (long long)gridDim.x * blockDim.x) {
@@ -462,6 +724,10 @@ __global__ void k_corr_add_pos(float* __restrict__ y, const float* __restrict__ 
 // xj[(b T' + i)][0 .. d) = state[b][i][.], xj[(b T' + i)][d .. 2d) = summary[b][.].
 __global__ void k_corr_join(const float* __restrict__ state, const float* __restrict__ summary,
                             float* __restrict__ xj, int B, int T, int d) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     const long long total = (long long)B * T * 2 * d;
     for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
          idx += (long long)gridDim.x * blockDim.x) {
@@ -476,6 +742,10 @@ __global__ void k_corr_join(const float* __restrict__ state, const float* __rest
 __global__ void __launch_bounds__(256) k_corr_confidence(const float* __restrict__ u, const float* __restrict__ w,
                                                          const float* __restrict__ bias, float* __restrict__ conf,
                                                          int T, int d) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     __shared__ float red[8];
     const int b = blockIdx.x;
     float s = 0.f;
@@ -497,6 +767,10 @@ __global__ void k_corr_cast(const float* __restrict__ src, __nv_bfloat16* __rest
 // dst[r n + i] = src[i] for r < reps, i < n. src may be the start of dst: the first n elements are
 // rewritten with their own values.
 __global__ void k_corr_repeat(const float* src, float* dst, long long n, int reps) {
+    // Launched with programmatic dependent launch: wait for the previous kernel's results, then
+    // let the next kernel's CTAs be scheduled (they wait in turn).
+    jpi::ptx::grid_dep_wait();
+    jpi::ptx::grid_dep_launch();
     const long long total = n * reps;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x)
@@ -529,6 +803,7 @@ struct BlockDev {
 struct jpi_corr_handle {
     jpi_corr_config cfg;
     bool bf16 = true;
+    int num_sms = 0;   // persistent CTAs of the streamed products
     int d = 0, H = 0, Dh = 0, F = 0, dv = 0, Ti = 0, A = 0, Dm = 0, J = 0, B = 0, Tm = 0, M = 0;
     std::vector<void*> allocs;
     size_t bytes = 0;
@@ -682,6 +957,24 @@ jpi_status put_block(jpi_corr_handle* h, bool dev, BlockDev* out, const jpi_corr
 
 // ---------------------------------------------------------------- launchers
 
+// Every kernel of a call is launched with programmatic dependent launch (each waits for its
+// predecessor at its start), so in the captured graph a kernel's launch overlaps the previous
+// kernel's tail. A failed launch leaves its error for the cudaGetLastError check that follows.
+template <typename... KArgs, typename... Args>
+void pdl(cudaStream_t st, dim3 grid, dim3 block, size_t smem, void (*k)(KArgs...), Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at;
+    at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &at;
+    cfg.numAttrs = 1;
+    (void)cudaLaunchKernelEx(&cfg, k, std::forward<Args>(args)...);
+}
+
 jpi_status linear(const jpi_corr_handle* h, cudaStream_t st, const float* x, int ldx, const void* w,
                   const float* bias, const float* res, int ldr, float* y, int ldy, int rows, int in,
                   int out, bool gelu, int hs_items = 0) {
@@ -704,13 +997,39 @@ jpi_status linear(const jpi_corr_handle* h, cudaStream_t st, const float* x, int
     a.hs_dh = h->Dh;
     const bool vec = in % 4 == 0 && ldx % 4 == 0 && ((uintptr_t)x & 15) == 0 &&
                      ((uintptr_t)w & (h->bf16 ? 7 : 15)) == 0;
+    // bf16 rows of 16-byte chunks up to LP_MAX_IN, no head-select: streamed through shared memory
+    // by persistent CTAs, one per SM at most.
+    if (h->bf16 && hs_items == 0 && in % 8 == 0 && in <= LP_MAX_IN && ldx % 4 == 0 && ((uintptr_t)x & 15) == 0 &&
+        ((uintptr_t)w & 15) == 0) {
+        const int groups = (out + LP_ROWS - 1) / LP_ROWS;
+        const int nb = groups < h->num_sms ? groups : h->num_sms;
+        const int nst = lp_stages(in);
+        const size_t smem = (size_t)nst * LP_ROWS * in * 2;
+        if (nst == 4) pdl(st, dim3(nb), dim3(256), smem, k_corr_linear_pipe<4>, a);
+        else pdl(st, dim3(nb), dim3(256), smem, k_corr_linear_pipe<3>, a);
+        JPI_CUDA_TRY(cudaGetLastError());
+        return JPI_OK;
+    }
+    // Other bf16 rows of 16-byte chunks: the streaming kernel, with 2 or 4 warps per output
+    // feature while that keeps at least 256 inputs a warp and brings the launch towards 2048 warps.
+    if (h->bf16 && in % 8 == 0 && ldx % 4 == 0 && ((uintptr_t)x & 15) == 0 && ((uintptr_t)w & 15) == 0) {
+        int ks = 1;
+        while (ks < 4 && (long long)out * ks < 2048 && in % (16 * ks) == 0 && in / (2 * ks) >= 256) ks *= 2;
+        const int groups = (out + 8 / ks - 1) / (8 / ks);
+        const int nb = groups < 4096 ? groups : 4096;
+        if (ks == 4) pdl(st, dim3(nb), dim3(256), 0, k_corr_linear16<4>, a);
+        else if (ks == 2) pdl(st, dim3(nb), dim3(256), 0, k_corr_linear16<2>, a);
+        else pdl(st, dim3(nb), dim3(256), 0, k_corr_linear16<1>, a);
+        JPI_CUDA_TRY(cudaGetLastError());
+        return JPI_OK;
+    }
     const int blocks = grid_for((long long)out * 32, 256, 4096);
     if (h->bf16) {
-        if (vec) k_corr_linear<__nv_bfloat16, true><<<blocks, 256, 0, st>>>(a);
-        else k_corr_linear<__nv_bfloat16, false><<<blocks, 256, 0, st>>>(a);
+        if (vec) pdl(st, dim3(blocks), dim3(256), 0, k_corr_linear<__nv_bfloat16, true>, a);
+        else pdl(st, dim3(blocks), dim3(256), 0, k_corr_linear<__nv_bfloat16, false>, a);
     } else {
-        if (vec) k_corr_linear<float, true><<<blocks, 256, 0, st>>>(a);
-        else k_corr_linear<float, false><<<blocks, 256, 0, st>>>(a);
+        if (vec) pdl(st, dim3(blocks), dim3(256), 0, k_corr_linear<float, true>, a);
+        else pdl(st, dim3(blocks), dim3(256), 0, k_corr_linear<float, false>, a);
     }
     JPI_CUDA_TRY(cudaGetLastError());
     return JPI_OK;
@@ -722,10 +1041,10 @@ jpi_status layernorm(const jpi_corr_handle* h, cudaStream_t st, const float* x, 
     const bool vec = h->d % 4 == 0 && ldx % 4 == 0 && ldy % 4 == 0 &&
                      (((uintptr_t)x | (uintptr_t)y | (uintptr_t)g | (uintptr_t)b) & 15) == 0;
     if (vec)
-        k_corr_layernorm<true><<<grid_for((long long)rows * 32), 256, 0, st>>>(x, ldx, g, b, y, ldy, rows, h->d,
+        pdl(st, dim3(grid_for((long long)rows * 32)), dim3(256), 0, k_corr_layernorm<true>, x, ldx, g, b, y, ldy, rows, h->d,
                                                                            h->cfg.ln_eps);
     else
-        k_corr_layernorm<false><<<grid_for((long long)rows * 32), 256, 0, st>>>(x, ldx, g, b, y, ldy, rows, h->d,
+        pdl(st, dim3(grid_for((long long)rows * 32)), dim3(256), 0, k_corr_layernorm<false>, x, ldx, g, b, y, ldy, rows, h->d,
                                                                             h->cfg.ln_eps);
     JPI_CUDA_TRY(cudaGetLastError());
     return JPI_OK;
@@ -749,7 +1068,7 @@ jpi_status attention(const jpi_corr_handle* h, cudaStream_t st, const float* q, 
     a.Dh = h->Dh;
     a.scale = 1.f / sqrtf((float)h->Dh);
     const long long warps = (long long)B * h->H * nq;
-    k_corr_attn<<<(int)((warps + 7) / 8), 256, 0, st>>>(a);
+    pdl(st, dim3((int)((warps + 7) / 8)), dim3(256), 0, k_corr_attn, a);
     JPI_CUDA_TRY(cudaGetLastError());
     return JPI_OK;
 }
@@ -781,14 +1100,14 @@ jpi_status prepare(jpi_corr_handle* h, cudaStream_t st) {
     const dim3 grid((unsigned)((h->dv + 255) / 256), (unsigned)h->H);
     const float scale = 1.f / sqrtf((float)h->Dh);
     if (h->bf16)
-        k_corr_qk<__nv_bfloat16><<<grid, 256, 0, st>>>(h->o, static_cast<const __nv_bfloat16*>(h->qf_ca_wk),
+        pdl(st, dim3(grid), dim3(256), 0, k_corr_qk<__nv_bfloat16>, h->o, static_cast<const __nv_bfloat16*>(h->qf_ca_wk),
                                                         h->qk, T, h->Dh, d, h->dv, scale);
     else
-        k_corr_qk<float><<<grid, 256, 0, st>>>(h->o, static_cast<const float*>(h->qf_ca_wk), h->qk, T, h->Dh,
+        pdl(st, dim3(grid), dim3(256), 0, k_corr_qk<float>, h->o, static_cast<const float*>(h->qf_ca_wk), h->qk, T, h->Dh,
                                                d, h->dv, scale);
     JPI_CUDA_TRY(cudaGetLastError());
     const long long n = (long long)T * d;
-    k_corr_repeat<<<grid_for(n * h->B), 256, 0, st>>>(h->x1b, h->x1b, n, h->B);
+    pdl(st, dim3(grid_for(n * h->B)), dim3(256), 0, k_corr_repeat, h->x1b, h->x1b, n, h->B);
     JPI_CUDA_TRY(cudaGetLastError());
     return JPI_OK;
 }
@@ -919,6 +1238,15 @@ jpi_status setup(jpi_corr_handle* h, const jpi_corr_config* c, const jpi_corr_we
                                       (int)CORR_SCORES_SMEM));
     JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       (int)CORR_SCORES_SMEM));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_linear_pipe<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      4 * LP_ROWS * 2048 * 2));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_linear_pipe<3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      3 * LP_ROWS * LP_MAX_IN * 2));
+    {
+        int dev = 0;
+        JPI_CUDA_TRY(cudaGetDevice(&dev));
+        JPI_CUDA_TRY(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev));
+    }
     JPI_TRY(corr_alloc(h, &h->conf_scratch, B));
 
     JPI_TRY(prepare(h, nullptr));
@@ -940,16 +1268,16 @@ jpi_status enqueue_compress(jpi_corr_handle* h, const void* hvlm, int vlm_is_fp3
     const int red_grid = grid_for((long long)batch * M * dv);
     if (vlm_is_fp32) {
         const float* hv = static_cast<const float*>(hvlm);
-        k_corr_scores<float><<<gs, 256, CORR_SCORES_SMEM, st>>>(h->qk, hv, h->scp, M, n_tokens, dv);
-        k_corr_softmax_sum<<<batch * M, 256, 0, st>>>(h->scp, h->sc, M, n_tokens, nkc);
-        k_corr_wsum<float><<<gw, 256, 0, st>>>(h->sc, hv, h->gsp, M, n_tokens, dv);
+        pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<float>, h->qk, hv, h->scp, M, n_tokens, dv);
+        pdl(st, dim3(batch * M), dim3(256), 0, k_corr_softmax_sum, h->scp, h->sc, M, n_tokens, nkc);
+        pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<float>, h->sc, hv, h->gsp, M, n_tokens, dv);
     } else {
         const __nv_bfloat16* hv = static_cast<const __nv_bfloat16*>(hvlm);
-        k_corr_scores<__nv_bfloat16><<<gs, 256, CORR_SCORES_SMEM, st>>>(h->qk, hv, h->scp, M, n_tokens, dv);
-        k_corr_softmax_sum<<<batch * M, 256, 0, st>>>(h->scp, h->sc, M, n_tokens, nkc);
-        k_corr_wsum<__nv_bfloat16><<<gw, 256, 0, st>>>(h->sc, hv, h->gsp, M, n_tokens, dv);
+        pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<__nv_bfloat16>, h->qk, hv, h->scp, M, n_tokens, dv);
+        pdl(st, dim3(batch * M), dim3(256), 0, k_corr_softmax_sum, h->scp, h->sc, M, n_tokens, nkc);
+        pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<__nv_bfloat16>, h->sc, hv, h->gsp, M, n_tokens, dv);
     }
-    k_corr_wsum_reduce<<<red_grid, 256, 0, st>>>(h->gsp, h->gs, batch, M, dv, ntc);
+    pdl(st, dim3(red_grid), dim3(256), 0, k_corr_wsum_reduce, h->gsp, h->gs, batch, M, dv, ntc);
     JPI_CUDA_TRY(cudaGetLastError());
     // out_hi = W_v,h g_hi + b_v (head-select rows of gs), then the output projection onto the
     // queries' residual, the MLP, and the output LayerNorm.
@@ -970,7 +1298,7 @@ jpi_status enqueue_predict(jpi_corr_handle* h, const float* state, const float* 
     // Action tokens: MLP, plus the position row of each action.
     JPI_TRY(linear(h, st, actions, h->A, h->act_w1, h->act_b1, nullptr, 0, h->t1, d, ra, h->A, d, true));
     JPI_TRY(linear(h, st, h->t1, d, h->act_w2, h->act_b2, nullptr, 0, h->xa, d, ra, d, d, false));
-    k_corr_add_pos<<<grid_for((long long)ra * d), 256, 0, st>>>(h->xa, h->act_pos, batch, delta, d);
+    pdl(st, dim3(grid_for((long long)ra * d)), dim3(256), 0, k_corr_add_pos, h->xa, h->act_pos, batch, delta, d);
     JPI_CUDA_TRY(cudaGetLastError());
     // Block ab, kept at the last action of each request only: keys and values of every action,
     // the query, attention output, residual and MLP of the last.
@@ -985,14 +1313,14 @@ jpi_status enqueue_predict(jpi_corr_handle* h, const float* state, const float* 
     JPI_TRY(linear(h, st, h->ul, d, ab.w1, ab.b1, nullptr, 0, h->hidl, F, batch, d, F, true));
     JPI_TRY(linear(h, st, h->hidl, F, ab.w2, ab.b2, h->xl, d, h->xl, d, batch, F, d, false));
     // Join: [compressed token ; action summary] projected back to the module width.
-    k_corr_join<<<grid_for((long long)rows * 2 * d), 256, 0, st>>>(state, h->xl, h->xj, batch, T, d);
+    pdl(st, dim3(grid_for((long long)rows * 2 * d)), dim3(256), 0, k_corr_join, state, h->xl, h->xj, batch, T, d);
     JPI_CUDA_TRY(cudaGetLastError());
     JPI_TRY(linear(h, st, h->xj, 2 * d, h->fuse_w, h->fuse_b, nullptr, 0, h->xf, d, rows, 2 * d, d, false));
     for (int i = 0; i < h->J; ++i) JPI_TRY(block(h, st, h->jb[(size_t)i], h->xf, batch, T));
     // Heads.
     JPI_TRY(layernorm(h, st, h->xf, d, h->head_ln_w, h->head_ln_b, h->u, d, rows));
     JPI_TRY(linear(h, st, h->u, d, h->corr_w, h->corr_b, nullptr, 0, out, d, rows, d, d, false));
-    k_corr_confidence<<<batch, 256, 0, st>>>(h->u, h->conf_w, h->conf_b, conf, T, d);
+    pdl(st, dim3(batch), dim3(256), 0, k_corr_confidence, h->u, h->conf_w, h->conf_b, conf, T, d);
     JPI_CUDA_TRY(cudaGetLastError());
     return JPI_OK;
 }
