@@ -283,31 +283,85 @@ jpi_status launch_gemm(jpi_handle* h, const GemmPlan& pl, const CUtensorMap& wma
     return JPI_OK;
 }
 
-// Large-M variant: grid (weight tiles, 128-row operand tiles), no cluster, full K per CTA.
-template <int KIND>
-jpi_status launch_gemm_big(jpi_handle* h, const GemmPlan& pl, const CUtensorMap& wmap,
-                           const CUtensorMap& xmap, const GemmArgs& a, cudaStream_t st) {
-    constexpr int TT = (KIND == G_QKV || KIND == G_GU) ? 2 * XS_TOKENS : BIG_NT;
-    // Persistent: one CTA per SM (at most one per tile).
-    const int total = pl.ntiles * std::max(1, (a.Mt + TT - 1) / TT);
-    GemmArgs ab = a;
-    ab.ntiles = pl.ntiles;
+// Large-M variant: persistent CTAs over (weight tile, 128-row operand tile) units. The residual
+// kinds (few weight tiles, long K) may split each unit's K range over a cluster of S CTAs so that
+// the units fill the GPU: S is the one of 1, 2, 4, 8 with the fewest estimated K blocks per SM,
+// counting waves of S x units CTAs and an exchange worth BIG_SPLIT_COST K blocks for S > 1.
+constexpr int BIG_SPLIT_COST = 4;
+
+// Clusters of S large-M CTAs that can run at once (one CTA per SM; clusters of 8 leave some SMs
+// of each GPC idle), from the occupancy query at prepare time.
+int big_clusters(const jpi_handle* h, int S) {
+    const int i = S == 1 ? 0 : S == 2 ? 1 : S == 4 ? 2 : 3;
+    return h->big_clusters[i] > 0 ? h->big_clusters[i] : h->num_sms / S;
+}
+
+int big_split(const jpi_handle* h, int kind, int units, int nkb) {
+    if (kind != G_O && kind != G_DOWN) return 1;
+    if (h->big_split > 0) return nkb % h->big_split == 0 ? h->big_split : 1;
+    int best = 1;
+    long best_cost = -1;
+    for (int S = 1; S <= 8; S *= 2) {
+        if (nkb % S || nkb / S < 2) continue;
+        const long waves = (units + big_clusters(h, S) - 1) / big_clusters(h, S);
+        const long cost = waves * (nkb / S + (S > 1 ? BIG_SPLIT_COST : 0));
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = S;
+        }
+    }
+    return best;
+}
+
+template <int KIND, int S>
+jpi_status launch_big_s(jpi_handle* h, int units, const CUtensorMap& wmap, const CUtensorMap& xmap,
+                        const GemmArgs& a, cudaStream_t st) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)std::min(total, h->num_sms));
+    // Persistent: one CTA per SM (clusters of S that all run at once, at most one per unit).
+    cfg.gridDim = dim3((unsigned)(S * std::min(units, big_clusters(h, S))));
     cfg.blockDim = dim3(BIG_THREADS);
-    cfg.dynamicSmemBytes = 1024 + big_smem_bytes();
+    cfg.dynamicSmemBytes = 1024 + big_smem_bytes<S>();
     cfg.stream = st;
-    cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr.val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = &attr;
-    cfg.numAttrs = h->pdl ? 1 : 0;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_big<KIND>, wmap, xmap, ab);
+    cudaLaunchAttribute attrs[2];
+    int n = 0;
+    if (S > 1) {
+        attrs[n].id = cudaLaunchAttributeClusterDimension;
+        attrs[n].val.clusterDim.x = S;
+        attrs[n].val.clusterDim.y = 1;
+        attrs[n].val.clusterDim.z = 1;
+        ++n;
+    }
+    if (h->pdl) {
+        attrs[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attrs[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    cfg.attrs = attrs;
+    cfg.numAttrs = n;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm_big<KIND, S>, wmap, xmap, a);
     if (e != cudaSuccess) {
         set_error("tensor-core GEMM launch failed: %s", cudaGetErrorString(e));
         return JPI_ERR_CUDA;
     }
     return JPI_OK;
+}
+
+template <int KIND>
+jpi_status launch_gemm_big(jpi_handle* h, const GemmPlan& pl, const CUtensorMap& wmap,
+                           const CUtensorMap& xmap, const GemmArgs& a, cudaStream_t st) {
+    constexpr int TT = (KIND == G_QKV || KIND == G_GU) ? 2 * XS_TOKENS : BIG_NT;
+    const int units = pl.ntiles * std::max(1, (a.Mt + TT - 1) / TT);
+    GemmArgs ab = a;
+    ab.ntiles = pl.ntiles;
+    if constexpr (KIND == G_O || KIND == G_DOWN) {
+        switch (big_split(h, KIND, units, pl.nkb)) {
+            case 2: return launch_big_s<KIND, 2>(h, units, wmap, xmap, ab, st);
+            case 4: return launch_big_s<KIND, 4>(h, units, wmap, xmap, ab, st);
+            case 8: return launch_big_s<KIND, 8>(h, units, wmap, xmap, ab, st);
+            default: break;
+        }
+    }
+    return launch_big_s<KIND, 1>(h, units, wmap, xmap, ab, st);
 }
 
 GemmArgs base_args(jpi_handle* h, int B, int C, const GemmPlan& pl) {
@@ -408,9 +462,43 @@ jpi_status tc_prepare(jpi_handle* h) {
         }
         JPI_CUDA_TRY(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024));
     }
-    auto big_kernels = {k_tc_gemm_big<G_QKV>, k_tc_gemm_big<G_O>, k_tc_gemm_big<G_GU>, k_tc_gemm_big<G_DOWN>};
-    for (auto k : big_kernels)
-        JPI_CUDA_TRY(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes()));
+    auto big1 = {k_tc_gemm_big<G_QKV, 1>, k_tc_gemm_big<G_O, 1>, k_tc_gemm_big<G_GU, 1>, k_tc_gemm_big<G_DOWN, 1>};
+    for (auto k : big1)
+        JPI_CUDA_TRY(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes<1>()));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_tc_gemm_big<G_O, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes<2>()));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_tc_gemm_big<G_DOWN, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes<2>()));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_tc_gemm_big<G_O, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes<4>()));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_tc_gemm_big<G_DOWN, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes<4>()));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_tc_gemm_big<G_O, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes<8>()));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_tc_gemm_big<G_DOWN, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 1024 + big_smem_bytes<8>()));
+    {
+        auto query = [&](const void* fn, int S, int smem) {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3((unsigned)(S * (sms / S)));
+            cfg.blockDim = dim3(BIG_THREADS);
+            cfg.dynamicSmemBytes = (size_t)smem;
+            cudaLaunchAttribute at;
+            at.id = cudaLaunchAttributeClusterDimension;
+            at.val.clusterDim.x = S;
+            at.val.clusterDim.y = 1;
+            at.val.clusterDim.z = 1;
+            cfg.attrs = &at;
+            cfg.numAttrs = 1;
+            int n = 0;
+            if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) {
+                cudaGetLastError();
+                n = 0;
+            }
+            return n;
+        };
+        h->big_clusters[0] = sms;
+        h->big_clusters[1] = query((const void*)k_tc_gemm_big<G_DOWN, 2>, 2, 1024 + big_smem_bytes<2>());
+        h->big_clusters[2] = query((const void*)k_tc_gemm_big<G_DOWN, 4>, 4, 1024 + big_smem_bytes<4>());
+        h->big_clusters[3] = query((const void*)k_tc_gemm_big<G_DOWN, 8>, 8, 1024 + big_smem_bytes<8>());
+    }
+    // JPI_BIG_SPLIT=S fixes the K split of the large-M residual projections (1, 2, 4 or 8).
+    const char* split_env = std::getenv("JPI_BIG_SPLIT");
+    if (split_env) h->big_split = std::atoi(split_env);
     // Launches with at least this many tokens use the large-M kernels (full K per CTA). The
     // gate/up projection (64 weight tiles at pi0.5 sizes) fills the GPU with them from 128 tokens;
     // the narrower ones (8-20 weight tiles) keep the K-split kernel up to 512 tokens (measured).

@@ -211,6 +211,43 @@ def test_odd_weight_tile_count_large_m_path(large_m_everywhere, B, P, C):
         ex.close()
 
 
+# The large-M residual projections (O, down) may split each unit's K range over a cluster of
+# 1, 2, 4 or 8 CTAs, exchanging fp32 partials and summing them in rank order (JPI_BIG_SPLIT fixes
+# the split). Every split must match the oracle; between splits only the order of the fp32 sums
+# of the partials differs, which can move a bf16 rounding of the next projection's operand (2^-9
+# relative), so two layers' hidden states must agree to 2e-3 of their largest magnitude.
+BIG_SPLITS = (1, 2, 4, 8)
+
+
+def test_pi05_large_m_k_splits(large_m_everywhere, monkeypatch):
+    cfg = PI05.with_(n_layers=2)
+    w = make_weights(cfg, 2280)
+    r = make_requests(cfg, 2281, 4, 816, 50)
+    t = 0.6
+    want_v, want_h = oracle.forward_batch(r["noise"], r["state"], t, r["prefix_k"], r["prefix_v"], w, cfg)
+    got = {}
+    for S in BIG_SPLITS:
+        monkeypatch.setenv("JPI_BIG_SPLIT", str(S))
+        ex = make_expert(cfg, w, max_batch=4, max_prefix=816, max_chunk=50, max_steps=1)
+        try:
+            k, v = to_dev_kv(r, cfg)
+            ex.set_prefix_kv(k, v)
+            vel, hid = ex.forward(torch.from_numpy(r["state"]).cuda(), torch.from_numpy(r["noise"]).cuda(), t)
+            torch.cuda.synchronize()
+            ex.device_status()
+            got[S] = (vel.cpu().numpy(), hid.cpu().numpy())
+        finally:
+            ex.close()
+        assert_close(got[S][0], want_v, cfg, f"pi0.5 2 layers B4, large-M K split {S}")
+        _, rel = errors(got[S][1], want_h)
+        assert rel <= 1e-2, f"K split {S}: hidden rel-L2 {rel:.3g}"
+    scale = float(np.abs(want_h).max())
+    for S in BIG_SPLITS[1:]:
+        dh = float(np.abs(got[S][1] - got[1][1]).max()) / scale
+        print(f"K split {S} vs 1: hidden {dh:.3g} of max |h|")
+        assert dh <= 2e-3, f"K split {S} vs 1: hidden state differs by {dh:.3g} of max |h|"
+
+
 def test_pi05_large_m_projection_path(large_m_everywhere):
     w = make_weights(PI05, 2000)
     ex = make_expert(PI05, w, max_batch=3, max_prefix=816, max_chunk=50, max_steps=10)
