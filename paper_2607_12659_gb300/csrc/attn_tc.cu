@@ -374,11 +374,12 @@ __global__ void __launch_bounds__(AT_THREADS) k_attn_tc(const __grid_constant__ 
 
     // ---- exchange: push every other split's rows into its receive buffer ----
     ptx::cluster_wait();
-    if (tid == 0) {
-        const uint32_t bar_u = ptx::smem_u32(rbar);
-        for (int s = 0; s < ns; ++s) {
-            const int lo = min(AT_ROWS, s * rows_per), hi = min(AT_ROWS, lo + rows_per);
-            if (hi <= lo || s == rank) continue;
+    // Lane s of warp 0 sends split s its rows (the copies to all splits issue together).
+    if (warp == 0 && lane < ns && lane != rank) {
+        const int s = lane;
+        const int lo = min(AT_ROWS, s * rows_per), hi = min(AT_ROWS, lo + rows_per);
+        if (hi > lo) {
+            const uint32_t bar_u = ptx::smem_u32(rbar);
             const int slot = rank < s ? rank : rank - 1;   // split s stores senders != s in order
             const uint32_t dst = ptx::smem_u32(recv + (size_t)slot * rows_per * ROWB);
             ptx::bulk_copy_to_cluster(ptx::dsmem_map(dst, (uint32_t)s), opart + (size_t)lo * ROWB,

@@ -386,18 +386,19 @@ __global__ void __launch_bounds__(BIG_THREADS, 1) k_tc_gemm_big(const __grid_con
                         ptx::mbar_arrive(&acce[buf]);
                         ptx::fence_proxy_async_smem();   // the outgoing slices, for the bulk copies
                         ptx::named_bar_sync(1, BIG_EPI);
-                        if (tid == 64) {
-                            // Slices of this unit from the S - 1 peers, then this CTA's slices out.
-                            ptx::mbar_expect_tx(recvf, (uint32_t)((S - 1) * CF::SLICE));
-                            const uint32_t own_slot = ptx::smem_u32(recvb + (size_t)rank * TOK * BIG_NT);
-                            const uint32_t rbar = ptx::smem_u32(recvf);
-                            for (int q = 0; q < S; ++q) {
-                                if (q == rank) continue;
+                        if (ew == 0) {
+                            // Slices of this unit from the S - 1 peers (lane 0), then this CTA's
+                            // slices out, lane q to peer q (the copies issue together).
+                            if (lane == 0) ptx::mbar_expect_tx(recvf, (uint32_t)((S - 1) * CF::SLICE));
+                            if (lane < S && lane != rank) {
+                                const int q = lane;
+                                const uint32_t own_slot = ptx::smem_u32(recvb + (size_t)rank * TOK * BIG_NT);
+                                const uint32_t rbar = ptx::smem_u32(recvf);
                                 ptx::bulk_copy_to_cluster(ptx::dsmem_map(own_slot, (uint32_t)q),
                                                           sendb + (size_t)(q < rank ? q : q - 1) * TOK * BIG_NT,
                                                           (uint32_t)CF::SLICE, ptx::dsmem_map(rbar, (uint32_t)q));
                             }
-                            if (!ptx::mbar_wait_bounded(recvf, j & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
+                            if (lane == 0 && !ptx::mbar_wait_bounded(recvf, j & 1, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
                         }
                         ptx::named_bar_sync(1, BIG_EPI);   // every partial of this CTA's tokens is here
                         // n = h + gamma * (sum of the S partials in rank order) for tokens cc of this

@@ -238,17 +238,16 @@ __global__ void __launch_bounds__(GEMM_THREADS, 2) k_tc_gemm(const __grid_consta
 
         // ---- 3b. push each other rank's rows (pairs r*npairs.. and +64) to that rank ----
         ptx::cluster_wait();   // receive barriers initialised everywhere
-        if (tid == 0) {
+        // Lane r of warp 0 sends rank r its rows (the copies to all ranks issue together).
+        if (warp == 0 && lane < a.splits && lane != rank) {
+            const int r = lane;
             const uint32_t chunk = (uint32_t)(npairs * 128);
             const uint32_t bar_u = ptx::smem_u32(&bars[3]);
-            for (int r = 0; r < a.splits; ++r) {
-                if (r == rank) continue;
-                const int slot = rank < r ? rank : rank - 1;   // owner r stores senders != r in order
-                const uint32_t dst = ptx::dsmem_map(ptx::smem_u32(recv + (size_t)slot * 2 * npairs * 64), (uint32_t)r);
-                const uint32_t rbar = ptx::dsmem_map(bar_u, (uint32_t)r);
-                ptx::bulk_copy_to_cluster(dst, part + (size_t)r * npairs * 64, chunk, rbar);
-                ptx::bulk_copy_to_cluster(dst + chunk, part + (size_t)(r * npairs + 64) * 64, chunk, rbar);
-            }
+            const int slot = rank < r ? rank : rank - 1;   // owner r stores senders != r in order
+            const uint32_t dst = ptx::dsmem_map(ptx::smem_u32(recv + (size_t)slot * 2 * npairs * 64), (uint32_t)r);
+            const uint32_t rbar = ptx::dsmem_map(bar_u, (uint32_t)r);
+            ptx::bulk_copy_to_cluster(dst, part + (size_t)r * npairs * 64, chunk, rbar);
+            ptx::bulk_copy_to_cluster(dst + chunk, part + (size_t)(r * npairs + 64) * 64, chunk, rbar);
         }
         if (!ptx::mbar_wait_bounded(&bars[3], 0, WAIT_LIMIT_NS)) *flag = DEV_TIMEOUT_MMA;
         // Everything addressed to this CTA has landed (seen through its own mbarrier); once all
