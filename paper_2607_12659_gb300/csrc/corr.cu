@@ -304,6 +304,16 @@ __global__ void __launch_bounds__(256) k_corr_linear_pipe(const LinArgs a) {
         const uint4* wst = reinterpret_cast<const uint4*>(lp_smem + (size_t)(k % NST) * sbytes);
         for (int r0 = 0; r0 < a.rows; r0 += LP_XR) {
             const int nr = min(LP_XR, a.rows - r0);
+            // The bias and residual of this thread's output (thread o LP_XR + q writes feature
+            // o0 + o of row r0 + q), fetched before the products so their latency hides there.
+            float bias_v = 0.f, res_v = 0.f;
+            if (tid < LP_ROWS * LP_XR) {
+                const int o = tid / LP_XR, q = tid % LP_XR;
+                if (o < nout && q < nr) {
+                    if (a.bias) bias_v = a.bias[o0 + o];
+                    if (a.res) res_v = a.res[(size_t)(r0 + q) * a.ldr + o0 + o];
+                }
+            }
             float acc[LP_ROWS][LP_XR];
 #pragma unroll
             for (int o = 0; o < LP_ROWS; ++o)
@@ -343,16 +353,28 @@ __global__ void __launch_bounds__(256) k_corr_linear_pipe(const LinArgs a) {
                     }
                 }
             }
-            // (feature o, row q) sums: over the warp's lanes, then over the 8 warps in order.
-            float mine = 0.f;   // lane o * LP_XR + q keeps pair (o, q)
+            // (feature o, row q) sums: over the warp's lanes, then over the 8 warps in order. The
+            // warp sum is a reduce-scatter: at offset 16, 8, .., 1 each lane keeps the half of its
+            // pairs whose bit matches its own and adds its partner's partial of them (the same
+            // pairwise sums as a butterfly per pair, 31 shuffles instead of 160); lane p ends
+            // with pair p = o LP_XR + q.
+            static_assert(LP_ROWS * LP_XR == 32, "one pair per lane");
+            float pv[32];
 #pragma unroll
             for (int o = 0; o < LP_ROWS; ++o)
 #pragma unroll
-                for (int q = 0; q < LP_XR; ++q) {
-                    const float v = warp_sum(acc[o][q]);
-                    if (lane == o * LP_XR + q) mine = v;
+                for (int q = 0; q < LP_XR; ++q) pv[o * LP_XR + q] = acc[o][q];
+#pragma unroll
+            for (int sh = 16; sh > 0; sh >>= 1) {
+                const bool hi = (lane & sh) != 0;
+#pragma unroll
+                for (int i = 0; i < sh; ++i) {
+                    const float send = hi ? pv[i] : pv[i + sh];
+                    const float keep = hi ? pv[i + sh] : pv[i];
+                    pv[i] = keep + __shfl_xor_sync(0xffffffffu, send, sh);
                 }
-            red[warp][lane] = mine;
+            }
+            red[warp][lane] = pv[0];
             __syncthreads();
             if (tid < LP_ROWS * LP_XR) {
                 const int o = tid / LP_XR, q = tid % LP_XR;
@@ -361,9 +383,9 @@ __global__ void __launch_bounds__(256) k_corr_linear_pipe(const LinArgs a) {
                 for (int w8 = 0; w8 < 8; ++w8) v += red[w8][tid];
                 const int of = o0 + o, r = r0 + q;
                 if (o < nout && q < nr) {
-                    v += a.bias ? a.bias[of] : 0.f;
+                    v += bias_v;
                     if (a.gelu) v = gelu_tanh_f(v);
-                    if (a.res) v += a.res[(size_t)r * a.ldr + of];
+                    if (a.res) v += res_v;
                     a.y[(size_t)r * a.ldy + of] = v;
                 }
             }
@@ -394,7 +416,7 @@ __global__ void __launch_bounds__(256) k_corr_layernorm(const float* __restrict_
             const int d4 = d >> 2;
             const float4* x4 = reinterpret_cast<const float4*>(xr);
             float s = 0.f;
-#pragma unroll 4
+#pragma unroll 8
             for (int i = lane; i < d4; i += 32) {
                 const float4 v = x4[i];
                 s += (v.x + v.y) + (v.z + v.w);
@@ -464,18 +486,34 @@ __global__ void __launch_bounds__(256) k_corr_attn(const AttnSmallArgs a) {
         const int d = lane + 32 * t;
         qf[t] = d < a.Dh ? qr[d] : 0.f;
     }
+    // Keys (and below, values) four rows at a time: their loads are in flight together.
     float mx = -INFINITY;
-    for (int j = 0; j < a.nk; ++j) {
-        const float* kr = a.k + (size_t)(b * a.nk + j) * a.ldk + h * a.Dh;
-        float s = 0.f;
+    for (int j0 = 0; j0 < a.nk; j0 += 4) {
+        float kv[4][8];
 #pragma unroll
-        for (int t = 0; t < 8; ++t) {
-            const int d = lane + 32 * t;
-            if (d < a.Dh) s = fmaf(qf[t], kr[d], s);
+        for (int u = 0; u < 4; ++u) {
+            const int j = j0 + u < a.nk ? j0 + u : j0;
+            const float* kr = a.k + (size_t)(b * a.nk + j) * a.ldk + h * a.Dh;
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                const int d = lane + 32 * t;
+                kv[u][t] = d < a.Dh ? kr[d] : 0.f;
+            }
         }
-        s = warp_sum(s) * a.scale;
-        if (lane == 0) sp[wib][j] = s;
-        mx = fmaxf(mx, s);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int j = j0 + u;
+            if (j >= a.nk) break;
+            float s = 0.f;
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                const int d = lane + 32 * t;
+                if (d < a.Dh) s = fmaf(qf[t], kv[u][t], s);
+            }
+            s = warp_sum(s) * a.scale;
+            if (lane == 0) sp[wib][j] = s;
+            mx = fmaxf(mx, s);
+        }
     }
     __syncwarp();
     float den = 0.f;
@@ -489,13 +527,28 @@ __global__ void __launch_bounds__(256) k_corr_attn(const AttnSmallArgs a) {
     float of[8];
 #pragma unroll
     for (int t = 0; t < 8; ++t) of[t] = 0.f;
-    for (int j = 0; j < a.nk; ++j) {
-        const float p = sp[wib][j];
-        const float* vr = a.v + (size_t)(b * a.nk + j) * a.ldv + h * a.Dh;
+    for (int j0 = 0; j0 < a.nk; j0 += 4) {
+        float vv[4][8];
 #pragma unroll
-        for (int t = 0; t < 8; ++t) {
-            const int d = lane + 32 * t;
-            if (d < a.Dh) of[t] = fmaf(p, vr[d], of[t]);
+        for (int u = 0; u < 4; ++u) {
+            const int j = j0 + u < a.nk ? j0 + u : j0;
+            const float* vr = a.v + (size_t)(b * a.nk + j) * a.ldv + h * a.Dh;
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                const int d = lane + 32 * t;
+                vv[u][t] = d < a.Dh ? vr[d] : 0.f;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int j = j0 + u;
+            if (j >= a.nk) break;
+            const float p = sp[wib][j];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                const int d = lane + 32 * t;
+                if (d < a.Dh) of[t] = fmaf(p, vv[u][t], of[t]);
+            }
         }
     }
     const float inv = 1.f / den;
