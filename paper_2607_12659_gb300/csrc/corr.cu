@@ -592,12 +592,14 @@ __global__ void __launch_bounds__(256) k_corr_qk(const float* __restrict__ qc, c
 
 // Partial scores over one chunk of the VLM features: part[b][kc][m][j] = sum over c in chunk kc
 // (CORR_KCHUNK features) of qk[m][c] hv[b][j][c], m < M, j < T. Grid (ceil(T / 32), chunks, B):
-// 32 tokens per CTA; the chunk's query rows and token rows are staged in shared memory with all
-// their loads in flight together, then warp w computes rows w, w + 8, ... for lane = token.
-// Splitting the feature sum over CTAs keeps the whole GPU busy at batch 1 (26 token tiles alone
-// would not); the chunks are added in order by k_corr_softmax_sum.
+// 32 tokens per CTA; the chunk's query rows and token rows are staged in shared memory (fp32) with
+// all their loads in flight together, then thread (mg, jg) = (tid / 16, tid mod 16) computes the
+// register tile of rows mg, mg + 16, .. (< M) x tokens jg, jg + 16 from 16-byte loads of both
+// operands (four features at a time, summed in feature order). Splitting the feature sum over
+// CTAs keeps the whole GPU busy at batch 1 (26 token tiles alone would not); the chunks are added
+// in order by k_corr_softmax_sum.
 constexpr int CORR_KCHUNK = 256;
-constexpr int CORR_KPAD = CORR_KCHUNK + 1;
+constexpr int CORR_KPAD = CORR_KCHUNK + 4;   // 16-byte rows; 8 consecutive rows hit distinct banks
 constexpr size_t CORR_SCORES_SMEM = (size_t)(CORR_MAX_M + 32) * CORR_KPAD * sizeof(float);
 
 template <typename THV>
@@ -607,11 +609,10 @@ __global__ void __launch_bounds__(256) k_corr_scores(const float* __restrict__ q
     // let the next kernel's CTAs be scheduled (they wait in turn).
     jpi::ptx::grid_dep_wait();
     jpi::ptx::grid_dep_launch();
-    extern __shared__ float sm_scores[];
-    float* as = sm_scores;                       // [M][CORR_KPAD]
-    float* bs = sm_scores + CORR_MAX_M * CORR_KPAD;   // [32][CORR_KPAD]
+    extern __shared__ float4 sm_scores4[];
+    float* as = reinterpret_cast<float*>(sm_scores4);   // [M][CORR_KPAD]
+    float* bs = as + CORR_MAX_M * CORR_KPAD;            // [32][CORR_KPAD]
     const int b = blockIdx.z, kc = blockIdx.y, j0 = blockIdx.x * 32;
-    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int c0 = kc * CORR_KCHUNK, cn = min(CORR_KCHUNK, dv - c0);
     const THV* hb = hv + (size_t)b * T * dv;
     for (int idx = threadIdx.x; idx < M * CORR_KCHUNK; idx += 256) {
@@ -623,25 +624,36 @@ __global__ void __launch_bounds__(256) k_corr_scores(const float* __restrict__ q
         bs[t * CORR_KPAD + kk] = (j < T && kk < cn) ? to_f(hb[(size_t)j * dv + c0 + kk]) : 0.f;
     }
     __syncthreads();
-    float acc[CORR_MAX_M / 8];
+    constexpr int RM = CORR_MAX_M / 16;   // rows per thread at most
+    const int mg = threadIdx.x >> 4, jg = threadIdx.x & 15;
+    float acc[RM][2];
 #pragma unroll
-    for (int r = 0; r < CORR_MAX_M / 8; ++r) acc[r] = 0.f;
-#pragma unroll 8
-    for (int kk = 0; kk < CORR_KCHUNK; ++kk) {
-        const float bv = bs[tx * CORR_KPAD + kk];
+    for (int r = 0; r < RM; ++r) acc[r][0] = acc[r][1] = 0.f;
+    const float4* b0 = reinterpret_cast<const float4*>(bs + jg * CORR_KPAD);
+    const float4* b1 = reinterpret_cast<const float4*>(bs + (jg + 16) * CORR_KPAD);
+#pragma unroll 4
+    for (int k4 = 0; k4 < CORR_KCHUNK / 4; ++k4) {
+        const float4 x0 = b0[k4], x1 = b1[k4];
 #pragma unroll
-        for (int r = 0; r < CORR_MAX_M / 8; ++r) {
-            const int m = ty + 8 * r;
-            if (m < M) acc[r] = fmaf(as[m * CORR_KPAD + kk], bv, acc[r]);
+        for (int r = 0; r < RM; ++r) {
+            const int m = mg + 16 * r;
+            if (m < M) {
+                const float4 q = reinterpret_cast<const float4*>(as + m * CORR_KPAD)[k4];
+                acc[r][0] = fmaf(q.w, x0.w, fmaf(q.z, x0.z, fmaf(q.y, x0.y, fmaf(q.x, x0.x, acc[r][0]))));
+                acc[r][1] = fmaf(q.w, x1.w, fmaf(q.z, x1.z, fmaf(q.y, x1.y, fmaf(q.x, x1.x, acc[r][1]))));
+            }
         }
     }
-    const int j = j0 + tx;
-    if (j < T)
 #pragma unroll
-        for (int r = 0; r < CORR_MAX_M / 8; ++r) {
-            const int m = ty + 8 * r;
-            if (m < M) part[(((size_t)b * gridDim.y + kc) * M + m) * T + j] = acc[r];
+    for (int r = 0; r < RM; ++r) {
+        const int m = mg + 16 * r;
+        if (m >= M) continue;
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int j = j0 + jg + 16 * u;
+            if (j < T) part[(((size_t)b * gridDim.y + kc) * M + m) * T + j] = acc[r][u];
         }
+    }
 }
 
 // Block-wide reductions over 256 threads (8 warps), through `red` [8] in shared memory.
@@ -698,47 +710,88 @@ __global__ void __launch_bounds__(256) k_corr_softmax_sum(const float* __restric
 }
 
 // Partial weighted sums over one chunk of CORR_TCHUNK tokens: part[b][tc][m][c] = sum over j in
-// chunk tc of p[b][m][j] hv[b][j][c]. Grid (ceil(dv / 256), chunks, B): one column per thread,
-// all M rows, the chunk's probabilities staged in shared memory (read as broadcasts). The token
-// chunks are added in order by k_corr_wsum_reduce.
+// chunk tc of p[b][m][j] hv[b][j][c]. Grid (ceil(dv / 256), chunks, B): thread (cg, mg) =
+// (tid mod 128, tid / 128) takes columns 2 cg, 2 cg + 1 of the CTA's 256 and rows mg RH .. + RH - 1
+// (RH = 16 for M <= 32, else 32), token after token in order; the chunk's probabilities sit in
+// shared memory transposed ([token][row], read as 16-byte broadcasts) and each token's two values
+// come in one load, eight tokens' loads in flight together. The token chunks are added in order
+// by k_corr_wsum_reduce.
 constexpr int CORR_TCHUNK = 64;
+constexpr int CORR_PTS = CORR_MAX_M + 4;   // row stride of the transposed probabilities
 
 template <typename THV>
+__device__ __forceinline__ float2 load2(const THV* p);
+template <>
+__device__ __forceinline__ float2 load2<float>(const float* p) { return __ldg(reinterpret_cast<const float2*>(p)); }
+template <>
+__device__ __forceinline__ float2 load2<__nv_bfloat16>(const __nv_bfloat16* p) {
+    const uint32_t u = __ldg(reinterpret_cast<const unsigned int*>(p));
+    return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u));
+}
+
+// PAIR: dv even and hv aligned to two elements, so a thread's two columns load together; else
+// each value on its own (and a last odd column alone).
+template <typename THV, int RH, bool PAIR>
 __global__ void __launch_bounds__(256) k_corr_wsum(const float* __restrict__ p, const THV* __restrict__ hv,
                                                    float* __restrict__ part, int M, int T, int dv) {
     // Launched with programmatic dependent launch: wait for the previous kernel's results, then
     // let the next kernel's CTAs be scheduled (they wait in turn).
     jpi::ptx::grid_dep_wait();
     jpi::ptx::grid_dep_launch();
-    __shared__ float ps[CORR_MAX_M][CORR_TCHUNK];
-    const int b = blockIdx.z, tc = blockIdx.y, c = blockIdx.x * 256 + threadIdx.x;
+    __shared__ __align__(16) float pt[CORR_TCHUNK][CORR_PTS];
+    const int b = blockIdx.z, tc = blockIdx.y;
     const int j0 = tc * CORR_TCHUNK, jn = min(CORR_TCHUNK, T - j0);
-    for (int idx = threadIdx.x; idx < M * CORR_TCHUNK; idx += 256) {
-        const int r = idx / CORR_TCHUNK, jj = idx % CORR_TCHUNK;
-        ps[r][jj] = jj < jn ? p[((size_t)b * M + r) * T + j0 + jj] : 0.f;
+    for (int idx = threadIdx.x; idx < CORR_TCHUNK * CORR_PTS; idx += 256) {
+        const int jj = idx / CORR_PTS, r = idx % CORR_PTS;
+        pt[jj][r] = (jj < jn && r < M) ? p[((size_t)b * M + r) * T + j0 + jj] : 0.f;
     }
     __syncthreads();
+    const int cg = threadIdx.x & 127, mg = threadIdx.x >> 7;
+    const int c = blockIdx.x * 256 + 2 * cg;
     if (c >= dv) return;
-    float acc[CORR_MAX_M];
+    const int m0 = mg * RH;
+    float acc[RH][2];
 #pragma unroll
-    for (int r = 0; r < CORR_MAX_M; ++r) acc[r] = 0.f;
+    for (int i = 0; i < RH; ++i) acc[i][0] = acc[i][1] = 0.f;
     const THV* hb = hv + ((size_t)b * T + j0) * dv + c;
-    // Eight tokens' values loaded together, then their products (loads of the next eight in
-    // flight behind them).
     for (int jb = 0; jb < jn; jb += 8) {
-        float hvv[8];
+        float2 hvv[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) hvv[u] = jb + u < jn ? to_f(hb[(size_t)(jb + u) * dv]) : 0.f;
+        for (int u = 0; u < 8; ++u) {
+            hvv[u] = make_float2(0.f, 0.f);
+            if (jb + u < jn) {
+                const THV* hp = hb + (size_t)(jb + u) * dv;
+                if (PAIR) hvv[u] = load2(hp);
+                else hvv[u] = make_float2(load1(hp), c + 1 < dv ? load1(hp + 1) : 0.f);
+            }
+        }
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
+        for (int u = 0; u < 8; ++u) {
+            const float4* prow = reinterpret_cast<const float4*>(&pt[jb + u][m0]);
 #pragma unroll
-            for (int r = 0; r < CORR_MAX_M; ++r)
-                if (r < M) acc[r] = fmaf(ps[r][jb + u], hvv[u], acc[r]);
+            for (int i4 = 0; i4 < RH / 4; ++i4) {
+                const float4 pw = prow[i4];
+                const float w4[4] = {pw.x, pw.y, pw.z, pw.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    acc[4 * i4 + e][0] = fmaf(w4[e], hvv[u].x, acc[4 * i4 + e][0]);
+                    acc[4 * i4 + e][1] = fmaf(w4[e], hvv[u].y, acc[4 * i4 + e][1]);
+                }
+            }
+        }
     }
     float* out = part + ((size_t)b * gridDim.y + tc) * M * dv + c;
 #pragma unroll
-    for (int r = 0; r < CORR_MAX_M; ++r)
-        if (r < M) out[(size_t)r * dv] = acc[r];
+    for (int i = 0; i < RH; ++i) {
+        const int m = m0 + i;
+        if (m >= M) continue;
+        if (PAIR) {
+            *reinterpret_cast<float2*>(out + (size_t)m * dv) = make_float2(acc[i][0], acc[i][1]);
+        } else {
+            out[(size_t)m * dv] = acc[i][0];
+            if (c + 1 < dv) out[(size_t)m * dv + 1] = acc[i][1];
+        }
+    }
 }
 
 // g[b][m][c] = the ntc token-chunk partials added in order.
@@ -1323,12 +1376,26 @@ jpi_status enqueue_compress(jpi_corr_handle* h, const void* hvlm, int vlm_is_fp3
         const float* hv = static_cast<const float*>(hvlm);
         pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<float>, h->qk, hv, h->scp, M, n_tokens, dv);
         pdl(st, dim3(batch * M), dim3(256), 0, k_corr_softmax_sum, h->scp, h->sc, M, n_tokens, nkc);
-        pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<float>, h->sc, hv, h->gsp, M, n_tokens, dv);
+        const bool pair = dv % 2 == 0 && ((uintptr_t)hv & 7) == 0;
+        if (M <= 32) {
+            if (pair) pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<float, 16, true>, h->sc, hv, h->gsp, M, n_tokens, dv);
+            else pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<float, 16, false>, h->sc, hv, h->gsp, M, n_tokens, dv);
+        } else {
+            if (pair) pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<float, 32, true>, h->sc, hv, h->gsp, M, n_tokens, dv);
+            else pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<float, 32, false>, h->sc, hv, h->gsp, M, n_tokens, dv);
+        }
     } else {
         const __nv_bfloat16* hv = static_cast<const __nv_bfloat16*>(hvlm);
         pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<__nv_bfloat16>, h->qk, hv, h->scp, M, n_tokens, dv);
         pdl(st, dim3(batch * M), dim3(256), 0, k_corr_softmax_sum, h->scp, h->sc, M, n_tokens, nkc);
-        pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<__nv_bfloat16>, h->sc, hv, h->gsp, M, n_tokens, dv);
+        const bool pair = dv % 2 == 0 && ((uintptr_t)hv & 3) == 0;
+        if (M <= 32) {
+            if (pair) pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<__nv_bfloat16, 16, true>, h->sc, hv, h->gsp, M, n_tokens, dv);
+            else pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<__nv_bfloat16, 16, false>, h->sc, hv, h->gsp, M, n_tokens, dv);
+        } else {
+            if (pair) pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<__nv_bfloat16, 32, true>, h->sc, hv, h->gsp, M, n_tokens, dv);
+            else pdl(st, dim3(gw), dim3(256), 0, k_corr_wsum<__nv_bfloat16, 32, false>, h->sc, hv, h->gsp, M, n_tokens, dv);
+        }
     }
     pdl(st, dim3(red_grid), dim3(256), 0, k_corr_wsum_reduce, h->gsp, h->gs, batch, M, dv, ntc);
     JPI_CUDA_TRY(cudaGetLastError());
