@@ -602,7 +602,10 @@ constexpr int CORR_KCHUNK = 256;
 constexpr int CORR_KPAD = CORR_KCHUNK + 4;   // 16-byte rows; 8 consecutive rows hit distinct banks
 constexpr size_t CORR_SCORES_SMEM = (size_t)(CORR_MAX_M + 32) * CORR_KPAD * sizeof(float);
 
-template <typename THV>
+// VEC: dv a multiple of 4 and hv aligned to four elements, so the staging moves four features
+// per load; every thread's staging loads are issued before any of its stores (one at a time, each
+// store would hold the next load back for a full L2 round trip).
+template <typename THV, bool VEC>
 __global__ void __launch_bounds__(256) k_corr_scores(const float* __restrict__ qk, const THV* __restrict__ hv,
                                                      float* __restrict__ part, int M, int T, int dv) {
     // Launched with programmatic dependent launch: wait for the previous kernel's results, then
@@ -615,13 +618,39 @@ __global__ void __launch_bounds__(256) k_corr_scores(const float* __restrict__ q
     const int b = blockIdx.z, kc = blockIdx.y, j0 = blockIdx.x * 32;
     const int c0 = kc * CORR_KCHUNK, cn = min(CORR_KCHUNK, dv - c0);
     const THV* hb = hv + (size_t)b * T * dv;
-    for (int idx = threadIdx.x; idx < M * CORR_KCHUNK; idx += 256) {
-        const int m = idx / CORR_KCHUNK, kk = idx % CORR_KCHUNK;
-        as[m * CORR_KPAD + kk] = kk < cn ? qk[(size_t)m * dv + c0 + kk] : 0.f;
-    }
-    for (int idx = threadIdx.x; idx < 32 * CORR_KCHUNK; idx += 256) {
-        const int t = idx / CORR_KCHUNK, kk = idx % CORR_KCHUNK, j = j0 + t;
-        bs[t * CORR_KPAD + kk] = (j < T && kk < cn) ? to_f(hb[(size_t)j * dv + c0 + kk]) : 0.f;
+    if (VEC) {
+        // Thread t takes feature quad t mod 64 of rows t / 64, t / 64 + 4, ..: CORR_MAX_M / 4 query
+        // rows and 8 token rows at most.
+        const int k4 = threadIdx.x & 63, r0 = threadIdx.x >> 6, kk = 4 * k4;
+        const bool kin = kk < cn;
+        float4 qa[CORR_MAX_M / 4], hb4[8];
+#pragma unroll
+        for (int i = 0; i < CORR_MAX_M / 4; ++i) {
+            const int m = r0 + 4 * i;
+            qa[i] = (m < M && kin) ? *reinterpret_cast<const float4*>(qk + (size_t)m * dv + c0 + kk)
+                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int j = j0 + r0 + 4 * i;
+            hb4[i] = (j < T && kin) ? load4(hb + (size_t)j * dv + c0 + kk) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int i = 0; i < CORR_MAX_M / 4; ++i) {
+            const int m = r0 + 4 * i;
+            if (m < M) *reinterpret_cast<float4*>(as + m * CORR_KPAD + kk) = qa[i];
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) *reinterpret_cast<float4*>(bs + (r0 + 4 * i) * CORR_KPAD + kk) = hb4[i];
+    } else {
+        for (int idx = threadIdx.x; idx < M * CORR_KCHUNK; idx += 256) {
+            const int m = idx / CORR_KCHUNK, kk = idx % CORR_KCHUNK;
+            as[m * CORR_KPAD + kk] = kk < cn ? qk[(size_t)m * dv + c0 + kk] : 0.f;
+        }
+        for (int idx = threadIdx.x; idx < 32 * CORR_KCHUNK; idx += 256) {
+            const int t = idx / CORR_KCHUNK, kk = idx % CORR_KCHUNK, j = j0 + t;
+            bs[t * CORR_KPAD + kk] = (j < T && kk < cn) ? to_f(hb[(size_t)j * dv + c0 + kk]) : 0.f;
+        }
     }
     __syncthreads();
     constexpr int RM = CORR_MAX_M / 16;   // rows per thread at most
@@ -741,9 +770,18 @@ __global__ void __launch_bounds__(256) k_corr_wsum(const float* __restrict__ p, 
     __shared__ __align__(16) float pt[CORR_TCHUNK][CORR_PTS];
     const int b = blockIdx.z, tc = blockIdx.y;
     const int j0 = tc * CORR_TCHUNK, jn = min(CORR_TCHUNK, T - j0);
-    for (int idx = threadIdx.x; idx < CORR_TCHUNK * CORR_PTS; idx += 256) {
-        const int jj = idx / CORR_PTS, r = idx % CORR_PTS;
-        pt[jj][r] = (jj < jn && r < M) ? p[((size_t)b * M + r) * T + j0 + jj] : 0.f;
+    {
+        // Thread t loads token t mod 64 of rows t / 64, t / 64 + 4, .. (coalesced along the
+        // tokens, all loads before the transposed stores); rows past M are zero.
+        const int jj = threadIdx.x & 63, r0 = threadIdx.x >> 6;
+        float pv[CORR_PTS / 4];
+#pragma unroll
+        for (int i = 0; i < CORR_PTS / 4; ++i) {
+            const int r = r0 + 4 * i;
+            pv[i] = (jj < jn && r < M) ? p[((size_t)b * M + r) * T + j0 + jj] : 0.f;
+        }
+#pragma unroll
+        for (int i = 0; i < CORR_PTS / 4; ++i) pt[jj][r0 + 4 * i] = pv[i];
     }
     __syncthreads();
     const int cg = threadIdx.x & 127, mg = threadIdx.x >> 7;
@@ -1340,9 +1378,13 @@ jpi_status setup(jpi_corr_handle* h, const jpi_corr_config* c, const jpi_corr_we
     JPI_TRY(corr_alloc(h, &h->out_st, B * (size_t)h->Ti * h->d));
     JPI_TRY(corr_alloc(h, &h->out_conf, (size_t)B));
     JPI_CUDA_TRY(cudaStreamCreateWithFlags(&h->cap, cudaStreamNonBlocking));
-    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<float, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       (int)CORR_SCORES_SMEM));
-    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<float, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)CORR_SCORES_SMEM));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<__nv_bfloat16, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)CORR_SCORES_SMEM));
+    JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_scores<__nv_bfloat16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       (int)CORR_SCORES_SMEM));
     JPI_CUDA_TRY(cudaFuncSetAttribute(k_corr_linear_pipe<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       4 * LP_ROWS * 2048 * 2));
@@ -1374,7 +1416,10 @@ jpi_status enqueue_compress(jpi_corr_handle* h, const void* hvlm, int vlm_is_fp3
     const int red_grid = grid_for((long long)batch * M * dv);
     if (vlm_is_fp32) {
         const float* hv = static_cast<const float*>(hvlm);
-        pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<float>, h->qk, hv, h->scp, M, n_tokens, dv);
+        if (dv % 4 == 0 && ((uintptr_t)hv & 15) == 0)
+            pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<float, true>, h->qk, hv, h->scp, M, n_tokens, dv);
+        else
+            pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<float, false>, h->qk, hv, h->scp, M, n_tokens, dv);
         pdl(st, dim3(batch * M), dim3(256), 0, k_corr_softmax_sum, h->scp, h->sc, M, n_tokens, nkc);
         const bool pair = dv % 2 == 0 && ((uintptr_t)hv & 7) == 0;
         if (M <= 32) {
@@ -1386,7 +1431,10 @@ jpi_status enqueue_compress(jpi_corr_handle* h, const void* hvlm, int vlm_is_fp3
         }
     } else {
         const __nv_bfloat16* hv = static_cast<const __nv_bfloat16*>(hvlm);
-        pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<__nv_bfloat16>, h->qk, hv, h->scp, M, n_tokens, dv);
+        if (dv % 4 == 0 && ((uintptr_t)hv & 7) == 0)
+            pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<__nv_bfloat16, true>, h->qk, hv, h->scp, M, n_tokens, dv);
+        else
+            pdl(st, dim3(gs), dim3(256), CORR_SCORES_SMEM, k_corr_scores<__nv_bfloat16, false>, h->qk, hv, h->scp, M, n_tokens, dv);
         pdl(st, dim3(batch * M), dim3(256), 0, k_corr_softmax_sum, h->scp, h->sc, M, n_tokens, nkc);
         const bool pair = dv % 2 == 0 && ((uintptr_t)hv & 3) == 0;
         if (M <= 32) {
