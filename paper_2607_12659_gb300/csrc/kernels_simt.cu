@@ -6,6 +6,7 @@
 
 #include "jpi_internal.h"
 #include "tc_path.h"
+#include "ptx.h"
 
 #include <cmath>
 #include <type_traits>
@@ -197,6 +198,10 @@ __global__ void __launch_bounds__(128) k_embed(
     const float* __restrict__ x, const float* __restrict__ Ws, const float* __restrict__ bs,
     const float* __restrict__ Wa, const float* __restrict__ ba, const float* __restrict__ corr, int nctx,
     int S, int C, int W, int Sd, int A) {
+    // Launched with programmatic dependent launch: x comes from the previous step's final kernel;
+    // the next kernel may start its weight prefetch at once.
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     __shared__ float scratch[32];
     const int m = blockIdx.y;
     const int b = m / S, i = m % S;
@@ -423,6 +428,9 @@ __global__ void k_final(const float* __restrict__ hres, const float* __restrict_
                         const float* __restrict__ bout, float* __restrict__ x,
                         float* __restrict__ vout, float* __restrict__ outcopy, int S, int nctx, int C,
                         int W, int A, float eps, float delta) {
+    // Launched with programmatic dependent launch: h comes from the last layer's down projection.
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     extern __shared__ float us[];        // [W]
     __shared__ float scratch[32];
     const int bj = blockIdx.x;           // request b, action j
@@ -462,6 +470,25 @@ __global__ void k_convert_kv(const TS* __restrict__ src, TD* __restrict__ dst, i
         const long long d = idx % D, p = (idx / D) % P, b = idx / ((long long)D * P);
         dst[((size_t)b * kv_rows + p) * D + d] = cvt<TD>(ldf(src + idx));
     }
+}
+
+// Launch with programmatic dependent launch when the handle uses it (the kernel waits for its
+// predecessor with griddepcontrol.wait before reading what that wrote); a failed launch leaves its
+// error for check_launch.
+template <typename... KArgs, typename... Args>
+void launch_pdl(const jpi_handle* h, dim3 grid, dim3 block, size_t smem, cudaStream_t st, void (*k)(KArgs...),
+                Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at;
+    at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &at;
+    cfg.numAttrs = h->pdl ? 1 : 0;
+    (void)cudaLaunchKernelEx(&cfg, k, args...);
 }
 
 inline jpi_status check_launch(const char* what) {
@@ -661,11 +688,11 @@ jpi_status launch_embed(jpi_handle* h, int step, int B, int C, const float* x, c
     const int S = C + h->n_ctx();
     // Scale and shift of layer 0's attention norm at this step.
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * h->W;
-    k_embed<<<dim3((h->W + 127) / 128, B * S), 128, 0, st>>>(
-        h->h, h->tc ? (__nv_bfloat16*)h->hx : nullptr, ms, ms + h->W, h->tc ? h->ss : nullptr, h->maxMt,
-        h->state,
-        x, h->state_in_w, h->state_in_b,
-        h->action_in_w, h->action_in_b, h->corr, h->n_ctx(), S, C, h->W, h->Sd, h->A);
+    launch_pdl(h, dim3((h->W + 127) / 128, B * S), dim3(128), 0, st, k_embed,
+               h->h, h->tc ? (__nv_bfloat16*)h->hx : nullptr, ms, ms + h->W, h->tc ? h->ss : nullptr, h->maxMt,
+               (const float*)h->state, x, (const float*)h->state_in_w, (const float*)h->state_in_b,
+               (const float*)h->action_in_w, (const float*)h->action_in_b, (const float*)h->corr, h->n_ctx(), S, C,
+               h->W, h->Sd, h->A);
     return check_launch("embed");
 }
 
@@ -684,9 +711,9 @@ jpi_status launch_final(jpi_handle* h, int step, int B, int C, float delta, floa
                         float* v_out, float* out_copy, cudaStream_t st) {
     const int W = h->W;
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * W + (size_t)6 * h->L * W;
-    k_final<<<B * C, 256, sizeof(float) * W, st>>>(h->h, ms, ms + W, h->action_out_w,
-                                                   h->action_out_b, x_inout, v_out, out_copy,
-                                                   C + h->n_ctx(), h->n_ctx(), C, W, h->A, h->cfg.rms_eps, delta);
+    launch_pdl(h, dim3(B * C), dim3(256), sizeof(float) * W, st, k_final, (const float*)h->h, ms, ms + W,
+               (const float*)h->action_out_w, (const float*)h->action_out_b, x_inout, v_out, out_copy,
+               C + h->n_ctx(), h->n_ctx(), C, W, h->A, h->cfg.rms_eps, delta);
     return check_launch("final norm + Euler");
 }
 
