@@ -198,10 +198,6 @@ __global__ void __launch_bounds__(128) k_embed(
     const float* __restrict__ x, const float* __restrict__ Ws, const float* __restrict__ bs,
     const float* __restrict__ Wa, const float* __restrict__ ba, const float* __restrict__ corr, int nctx,
     int S, int C, int W, int Sd, int A) {
-    // Launched with programmatic dependent launch: x comes from the previous step's final kernel;
-    // the next kernel may start its weight prefetch at once.
-    ptx::grid_dep_wait();
-    ptx::grid_dep_launch();
     __shared__ float scratch[32];
     const int m = blockIdx.y;
     const int b = m / S, i = m % S;
@@ -215,19 +211,45 @@ __global__ void __launch_bounds__(128) k_embed(
         in = x + ((size_t)b * C + (i - nctx)) * A; Wm = Wa; bias = ba; K = A;
     }
     const int n = blockIdx.x * 128 + threadIdx.x;
+    // Everything but x (the previous step's actions) is ready before the dependency wait: the
+    // first EMB_K weights of this feature's row, its bias and the norm's scale and shift.
+    constexpr int EMB_K = 32;
+    float wv[EMB_K];
+    float bv = 0.f, sg = 0.f, bt = 0.f;
+    const bool lin = n < W && !(i > 0 && i < nctx);
+    if (lin) {
+#pragma unroll
+        for (int k = 0; k < EMB_K; ++k) wv[k] = k < K ? Wm[(size_t)n * K + k] : 0.f;
+        bv = bias[n];
+    }
+    if (n < W && xs) {
+        sg = sigma[n];
+        bt = beta[n];
+    }
+    // Launched with programmatic dependent launch: x comes from the previous step's final kernel;
+    // the next kernel may start its weight prefetch at once.
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     float v = 0.f;
     if (n < W) {
-        if (i > 0 && i < nctx) {
+        if (!lin) {
             v = corr[((size_t)b * (nctx - 1) + (i - 1)) * W + n];
         } else {
+            // The inputs of this row loaded together, then summed in k order.
             float acc = 0.f;
-            for (int k = 0; k < K; ++k) acc = fmaf(Wm[(size_t)n * K + k], in[k], acc);
-            v = acc + bias[n];
+            float iv[EMB_K];
+#pragma unroll
+            for (int k = 0; k < EMB_K; ++k) iv[k] = k < K ? in[k] : 0.f;
+#pragma unroll
+            for (int k = 0; k < EMB_K; ++k)
+                if (k < K) acc = fmaf(wv[k], iv[k], acc);
+            for (int k = EMB_K; k < K; ++k) acc = fmaf(Wm[(size_t)n * K + k], in[k], acc);
+            v = acc + bv;
         }
         hres[(size_t)m * W + n] = v;
         if (xs) {
-            xs[(size_t)xs_row(m) * W + n] = __float2bfloat16_rn((1.f + sigma[n]) * v);
-            if (m < xs_tiles(gridDim.y)) xs[((size_t)m * 64 + 63) * W + n] = __float2bfloat16_rn(beta[n]);
+            xs[(size_t)xs_row(m) * W + n] = __float2bfloat16_rn((1.f + sg) * v);
+            if (m < xs_tiles(gridDim.y)) xs[((size_t)m * 64 + 63) * W + n] = __float2bfloat16_rn(bt);
         }
     }
     if (ss) {
@@ -423,32 +445,73 @@ __global__ void k_attn_simt(const TQ* __restrict__ q, const TKV* __restrict__ ks
 // ---------------------------------------------------------------------------------------------
 // Final adaptive RMSNorm of an action row, velocity v = u W_out^T + b_out, Euler update
 // x <- x + delta v (or, for a single forward, v itself).
-__global__ void k_final(const float* __restrict__ hres, const float* __restrict__ sigma,
+// One CTA of FIN_THREADS per action row. The row's values (FIN_CAP per thread at most, all loads
+// in flight together) give the norm; the normalised row goes to shared memory; then thread t
+// takes output a0 + t / 8 over the 16-byte column chunks t mod 8, t mod 8 + 8, .. (a group of 8
+// threads reads 128 contiguous bytes per step) and the group adds its 8 partial sums.
+constexpr int FIN_THREADS = 256;
+constexpr int FIN_CAP = 16;   // W <= 4096
+__global__ void __launch_bounds__(FIN_THREADS) k_final(const float* __restrict__ hres, const float* __restrict__ sigma,
                         const float* __restrict__ beta, const float* __restrict__ Wout,
                         const float* __restrict__ bout, float* __restrict__ x,
                         float* __restrict__ vout, float* __restrict__ outcopy, int S, int nctx, int C,
                         int W, int A, float eps, float delta) {
+    extern __shared__ float us[];        // [W]
+    __shared__ float scratch[32];
+    const int tid = threadIdx.x;
+    const int bj = blockIdx.x;           // request b, action j
+    const int b = bj / C, j = bj % C;
+    // The modulation (scale, shift) of this thread's features, before the dependency wait.
+    float sg[FIN_CAP], bt[FIN_CAP];
+#pragma unroll
+    for (int q = 0; q < FIN_CAP; ++q) {
+        const int k = tid + FIN_THREADS * q;
+        sg[q] = k < W ? sigma[k] : 0.f;
+        bt[q] = k < W ? beta[k] : 0.f;
+    }
     // Launched with programmatic dependent launch: h comes from the last layer's down projection.
     ptx::grid_dep_wait();
     ptx::grid_dep_launch();
-    extern __shared__ float us[];        // [W]
-    __shared__ float scratch[32];
-    const int bj = blockIdx.x;           // request b, action j
-    const int b = bj / C, j = bj % C;
     const float* hr = hres + ((size_t)b * S + nctx + j) * W;
+    float hv[FIN_CAP];
+#pragma unroll
+    for (int q = 0; q < FIN_CAP; ++q) {
+        const int k = tid + FIN_THREADS * q;
+        hv[q] = k < W ? hr[k] : 0.f;
+    }
     float ss = 0.f;
-    for (int k = threadIdx.x; k < W; k += blockDim.x) ss = fmaf(hr[k], hr[k], ss);
+#pragma unroll
+    for (int q = 0; q < FIN_CAP; ++q) ss = fmaf(hv[q], hv[q], ss);
+    for (int k = tid + FIN_THREADS * FIN_CAP; k < W; k += FIN_THREADS) ss = fmaf(hr[k], hr[k], ss);   // W > 4096
     ss = block_sum(ss, scratch);
     const float rinv = rsqrtf(ss / (float)W + eps);
-    for (int k = threadIdx.x; k < W; k += blockDim.x)
+#pragma unroll
+    for (int q = 0; q < FIN_CAP; ++q) {
+        const int k = tid + FIN_THREADS * q;
+        if (k < W) us[k] = hv[q] * rinv * (1.f + sg[q]) + bt[q];
+    }
+    for (int k = tid + FIN_THREADS * FIN_CAP; k < W; k += FIN_THREADS)
         us[k] = hr[k] * rinv * (1.f + sigma[k]) + beta[k];
     __syncthreads();
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-    for (int a = warp; a < A; a += nw) {
+    const int ks = tid & 7;
+    const int n4 = W >> 2;   // W is a multiple of 32 (checked at create)
+    const float4* us4 = reinterpret_cast<const float4*>(us);
+    for (int a0 = 0; a0 < A; a0 += FIN_THREADS / 8) {
+        const int a = a0 + (tid >> 3);
         float acc = 0.f;
-        for (int k = lane; k < W; k += 32) acc = fmaf(us[k], Wout[(size_t)a * W + k], acc);
-        const float v = warp_sum(acc) + bout[a];
-        if (lane == 0) {
+        if (a < A) {
+            const float4* wr = reinterpret_cast<const float4*>(Wout + (size_t)a * W);
+#pragma unroll 8
+            for (int c = ks; c < n4; c += 8) {
+                const float4 w4 = __ldg(wr + c), u4 = us4[c];
+                acc = fmaf(u4.x, w4.x, fmaf(u4.y, w4.y, fmaf(u4.z, w4.z, fmaf(u4.w, w4.w, acc))));
+            }
+        }
+        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+        acc += __shfl_xor_sync(0xffffffffu, acc, 4);
+        if (ks == 0 && a < A) {
+            const float v = acc + bout[a];
             const size_t idx = (size_t)bj * A + a;
             if (vout) vout[idx] = v;
             if (x) {
@@ -711,7 +774,7 @@ jpi_status launch_final(jpi_handle* h, int step, int B, int C, float delta, floa
                         float* v_out, float* out_copy, cudaStream_t st) {
     const int W = h->W;
     const float* ms = h->mods + (size_t)step * mod_rows(h->L) * W + (size_t)6 * h->L * W;
-    launch_pdl(h, dim3(B * C), dim3(256), sizeof(float) * W, st, k_final, (const float*)h->h, ms, ms + W,
+    launch_pdl(h, dim3(B * C), dim3(FIN_THREADS), sizeof(float) * W, st, k_final, (const float*)h->h, ms, ms + W,
                (const float*)h->action_out_w, (const float*)h->action_out_b, x_inout, v_out, out_copy,
                C + h->n_ctx(), h->n_ctx(), C, W, h->A, h->cfg.rms_eps, delta);
     return check_launch("final norm + Euler");
