@@ -61,12 +61,14 @@ __device__ float block_sum(float v, float* scratch /* >= 32 floats */) {
 // by a two-layer swish MLP; the per-layer modulation vectors are a linear map of the result.
 // All of it depends on t alone, so it is evaluated once per call for every step time.
 
+// Grid (steps, ceil(half / blockDim)): one frequency i of one step time per thread (the fp64
+// pow/sin/cos are slow on this GPU; spread over the grid they run side by side).
 __global__ void k_time_embed(float* temb, int nsteps, int dt, double pmin, double pmax,
                              double t_override) {
     const int k = blockIdx.x;
     const double t = t_override >= 0.0 ? t_override : (double)k / (double)nsteps;
     const int half = dt / 2;
-    for (int i = threadIdx.x; i < half; i += blockDim.x) {
+    for (int i = blockIdx.y * blockDim.x + threadIdx.x; i < half; i += gridDim.y * blockDim.x) {
         const double frac = (double)i / (double)(half - 1);
         const double period = pmin * pow(pmax / pmin, frac);
         const double theta = 2.0 * 3.14159265358979323846 * t / period;
@@ -82,7 +84,21 @@ __global__ void k_gemv_multi(const TW* __restrict__ Wm, const float* __restrict_
                              const float* __restrict__ X, float* __restrict__ Y, int R, int K,
                              int N) {
     extern __shared__ float xs[];
-    for (int i = threadIdx.x; i < N * K; i += blockDim.x) xs[i] = X[i];
+    // Eight loads of each thread in flight before their stores (one at a time, every store would
+    // hold the next load back for a full round trip).
+    for (int i0 = threadIdx.x; i0 < N * K; i0 += 8 * blockDim.x) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int i = i0 + u * blockDim.x;
+            v[u] = i < N * K ? X[i] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int i = i0 + u * blockDim.x;
+            if (i < N * K) xs[i] = v[u];
+        }
+    }
     __syncthreads();
     const int lane = threadIdx.x & 31;
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -93,11 +109,23 @@ __global__ void k_gemv_multi(const TW* __restrict__ Wm, const float* __restrict_
             float acc[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) acc[j] = 0.f;
-            for (int k = lane; k < K; k += 32) {
-                const float wv = ldf(wr + k);
+            // Eight weights of the row loaded together, then their products in k order.
+            for (int k0 = lane; k0 < K; k0 += 32 * 8) {
+                float wv[8];
 #pragma unroll
-                for (int j = 0; j < 8; ++j)
-                    if (n0 + j < N) acc[j] = fmaf(wv, xs[(n0 + j) * K + k], acc[j]);
+                for (int u = 0; u < 8; ++u) {
+                    const int k = k0 + 32 * u;
+                    wv[u] = k < K ? ldf(wr + k) : 0.f;
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int k = k0 + 32 * u;
+                    if (k < K) {
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            if (n0 + j < N) acc[j] = fmaf(wv[u], xs[(n0 + j) * K + k], acc[j]);
+                    }
+                }
             }
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
@@ -711,8 +739,8 @@ jpi_status configure_simt_kernels(jpi_handle* h) {
 }
 
 jpi_status launch_time_embed(jpi_handle* h, int nsteps, double t_override, cudaStream_t st) {
-    k_time_embed<<<nsteps, 128, 0, st>>>(h->temb, nsteps, h->dt, h->cfg.t_min_period,
-                                         h->cfg.t_max_period, t_override);
+    k_time_embed<<<dim3(nsteps, (h->dt / 2 + 127) / 128), 128, 0, st>>>(h->temb, nsteps, h->dt, h->cfg.t_min_period,
+                                                                      h->cfg.t_max_period, t_override);
     return check_launch("time embedding");
 }
 
@@ -727,7 +755,7 @@ jpi_status launch_time_conditioning_into(jpi_handle* h, double t, float* temb, f
                                          float* cond, cudaStream_t st) {
     const int W = h->W, dt = h->dt;
     const int R = mod_rows(h->L) * W;
-    k_time_embed<<<1, 128, 0, st>>>(temb, 1, dt, h->cfg.t_min_period, h->cfg.t_max_period, t);
+    k_time_embed<<<dim3(1, (dt / 2 + 127) / 128), 128, 0, st>>>(temb, 1, dt, h->cfg.t_min_period, h->cfg.t_max_period, t);
     const dim3 blk(256);
     if (h->bf16) {
         using T = __nv_bfloat16;
