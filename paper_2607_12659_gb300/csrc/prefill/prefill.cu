@@ -153,24 +153,42 @@ __global__ void k_pf_rope_scatter(const float* __restrict__ qkv, const float2* _
                                   __nv_bfloat16* __restrict__ vd, long long stride, int B, int P, int H,
                                   int D) {
     const int half = D / 2, secs = H + 2, slots = secs * half;
+    constexpr int RS_BATCH = 8;   // slots of a thread whose loads are in flight together
     for (long long r = blockIdx.x; r < (long long)B * P; r += gridDim.x) {   // r = b P + p
         const int p = (int)(r % P), b = (int)(r / P);
         const float* row = qkv + r * (long long)secs * D;
-        for (int t = threadIdx.x; t < slots; t += blockDim.x) {
-            const int s = t / half, j = t - s * half;
-            const float* src = row + s * D;
-            float x1 = src[j], x2 = src[j + half];
-            if (s <= H) {
-                const float2 cs = rope[(size_t)p * half + j];
-                const float r1 = x1 * cs.x - x2 * cs.y, r2 = x2 * cs.x + x1 * cs.y;
-                x1 = r1;
-                x2 = r2;
+        for (int t0 = threadIdx.x; t0 < slots; t0 += RS_BATCH * blockDim.x) {
+            float x1[RS_BATCH], x2[RS_BATCH];
+            float2 cs[RS_BATCH];
+#pragma unroll
+            for (int u = 0; u < RS_BATCH; ++u) {
+                const int t = t0 + u * blockDim.x;
+                x1[u] = x2[u] = 0.f;
+                cs[u] = make_float2(1.f, 0.f);
+                if (t < slots) {
+                    const int s = t / half, j = t - s * half;
+                    const float* src = row + s * D;
+                    x1[u] = src[j];
+                    x2[u] = src[j + half];
+                    if (s <= H) cs[u] = rope[(size_t)p * half + j];
+                }
             }
-            __nv_bfloat16* dst;
-            if (s < H) dst = q + (r * H + s) * (long long)D;
-            else dst = (s == H ? kd : vd) + b * stride + (long long)p * D;
-            dst[j] = __float2bfloat16_rn(x1);
-            dst[j + half] = __float2bfloat16_rn(x2);
+#pragma unroll
+            for (int u = 0; u < RS_BATCH; ++u) {
+                const int t = t0 + u * blockDim.x;
+                if (t >= slots) break;
+                const int s = t / half, j = t - s * half;
+                float y1 = x1[u], y2 = x2[u];
+                if (s <= H) {
+                    y1 = x1[u] * cs[u].x - x2[u] * cs[u].y;
+                    y2 = x2[u] * cs[u].x + x1[u] * cs[u].y;
+                }
+                __nv_bfloat16* dst;
+                if (s < H) dst = q + (r * H + s) * (long long)D;
+                else dst = (s == H ? kd : vd) + b * stride + (long long)p * D;
+                dst[j] = __float2bfloat16_rn(y1);
+                dst[j + half] = __float2bfloat16_rn(y2);
+            }
         }
     }
 }
@@ -266,12 +284,18 @@ __global__ void __launch_bounds__(RB) k_pf_residual_norm(float* __restrict__ h, 
                     }
                 }
             }
+            // The residual row: every load before the stores that update it.
+            float4 o[RB_CAP];
+#pragma unroll
+            for (int k = 0; k < RB_CAP; ++k) {
+                const int i = t + RB * k;
+                o[k] = i < n4 ? hr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
 #pragma unroll
             for (int k = 0; k < RB_CAP; ++k) {
                 const int i = t + RB * k;
                 if (i < n4) {
-                    const float4 o = hr[i];
-                    v[k] = make_float4(o.x + v[k].x, o.y + v[k].y, o.z + v[k].z, o.w + v[k].w);
+                    v[k] = make_float4(o[k].x + v[k].x, o[k].y + v[k].y, o[k].z + v[k].z, o[k].w + v[k].w);
                     hr[i] = v[k];
                 }
             }
