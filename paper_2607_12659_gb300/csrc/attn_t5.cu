@@ -65,7 +65,7 @@ jpi_status attn_t5_prepare(jpi_handle* h) {
     // Smallest batch that takes this kernel (smaller ones keep the split-KV kernel); the
     // environment can move it, 0 turns the kernel off.
     const char* env = std::getenv("JPI_ATTN_T5_MIN_BATCH");
-    h->attn_t5_min_batch = env ? std::atoi(env) : 8;
+    h->attn_t5_min_batch = env ? std::atoi(env) : 6;
     // q [maxMt * H][D]; K and V of all layers [L * maxB * kv_rows][D].
     JPI_TRY(tc_make_tmap(h->q, (uint64_t)h->maxMt * h->H, h->D, T5_ROWS, &h->amaps[0]));
     const uint64_t kv_rows_all = (uint64_t)h->L * h->maxB * h->kv_rows;

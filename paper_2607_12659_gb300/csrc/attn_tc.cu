@@ -457,14 +457,18 @@ template <int D>
 jpi_status launch_attn_d(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     const int S = C + h->n_ctx(), nrows = S * h->H, nk = h->cur_prefix + S;
     const int rblocks = (nrows + AT_ROWS - 1) / AT_ROWS;
-    // Enough key splits for the launch to put about two CTAs on every SM, at most 16 (one
-    // cluster): 14 splits for one pi0.5-shaped request, one when many requests fill the GPU by
+    // Key splits: the largest power of two that keeps the launch within two CTAs per SM, at
+    // most 16 (one cluster): 16 asked (14 after rounding the chunk to whole 64-key blocks) for one
+    // pi0.5-shaped request, 8 for two, 4 for three to five, one when many requests fill the GPU by
     // themselves (then each CTA runs an online softmax over all keys and nothing is exchanged).
+    // Clusters of a power of two measured faster than the counts in between (batch 4: 4 splits
+    // 13.9 us, 3 splits 18.2, 6 splits 19.7 per launch; batch 2: 8 splits 9.3, 12 splits 13.0).
     // The split follows the launch's sizes, so a request's low-order bits depend on the batch
     // size it runs with; they never depend on timing.
     // In the batch-invariant mode the split is the one a single request gets, whatever B.
     const int blocks = rblocks * (h->batch_invariant ? 1 : B);
-    int want = (2 * h->num_sms + blocks - 1) / blocks;
+    int want = 1;
+    while (2 * want <= AT_MAX_SPLITS && (long long)blocks * want * 2 <= 2LL * h->num_sms) want *= 2;
     // A split count asked through the environment at create time replaces that choice.
     if (h->attn_force_splits > 0) want = h->attn_force_splits;
     want = want < 1 ? 1 : (want > h->attn_max_splits ? h->attn_max_splits : want);
