@@ -1,12 +1,16 @@
 // Launchers of the tcgen05 attention kernel (attn_t5_kernel.cuh) for the expert's batched
-// denoise: one CTA per 128 query rows of a request over its prefix and suffix keys, no key split.
+// denoise: one CTA per 128 query rows of a request and key split. The keys are split four ways
+// when (row blocks x requests x 4) CTAs fit on the SMs, else not at all: 4 at 6-9 requests, 1 from
+// 10 (pi0.5 shapes: 4 row blocks per request).
 
 #include "jpi_internal.h"
 #include "ptx.h"
 #include "tc_path.h"
 #include "attn_t5_kernel.cuh"
 
+#include <algorithm>
 #include <cmath>
+#include <cstdint>
 #include <cstdlib>
 
 namespace jpi {
@@ -14,6 +18,21 @@ namespace {
 
 static_assert(T5_ERR_LOAD == DEV_TIMEOUT_WEIGHTS && T5_ERR_MMA == DEV_TIMEOUT_MMA,
               "the attention kernel reports the library's device error codes");
+
+constexpr int T5_MAX_SPLIT = 4;
+
+int t5_splits(const jpi_handle* h, int blocks, int nb_all) {
+    if (h->attn_t5_splits > 0) {
+        // A fixed split, within the key blocks and the workspace (one slot per SM).
+        int s = std::max(1, std::min({h->attn_t5_splits, T5_MAX_SPLIT, nb_all}));
+        while (s > 1 && (long long)blocks * s > h->num_sms) --s;
+        return s;
+    }
+    // Four splits where they fit on the SMs, else none: on pi0.5 shapes (14 key blocks) two splits
+    // were slower than one, the exchange's 256 KB per CTA of L2 traffic costing more than the
+    // seven key blocks it saves.
+    return nb_all >= T5_MAX_SPLIT && (long long)blocks * T5_MAX_SPLIT <= h->num_sms ? T5_MAX_SPLIT : 1;
+}
 
 template <int D>
 jpi_status prepare_t5(jpi_handle* h) {
@@ -36,16 +55,30 @@ jpi_status launch_t5(jpi_handle* h, int l, int B, int C, cudaStream_t st) {
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)D);
     a.o = (__nv_bfloat16*)h->o;
     a.err = h->dev_err;
+    const int splits = h->t5_ws ? t5_splits(h, rblocks * B, (a.P + a.S + T5_KEYS - 1) / T5_KEYS) : 1;
+    a.ws = reinterpret_cast<float4*>(h->t5_ws);
+    a.wml = reinterpret_cast<float2*>(h->t5_wml);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(rblocks, B);
+    cfg.gridDim = dim3(rblocks, B, splits);
     cfg.blockDim = dim3(T5_THREADS);
     cfg.dynamicSmemBytes = 1024 + T5Smem<D>::TOTAL;
     cfg.stream = st;
-    cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr.val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = &attr;
-    cfg.numAttrs = h->pdl ? 1 : 0;
+    cudaLaunchAttribute attrs[2];
+    int n = 0;
+    if (h->pdl) {
+        attrs[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attrs[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    if (splits > 1) {
+        attrs[n].id = cudaLaunchAttributeClusterDimension;
+        attrs[n].val.clusterDim.x = 1;
+        attrs[n].val.clusterDim.y = 1;
+        attrs[n].val.clusterDim.z = (unsigned)splits;
+        ++n;
+    }
+    cfg.attrs = attrs;
+    cfg.numAttrs = n;
     cudaError_t e = cudaLaunchKernelEx(&cfg, k_attn_t5<D>, h->amaps[0], h->amaps[1], h->amaps[2], a);
     if (e != cudaSuccess) {
         set_error("attention launch failed: %s", cudaGetErrorString(e));
@@ -66,6 +99,24 @@ jpi_status attn_t5_prepare(jpi_handle* h) {
     // environment can move it, 0 turns the kernel off.
     const char* env = std::getenv("JPI_ATTN_T5_MIN_BATCH");
     h->attn_t5_min_batch = env ? std::atoi(env) : 6;
+    // JPI_ATTN_T5_SPLITS fixes its key split (1, 2 or 4; 0 or unset: chosen per launch).
+    const char* split_env = std::getenv("JPI_ATTN_T5_SPLITS");
+    h->attn_t5_splits = split_env ? std::atoi(split_env) : 0;
+    // Workspace of the key splits: a slot per CTA of a launch that splits (at most one CTA per SM).
+    {
+        const size_t part = (size_t)h->num_sms * (h->D / 4) * T5_ROWS * sizeof(float4);
+        const size_t ml = (size_t)h->num_sms * T5_ROWS * sizeof(float2);
+        void* p = nullptr;
+        if (cudaMalloc(&p, part + ml) != cudaSuccess) {
+            cudaGetLastError();
+            set_error("cudaMalloc of %zu bytes failed", part + ml);
+            return JPI_ERR_OOM;
+        }
+        h->allocations.push_back(p);
+        h->device_bytes += part + ml;
+        h->t5_ws = p;
+        h->t5_wml = static_cast<uint8_t*>(p) + part;
+    }
     // q [maxMt * H][D]; K and V of all layers [L * maxB * kv_rows][D].
     JPI_TRY(tc_make_tmap(h->q, (uint64_t)h->maxMt * h->H, h->D, T5_ROWS, &h->amaps[0]));
     const uint64_t kv_rows_all = (uint64_t)h->L * h->maxB * h->kv_rows;

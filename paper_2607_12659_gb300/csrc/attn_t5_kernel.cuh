@@ -26,6 +26,13 @@
 //           The running maximum is only moved, and O rescaled in TMEM, when a block's maximum
 //           exceeds it by more than 8 (log2 units), so probabilities stay below 2^8.
 // At the end every row is divided by its sum and written as bf16. All waits are bounded.
+// Key splits (gridDim.z = S > 1, the S CTAs of a row block forming a cluster along z): CTA s takes
+// the key blocks [s nb / S, (s + 1) nb / S). Past its key loop each CTA writes its rows'
+// unnormalised fp32 outputs and (m, l) to its slot of a workspace in global memory (row-fastest,
+// so a warp's 16-byte stores are contiguous); after a cluster barrier (release / acquire at
+// cluster scope) CTA s combines rows [s ceil(128 / S), ..) over the splits in split order,
+// o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, and writes bf16. The exchange goes through
+// L2 because the distributed shared memory takes a CTA's 128 rows at about 21 GB/s per SM.
 // The LLM prefill runs the same kernel with no separate prefix (P = 0) and its prompt tokens as
 // the S query tokens, every key visible (nctx = 0).
 
@@ -53,6 +60,10 @@ struct T5Args {
     float scale_log2;   // log2(e) / sqrt(D)
     __nv_bfloat16* o;   // [Mt][H][D]
     int* err;
+    // Key splits: [CTA][D / 4][128] partial outputs and [CTA][128] (m, l), CTA = (row block,
+    // request, split) in launch order; unused (null) without splits.
+    float4* ws = nullptr;
+    float2* wml = nullptr;
 };
 
 template <int D>
@@ -111,7 +122,12 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     const int rb = blockIdx.x, b = blockIdx.y;
     const int nrows = a.S * a.H, nk = a.P + a.S;
     const int row0 = rb * T5_ROWS;
-    const int nb = (nk + T5_KEYS - 1) / T5_KEYS;
+    // Key split: this CTA's key blocks blk0 .. blk0 + nb - 1 of the request's nb_all.
+    const int nsplit = (int)gridDim.z, split = (int)blockIdx.z;
+    const int nb_all = (nk + T5_KEYS - 1) / T5_KEYS;
+    const int blk0 = split * nb_all / nsplit;
+    const int nb = (split + 1) * nb_all / nsplit - blk0;
+    float x_m = -INFINITY, x_l = 0.f;   // the row's running maximum and sum (softmax threads)
 
     if (warp == 1) {
         ptx::tmem_alloc(tmem_slot, L::TMEM_COLS);
@@ -154,12 +170,13 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                 uint8_t* base = stages + sl * L::STAGE + (is_v ? L::KVBYTES : 0);
                 ptx::mbar_expect_tx(&fullb[sl], (uint32_t)L::KVBYTES);
                 for (int db = 0; db < NDB; ++db)
-                    ptx::tma_load_2d(base + db * (T5_KEYS * 128), map, &fullb[sl], db * 64, kv0 + i * T5_KEYS, pol);
+                    ptx::tma_load_2d(base + db * (T5_KEYS * 128), map, &fullb[sl], db * 64,
+                                     kv0 + (blk0 + i) * T5_KEYS, pol);
             };
             // First use of both slots: blocks made only of prefix keys were written before this
             // graph ran and are fetched before the dependency wait.
             int first = 0;
-            while (first < T5_STAGES && first < nb && (first + 1) * T5_KEYS <= a.P) load(first++);
+            while (first < T5_STAGES && first < nb && (blk0 + first + 1) * T5_KEYS <= a.P) load(first++);
             if (!is_v) ptx::prefetch_tmap(&qmap);
             ptx::grid_dep_wait();
             if (!is_v) {
@@ -199,7 +216,7 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                 ptx::mma_commit(&sfull[i & 1]);
                 if (i + T5_STAGES < nb) ptx::mma_commit(&kempty[sl]);
             };
-            issue_s(0);
+            if (nb > 0) issue_s(0);
             if (nb > 1) issue_s(1);
             // S_{i+2} once P_i is written: the softmax of block i has read score buffer i mod 2.
             for (int i = 0; i + 2 < nb; ++i) {
@@ -256,7 +273,7 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                 ptx::tmem_ld_wait();
             }
             // Keys of this block the row sees: all of them except in the last block(s).
-            const int vis = nvis - i * T5_KEYS;
+            const int vis = nvis - (blk0 + i) * T5_KEYS;
             const bool full = vis >= T5_KEYS;
             // Block maximum in log2 units (the scale is positive, so it commutes with the max);
             // four independent chains.
@@ -324,14 +341,16 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
         }
         // Every P V is done (both buffers' last commits observed, so none arrives after exit).
         if (nb >= 2 && !ptx::mbar_wait_bounded(&odone[(nb - 2) & 1], ((nb - 2) >> 1) & 1, T5_WAIT_NS)) good = false;
-        if (!ptx::mbar_wait_bounded(&odone[(nb - 1) & 1], ((nb - 1) >> 1) & 1, T5_WAIT_NS)) good = false;
+        if (nb >= 1 && !ptx::mbar_wait_bounded(&odone[(nb - 1) & 1], ((nb - 1) >> 1) & 1, T5_WAIT_NS)) good = false;
         ptx::tc_fence_after();
         ptx::grid_dep_launch();
         if (!good) *flag = T5_ERR_MMA;
+        x_m = m_used;
+        x_l = l;
         const float inv = l > 0.f ? 1.f / l : 0.f;
         __nv_bfloat16* orow = a.o + ((size_t)b * nrows + R) * D;
 #pragma unroll 1
-        for (int c0 = 0; c0 < D; c0 += 32) {
+        for (int c0 = 0; c0 < D && nsplit == 1; c0 += 32) {
             uint32_t r[2][16];
             ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)c0, r[0]);
             ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)(c0 + 16), r[1]);
@@ -349,6 +368,70 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                     dst[1] = make_uint4(w8[4], w8[5], w8[6], w8[7]);
                 }
             }
+        }
+    }
+
+    if (nsplit > 1) {
+        // ---- combine the key splits of this row block through the workspace ----
+        const size_t cta = ((size_t)blockIdx.y * gridDim.x + blockIdx.x) * nsplit;   // split 0 of the row block
+        if (warp >= 4) {
+            const int row = (warp & 3) * 32 + lane;
+            const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+            float4* dst = a.ws + (cta + split) * (size_t)(D / 4) * T5_ROWS + row;
+#pragma unroll 1
+            for (int c0 = 0; c0 < D; c0 += 32) {
+                uint32_t r[2][16];
+                ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)c0, r[0]);
+                ptx::tmem_ld_x16(lane_base + 128u + (uint32_t)(c0 + 16), r[1]);
+                ptx::tmem_ld_wait();
+#pragma unroll
+                for (int v = 0; v < 8; ++v)
+                    dst[(size_t)(c0 / 4 + v) * T5_ROWS] =
+                        make_float4(__uint_as_float(r[v >> 2][4 * (v & 3)]), __uint_as_float(r[v >> 2][4 * (v & 3) + 1]),
+                                    __uint_as_float(r[v >> 2][4 * (v & 3) + 2]), __uint_as_float(r[v >> 2][4 * (v & 3) + 3]));
+            }
+            a.wml[(cta + split) * T5_ROWS + row] = make_float2(x_m, x_l);
+        }
+        // Every split's rows are in the workspace (the barrier orders global memory at cluster scope;
+        // the reads below go to L2, past this SM's L1).
+        ptx::tc_fence_before();
+        ptx::cluster_sync_all();
+        ptx::tc_fence_after();
+        float* wsm = reinterpret_cast<float*>(smem);   // [rps][S] weights, over the query tile
+        const int rps = (T5_ROWS + nsplit - 1) / nsplit;
+        const int r_lo = split * rps;
+        const int nown = max(0, min(T5_ROWS, r_lo + rps) - r_lo);
+        if (tid < nown) {
+            float M = -INFINITY;
+            for (int sp = 0; sp < nsplit; ++sp) M = fmaxf(M, __ldcg(&a.wml[(cta + sp) * T5_ROWS + r_lo + tid]).x);
+            float Lsum = 0.f;
+            for (int sp = 0; sp < nsplit; ++sp) {
+                const float2 ml = __ldcg(&a.wml[(cta + sp) * T5_ROWS + r_lo + tid]);
+                const float w = ml.x == -INFINITY ? 0.f : ex2(ml.x - M);
+                wsm[tid * nsplit + sp] = w;
+                Lsum += w * ml.y;
+            }
+            const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+            for (int sp = 0; sp < nsplit; ++sp) wsm[tid * nsplit + sp] *= inv;
+        }
+        __syncthreads();
+        const bool ok_all = *flag == 0;
+        // Item (chunk c, owned row rr), rows fastest: a warp reads 32 consecutive rows of a chunk.
+        for (int idx = tid; idx < nown * (D / 4); idx += T5_THREADS) {
+            const int c = idx / nown, rr = idx - c * nown;
+            const int R = row0 + r_lo + rr;
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int sp = 0; sp < nsplit; ++sp) {
+                const float w = wsm[rr * nsplit + sp];
+                const float4 v = __ldcg(&a.ws[((cta + sp) * (size_t)(D / 4) + c) * T5_ROWS + r_lo + rr]);
+                acc.x = fmaf(w, v.x, acc.x);
+                acc.y = fmaf(w, v.y, acc.y);
+                acc.z = fmaf(w, v.z, acc.z);
+                acc.w = fmaf(w, v.w, acc.w);
+            }
+            if (R < nrows && ok_all)
+                *(uint2*)(a.o + ((size_t)b * nrows + R) * D + c * 4) =
+                    make_uint2(pack_bf16x2_t5(acc.x, acc.y), pack_bf16x2_t5(acc.z, acc.w));
         }
     }
 

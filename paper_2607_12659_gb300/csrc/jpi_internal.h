@@ -166,6 +166,9 @@ struct jpi_handle {
     int big_clusters[4] = {0, 0, 0, 0};   // co-resident large-M clusters of 1, 2, 4, 8 CTAs
     int attn_t5_min_batch = 6;  // batches of at least this many requests use the unsplit attention
     bool attn_t5 = false;       // its tensor maps and attributes are ready
+    int attn_t5_splits = 0;     // its key split (0: chosen per launch)
+    void* t5_ws = nullptr;      // its key-split workspace: partial outputs, then (m, l)
+    void* t5_wml = nullptr;
     CUtensorMap amaps[3];       // attention operands: q, prefix/suffix K, V (all layers)
     CUtensorMap qmap_at;        // q as 32-row boxes for the split-KV attention
     CUtensorMap kmap_at, vmap_at;   // K, V of all layers as 32-row boxes for it

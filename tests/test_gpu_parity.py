@@ -358,6 +358,58 @@ def test_split_counts_agree_on_one_pi05_shaped_layer(monkeypatch):
         assert dh <= SPLIT_AGREEMENT, f"{s} key splits: hidden state differs by {dh:.3g} of max |h|"
 
 
+# The tcgen05 attention's key split: the key blocks of each 128-row block spread over a cluster of
+# 1, 2 or 4 CTAs whose fp32 partial rows are combined in split order through a workspace in
+# global memory (JPI_ATTN_T5_SPLITS fixes the count). Every count must match the oracle; between
+# counts only the fp32 rounding of the combine differs.
+T5_SPLITS = (1, 2, 4)
+
+
+def _forward_t5_splits(monkeypatch, cfg, w, r, t, splits):
+    monkeypatch.setenv("JPI_ATTN_T5_MIN_BATCH", "1")
+    monkeypatch.setenv("JPI_ATTN_T5_SPLITS", str(splits))
+    B, P, C = r["noise"].shape[0], r["prefix_k"].shape[2], r["noise"].shape[1]
+    ex = make_expert(cfg, w, max_batch=B, max_prefix=P, max_chunk=C, max_steps=1)
+    try:
+        k, v = to_dev_kv(r, cfg)
+        ex.set_prefix_kv(k, v)
+        vel, hid = ex.forward(torch.from_numpy(r["state"]).cuda(), torch.from_numpy(r["noise"]).cuda(), t)
+        torch.cuda.synchronize()
+        ex.device_status()
+        return vel.cpu().numpy(), hid.cpu().numpy()
+    finally:
+        ex.close()
+
+
+def test_tcgen05_attention_key_splits_on_one_pi05_layer(monkeypatch):
+    cfg = PI05.with_(n_layers=1)
+    w = make_weights(cfg, 2620)
+    r = make_requests(cfg, 2621, 2, 816, 50)
+    t = 0.4
+    want_v, want_h = oracle.forward_batch(r["noise"], r["state"], t, r["prefix_k"], r["prefix_v"], w, cfg)
+    got = {s: _forward_t5_splits(monkeypatch, cfg, w, r, t, s) for s in T5_SPLITS}
+    scale = float(np.abs(want_h).max())
+    for s in T5_SPLITS:
+        assert_close(got[s][0], want_v, cfg, f"one pi0.5 layer B2, tcgen05 attention, {s} key splits")
+    for s in T5_SPLITS[1:]:
+        dh = float(np.abs(got[s][1] - got[1][1]).max()) / scale
+        print(f"tcgen05 attention {s} splits vs 1: hidden {dh:.3g} of max |h|")
+        assert dh <= SPLIT_AGREEMENT, f"{s} key splits: hidden state differs by {dh:.3g} of max |h|"
+
+
+@pytest.mark.parametrize("splits", [2, 4])
+def test_tcgen05_attention_key_splits_small_and_ragged(monkeypatch, splits):
+    # Prefix 70 + suffix 14 = 84 keys: two 64-key blocks, so 4 splits are capped at 2; the state
+    # row sees the prefix and itself only.
+    w = make_weights(SMALL_BF16, 2630)
+    r = make_requests(SMALL_BF16, 2631, 3, 70, 13)
+    t = 0.8
+    want_v, _ = oracle.forward_batch(r["noise"], r["state"], t, r["prefix_k"], r["prefix_v"],
+                                     oracle.to_f64(w), SMALL_BF16)
+    vel, _ = _forward_t5_splits(monkeypatch, SMALL_BF16, w, r, t, splits)
+    assert_close(vel, want_v, SMALL_BF16, f"small bf16 B3 P70, tcgen05 attention, {splits} key splits")
+
+
 # Batch invariance, bit for bit: with JPI_BATCH_INVARIANT=1 every launch makes the choices it makes
 # for a single request (the K-split projections with their fixed K split, the split-KV attention
 # with one request's key split), so request b of a batch gets exactly the actions it gets alone.
