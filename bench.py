@@ -564,6 +564,61 @@ def prefill_arm(args):
     pre.close()
 
 
+SWEEP = dict(prefix=(256, 512, 816, 1536), chunk=(10, 50), steps=(1, 5, 10))
+
+
+def sweep_arm(args):
+    """The batch-1 sweep over prefix length, chunk length and Euler steps (24 cases) in one
+    process: one expert sized for the largest case, a graph per case (captured on its first
+    call, untimed), then `--steps` timed calls. One JSON line with every case's median time
+    against its HBM roofline (a table beside the bench line, not a bench line)."""
+    import torch
+    from paper_2607_12659_gb300 import build, jpi
+    from synth import PI05, make_requests, make_weights
+    build.build()
+    jpi.load()
+    torch.cuda.set_device(0)
+    cfg = PI05
+    ex = jpi.Expert(cfg, make_weights(cfg, 2000), max_batch=1, max_prefix=max(SWEEP["prefix"]),
+                    max_chunk=max(SWEEP["chunk"]), max_steps=max(SWEEP["steps"]))
+    hbm_peak, _, peak_src = measured_peaks()
+    stream = torch.cuda.current_stream()
+    cases = []
+    with ClockSampler(0) as clk:
+        for P in SWEEP["prefix"]:
+            for C in SWEEP["chunk"]:
+                r = make_requests(cfg, 3000 + P + C, 1, P, C)
+                ex.set_prefix_kv(torch.from_numpy(r["prefix_k"]).cuda().to(torch.bfloat16),
+                                 torch.from_numpy(r["prefix_v"]).cuda().to(torch.bfloat16))
+                state = torch.from_numpy(r["state"]).cuda()
+                noise = torch.from_numpy(r["noise"]).cuda()
+                out = torch.empty_like(noise)
+                for N in SWEEP["steps"]:
+                    for _ in range(args.warmup):
+                        ex.denoise(state, noise, N, out)
+                    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+                    torch.cuda.synchronize()
+                    ev[0].record(stream)
+                    for i in range(args.steps):
+                        ex.denoise(state, noise, N, out)
+                        ev[i + 1].record(stream)
+                    torch.cuda.synchronize()
+                    ex.device_status()
+                    us = statistics.median([ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]) * 1e3
+                    roof_us = algorithmic_bytes(cfg, 1, P, C, N) / (hbm_peak * 1e9) * 1e6
+                    cases.append({"prefix": P, "chunk": C, "steps": N, "us_per_denoise": round(us, 1),
+                                  "chunks_per_s": round(1e6 / us, 1), "roofline_us": round(roof_us, 1),
+                                  "frac": round(roof_us / us, 4)})
+    print(json.dumps({
+        "metric": "us per denoise, batch 1, prefix x chunk x Euler-step sweep (pi0.5-shaped expert)",
+        "cases": cases, "steps": args.steps, "warmup": args.warmup,
+        "roofline": {"bound": "hbm", "peak": hbm_peak, "unit": "GB/s", "peak_source": peak_src},
+        "dtype": "bf16 GEMM operands, fp32 accumulation and residual stream", "data": "synthetic",
+        "clocks": clk.summary(),
+    }), flush=True)
+    ex.close()
+
+
 def profile_forward(args):
     """Small case for kernel captures: the workload's expert, eager expert passes (batch and
     prefix as given, else the workload's)."""
@@ -613,6 +668,8 @@ def main():
     ap.add_argument("--correction", action="store_true",
                     help="time the future correction module alone (compress + predict)")
     ap.add_argument("--prefill", action="store_true", help="time the Gemma-2B-shaped prefix prefill alone")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time the batch-1 prefix x chunk x Euler-step sweep (24 cases, one JSON line)")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
@@ -640,6 +697,8 @@ def main():
         correction_arm(args)
     elif args.prefill:
         prefill_arm(args)
+    elif args.sweep:
+        sweep_arm(args)
     elif args.impl == "reference":
         reference_arm(args)
     else:
