@@ -1,7 +1,7 @@
 // Launchers of the tcgen05 attention kernel (attn_t5_kernel.cuh) for the expert's batched
 // denoise: one CTA per 128 query rows of a request and key split. The keys are split four ways
-// when (row blocks x requests x 4) CTAs fit on the SMs, else not at all: 4 at 6-9 requests, 1 from
-// 10 (pi0.5 shapes: 4 row blocks per request).
+// when the (row blocks x requests) clusters of 4 CTAs are co-resident, else not at all: 4 at 6-9
+// requests, 1 from 10 (pi0.5 shapes: 4 row blocks per request).
 
 #include "jpi_internal.h"
 #include "ptx.h"
@@ -21,23 +21,49 @@ static_assert(T5_ERR_LOAD == DEV_TIMEOUT_WEIGHTS && T5_ERR_MMA == DEV_TIMEOUT_MM
 
 constexpr int T5_MAX_SPLIT = 4;
 
+// Whether `blocks` clusters of s CTAs are co-resident (one wave) and fit the workspace.
+bool t5_fits(const jpi_handle* h, int blocks, int s) {
+    return (long long)blocks * s <= h->num_sms && blocks <= h->t5_clusters[s];
+}
+
 int t5_splits(const jpi_handle* h, int blocks, int nb_all) {
     if (h->attn_t5_splits > 0) {
-        // A fixed split, within the key blocks and the workspace (one slot per SM).
+        // A fixed split, within the key blocks and one wave of clusters.
         int s = std::max(1, std::min({h->attn_t5_splits, T5_MAX_SPLIT, nb_all}));
-        while (s > 1 && (long long)blocks * s > h->num_sms) --s;
+        while (s > 1 && !t5_fits(h, blocks, s)) --s;
         return s;
     }
-    // Four splits where they fit on the SMs, else none: on pi0.5 shapes (14 key blocks) two splits
-    // were slower than one, the exchange's 256 KB per CTA of L2 traffic costing more than the
-    // seven key blocks it saves.
-    return nb_all >= T5_MAX_SPLIT && (long long)blocks * T5_MAX_SPLIT <= h->num_sms ? T5_MAX_SPLIT : 1;
+    // Four splits where the clusters fit in one wave, else none: on pi0.5 shapes (14 key blocks)
+    // two splits measured no faster than one, and three or four past one wave of clusters took
+    // twice as long.
+    return nb_all >= T5_MAX_SPLIT && t5_fits(h, blocks, T5_MAX_SPLIT) ? T5_MAX_SPLIT : 1;
 }
 
 template <int D>
 jpi_status prepare_t5(jpi_handle* h) {
     JPI_CUDA_TRY(cudaFuncSetAttribute(k_attn_t5<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       1024 + T5Smem<D>::TOTAL));
+    // Co-resident clusters of s CTAs along z (the key splits of one row block).
+    h->t5_clusters[1] = h->num_sms;
+    for (int s = 2; s <= T5_MAX_SPLIT; ++s) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)(h->num_sms / s), 1, (unsigned)s);
+        cfg.blockDim = dim3(T5_THREADS);
+        cfg.dynamicSmemBytes = 1024 + T5Smem<D>::TOTAL;
+        cudaLaunchAttribute at;
+        at.id = cudaLaunchAttributeClusterDimension;
+        at.val.clusterDim.x = 1;
+        at.val.clusterDim.y = 1;
+        at.val.clusterDim.z = (unsigned)s;
+        cfg.attrs = &at;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, k_attn_t5<D>, &cfg) != cudaSuccess) {
+            cudaGetLastError();
+            n = 0;
+        }
+        h->t5_clusters[s] = n;
+    }
     return JPI_OK;
 }
 

@@ -90,6 +90,70 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
+// Combine of S key splits for rows [r_lo, r_lo + nown) of a row block whose split 0 has workspace
+// slot `cta`: each row's weights 2^(m_s - M) / sum_s 2^(m_s - M) l_s into `wsm`, then items
+// (16-byte chunk c, owned row rr), rows fastest, summed over the splits in split order. A thread
+// fetches the partials of IB items for all splits before it combines and stores any of them:
+// with a store between them, the next item's loads would wait for it (the compiler cannot tell
+// the workspace from the output), one L2 round trip per item.
+template <int D, int S>
+__device__ __forceinline__ void t5_combine(const T5Args& a, size_t cta, int r_lo, int nown, float* wsm, int row0,
+                                           int nrows, int b, bool ok_all, int tid) {
+    if (tid < nown) {
+        float2 ml[S];
+#pragma unroll
+        for (int sp = 0; sp < S; ++sp) ml[sp] = __ldcg(&a.wml[(cta + sp) * T5_ROWS + r_lo + tid]);
+        float M = -INFINITY;
+#pragma unroll
+        for (int sp = 0; sp < S; ++sp) M = fmaxf(M, ml[sp].x);
+        float w[S], lsum = 0.f;
+#pragma unroll
+        for (int sp = 0; sp < S; ++sp) {
+            w[sp] = ml[sp].x == -INFINITY ? 0.f : ex2(ml[sp].x - M);
+            lsum += w[sp] * ml[sp].y;
+        }
+        const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+#pragma unroll
+        for (int sp = 0; sp < S; ++sp) wsm[tid * S + sp] = w[sp] * inv;
+    }
+    __syncthreads();
+    constexpr int IB = 32 / S;
+    const int nitems = nown * (D / 4);
+    for (int base = tid; base < nitems; base += IB * T5_THREADS) {
+        float4 v[IB][S];
+#pragma unroll
+        for (int i = 0; i < IB; ++i) {
+            const int idx = base + i * T5_THREADS;
+            if (idx < nitems) {
+                const int c = idx / nown, rr = idx - c * nown;
+#pragma unroll
+                for (int sp = 0; sp < S; ++sp)
+                    v[i][sp] = __ldcg(&a.ws[((cta + sp) * (size_t)(D / 4) + c) * T5_ROWS + r_lo + rr]);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < IB; ++i) {
+            const int idx = base + i * T5_THREADS;
+            if (idx < nitems) {
+                const int c = idx / nown, rr = idx - c * nown;
+                const int R = row0 + r_lo + rr;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int sp = 0; sp < S; ++sp) {
+                    const float w = wsm[rr * S + sp];
+                    acc.x = fmaf(w, v[i][sp].x, acc.x);
+                    acc.y = fmaf(w, v[i][sp].y, acc.y);
+                    acc.z = fmaf(w, v[i][sp].z, acc.z);
+                    acc.w = fmaf(w, v[i][sp].w, acc.w);
+                }
+                if (R < nrows && ok_all)
+                    *(uint2*)(a.o + ((size_t)b * nrows + R) * D + c * 4) =
+                        make_uint2(pack_bf16x2_t5(acc.x, acc.y), pack_bf16x2_t5(acc.z, acc.w));
+            }
+        }
+    }
+}
+
 template <int D>
 __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant__ CUtensorMap qmap,
                                                            const __grid_constant__ CUtensorMap kmap,
@@ -397,42 +461,15 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
         ptx::tc_fence_before();
         ptx::cluster_sync_all();
         ptx::tc_fence_after();
-        float* wsm = reinterpret_cast<float*>(smem);   // [rps][S] weights, over the query tile
+        float* wsm = reinterpret_cast<float*>(smem);   // [rows][S] weights, over the query tile
         const int rps = (T5_ROWS + nsplit - 1) / nsplit;
         const int r_lo = split * rps;
         const int nown = max(0, min(T5_ROWS, r_lo + rps) - r_lo);
-        if (tid < nown) {
-            float M = -INFINITY;
-            for (int sp = 0; sp < nsplit; ++sp) M = fmaxf(M, __ldcg(&a.wml[(cta + sp) * T5_ROWS + r_lo + tid]).x);
-            float Lsum = 0.f;
-            for (int sp = 0; sp < nsplit; ++sp) {
-                const float2 ml = __ldcg(&a.wml[(cta + sp) * T5_ROWS + r_lo + tid]);
-                const float w = ml.x == -INFINITY ? 0.f : ex2(ml.x - M);
-                wsm[tid * nsplit + sp] = w;
-                Lsum += w * ml.y;
-            }
-            const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-            for (int sp = 0; sp < nsplit; ++sp) wsm[tid * nsplit + sp] *= inv;
-        }
-        __syncthreads();
-        const bool ok_all = *flag == 0;
-        // Item (chunk c, owned row rr), rows fastest: a warp reads 32 consecutive rows of a chunk.
-        for (int idx = tid; idx < nown * (D / 4); idx += T5_THREADS) {
-            const int c = idx / nown, rr = idx - c * nown;
-            const int R = row0 + r_lo + rr;
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int sp = 0; sp < nsplit; ++sp) {
-                const float w = wsm[rr * nsplit + sp];
-                const float4 v = __ldcg(&a.ws[((cta + sp) * (size_t)(D / 4) + c) * T5_ROWS + r_lo + rr]);
-                acc.x = fmaf(w, v.x, acc.x);
-                acc.y = fmaf(w, v.y, acc.y);
-                acc.z = fmaf(w, v.z, acc.z);
-                acc.w = fmaf(w, v.w, acc.w);
-            }
-            if (R < nrows && ok_all)
-                *(uint2*)(a.o + ((size_t)b * nrows + R) * D + c * 4) =
-                    make_uint2(pack_bf16x2_t5(acc.x, acc.y), pack_bf16x2_t5(acc.z, acc.w));
-        }
+        const bool ok_all = *flag == 0;   // written before the cluster barrier
+        // The launcher splits 2, 3 or 4 ways.
+        if (nsplit == 2) t5_combine<D, 2>(a, cta, r_lo, nown, wsm, row0, nrows, b, ok_all, tid);
+        else if (nsplit == 3) t5_combine<D, 3>(a, cta, r_lo, nown, wsm, row0, nrows, b, ok_all, tid);
+        else t5_combine<D, 4>(a, cta, r_lo, nown, wsm, row0, nrows, b, ok_all, tid);
     }
 
     ptx::tc_fence_before();

@@ -167,6 +167,7 @@ struct jpi_handle {
     int attn_t5_min_batch = 6;  // batches of at least this many requests use the unsplit attention
     bool attn_t5 = false;       // its tensor maps and attributes are ready
     int attn_t5_splits = 0;     // its key split (0: chosen per launch)
+    int t5_clusters[5] = {};    // co-resident clusters of s CTAs of it, s = 1..4
     void* t5_ws = nullptr;      // its key-split workspace: partial outputs, then (m, l)
     void* t5_wml = nullptr;
     CUtensorMap amaps[3];       // attention operands: q, prefix/suffix K, V (all layers)
