@@ -124,7 +124,10 @@ typedef struct jpi_weights {
  * a request's actions are identical bit for bit alone and inside any batch (slower from batch 4);
  * JPI_ATTN_SPLITS=n fixes the key splits of the small-batch attention (results agree across
  * split counts to rounding only); JPI_ATTN_T5_MIN_BATCH and JPI_BIG_GEMM_MIN_TOKENS move the
- * batch / token thresholds of the large-batch attention and projection kernels (0 disables them).
+ * batch / token thresholds of the large-batch attention and projection kernels (0 disables them);
+ * JPI_ATTN_T5_SPLITS=n fixes the key splits of the large-batch attention (1-4, within one wave of
+ * clusters; the same rounding-only agreement); JPI_BIG_SPLIT=n fixes the K split of the large-batch
+ * O and down projections (1, 2, 4 or 8).
  */
 JPI_API jpi_status jpi_expert_create(const jpi_config* cfg, const jpi_weights* w, jpi_handle** out);
 

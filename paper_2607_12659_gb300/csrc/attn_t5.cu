@@ -1,6 +1,6 @@
 // Launchers of the tcgen05 attention kernel (attn_t5_kernel.cuh) for the expert's batched
 // denoise: one CTA per 128 query rows of a request and key split. The keys are split four ways
-// when the (row blocks x requests) clusters of 4 CTAs are co-resident, else not at all: 4 at 6-9
+// when the (row blocks x requests) clusters of 4 CTAs are co-resident, else not at all: 4 at 3-9
 // requests, 1 from 10 (pi0.5 shapes: 4 row blocks per request).
 
 #include "jpi_internal.h"
@@ -124,7 +124,7 @@ jpi_status attn_t5_prepare(jpi_handle* h) {
     // Smallest batch that takes this kernel (smaller ones keep the split-KV kernel); the
     // environment can move it, 0 turns the kernel off.
     const char* env = std::getenv("JPI_ATTN_T5_MIN_BATCH");
-    h->attn_t5_min_batch = env ? std::atoi(env) : 6;
+    h->attn_t5_min_batch = env ? std::atoi(env) : 3;
     // JPI_ATTN_T5_SPLITS fixes its key split (1, 2 or 4; 0 or unset: chosen per launch).
     const char* split_env = std::getenv("JPI_ATTN_T5_SPLITS");
     h->attn_t5_splits = split_env ? std::atoi(split_env) : 0;

@@ -164,7 +164,7 @@ struct jpi_handle {
     int big_min_tokens[4] = {512, 128, 128, 128};   // per projection kind: from this many tokens the large-M GEMM
     int big_split = 0;          // K split of the large-M residual projections (0: chosen per launch)
     int big_clusters[4] = {0, 0, 0, 0};   // co-resident large-M clusters of 1, 2, 4, 8 CTAs
-    int attn_t5_min_batch = 6;  // batches of at least this many requests use the unsplit attention
+    int attn_t5_min_batch = 3;  // batches of at least this many requests use the tcgen05 attention
     bool attn_t5 = false;       // its tensor maps and attributes are ready
     int attn_t5_splits = 0;     // its key split (0: chosen per launch)
     int t5_clusters[5] = {};    // co-resident clusters of s CTAs of it, s = 1..4

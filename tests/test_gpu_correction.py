@@ -58,11 +58,11 @@ def test_tiny_fp32_forward_and_denoise_with_items():
         ex.close()
 
 
-@pytest.mark.parametrize("attn", ["split", "unsplit"])
+@pytest.mark.parametrize("attn", ["split_kv", "tcgen05"])
 @pytest.mark.parametrize("B,P,C,T,N", [(2, 100, 13, 3, 2), (1, 257, 50, 4, 1), (3, 1, 1, 1, 2)])
 def test_small_bf16_items(attn, B, P, C, T, N, monkeypatch):
-    if attn == "unsplit":
-        monkeypatch.setenv("JPI_ATTN_T5_MIN_BATCH", "1")
+    # Either attention kernel at every batch: 0 turns the tcgen05 kernel off, 1 takes it from one request.
+    monkeypatch.setenv("JPI_ATTN_T5_MIN_BATCH", "1" if attn == "tcgen05" else "0")
     w = make_weights(SMALL_BF16, 2600, mod_bias_std=0.5)
     ex = make_expert(SMALL_BF16, w, max_batch=3, max_prefix=300, max_chunk=70, max_steps=3)
     try:

@@ -260,25 +260,26 @@ def test_pi05_large_m_projection_path(large_m_everywhere):
 
 
 @pytest.fixture
-def unsplit_attention_everywhere(monkeypatch):
-    """Handles created under this fixture take the unsplit tensor-core attention at any batch."""
+def tcgen05_attention_everywhere(monkeypatch):
+    """Handles created under this fixture take the tcgen05 attention at any batch (its keys split
+    four ways where the clusters fit, as chosen per launch)."""
     monkeypatch.setenv("JPI_ATTN_T5_MIN_BATCH", "1")
 
 
 @pytest.mark.parametrize("B,P,C,N", [(1, 100, 13, 2), (3, 257, 50, 1), (2, 64, 70, 3), (1, 1, 1, 2)])
-def test_small_bf16_unsplit_tensor_core_attention(unsplit_attention_everywhere, B, P, C, N):
+def test_small_bf16_tcgen05_attention(tcgen05_attention_everywhere, B, P, C, N):
     w = make_weights(SMALL_BF16, 2400)
     ex = make_expert(SMALL_BF16, w, max_batch=3, max_prefix=300, max_chunk=70, max_steps=3)
     try:
         r = make_requests(SMALL_BF16, 2401 + B, B, P, C)
         got = gpu_denoise(ex, SMALL_BF16, r, N)
         assert_close(got, oracle_denoise(SMALL_BF16, oracle.to_f64(w), r, N), SMALL_BF16,
-                     f"small bf16 unsplit attention B{B} P{P} C{C} N{N}")
+                     f"small bf16 tcgen05 attention B{B} P{P} C{C} N{N}")
     finally:
         ex.close()
 
 
-def test_small_bf16_unsplit_attention_rescales(unsplit_attention_everywhere):
+def test_small_bf16_tcgen05_attention_rescales(tcgen05_attention_everywhere):
     """O(1) modulation gains give score spreads wide enough that the running maximum moves by
     more than the lazy-rescale threshold inside a row."""
     w = make_weights(SMALL_BF16, 2410, mod_bias_std=1.0)
@@ -287,19 +288,19 @@ def test_small_bf16_unsplit_attention_rescales(unsplit_attention_everywhere):
         r = make_requests(SMALL_BF16, 2411, 2, 300, 70)
         got = gpu_denoise(ex, SMALL_BF16, r, 2)
         assert_close(got, oracle_denoise(SMALL_BF16, oracle.to_f64(w), r, 2), SMALL_BF16,
-                     "small bf16 unsplit attention high gain", max_abs_tol=3e-2)
+                     "small bf16 tcgen05 attention high gain", max_abs_tol=3e-2)
     finally:
         ex.close()
 
 
-def test_pi05_unsplit_tensor_core_attention(unsplit_attention_everywhere):
+def test_pi05_tcgen05_attention(tcgen05_attention_everywhere):
     w = make_weights(PI05, 2000)
     ex = make_expert(PI05, w, max_batch=2, max_prefix=1536, max_chunk=50, max_steps=10)
     try:
         for P in (816, 1536):
             r = make_requests(PI05, 2500 + P, 2, P, 50)
             got = gpu_denoise(ex, PI05, r, 10)
-            assert_close(got[[1]], oracle_denoise(PI05, w, r, 10, [1]), PI05, f"pi0.5 unsplit B2 P{P}")
+            assert_close(got[[1]], oracle_denoise(PI05, w, r, 10, [1]), PI05, f"pi0.5 tcgen05 attention B2 P{P}")
     finally:
         ex.close()
 
