@@ -154,6 +154,69 @@ __device__ __forceinline__ void t5_combine(const T5Args& a, size_t cta, int r_lo
     }
 }
 
+// The same combine for S = 2 or 4, where rows [r_lo, r_lo + 128 / S) are exactly the rows of
+// 4 / S softmax warps: those warps left this CTA's own partial rows in shared memory (`own`,
+// [chunk][row], and `own_ml`), and every combine thread keeps one row (tid mod 128 / S) for all its
+// chunks, so it fetches that row's (m, l) of every split together with the partials (one L2 round
+// trip, no block barrier) and forms the weights itself.
+template <int D, int S>
+__device__ __forceinline__ void t5_combine_rows(const T5Args& a, size_t cta, int split, const float4* own,
+                                                const float2* own_ml, int row0, int nrows, int b, bool ok_all,
+                                                int tid) {
+    constexpr int NOWN = T5_ROWS / S;          // rows per split: 64 or 32
+    constexpr int CSTEP = T5_THREADS / NOWN;   // chunks one pass of the block covers
+    constexpr int NI = (D / 4) / CSTEP;        // chunks per thread
+    static_assert(T5_THREADS % NOWN == 0 && (D / 4) % CSTEP == 0, "rows and chunks tile the block");
+    const int rr = tid % NOWN, cb = tid / NOWN, r_lo = split * NOWN;
+    float2 ml[S];
+    float4 v[NI][S];
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) {
+        if (sp == split) {
+            ml[sp] = own_ml[rr];
+        } else {
+            ml[sp] = __ldcg(&a.wml[(cta + sp) * T5_ROWS + r_lo + rr]);
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < NI; ++i) {
+        const int c = cb + i * CSTEP;
+#pragma unroll
+        for (int sp = 0; sp < S; ++sp) {
+            if (sp == split) v[i][sp] = own[c * NOWN + rr];
+            else v[i][sp] = __ldcg(&a.ws[((cta + sp) * (size_t)(D / 4) + c) * T5_ROWS + r_lo + rr]);
+        }
+    }
+    float M = -INFINITY;
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) M = fmaxf(M, ml[sp].x);
+    float w[S], lsum = 0.f;
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) {
+        w[sp] = ml[sp].x == -INFINITY ? 0.f : ex2(ml[sp].x - M);
+        lsum += w[sp] * ml[sp].y;
+    }
+    const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) w[sp] *= inv;
+    const int R = row0 + r_lo + rr;
+    if (R >= nrows || !ok_all) return;
+    __nv_bfloat16* orow = a.o + ((size_t)b * nrows + R) * D;
+#pragma unroll
+    for (int i = 0; i < NI; ++i) {
+        const int c = cb + i * CSTEP;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int sp = 0; sp < S; ++sp) {
+            acc.x = fmaf(w[sp], v[i][sp].x, acc.x);
+            acc.y = fmaf(w[sp], v[i][sp].y, acc.y);
+            acc.z = fmaf(w[sp], v[i][sp].z, acc.z);
+            acc.w = fmaf(w[sp], v[i][sp].w, acc.w);
+        }
+        *(uint2*)(orow + c * 4) = make_uint2(pack_bf16x2_t5(acc.x, acc.y), pack_bf16x2_t5(acc.z, acc.w));
+    }
+}
+
 template <int D>
 __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant__ CUtensorMap qmap,
                                                            const __grid_constant__ CUtensorMap kmap,
@@ -438,10 +501,19 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
     if (nsplit > 1) {
         // ---- combine the key splits of this row block through the workspace ----
         const size_t cta = ((size_t)blockIdx.y * gridDim.x + blockIdx.x) * nsplit;   // split 0 of the row block
+        // With 2 or 4 splits the rows this CTA combines are whole warps' rows: those warps keep
+        // their partials in shared memory (over the query tile; every MMA is done) and their
+        // (m, l) over the P buffers.
+        const bool rows_fixed = nsplit == 2 || nsplit == 4;
+        const int nown_fixed = rows_fixed ? T5_ROWS / nsplit : 0;
+        float4* own = reinterpret_cast<float4*>(smem);
+        float2* own_ml = reinterpret_cast<float2*>(ps);
         if (warp >= 4) {
             const int row = (warp & 3) * 32 + lane;
             const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-            float4* dst = a.ws + (cta + split) * (size_t)(D / 4) * T5_ROWS + row;
+            const bool mine = rows_fixed && row / nown_fixed == split;   // warp-uniform
+            float4* dst = mine ? own + (row - split * nown_fixed) : a.ws + (cta + split) * (size_t)(D / 4) * T5_ROWS + row;
+            const int stride = mine ? nown_fixed : T5_ROWS;
 #pragma unroll 1
             for (int c0 = 0; c0 < D; c0 += 32) {
                 uint32_t r[2][16];
@@ -450,11 +522,12 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
                 ptx::tmem_ld_wait();
 #pragma unroll
                 for (int v = 0; v < 8; ++v)
-                    dst[(size_t)(c0 / 4 + v) * T5_ROWS] =
+                    dst[(size_t)(c0 / 4 + v) * stride] =
                         make_float4(__uint_as_float(r[v >> 2][4 * (v & 3)]), __uint_as_float(r[v >> 2][4 * (v & 3) + 1]),
                                     __uint_as_float(r[v >> 2][4 * (v & 3) + 2]), __uint_as_float(r[v >> 2][4 * (v & 3) + 3]));
             }
-            a.wml[(cta + split) * T5_ROWS + row] = make_float2(x_m, x_l);
+            if (mine) own_ml[row - split * nown_fixed] = make_float2(x_m, x_l);
+            else a.wml[(cta + split) * T5_ROWS + row] = make_float2(x_m, x_l);
         }
         // Every split's rows are in the workspace (the barrier orders global memory at cluster scope;
         // the reads below go to L2, past this SM's L1).
@@ -467,9 +540,9 @@ __global__ void __launch_bounds__(T5_THREADS, 1) k_attn_t5(const __grid_constant
         const int nown = max(0, min(T5_ROWS, r_lo + rps) - r_lo);
         const bool ok_all = *flag == 0;   // written before the cluster barrier
         // The launcher splits 2, 3 or 4 ways.
-        if (nsplit == 2) t5_combine<D, 2>(a, cta, r_lo, nown, wsm, row0, nrows, b, ok_all, tid);
-        else if (nsplit == 3) t5_combine<D, 3>(a, cta, r_lo, nown, wsm, row0, nrows, b, ok_all, tid);
-        else t5_combine<D, 4>(a, cta, r_lo, nown, wsm, row0, nrows, b, ok_all, tid);
+        if (nsplit == 2) t5_combine_rows<D, 2>(a, cta, split, own, own_ml, row0, nrows, b, ok_all, tid);
+        else if (nsplit == 4) t5_combine_rows<D, 4>(a, cta, split, own, own_ml, row0, nrows, b, ok_all, tid);
+        else t5_combine<D, 3>(a, cta, r_lo, nown, wsm, row0, nrows, b, ok_all, tid);
     }
 
     ptx::tc_fence_before();
