@@ -1,7 +1,8 @@
 // Launchers of the tcgen05 attention kernel (attn_t5_kernel.cuh) for the expert's batched
 // denoise: one CTA per 128 query rows of a request and key split. The keys are split four ways
-// when the (row blocks x requests) clusters of 4 CTAs are co-resident, else not at all: 4 at 3-9
-// requests, 1 from 10 (pi0.5 shapes: 4 row blocks per request).
+// when the (row blocks x requests) clusters of 4 CTAs are co-resident, else two ways when clusters
+// of 2 are, else not at all (pi0.5 shapes, 4 row blocks per request: 4 at 3-9 requests, 2 at
+// 10-19, 1 from 20).
 
 #include "jpi_internal.h"
 #include "ptx.h"
@@ -33,10 +34,12 @@ int t5_splits(const jpi_handle* h, int blocks, int nb_all) {
         while (s > 1 && !t5_fits(h, blocks, s)) --s;
         return s;
     }
-    // Four splits where the clusters fit in one wave, else none: on pi0.5 shapes (14 key blocks)
-    // two splits measured no faster than one, and three or four past one wave of clusters took
-    // twice as long.
-    return nb_all >= T5_MAX_SPLIT && t5_fits(h, blocks, T5_MAX_SPLIT) ? T5_MAX_SPLIT : 1;
+    // Four splits, else two, where the clusters fit in one wave; else none. A cluster past one
+    // wave makes the launch take twice as long, and three splits pack fewer clusters than two or
+    // four and keep no rows on chip.
+    for (int s = T5_MAX_SPLIT; s >= 2; s /= 2)
+        if (nb_all >= s && t5_fits(h, blocks, s)) return s;
+    return 1;
 }
 
 template <int D>
