@@ -37,11 +37,11 @@ OP_NAMES = {2: "norm+qkv+rope", 3: "attention", 4: "o_proj+residual", 5: "norm+g
 # valid only while the kernel sources hash to `source_sha256`.
 NCU_TRAFFIC = {
     # profiles/layer_kernels_pi05_forward.md (layer 1 of one eager forward, batch 1, P 816).
-    "norm+qkv+rope": {"bytes": 5492224, "source_sha256": "b767bbcf1dfc9c66"},
-    "attention": {"bytes": 1181696, "source_sha256": "b767bbcf1dfc9c66"},
-    "o_proj+residual": {"bytes": 4697600, "source_sha256": "b767bbcf1dfc9c66"},
-    "norm+gate_up+geglu": {"bytes": 16961792, "source_sha256": "b767bbcf1dfc9c66"},
-    "down_proj+residual": {"bytes": 9133568, "source_sha256": "b767bbcf1dfc9c66"},
+    "norm+qkv+rope": {"bytes": 5489664, "source_sha256": "eb98c3678ac8178d"},
+    "attention": {"bytes": 1179648, "source_sha256": "eb98c3678ac8178d"},
+    "o_proj+residual": {"bytes": 4695808, "source_sha256": "eb98c3678ac8178d"},
+    "norm+gate_up+geglu": {"bytes": 16959744, "source_sha256": "eb98c3678ac8178d"},
+    "down_proj+residual": {"bytes": 9131776, "source_sha256": "eb98c3678ac8178d"},
 }
 
 
