@@ -34,14 +34,14 @@ OP_NAMES = {2: "norm+qkv+rope", 3: "attention", 4: "o_proj+residual", 5: "norm+g
             6: "down_proj+residual"}
 
 # DRAM bytes per launch from an ncu capture (dram__bytes_read.sum + dram__bytes_write.sum),
-# valid only while the kernel sources hash to `source_sha256`.
+# valid only while TRAFFIC_SOURCES hash to `source_sha256`.
 NCU_TRAFFIC = {
     # profiles/layer_kernels_pi05_forward.md (layer 1 of one eager forward, batch 1, P 816).
-    "norm+qkv+rope": {"bytes": 5489664, "source_sha256": "eb98c3678ac8178d"},
-    "attention": {"bytes": 1179648, "source_sha256": "eb98c3678ac8178d"},
-    "o_proj+residual": {"bytes": 4695808, "source_sha256": "eb98c3678ac8178d"},
-    "norm+gate_up+geglu": {"bytes": 16959744, "source_sha256": "eb98c3678ac8178d"},
-    "down_proj+residual": {"bytes": 9131776, "source_sha256": "eb98c3678ac8178d"},
+    "norm+qkv+rope": {"bytes": 5489664, "source_sha256": "39321630f8ff0a0e"},
+    "attention": {"bytes": 1179648, "source_sha256": "39321630f8ff0a0e"},
+    "o_proj+residual": {"bytes": 4695808, "source_sha256": "39321630f8ff0a0e"},
+    "norm+gate_up+geglu": {"bytes": 16959744, "source_sha256": "39321630f8ff0a0e"},
+    "down_proj+residual": {"bytes": 9131776, "source_sha256": "39321630f8ff0a0e"},
 }
 
 
@@ -53,10 +53,17 @@ EXPERT_SOURCES = ("api.cu", "attn_t5.cu", "attn_t5_kernel.cuh", "attn_tc.cu", "g
 CORRECTION_SOURCES = ("corr.cu",)
 
 
-def source_sha() -> str:
+# The sources the five batch-1 layer kernels of NCU_TRAFFIC are built and launched from (the
+# projection kernel, the split-KV attention, their launcher and shared headers): their counters
+# stay valid while these are unchanged, whatever changes elsewhere (the large-batch attention).
+TRAFFIC_SOURCES = ("attn_tc.cu", "gemm_big.cuh", "gemm_kernel.cuh", "jpi_internal.h", "ptx.h", "tc_path.cu",
+                   "tc_path.h")
+
+
+def source_sha(files=EXPERT_SOURCES) -> str:
     d = os.path.join(ROOT, "paper_2607_12659_gb300", "csrc")
     h = hashlib.sha256()
-    for f in sorted(EXPERT_SOURCES):
+    for f in sorted(files):
         h.update(open(os.path.join(d, f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -384,7 +391,8 @@ def our_arm(args):
     achieved = dom_bytes / (op_ms[dom] * 1e-3) / 1e9
     sha = source_sha()
     tr = NCU_TRAFFIC.get(OP_NAMES[dom])
-    traffic = tr["bytes"] if tr and tr.get("source_sha256") == sha and default_workload else None
+    traffic = (tr["bytes"] if tr and tr.get("source_sha256") == source_sha(TRAFFIC_SOURCES) and default_workload
+               else None)
 
     n_kernels = jpi.jpi_graph_kernel_count(ex.handle, B, C, N)
     alg = algorithmic_bytes(cfg, B, P, C, N, args.items)
