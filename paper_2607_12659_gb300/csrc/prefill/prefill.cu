@@ -2,14 +2,15 @@
 // Sec. 4.3): Gemma-shaped blocks over the prefix tokens, writing each layer's rotated keys and
 // values straight into the action expert's KV store.
 //
-// Every product here is a plain GEMM with batch * prefix rows (816 per request): the Q/K/V, output,
-// gate/up and down projections, and per request the scores q K^T (all heads stacked as rows,
-// since the single KV head is shared) and the probabilities times V. They run on this file's
-// tcgen05 GEMM (bf16 operands by bulk tensor copies, fp32 accumulation in TMEM, see k_pf_gemm);
-// the residual stream stays fp32 and the two residual projections accumulate into it in place.
-// This file's other kernels do the rest: RMSNorm to a bf16 operand, rotary coding of q and k from
-// a table built once in double precision (with k and v scattered into the store), the row
-// softmax, the per-request transpose of V, and GeGLU.
+// The Q/K/V, output, gate/up and down projections are plain GEMMs with batch * prefix rows (816
+// per request) on this file's tcgen05 GEMM (bf16 operands by bulk tensor copies, fp32
+// accumulation in TMEM, see k_pf_gemm); the residual stream stays fp32 and the two residual
+// projections accumulate into it in place. Attention (all heads stacked as query rows, since the
+// single KV head is shared) runs on the expert's tcgen05 attention kernel with every key visible;
+// for head dims or store strides that kernel does not take, it falls back to per-request GEMMs:
+// the scores q K^T, a row softmax, V transposed, and the probabilities times V. This file's other
+// kernels do the rest: RMSNorm to a bf16 operand, rotary coding of q and k from a table built
+// once in double precision (with k and v scattered into the store), and GeGLU.
 
 #include <cuda.h>
 #include <cudaTypedefs.h>
