@@ -99,13 +99,39 @@ def test_reference_arm_json_line():
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
 
 
-def test_every_kernel_source_is_accounted_for_by_the_traffic_hash():
-    # A source the measured kernels are built from must change `source_sha` (and so null the
-    # recorded DRAM traffic) when it changes; only the correction module's files stay outside.
+def test_every_kernel_source_is_accounted_for_by_the_source_hash():
+    # Every source of the expert's kernels changes `source_sha`, the build's identity in the bench
+    # line; only the correction module's files stay outside.
     d = os.path.join(bench.ROOT, "paper_2607_12659_gb300", "csrc")
     files = {f for f in os.listdir(d) if f.endswith((".cu", ".cuh", ".h"))}
     assert files == set(bench.EXPERT_SOURCES) | set(bench.CORRECTION_SOURCES)
     assert not set(bench.EXPERT_SOURCES) & set(bench.CORRECTION_SOURCES)
+
+
+def _local_include_closure(d, roots):
+    seen, todo = set(), list(roots)
+    while todo:
+        f = todo.pop()
+        if f in seen or not os.path.exists(os.path.join(d, f)):
+            continue   # headers outside the kernel directory (the public ABI header) are not hashed
+        seen.add(f)
+        for line in open(os.path.join(d, f)):
+            line = line.strip()
+            if line.startswith('#include "'):
+                todo.append(line.split('"')[1])
+    return seen
+
+
+def test_traffic_hash_covers_the_batch1_layer_kernels_and_their_headers():
+    # The recorded DRAM traffic of the five batch-1 layer kernels (the projection kernel in
+    # gemm_kernel.cuh, launched from tc_path.cu, and the split-KV attention in attn_tc.cu) stays
+    # valid exactly while these files and every local header they include are unchanged.
+    d = os.path.join(bench.ROOT, "paper_2607_12659_gb300", "csrc")
+    closure = _local_include_closure(d, ["tc_path.cu", "attn_tc.cu"])
+    assert closure == set(bench.TRAFFIC_SOURCES)
+    assert set(bench.TRAFFIC_SOURCES) <= set(bench.EXPERT_SOURCES)
+    for entry in bench.NCU_TRAFFIC.values():
+        assert len(entry["source_sha256"]) == 16 and entry["bytes"] > 0
 
 
 def test_correction_bytes_from_the_weight_shapes():
